@@ -1,0 +1,496 @@
+/*
+ * K-interval attention -- plain fp64 CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the tests, the package smoke check and the
+ * benchmark's CPU-baseline leg may load this library.  It shares no code with
+ * the CUDA path and is written for a reader who checks it against the paper
+ * ("Pretraining Transformers with Quantized Softmax in Attention"):
+ *
+ *   Sec. 3 "Objects and calibration" and App. A  -> scores, MinMax / FWM grids,
+ *                                                  interval index r, position t
+ *   Sec. 3 "Reconstruction" and App. A LERP/Nearest -> w^L, w^N, bin index l
+ *   App. A "Normalization"                        -> P = w / sum w, O = P V
+ *   App. B "Normalization Jacobian"               -> gamma = (g - <g>_P) / W
+ *   App. B "LERP own-score slope"                 -> Delta (secant)
+ *   Eq. (calgrad), Eq. (full), App. B "Full calibration gradient (MinMax)"
+ *   App. B "FWM" paragraph                        -> FWM calibration gradient
+ *   Eq. (wste) / Eq. (pste), App. B Weight-STE / Prob-STE paragraphs
+ *   App. B "Detach (legacy)"                      -> detached extrema
+ *   App. B "Softmax", App. A "Softmax"            -> the comparator
+ *   Table "Edge cases" (App. A)                   -> degenerate rows, ties,
+ *                                                  midpoint rounding, window edge
+ *
+ * Everything is computed per causal row in fp64 from the fp32 inputs (fp64
+ * inputs in the -DKOR_F64_INPUT build), with
+ * plain loops and no blocking.  Rows are independent; heads (b, h) are spread
+ * over POSIX threads, one head per thread at a time.
+ *
+ * Readings of points the paper leaves open (each is listed with its reason in
+ * the design notes of the repository):
+ *   - the score scale 1/sqrt(d) is applied once, inside the operator;
+ *   - tau is a parameter (the paper trains only tau = 6);
+ *   - ties among extrema split the extremum gradient evenly over the tie set;
+ *   - the Nearest midpoint t = 1/2 rounds up; the FWM cutoff is strict (z < -tau);
+ *   - the degenerate MinMax branch is M - m <= 1e-12 (fp64 here);
+ *   - the forward of Nearest returns P^N = w^N / W^N directly (strict hard forward).
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#include <unistd.h>
+
+#include "kint_oracle.h"
+
+#define DEGENERATE_EPS 1e-12
+
+typedef struct {
+  const kor_params* p;
+  const kor_in *Q, *K, *V, *dO;
+  const kor_fwd_out* fo;
+  const kor_bwd_out* bo;
+  const kor_override* ov;
+  int do_bwd;
+  int next_bh;
+  pthread_mutex_t lock;
+} job_t;
+
+/* Per-thread row workspace, sized T. */
+typedef struct {
+  double *s, *z, *t, *wL, *wN, *P, *Pst, *g, *dS;
+  int *r, *l, *tail, *code_l, *code_r;
+  double* e; /* K+1 grid values e^{b_r} */
+  double* margin;
+  /* scalars of the current row */
+  double M, m, h, b0, W_N, W_L, Wst;
+  int amax, amin, nmax, nmin, degenerate, n;
+} row_t;
+
+static double dot_in(const kor_in* a, const kor_in* b, int d) {
+  double acc = 0.0;
+  for (int k = 0; k < d; ++k) acc += (double)a[k] * (double)b[k];
+  return acc;
+}
+
+static double clampd(double x, double lo, double hi) { return x < lo ? lo : (x > hi ? hi : x); }
+
+/* Distance from u to the nearest point of {n + 1/2 : n = 0..K-1} (Nearest bin
+ * edges) and of {1..K-1} (LERP interval switches). */
+static double decision_distance_u(double u, int K) {
+  double best = INFINITY;
+  for (int n = 0; n < K; ++n) {
+    double dh = fabs(u - (n + 0.5));
+    if (dh < best) best = dh;
+    if (n >= 1) {
+      double di = fabs(u - n);
+      if (di < best) best = di;
+    }
+  }
+  return best;
+}
+
+/*
+ * Forward quantities of causal row i of head bh (App. A).  Fills R.
+ */
+static void row_forward(const job_t* J, int bh, int i, row_t* R) {
+  const kor_params* p = J->p;
+  const int T = p->T, d = p->d, K = p->Kint;
+  const kor_in* Qi = J->Q + ((size_t)bh * T + i) * d;
+  const kor_in* Kh = J->K + (size_t)bh * T * d;
+  const double scale = 1.0 / sqrt((double)d);
+  const int n = i + 1; /* causal: keys 0..i are valid, later keys get w = 0 */
+  R->n = n;
+
+  /* Scores S = Q K^T / sqrt(d_h)  (Sec. 3, App. A) */
+  for (int j = 0; j < n; ++j) R->s[j] = dot_in(Qi, Kh + (size_t)j * d, d) * scale;
+
+  /* Row extrema; lowest index among ties, and the size of the tie set. */
+  int amax = 0, amin = 0;
+  for (int j = 1; j < n; ++j) {
+    if (R->s[j] > R->s[amax]) amax = j;
+    if (R->s[j] < R->s[amin]) amin = j;
+  }
+  if (J->ov && J->ov->amax) amax = J->ov->amax[(size_t)bh * T + i];
+  if (J->ov && J->ov->amin) amin = J->ov->amin[(size_t)bh * T + i];
+  R->M = R->s[amax];
+  R->m = R->s[amin];
+  R->amax = amax;
+  R->amin = amin;
+  R->nmax = 0;
+  R->nmin = 0;
+  for (int j = 0; j < n; ++j) {
+    if (R->s[j] == R->M) R->nmax++;
+    if (R->s[j] == R->m) R->nmin++;
+  }
+
+  R->degenerate = 0;
+  R->h = 0.0;
+  R->b0 = 0.0;
+  for (int j = 0; j < n; ++j) {
+    R->z[j] = R->s[j] - R->M;
+    R->tail[j] = 0;
+    R->r[j] = 0;
+    R->l[j] = 0;
+    R->t[j] = 0.0;
+    R->margin[j] = INFINITY;
+    R->code_l[j] = KOR_CODE_NOGRID;
+    R->code_r[j] = KOR_CODE_NOGRID;
+  }
+
+  if (p->calib == KOR_SOFTMAX) {
+    /* w^E_j = e^{z_j} (App. A, Softmax) */
+    for (int j = 0; j < n; ++j) {
+      R->wL[j] = exp(R->z[j]);
+      R->wN[j] = R->wL[j];
+    }
+  } else if (p->calib == KOR_MINMAX && (R->M - R->m) <= DEGENERATE_EPS) {
+    /* Degenerate MinMax row: weights 1, P uniform (Table "Edge cases"). */
+    R->degenerate = 1;
+    for (int j = 0; j < n; ++j) {
+      R->wL[j] = 1.0;
+      R->wN[j] = 1.0;
+    }
+  } else {
+    /* Grid.  MinMax: z_min = m - M, h = (M - m)/K, b_r = z_min + r h.
+     *        FWM:    h = tau/K, b_r = -tau + r h.                     */
+    if (p->calib == KOR_MINMAX) {
+      R->b0 = R->m - R->M;
+      R->h = (R->M - R->m) / K;
+    } else {
+      R->b0 = -p->tau;
+      R->h = p->tau / K;
+    }
+    const double h = R->h, b0 = R->b0;
+    for (int rr = 0; rr <= K; ++rr) R->e[rr] = exp(b0 + rr * h);
+
+    for (int j = 0; j < n; ++j) {
+      const double z = R->z[j];
+      int tail = 0;
+      double zc = z;
+      if (p->calib == KOR_FWM) {
+        tail = (z < -p->tau);        /* zero tail below the window, strict */
+        zc = clampd(z, -p->tau, 0.0); /* z~ = clip(z, -tau, 0) */
+      }
+      /* r = clip(floor((z - b_0)/h), 0, K-1), t = clip((z - b_r)/h, 0, 1) */
+      const double u = (zc - b0) / h;
+      int r = (int)floor(u);
+      if (r < 0) r = 0;
+      if (r > K - 1) r = K - 1;
+      double t = clampd((zc - (b0 + r * h)) / h, 0.0, 1.0);
+      /* Nearest grid centre: l = r + [t >= 1/2] (midpoint rounds up) */
+      int l = r + (t >= 0.5 ? 1 : 0);
+
+      /* Distance to the nearest decision boundary, in score units. */
+      double mg = INFINITY;
+      if (p->calib == KOR_FWM) mg = fabs(z + p->tau);
+      if (!tail) {
+        double du = decision_distance_u(u, K) * h;
+        if (du < mg) mg = du;
+      }
+      R->margin[j] = mg;
+
+      if (J->ov && J->ov->bins) {
+        /* Decision-aligned re-run: take the given bin / interval / tail choice. */
+        const size_t idx = ((size_t)bh * T + i) * T + j;
+        const int cb = J->ov->bins[idx];
+        tail = (cb == KOR_CODE_TAIL);
+        if (!tail) {
+          l = cb;
+          if (J->ov->ivals) r = J->ov->ivals[idx];
+          t = clampd((zc - (b0 + r * h)) / h, 0.0, 1.0);
+        }
+      }
+      R->tail[j] = tail;
+      R->r[j] = r;
+      R->t[j] = t;
+      R->l[j] = l;
+      if (tail) {
+        R->wL[j] = 0.0;
+        R->wN[j] = 0.0;
+        R->code_l[j] = KOR_CODE_TAIL;
+        R->code_r[j] = KOR_CODE_TAIL;
+      } else {
+        R->wL[j] = (1.0 - t) * R->e[r] + t * R->e[r + 1]; /* LERP */
+        R->wN[j] = R->e[l];                               /* Nearest */
+        R->code_l[j] = l;
+        R->code_r[j] = r;
+      }
+    }
+  }
+
+  /* Normalization: W = sum_l w_l, P = w / W (App. A). */
+  double WN = 0.0, WL = 0.0;
+  for (int j = 0; j < n; ++j) {
+    WN += R->wN[j];
+    WL += R->wL[j];
+  }
+  R->W_N = WN;
+  R->W_L = WL;
+  const int hard = (p->calib != KOR_SOFTMAX && p->recon == KOR_NEAREST);
+  for (int j = 0; j < n; ++j) R->P[j] = hard ? R->wN[j] / WN : R->wL[j] / WL;
+}
+
+static void fwd_row_outputs(const job_t* J, int bh, int i, row_t* R) {
+  const kor_params* p = J->p;
+  const kor_fwd_out* fo = J->fo;
+  const int T = p->T, d = p->d, n = R->n;
+  const size_t row = (size_t)bh * T + i;
+  const kor_in* Vh = J->V + (size_t)bh * T * d;
+  const int hard = (p->calib != KOR_SOFTMAX && p->recon == KOR_NEAREST);
+  if (fo->O) {
+    double* O = fo->O + row * d;
+    for (int k = 0; k < d; ++k) O[k] = 0.0;
+    for (int j = 0; j < n; ++j)
+      for (int k = 0; k < d; ++k) O[k] += R->P[j] * (double)Vh[(size_t)j * d + k];
+  }
+  if (fo->OL) {
+    double* OL = fo->OL + row * d;
+    for (int k = 0; k < d; ++k) OL[k] = 0.0;
+    for (int j = 0; j < n; ++j)
+      for (int k = 0; k < d; ++k) OL[k] += (R->wL[j] / R->W_L) * (double)Vh[(size_t)j * d + k];
+  }
+  if (fo->M) fo->M[row] = R->M;
+  if (fo->m) fo->m[row] = R->m;
+  if (fo->amax) fo->amax[row] = R->amax;
+  if (fo->amin) fo->amin[row] = R->amin;
+  if (fo->nmax) fo->nmax[row] = R->nmax;
+  if (fo->nmin) fo->nmin[row] = R->nmin;
+  if (fo->W) fo->W[row] = hard ? R->W_N : R->W_L;
+  if (fo->WL) fo->WL[row] = R->W_L;
+  if (fo->bins || fo->ivals || fo->margin) {
+    for (int j = 0; j < T; ++j) {
+      const size_t idx = row * T + j;
+      const int valid = j < n;
+      if (fo->bins) fo->bins[idx] = (uint8_t)(valid ? R->code_l[j] : KOR_CODE_MASKED);
+      if (fo->ivals) fo->ivals[idx] = (uint8_t)(valid ? R->code_r[j] : KOR_CODE_MASKED);
+      if (fo->margin) fo->margin[idx] = valid ? R->margin[j] : INFINITY;
+    }
+  }
+  if (fo->row_margin) {
+    /* Gap between the extremum and the runner-up (a different score value),
+     * i.e. how far the arg-extremum decision is from flipping. */
+    double gmax = INFINITY, gmin = INFINITY;
+    for (int j = 0; j < n; ++j) {
+      if (R->s[j] != R->M && R->M - R->s[j] < gmax) gmax = R->M - R->s[j];
+      if (R->s[j] != R->m && R->s[j] - R->m < gmin) gmin = R->s[j] - R->m;
+    }
+    fo->row_margin[row] = gmax < gmin ? gmax : gmin;
+  }
+}
+
+/*
+ * Backward of causal row i (App. B).  Adds this row's contributions to
+ * dK, dV (rows 0..i of the head) and writes dQ_i.
+ */
+static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
+  const kor_params* p = J->p;
+  const kor_bwd_out* bo = J->bo;
+  const int T = p->T, d = p->d, K = p->Kint, n = R->n;
+  const size_t row = (size_t)bh * T + i;
+  const kor_in* Qi = J->Q + row * d;
+  const kor_in* dOi = J->dO + row * d;
+  const kor_in* Kh = J->K + (size_t)bh * T * d;
+  const kor_in* Vh = J->V + (size_t)bh * T * d;
+  const double scale = 1.0 / sqrt((double)d);
+
+  /* Upstream gradient at the probabilities: g_j = dO_i . V_j */
+  for (int j = 0; j < n; ++j) R->g[j] = dot_in(dOi, Vh + (size_t)j * d, d);
+
+  double cM = 0.0, cm = 0.0;
+  if (p->calib == KOR_SOFTMAX) {
+    /* dL/ds_j = P_j (g_j - sum_i P_i g_i)  (App. B, Softmax) */
+    double D = 0.0;
+    for (int j = 0; j < n; ++j) D += R->P[j] * R->g[j];
+    for (int j = 0; j < n; ++j) R->dS[j] = R->P[j] * (R->g[j] - D);
+  } else if (R->degenerate) {
+    /* Degenerate MinMax row: zero gradient (Table "Edge cases"). */
+    for (int j = 0; j < n; ++j) R->dS[j] = 0.0;
+  } else {
+    /* Point of the normalization Jacobian:
+     *   Nearest + Weight-STE: (P^N, W^N)   Eq. (wste)
+     *   Nearest + Prob-STE:   (P^L, W^L)   Eq. (pste)
+     *   LERP:                 (P^L, W^L)   exact Jacobian                 */
+    const int at_hard = (p->recon == KOR_NEAREST && p->ste == KOR_WEIGHT);
+    const double Wst = at_hard ? R->W_N : R->W_L;
+    double D = 0.0;
+    for (int j = 0; j < n; ++j) {
+      R->Pst[j] = at_hard ? R->wN[j] / R->W_N : R->wL[j] / R->W_L;
+      D += R->Pst[j] * R->g[j];
+    }
+    const double h = R->h;
+    for (int j = 0; j < n; ++j) {
+      if (R->tail[j]) {
+        R->dS[j] = 0.0; /* mask and clamp: zero gradient */
+        continue;
+      }
+      const int r = R->r[j];
+      const double t = R->t[j];
+      const double gamma = (R->g[j] - D) / Wst;           /* normalization Jacobian */
+      const double Delta = (R->e[r + 1] - R->e[r]) / h;   /* secant slope */
+      R->dS[j] = gamma * Delta;                           /* own-score term */
+      if (p->grad == KOR_FULL) {
+        if (p->calib == KOR_MINMAX) {
+          /* Eq. (calgrad) */
+          const double rho = (r + t) / K;
+          const double X = ((1.0 - t) * r * R->e[r] + t * (r + 1) * R->e[r + 1]) / K;
+          const double dwdM = -R->wL[j] - Delta * rho + X;
+          const double dwdm = -Delta * (1.0 - rho) + R->wL[j] - X;
+          cM += gamma * dwdM;
+          cm += gamma * dwdm;
+        } else {
+          /* FWM: dw/dM = -Delta for in-window keys, no m term. */
+          cM += gamma * (-Delta);
+        }
+      }
+    }
+    if (p->grad == KOR_FULL) {
+      /* Eq. (full): the extremum terms go to the arg-max / arg-min keys, split
+       * evenly among ties. */
+      for (int j = 0; j < n; ++j) {
+        if (R->s[j] == R->M) R->dS[j] += cM / R->nmax;
+        if (p->calib == KOR_MINMAX && R->s[j] == R->m) R->dS[j] += cm / R->nmin;
+      }
+    }
+  }
+
+  /* dQ_i = sum_j dS_j K_j / sqrt(d); dK_j += dS_j Q_i / sqrt(d); dV_j += P_j dO_i */
+  double* dQi = bo->dQ ? bo->dQ + row * d : NULL;
+  if (dQi)
+    for (int k = 0; k < d; ++k) dQi[k] = 0.0;
+  double dsum = 0.0, dabs = 0.0;
+  for (int j = 0; j < n; ++j) {
+    const double ds = R->dS[j];
+    dsum += ds;
+    dabs += fabs(ds);
+    const kor_in* Kj = Kh + (size_t)j * d;
+    if (dQi)
+      for (int k = 0; k < d; ++k) dQi[k] += ds * (double)Kj[k] * scale;
+    if (bo->dK) {
+      double* dKj = bo->dK + ((size_t)bh * T + j) * d;
+      for (int k = 0; k < d; ++k) dKj[k] += ds * (double)Qi[k] * scale;
+    }
+    if (bo->dV) {
+      double* dVj = bo->dV + ((size_t)bh * T + j) * d;
+      for (int k = 0; k < d; ++k) dVj[k] += R->P[j] * (double)dOi[k];
+    }
+  }
+  if (bo->dS) {
+    double* out = bo->dS + row * T;
+    for (int j = 0; j < T; ++j) out[j] = j < n ? R->dS[j] : 0.0;
+  }
+  if (bo->cM) bo->cM[row] = cM;
+  if (bo->cm) bo->cm[row] = cm;
+  if (bo->dsum) bo->dsum[row] = dsum;
+  if (bo->dabs) bo->dabs[row] = dabs;
+}
+
+static int row_alloc(row_t* R, int T, int K) {
+  memset(R, 0, sizeof(*R));
+  double** dptrs[] = {&R->s, &R->z, &R->t, &R->wL, &R->wN, &R->P, &R->Pst, &R->g, &R->dS, &R->margin};
+  for (size_t k = 0; k < sizeof(dptrs) / sizeof(dptrs[0]); ++k) {
+    *dptrs[k] = (double*)calloc((size_t)T, sizeof(double));
+    if (!*dptrs[k]) return -1;
+  }
+  int** iptrs[] = {&R->r, &R->l, &R->tail, &R->code_l, &R->code_r};
+  for (size_t k = 0; k < sizeof(iptrs) / sizeof(iptrs[0]); ++k) {
+    *iptrs[k] = (int*)calloc((size_t)T, sizeof(int));
+    if (!*iptrs[k]) return -1;
+  }
+  R->e = (double*)calloc((size_t)K + 2, sizeof(double));
+  return R->e ? 0 : -1;
+}
+
+static void row_free(row_t* R) {
+  double* dp[] = {R->s, R->z, R->t, R->wL, R->wN, R->P, R->Pst, R->g, R->dS, R->margin, R->e};
+  for (size_t k = 0; k < sizeof(dp) / sizeof(dp[0]); ++k) free(dp[k]);
+  int* ip[] = {R->r, R->l, R->tail, R->code_l, R->code_r};
+  for (size_t k = 0; k < sizeof(ip) / sizeof(ip[0]); ++k) free(ip[k]);
+}
+
+static void* worker(void* arg) {
+  job_t* J = (job_t*)arg;
+  const kor_params* p = J->p;
+  row_t R;
+  if (row_alloc(&R, p->T, p->Kint) != 0) {
+    row_free(&R);
+    return (void*)1;
+  }
+  const int nbh = p->B * p->H;
+  for (;;) {
+    pthread_mutex_lock(&J->lock);
+    const int bh = J->next_bh++;
+    pthread_mutex_unlock(&J->lock);
+    if (bh >= nbh) break;
+    if (J->do_bwd) {
+      const size_t base = (size_t)bh * p->T * p->d;
+      if (J->bo->dK) memset(J->bo->dK + base, 0, sizeof(double) * p->T * p->d);
+      if (J->bo->dV) memset(J->bo->dV + base, 0, sizeof(double) * p->T * p->d);
+    }
+    for (int i = 0; i < p->T; ++i) {
+      row_forward(J, bh, i, &R);
+      if (J->do_bwd)
+        bwd_row(J, bh, i, &R);
+      else
+        fwd_row_outputs(J, bh, i, &R);
+    }
+  }
+  row_free(&R);
+  return NULL;
+}
+
+static int check_params(const kor_params* p) {
+  if (!p || p->B < 1 || p->H < 1 || p->T < 1 || p->d < 1) return -1;
+  if (p->calib < 0 || p->calib > 2) return -1;
+  if (p->calib != KOR_SOFTMAX && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
+  if (p->calib == KOR_FWM && !(p->tau > 0.0)) return -1;
+  if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 1) return -1;
+  return 0;
+}
+
+static int run(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_in* V, const kor_in* dO,
+               const kor_fwd_out* fo, const kor_bwd_out* bo, const kor_override* ov) {
+  if (check_params(p) != 0) return -1;
+  /* the uint8 decision codes hold l in 0..K and need K + 1 < KOR_CODE_NOGRID */
+  if (fo && (fo->bins || fo->ivals) && p->Kint >= KOR_CODE_NOGRID - 1) return -1;
+  job_t J;
+  memset(&J, 0, sizeof(J));
+  J.p = p;
+  J.Q = Q;
+  J.K = K;
+  J.V = V;
+  J.dO = dO;
+  J.fo = fo;
+  J.bo = bo;
+  J.ov = ov;
+  J.do_bwd = bo != NULL;
+  pthread_mutex_init(&J.lock, NULL);
+  int nt = p->nthreads > 0 ? p->nthreads : (int)sysconf(_SC_NPROCESSORS_ONLN);
+  if (nt < 1) nt = 1;
+  if (nt > p->B * p->H) nt = p->B * p->H;
+  pthread_t* th = (pthread_t*)calloc((size_t)nt, sizeof(pthread_t));
+  int rc = 0;
+  for (int k = 0; k < nt; ++k) pthread_create(&th[k], NULL, worker, &J);
+  for (int k = 0; k < nt; ++k) {
+    void* ret = NULL;
+    pthread_join(th[k], &ret);
+    if (ret) rc = -2;
+  }
+  free(th);
+  pthread_mutex_destroy(&J.lock);
+  return rc;
+}
+
+int kor_forward(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_in* V, const kor_fwd_out* out,
+                const kor_override* ov) {
+  if (!Q || !K || !V || !out) return -1;
+  return run(p, Q, K, V, NULL, out, NULL, ov);
+}
+
+int kor_backward(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_in* V, const kor_in* dO,
+                 const kor_bwd_out* out, const kor_override* ov) {
+  if (!Q || !K || !V || !dO || !out) return -1;
+  return run(p, Q, K, V, dO, NULL, out, ov);
+}
+
+int kor_hardware_threads(void) { return (int)sysconf(_SC_NPROCESSORS_ONLN); }

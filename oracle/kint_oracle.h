@@ -1,0 +1,94 @@
+/*
+ * K-interval attention -- fp64 CPU oracle (TEST INFRASTRUCTURE ONLY).
+ * Interface of oracle/kint_oracle.c.  Not used by, and not sharing anything
+ * with, the CUDA library.
+ *
+ * Inputs are row-major [B, H, T, d] arrays (Q, K, V, dO); every output is
+ * fp64 (or int32 / uint8 for decisions), row-major, caller-allocated.  Any
+ * output pointer may be NULL.  Attention is causal: row i sees keys 0..i.
+ */
+#ifndef KINT_ORACLE_H
+#define KINT_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element type of Q, K, V, dO.  The default build takes fp32 (the operator's
+ * input type); building with -DKOR_F64_INPUT gives an otherwise identical
+ * library taking fp64 inputs, used by the finite-difference checks. */
+#ifdef KOR_F64_INPUT
+typedef double kor_in;
+#else
+typedef float kor_in;
+#endif
+
+enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2 };
+enum { KOR_LERP = 0, KOR_NEAREST = 1 };
+enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
+enum { KOR_FULL = 0, KOR_DETACH = 1 };
+
+/* Codes of the per-key decision arrays (bins: Nearest index l in 0..K,
+ * ivals: interval index r in 0..K-1). */
+enum { KOR_CODE_NOGRID = 253, KOR_CODE_TAIL = 254, KOR_CODE_MASKED = 255 };
+
+typedef struct {
+  int B, H, T, d;
+  int Kint;   /* K, number of intervals */
+  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX */
+  double tau; /* FWM window in nats */
+  int recon;  /* KOR_LERP / KOR_NEAREST */
+  int ste;    /* KOR_WEIGHT / KOR_PROB (ignored for LERP) */
+  int grad;   /* KOR_FULL / KOR_DETACH */
+  int nthreads; /* <= 0: all online cores */
+} kor_params;
+
+typedef struct {
+  double* O;          /* [B,H,T,d] forward output */
+  double* M;          /* [B,H,T] row max */
+  double* m;          /* [B,H,T] row min */
+  int32_t* amax;      /* [B,H,T] lowest arg-max */
+  int32_t* amin;      /* [B,H,T] lowest arg-min */
+  int32_t* nmax;      /* [B,H,T] size of the arg-max tie set */
+  int32_t* nmin;      /* [B,H,T] size of the arg-min tie set */
+  double* W;          /* [B,H,T] W^N (Nearest) or W^L (LERP); softmax: sum e^z */
+  double* WL;         /* [B,H,T] W^L */
+  double* OL;         /* [B,H,T,d] P^L V */
+  uint8_t* bins;      /* [B,H,T,T] Nearest index l / codes */
+  uint8_t* ivals;     /* [B,H,T,T] interval index r / codes */
+  double* margin;     /* [B,H,T,T] distance (score units) to the nearest decision boundary */
+  double* row_margin; /* [B,H,T] gap between an extremum and its runner-up */
+} kor_fwd_out;
+
+typedef struct {
+  double* dQ;   /* [B,H,T,d] */
+  double* dK;   /* [B,H,T,d] */
+  double* dV;   /* [B,H,T,d] */
+  double* cM;   /* [B,H,T] sum_j gamma_j dw_j/dM (0 under detach) */
+  double* cm;   /* [B,H,T] sum_j gamma_j dw_j/dm (MinMax, full) */
+  double* dsum; /* [B,H,T] sum_j dL/ds_ij */
+  double* dabs; /* [B,H,T] sum_j |dL/ds_ij| */
+  double* dS;   /* [B,H,T,T] dL/ds (optional, small cases) */
+} kor_bwd_out;
+
+/* Decision-aligned re-run: where given, the oracle takes these decisions
+ * instead of its own (used only for keys whose own decision lies within the
+ * rounding guard band of a boundary). */
+typedef struct {
+  const uint8_t* bins;  /* [B,H,T,T] */
+  const uint8_t* ivals; /* [B,H,T,T] */
+  const int32_t* amax;  /* [B,H,T] */
+  const int32_t* amin;  /* [B,H,T] */
+} kor_override;
+
+int kor_forward(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_in* V, const kor_fwd_out* out,
+                const kor_override* ov);
+int kor_backward(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_in* V, const kor_in* dO,
+                 const kor_bwd_out* out, const kor_override* ov);
+int kor_hardware_threads(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

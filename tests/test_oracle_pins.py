@@ -1,0 +1,434 @@
+"""Pins for the fp64 oracle, against what the paper and the mathematics fix.
+
+Each test names the passage it follows.  None of them compares the oracle with
+itself: the references are brute-force scans, closed forms, textbook error
+bounds of linear interpolation, finite differences, an independent PyTorch
+autograd restatement (tests/witness.py), and invariants (row sums, shift
+invariance, the zero-sum identity).
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+from oracle import Config, MINMAX, FWM, SOFTMAX, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH
+from tests import witness
+
+ALL_COMBOS = [(c, r, s, g) for c in (MINMAX, FWM) for r in (LERP, NEAREST) for s in (WEIGHT, PROB)
+              for g in (FULL, DETACH)]
+
+
+def rand_inputs(B, H, T, d, seed, scale=1.0, f64=False):
+    rng = np.random.default_rng(seed)
+    dt = np.float64 if f64 else np.float32
+    return [(rng.standard_normal((B, H, T, d)) * (scale if i == 0 else 1.0)).astype(dt) for i in range(4)]
+
+
+def eye_values(T, d):
+    """V = I (T <= d): then O_i = P_i, and g_ij = dO_i[j]."""
+    V = np.zeros((1, 1, T, d), np.float32)
+    V[0, 0, np.arange(T), np.arange(T)] = 1.0
+    return V
+
+
+def lattice_qk(targets, d=16):
+    """Q, K whose every row i sees the scores targets[0..i] exactly:
+    Q_i = (2, 0, ...), K_j = (2 t_j, 0, ...), scale 1/sqrt(16) = 1/4."""
+    T = len(targets)
+    Q = np.zeros((1, 1, T, d), np.float32)
+    K = np.zeros((1, 1, T, d), np.float32)
+    Q[0, 0, :, 0] = 2.0
+    K[0, 0, :, 0] = 2.0 * np.asarray(targets, np.float64)
+    return Q, K
+
+
+def scores_np(Q, K):
+    d = Q.shape[-1]
+    return np.einsum("bhid,bhjd->bhij", Q.astype(np.float64), K.astype(np.float64)) / math.sqrt(d)
+
+
+# --- P1: rows sum to one (App. A "Normalization") ------------------------------------------------
+
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + [(SOFTMAX, LERP, WEIGHT, FULL)])
+def test_rows_sum_to_one(calib, recon, ste, grad):
+    Q, K, _, _ = rand_inputs(2, 2, 40, 16, 1, scale=2.0)
+    V = np.ones_like(Q)
+    out = oracle.forward(Q, K, V, Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad))
+    assert np.max(np.abs(out["O"] - 1.0)) < 1e-13
+
+
+# --- two valid keys: both sit on grid points, so every MinMax operator is softmax -----------------
+
+@pytest.mark.parametrize("Kint", [1, 2, 4, 16])
+@pytest.mark.parametrize("recon", [LERP, NEAREST])
+def test_two_key_rows_equal_softmax(Kint, recon):
+    T = 16
+    Q, K, _, _ = rand_inputs(1, 1, T, 16, 2)
+    out = oracle.forward(Q, K, eye_values(T, 16), Config(Kint=Kint, calib=MINMAX, recon=recon))
+    s = scores_np(Q, K)[0, 0, 1, :2]
+    ref = np.exp(s - s.max()) / np.exp(s - s.max()).sum()
+    assert np.allclose(out["O"][0, 0, 1, :2], ref, rtol=0, atol=1e-15)
+
+
+# --- P2: brute-force bins on score lattices (Sec. 3 "Reconstruction", App. A, Table "Edge cases") --
+
+def brute_force_row(z, b, tail):
+    """Nearest index by scanning all K+1 grid points (ties go up), LERP weight
+    by scanning for an interval that contains z."""
+    K = len(b) - 1
+    ell, r_idx, wl, wn = [], [], [], []
+    for zj, tj in zip(z, tail):
+        if tj:
+            ell.append(254)
+            r_idx.append(254)
+            wl.append(0.0)
+            wn.append(0.0)
+            continue
+        best, best_l = math.inf, -1
+        for l in range(K + 1):
+            dist = abs(zj - b[l])
+            if dist < best or dist == best:  # equal distance: the larger index wins
+                best, best_l = dist, l
+        r = max(rr for rr in range(K) if b[rr] <= zj) if zj >= b[0] else 0
+        t = min(max((zj - b[r]) / (b[r + 1] - b[r]), 0.0), 1.0)
+        ell.append(best_l)
+        r_idx.append(r)
+        wn.append(math.exp(b[best_l]))
+        wl.append((1 - t) * math.exp(b[r]) + t * math.exp(b[r + 1]))
+    return np.array(ell), np.array(r_idx), np.array(wl), np.array(wn)
+
+
+@pytest.mark.parametrize("calib", [MINMAX, FWM])
+def test_brute_force_bins_on_lattice(calib):
+    rng = np.random.default_rng(3)
+    Kint, T, step = 4, 16, 0.125
+    for trial in range(60):
+        # max key 1.0; for MinMax a min key at 1 - 2 (span 2, h = 0.5); the rest on a 1/8 lattice that
+        # hits grid points, Nearest midpoints and (for FWM, tau = 2) the window edge and the tail.
+        depth = 16 if calib == MINMAX else 24
+        ks = rng.integers(0, depth + 1, size=T)
+        ks[rng.integers(0, T)] = 0
+        if calib == MINMAX:
+            ks[rng.integers(0, T)] = 16
+        targets = 1.0 - step * ks
+        Q, K = lattice_qk(targets)
+        cfg = Config(Kint=Kint, calib=calib, tau=2.0, recon=NEAREST)
+        out = oracle.forward(Q, K, eye_values(T, 16), cfg, decisions=True)
+        out_l = oracle.forward(Q, K, eye_values(T, 16), Config(Kint=Kint, calib=calib, tau=2.0, recon=LERP))
+        z = targets - targets.max()
+        if calib == MINMAX:
+            b = [z.min() + r * (0 - z.min()) / Kint for r in range(Kint + 1)]
+            tail = np.zeros(T, bool)
+        else:
+            b = [-2.0 + r * 0.5 for r in range(Kint + 1)]
+            tail = z < -2.0
+        ell, r_idx, wl, wn = brute_force_row(z, b, tail)
+        last = T - 1
+        assert np.array_equal(out["bins"][0, 0, last], ell), (trial, targets)
+        assert np.array_equal(out["ivals"][0, 0, last], r_idx), (trial, targets)
+        assert np.allclose(out["O"][0, 0, last, :T], wn / wn.sum(), rtol=0, atol=1e-15)
+        assert np.allclose(out_l["O"][0, 0, last, :T], wl / wl.sum(), rtol=0, atol=1e-15)
+
+
+def test_midpoint_rounds_up_and_window_edge_is_inside():
+    # MinMax K=4 over [-1, 1]: h = 0.5, grid z in {-2, -1.5, -1, -0.5, 0}; z = -0.25 sits exactly
+    # between b_3 = -0.5 and b_4 = 0 (rounds up to 4); z = -1.5 and z = -1 are grid points 1 and 2.
+    targets = [1.0, -1.0, 0.75, -0.5, 0.0]
+    Q, K = lattice_qk(targets)
+    out = oracle.forward(Q, K, eye_values(5, 16), Config(Kint=4, calib=MINMAX, recon=NEAREST), decisions=True)
+    assert list(out["bins"][0, 0, 4, :5]) == [4, 0, 4, 1, 2]
+    # FWM tau = 2: z = -2 is in the window (bin 0), z = -2.125 is in the tail.
+    targets = [1.0, -1.0, -1.125, 0.0]
+    Q, K = lattice_qk(targets)
+    out = oracle.forward(Q, K, eye_values(4, 16), Config(Kint=4, calib=FWM, tau=2.0, recon=NEAREST),
+                         decisions=True)
+    assert list(out["bins"][0, 0, 3, :4]) == [4, 0, 254, 2]
+
+
+# --- P3: closed form at K = 1 (App. A "LERP") ----------------------------------------------------
+
+def test_lerp_k1_closed_form():
+    T = 16
+    Q, K, _, _ = rand_inputs(1, 1, T, 16, 4, scale=2.0)
+    out = oracle.forward(Q, K, eye_values(T, 16), Config(Kint=1, calib=MINMAX, recon=LERP))
+    S = scores_np(Q, K)[0, 0]
+    for i in range(1, T):
+        s = S[i, : i + 1]
+        M, m = s.max(), s.min()
+        rho = (s - m) / (M - m)
+        w = (1 - rho) * math.exp(m - M) + rho
+        assert np.allclose(out["O"][0, 0, i, : i + 1], w / w.sum(), rtol=0, atol=1e-15)
+
+
+# --- P4: K -> infinity, against textbook interpolation bounds ------------------------------------
+
+@pytest.mark.parametrize("calib", [MINMAX, FWM])
+def test_convergence_to_softmax(calib):
+    T, d = 16, 16
+    Q, K, _, _ = rand_inputs(8, 1, T, d, 5, scale=2.5)
+    V = np.broadcast_to(eye_values(T, d), (8, 1, T, d)).copy()
+    S = scores_np(Q, K)
+    span = max(S[b, 0, i, : i + 1].max() - S[b, 0, i, : i + 1].min() for b in range(8) for i in range(T))
+    tau = span + 1.0  # FWM window covering every row: no tail
+    Ks = [2 ** k for k in range(2, 13)]
+    errs = {LERP: [], NEAREST: []}
+    for Kint in Ks:
+        for recon in (LERP, NEAREST):
+            out = oracle.forward(Q, K, V, Config(Kint=Kint, calib=calib, tau=tau, recon=recon))
+            worst_abs = 0.0
+            for b in range(8):
+                for i in range(1, T):
+                    s = S[b, 0, i, : i + 1]
+                    pe = np.exp(s - s.max())
+                    pe /= pe.sum()
+                    p = out["O"][b, 0, i, : i + 1]
+                    worst_abs = max(worst_abs, np.max(np.abs(p - pe)))
+                    h = (s.max() - s.min()) / Kint if calib == MINMAX else tau / Kint
+                    # chord of a convex function: e^z <= w^L <= e^z (1 + h^2/8 e^h);
+                    # nearest grid centre: |b_l - z| <= h/2, so w^N / e^z in [e^-h/2, e^h/2].
+                    bound = math.log1p(h * h / 8 * math.exp(h)) if recon == LERP else h / 2
+                    assert np.max(np.abs(np.log(p / pe))) <= 2 * bound + 1e-12
+            errs[recon].append(worst_abs)
+    # convergence order from a log-log fit over K >= 32: 2 for LERP, 1 for Nearest
+    sel = [k for k, K_ in enumerate(Ks) if K_ >= 32]
+    slope = {r: np.polyfit(np.log([Ks[k] for k in sel]), np.log([errs[r][k] for k in sel]), 1)[0]
+             for r in (LERP, NEAREST)}
+    assert -2.25 < slope[LERP] < -1.75, slope
+    assert -1.3 < slope[NEAREST] < -0.7, slope
+
+
+# --- P5: finite differences in fp64 (App. B; diagnostics A3/A4 of App. "detach") ------------------
+
+def _loss(Q, K, V, dO, cfg):
+    return float(np.sum(oracle.forward(Q, K, V, cfg, f64=True)["O"] * dO))
+
+
+def _fd_setup(seed, calib, tau):
+    # find a seed whose every decision is far from a boundary, so a 1e-6 step flips nothing
+    for s in range(seed, seed + 200):
+        Q, K, V, dO = rand_inputs(1, 1, 8, 4, s, scale=1.5, f64=True)
+        f = oracle.forward(Q, K, V, Config(Kint=4, calib=calib, tau=tau), decisions=True, f64=True)
+        if np.min(f["margin"]) > 1e-3 and np.min(f["row_margin"][0, 0, 1:]) > 1e-3:
+            return Q, K, V, dO
+    raise RuntimeError("no well-separated seed")
+
+
+@pytest.mark.parametrize("calib", [MINMAX, FWM, SOFTMAX])
+def test_lerp_full_gradient_matches_finite_differences(calib):
+    tau = 2.0
+    Q, K, V, dO = _fd_setup(10, calib, tau)
+    for recon_ste in ((LERP, WEIGHT), (NEAREST, PROB)) if calib != SOFTMAX else ((LERP, WEIGHT),):
+        cfg = Config(Kint=4, calib=calib, tau=tau, recon=recon_ste[0], ste=recon_ste[1])
+        g = oracle.backward(Q, K, V, dO, cfg, f64=True)
+        # Prob-STE's backward is the Jacobian of normalize(w^L): differentiate the LERP forward
+        lcfg = Config(Kint=4, calib=calib, tau=tau, recon=LERP)
+        eps = 1e-6
+        for name, X, G in (("Q", Q, g["dQ"]), ("K", K, g["dK"]), ("V", V, g["dV"] if recon_ste[0] == LERP else None)):
+            if G is None:
+                continue
+            fd = np.zeros_like(X)
+            for idx in np.ndindex(X.shape):
+                Xp, Xm = X.copy(), X.copy()
+                Xp[idx] += eps
+                Xm[idx] -= eps
+                args_p = {"Q": Q, "K": K, "V": V}
+                args_m = dict(args_p)
+                args_p[name], args_m[name] = Xp, Xm
+                fd[idx] = (_loss(args_p["Q"], args_p["K"], args_p["V"], dO, lcfg)
+                           - _loss(args_m["Q"], args_m["K"], args_m["V"], dO, lcfg)) / (2 * eps)
+            assert np.max(np.abs(fd - G)) <= 1e-7 * np.max(np.abs(G)) + 1e-9, (calib, recon_ste, name)
+
+
+def _dS_probe_inputs(T, seed, scale=1.5):
+    """K = 4 I and V = I with d = 16: s_ij = Q_i[j], dQ_i[j] = dL/ds_ij, g_ij = dO_i[j], O_i = P_i."""
+    d = 16
+    rng = np.random.default_rng(seed)
+    Q = np.zeros((1, 1, T, d))
+    Q[0, 0, :, :T] = rng.standard_normal((T, T)) * scale
+    K = np.zeros((1, 1, T, d))
+    K[0, 0, np.arange(T), np.arange(T)] = 4.0
+    V = np.zeros((1, 1, T, d))
+    V[0, 0, np.arange(T), np.arange(T)] = 1.0
+    dO = rng.standard_normal((1, 1, T, d))
+    return Q, K, V, dO
+
+
+@pytest.mark.parametrize("calib", [MINMAX, FWM])
+@pytest.mark.parametrize("grad", [FULL, DETACH])
+def test_weight_ste_is_lerp_jacobian_at_hard_normalization(calib, grad):
+    """Eq. (wste): dL/ds = J_{w^L}(s)^T gamma^W with gamma^W = (g - <g>_{P^N}) / W^N; under detach the
+    grid is frozen, so J is diagonal (Delta) -- checked on keys that are not extrema."""
+    T, tau, eps = 10, 2.0, 1e-6
+    for seed in range(20, 60):
+        Q, K, V, dO = _dS_probe_inputs(T, seed)
+        f = oracle.forward(Q, K, V, Config(Kint=4, calib=calib, tau=tau), decisions=True, f64=True)
+        if np.min(f["margin"]) > 1e-3 and np.min(f["row_margin"][0, 0, 1:]) > 1e-3:
+            break
+    lerp = Config(Kint=4, calib=calib, tau=tau, recon=LERP)
+    near = Config(Kint=4, calib=calib, tau=tau, recon=NEAREST, ste=WEIGHT, grad=grad)
+    fn = oracle.forward(Q, K, V, near, f64=True)
+    dS = oracle.backward(Q, K, V, dO, near, f64=True)["dQ"][0, 0, :, :T]
+    for i in range(1, T):
+        n = i + 1
+        PN, WN = fn["O"][0, 0, i, :n], fn["W"][0, 0, i]
+        g = dO[0, 0, i, :n]
+        gammaW = (g - PN @ g) / WN
+        J = np.zeros((n, n))  # J[k, j] = d w^L_k / d s_j
+        for j in range(n):
+            Qp, Qm = Q.copy(), Q.copy()
+            Qp[0, 0, i, j] += eps
+            Qm[0, 0, i, j] -= eps
+            fp = oracle.forward(Qp, K, V, lerp, f64=True)
+            fm = oracle.forward(Qm, K, V, lerp, f64=True)
+            wp = fp["O"][0, 0, i, :n] * fp["WL"][0, 0, i]
+            wm = fm["O"][0, 0, i, :n] * fm["WL"][0, 0, i]
+            J[:, j] = (wp - wm) / (2 * eps)
+        s = Q[0, 0, i, :n]
+        if grad == FULL:
+            expect = J.T @ gammaW
+            assert np.allclose(dS[i, :n], expect, rtol=0, atol=1e-7 * max(1.0, np.abs(expect).max()))
+        else:
+            inner = [j for j in range(n) if s[j] != s.max() and s[j] != s.min()]
+            if not inner:
+                continue
+            expect = np.diag(J)[inner] * gammaW[inner]
+            assert np.allclose(dS[i, inner], expect, rtol=0, atol=1e-7 * max(1.0, np.abs(expect).max()))
+
+
+# --- Witness: independent PyTorch autograd restatement -------------------------------------------
+
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + [(SOFTMAX, LERP, WEIGHT, FULL)])
+@pytest.mark.parametrize("Kint", [1, 4, 16])
+def test_matches_autograd_witness(calib, recon, ste, grad, Kint):
+    Q, K, V, dO = rand_inputs(1, 2, 12, 8, 7, scale=2.0)
+    cfg = Config(Kint=Kint, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad)
+    f = oracle.forward(Q, K, V, cfg)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+    for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+        assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+def test_ties_split_evenly_like_autograd():
+    """Duplicate keys give tied extrema; amax/amin split the extremum gradient evenly (Table "Edge cases")."""
+    Q, K, V, dO = rand_inputs(1, 1, 12, 8, 8, scale=2.0)
+    K[0, 0, 5] = K[0, 0, 2]
+    K[0, 0, 9] = K[0, 0, 2]
+    K[0, 0, 7] = K[0, 0, 3]
+    for calib, recon, ste in ((MINMAX, LERP, WEIGHT), (MINMAX, NEAREST, WEIGHT), (FWM, NEAREST, PROB)):
+        cfg = Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=FULL)
+        f = oracle.forward(Q, K, V, cfg)
+        assert f["nmax"].max() >= 2 or f["nmin"].max() >= 2
+        b = oracle.backward(Q, K, V, dO, cfg)
+        O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+        for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+            assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+# --- P6 / P8: zero-sum identity, shift invariance, the per-key calibration identity --------------
+
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS)
+def test_zero_sum_identity(calib, recon, ste, grad):
+    Q, K, V, dO = rand_inputs(1, 2, 48, 16, 9, scale=2.0)
+    cfg = Config(Kint=8, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    live = b["dabs"] > 0
+    rho = np.abs(b["dsum"][live]) / b["dabs"][live]
+    if grad == FULL:
+        assert rho.max() < 1e-13  # Eq. (full): the three per-key terms sum to zero
+    else:
+        assert np.median(rho) > 1e-3  # detach violates it (App. B "Detach")
+
+
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS)
+def test_key_shift_invariance(calib, recon, ste, grad):
+    """K' = K + 1 k0^T adds Q_i.k0/sqrt(d) to every score of row i: F(s + c1) = F(s), so O and dV are
+    unchanged; dQ' = dQ + (sum_j dS_ij) k0 / sqrt(d), which is dQ exactly under the full gradient."""
+    Q, K, V, dO = rand_inputs(1, 2, 24, 8, 11, scale=2.0, f64=True)
+    k0 = np.random.default_rng(12).standard_normal(8) * 0.7
+    cfg = Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad)
+    f, fs = oracle.forward(Q, K, V, cfg, f64=True), oracle.forward(Q, K + k0, V, cfg, f64=True)
+    b, bs = oracle.backward(Q, K, V, dO, cfg, f64=True), oracle.backward(Q, K + k0, V, dO, cfg, f64=True)
+    assert np.max(np.abs(f["O"] - fs["O"])) < 1e-12
+    assert np.max(np.abs(b["dV"] - bs["dV"])) < 1e-12
+    expect = b["dQ"] + b["dsum"][..., None] * k0 / math.sqrt(8)
+    assert np.max(np.abs(bs["dQ"] - expect)) < 1e-11
+    if grad == FULL:
+        assert np.max(np.abs(bs["dQ"] - b["dQ"])) < 1e-11
+
+
+@pytest.mark.parametrize("calib", [MINMAX, FWM])
+@pytest.mark.parametrize("recon,ste", [(LERP, WEIGHT), (NEAREST, WEIGHT), (NEAREST, PROB)])
+def test_calibration_sums_cancel_own_terms(calib, recon, ste):
+    """Delta_j + dw_j/dM + dw_j/dm = 0 per key (App. B), so c_M + c_m = -sum_j gamma_j Delta_j, which is
+    the row sum of the detached gradient; under FWM dw/dM = -Delta."""
+    Q, K, V, dO = rand_inputs(2, 2, 32, 16, 13, scale=2.0)
+    full = oracle.backward(Q, K, V, dO, Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=FULL))
+    det = oracle.backward(Q, K, V, dO, Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=DETACH))
+    assert np.max(np.abs(full["cM"] + full["cm"] + det["dsum"])) < 1e-12
+    if calib == FWM:
+        assert np.max(np.abs(full["cm"])) == 0.0
+
+
+def test_prob_ste_backward_is_lerp_backward():
+    """Eq. (pste): Prob-STE back-propagates the Jacobian of normalize(w^L); only the value path
+    (dV, with the hard forward P^N) differs from LERP."""
+    Q, K, V, dO = rand_inputs(1, 2, 32, 16, 14, scale=2.0)
+    for calib in (MINMAX, FWM):
+        a = oracle.backward(Q, K, V, dO, Config(Kint=4, calib=calib, tau=3.0, recon=NEAREST, ste=PROB))
+        b = oracle.backward(Q, K, V, dO, Config(Kint=4, calib=calib, tau=3.0, recon=LERP))
+        assert np.max(np.abs(a["dQ"] - b["dQ"])) < 1e-13 and np.max(np.abs(a["dK"] - b["dK"])) < 1e-13
+        assert np.max(np.abs(a["dV"] - b["dV"])) > 1e-6
+
+
+# --- P10: edge cases of Table "Edge cases" -------------------------------------------------------
+
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + [(SOFTMAX, LERP, WEIGHT, FULL)])
+def test_single_key(calib, recon, ste, grad):
+    Q, K, V, dO = rand_inputs(1, 1, 1, 8, 15)
+    cfg = Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad)
+    f = oracle.forward(Q, K, V, cfg)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    assert np.allclose(f["O"], V)
+    assert np.all(b["dQ"] == 0) and np.all(b["dK"] == 0)
+    assert np.allclose(b["dV"], dO)
+
+
+def test_degenerate_minmax_rows_are_uniform_with_zero_score_gradient():
+    _, K, V, dO = rand_inputs(1, 1, 12, 8, 16)
+    Q = np.zeros_like(K)
+    for recon in (LERP, NEAREST):
+        cfg = Config(Kint=4, calib=MINMAX, recon=recon)
+        f = oracle.forward(Q, K, V, cfg)
+        b = oracle.backward(Q, K, V, dO, cfg)
+        assert np.allclose(f["O"][0, 0], np.cumsum(V[0, 0], 0) / np.arange(1, 13)[:, None])
+        assert np.all(b["dQ"] == 0) and np.all(b["dK"] == 0)
+
+
+def test_fwm_equal_scores_and_far_tail_match_autograd():
+    _, K, V, dO = rand_inputs(1, 1, 12, 8, 17)
+    cases = [np.zeros_like(K), rand_inputs(1, 1, 12, 8, 18, scale=30.0)[0]]  # all z = 0; all but max in tail
+    for Q in cases:
+        for recon, ste in ((LERP, WEIGHT), (NEAREST, WEIGHT), (NEAREST, PROB)):
+            cfg = Config(Kint=4, calib=FWM, tau=3.0, recon=recon, ste=ste)
+            f = oracle.forward(Q, K, V, cfg)
+            b = oracle.backward(Q, K, V, dO, cfg)
+            O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+            for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+                assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+def test_decision_override_roundtrip():
+    Q, K, V, dO = rand_inputs(1, 1, 20, 8, 19, scale=2.0)
+    cfg = Config(Kint=4, calib=MINMAX, recon=NEAREST, ste=WEIGHT)
+    f = oracle.forward(Q, K, V, cfg, decisions=True)
+    ov = {"bins": f["bins"], "ivals": f["ivals"], "amax": f["amax"], "amin": f["amin"]}
+    g = oracle.forward(Q, K, V, cfg, override=ov)
+    assert np.array_equal(f["O"], g["O"])
+    bins = f["bins"].copy()
+    i, j = 15, 4
+    bins[0, 0, i, j] = bins[0, 0, i, j] + (1 if bins[0, 0, i, j] < 4 else -1)
+    h = oracle.forward(Q, K, V, cfg, override={**ov, "bins": bins})
+    changed = np.where(np.any(h["O"] != f["O"], axis=-1))
+    assert list(changed[2]) == [i]
