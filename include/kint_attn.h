@@ -1,0 +1,155 @@
+/*
+ * kint_attn.h -- C ABI of libkint, K-interval attention (forward and backward)
+ * on one NVIDIA GB300 (sm_103a).
+ *
+ * K-interval attention replaces the softmax of causal attention (paper: Sec. 3,
+ * App. A): scores S = Q K^T / sqrt(d) are calibrated per row (MinMax: the grid
+ * spans the row's own [m, M]; FWM: a fixed window [M - tau, M] anchored at the
+ * row maximum, zero weight below it), the exponential is rebuilt on K intervals
+ * from K + 1 grid values e^{b_r} (LERP interpolation or Nearest rounding), the
+ * weights are normalised, P = w / sum w, and O = P V.  The backward is the
+ * closed form of App. B: normalization Jacobian, LERP secant slope, and the
+ * calibration derivatives through the row extrema (Eqs. calgrad and full),
+ * placed by Weight-STE (Eq. wste) or Prob-STE (Eq. pste); the detached-extrema
+ * mode keeps only the own-score term.
+ *
+ * Conventions shared by every entry point
+ *   - Tensors are fp32, row-major, contiguous [B, H, T, d]; row statistics are
+ *     [B, H, T].  All tensor pointers are DEVICE pointers owned by the caller;
+ *     the library never allocates, frees or synchronises (except
+ *     kint_get_status, which synchronises the given stream).  Work is enqueued
+ *     on `stream` (a cudaStream_t; 0 = legacy default stream).
+ *   - Attention is causal (row i sees keys 0..i, App. A); causal must be 1.
+ *   - d must be 64 or 128; T >= 1 is arbitrary (ragged final tiles are masked);
+ *     B * H * ceil(T / 128) <= 2^31 - 1.
+ *   - Every device pointer must be 16-byte aligned.
+ *   - The score scale 1/sqrt(d) is applied inside the operator.
+ *   - Errors are returned as negative codes BEFORE any work is enqueued; no
+ *     output is touched then.  Faults detected on the device (a bounded wait
+ *     that ran out) are reported by kint_get_status().
+ *   - Calls on different streams that share a workspace race.
+ */
+#ifndef KINT_ATTN_H
+#define KINT_ATTN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Return codes. */
+#define KINT_OK 0
+#define KINT_ERR_ARG (-1)          /* null pointer, size < 1, K out of [1, 64], tau <= 0, bad enum, causal != 1 */
+#define KINT_ERR_UNSUPPORTED (-2)  /* d not in {64, 128}; sizes beyond the limits above */
+#define KINT_ERR_ALIGN (-3)        /* a device pointer is not 16-byte aligned */
+#define KINT_ERR_WORKSPACE (-4)    /* workspace NULL or smaller than kint_attn_workspace_bytes() */
+#define KINT_ERR_LAUNCH (-5)       /* the CUDA runtime refused a launch or a tensor-map encoding */
+#define KINT_ERR_DEVICE (-6)       /* kint_get_status: a kernel flagged a device-side fault */
+#define KINT_ERR_NO_DEVICE (-7)    /* no sm_103 device current, or the driver lacks tensor maps */
+
+/* Calibration (Sec. 3 "Objects and calibration"; App. A "MinMax grid", "FWM";
+ * App. A "Softmax" is the exact-exponential comparator). */
+typedef enum { KINT_CALIB_MINMAX = 0, KINT_CALIB_FWM = 1, KINT_CALIB_SOFTMAX = 2 } kint_calib;
+/* Reconstruction (Sec. 3 "Reconstruction"; App. A "LERP", "Nearest"). */
+typedef enum { KINT_RECON_LERP = 0, KINT_RECON_NEAREST = 1 } kint_recon;
+/* Surrogate placement (Sec. 3 Eqs. wste / pste).  Ignored under LERP, where the
+ * two placements coincide (w^N = w^L). */
+typedef enum { KINT_STE_WEIGHT = 0, KINT_STE_PROB = 1 } kint_ste;
+/* Backward mode: full calibration gradient (Eq. full) or detached extrema
+ * (App. B "Detach (legacy)").  The forward does not depend on it. */
+typedef enum { KINT_GRAD_FULL = 0, KINT_GRAD_DETACH = 1 } kint_grad;
+/* Tensor-core arithmetic: plain TF32 products (the precision the paper trains
+ * with, App. C "Numerics and hardware"), or 3xTF32 (hi/lo operand splitting,
+ * fp32-level accuracy). */
+typedef enum { KINT_PREC_TF32 = 0, KINT_PREC_3XTF32 = 1 } kint_prec;
+
+/* Row statistics written by kint_attn_fwd and read by kint_attn_bwd.  All
+ * arrays are caller-owned device memory of B*H*T elements unless noted. */
+typedef struct {
+  float* row_max;    /* M_i = max_j s_ij over valid keys (App. A) */
+  float* row_min;    /* m_i = min_j s_ij (written for FWM too, as a diagnostic) */
+  int32_t* arg_max;  /* lowest j with s_ij == M_i */
+  int32_t* arg_min;  /* lowest j with s_ij == m_i */
+  int32_t* n_max;    /* number of keys tied at M_i (the extremum gradient is split evenly) */
+  int32_t* n_min;    /* number of keys tied at m_i */
+  float* W;          /* W^N = sum w^N (Nearest) or W^L (LERP); softmax: sum e^{s - M} */
+  float* W_lerp;     /* W^L; required for Prob-STE, may be NULL otherwise */
+  float* O_lerp;     /* [B,H,T,d] P^L V; required for Prob-STE, may be NULL otherwise */
+} kint_rowstats;
+
+/*
+ * Workspace needed by kint_attn_fwd (is_bwd = 0) or kint_attn_bwd (is_bwd = 1)
+ * for these sizes and precision.  0 for invalid sizes.
+ */
+size_t kint_attn_workspace_bytes(int B, int H, int T, int d, kint_prec prec, int is_bwd);
+
+/*
+ * Forward: O = P V with P the K-interval probabilities (App. A).  For Nearest
+ * the forward returns the hard probabilities P^N = w^N / W^N directly
+ * (the strict hard forward of App. C.2 (iii)); for LERP P^L = w^L / W^L.
+ *   Q, K, V  in:  [B,H,T,d]
+ *   O        out: [B,H,T,d]
+ *   st       out: row statistics (struct itself is host memory, read during the call)
+ *   Kint     number of intervals K, 1..64 (ignored for softmax)
+ *   tau      FWM window in nats, > 0 (ignored otherwise)
+ *   workspace, workspace_bytes: device scratch of at least
+ *            kint_attn_workspace_bytes(B, H, T, d, prec, 0) bytes
+ */
+int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, const kint_rowstats* st, int B, int H,
+                  int T, int d, int Kint, kint_calib calib, float tau, kint_recon recon, kint_ste ste,
+                  kint_grad grad, int causal, kint_prec prec, void* workspace, size_t workspace_bytes,
+                  void* stream);
+
+/*
+ * Backward (App. B): dQ, dK, dV of L given dO = dL/dO, with the row statistics
+ * of the forward of the same inputs and configuration.
+ *   gamma_j = (g_j - <g>_{P*}) / W*, g_j = dO_i . V_j, where (P*, W*) is
+ *     (P^N, W^N) for Nearest + Weight-STE and (P^L, W^L) otherwise;
+ *   dS_ij = gamma_j Delta_j + [j tied at M_i] c_M / n_max + [j tied at m_i] c_m / n_min
+ *     (c_m only for MinMax; both zero under detach; FWM tail keys get 0;
+ *      degenerate MinMax rows get 0);
+ *   dQ = dS K / sqrt(d), dK = dS^T Q / sqrt(d), dV = P^T dO with the forward P.
+ * dQ, dK, dV are overwritten.
+ *   O        in:  forward output
+ *   dO       in:  [B,H,T,d]
+ *   st       in:  row statistics written by kint_attn_fwd
+ */
+int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O, const float* dO,
+                  const kint_rowstats* st, float* dQ, float* dK, float* dV, int B, int H, int T, int d, int Kint,
+                  kint_calib calib, float tau, kint_recon recon, kint_ste ste, kint_grad grad, int causal,
+                  kint_prec prec, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Decision dump for parity checks: for every (b, h, i, j) the Nearest index
+ * l_ij = r + [t >= 1/2] in 0..K (bins) and the interval index r_ij in 0..K-1
+ * (ivals), with 254 for FWM tail keys (z < -tau), 255 for masked keys (j > i)
+ * and 253 where no grid exists (degenerate MinMax rows, softmax).  Either
+ * output may be NULL.  Needs the row statistics of kint_attn_fwd on the same
+ * inputs and the forward's workspace size.  bins, ivals: [B,H,T,T] uint8.
+ */
+int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const kint_rowstats* st, uint8_t* bins,
+                         uint8_t* ivals, int B, int H, int T, int d, int Kint, kint_calib calib, float tau,
+                         kint_recon recon, kint_ste ste, int causal, kint_prec prec, void* workspace,
+                         size_t workspace_bytes, void* stream);
+
+/*
+ * Synchronises `stream`, then returns KINT_OK, or KINT_ERR_DEVICE if any kernel
+ * of this library flagged a device-side fault since the last call (the flag
+ * word is cleared).  *detail (may be NULL) receives the raw flag bits:
+ * 1 = TMA wait timed out, 2 = MMA wait timed out, 4 = CTA sync timed out.
+ */
+int kint_get_status(void* stream, unsigned* detail);
+
+/* Human-readable text for a return code (static storage). */
+const char* kint_strerror(int code);
+
+/* Wall-clock limit, in nanoseconds, of every bounded device-side wait
+ * (default 2e9).  Values < 1000 are clamped to 1000. */
+void kint_set_wait_timeout_ns(unsigned long long ns);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

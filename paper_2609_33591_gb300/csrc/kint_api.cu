@@ -1,0 +1,491 @@
+// C ABI of libkint (include/kint_attn.h): argument checks, workspace layout,
+// TMA descriptors, shared-memory plans and the launch sequence of each entry
+// point.  Nothing here allocates device memory or synchronises, except
+// kint_get_status.
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include "../../include/kint_attn.h"
+#include "kint_launch.h"
+#include "kint_params.h"
+
+namespace kint {
+
+// Device-side fault flags (see tc.cuh); read and cleared by kint_get_status.
+__device__ unsigned g_status_word = 0;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+unsigned* g_status_ptr[kMaxDevices] = {nullptr};
+int g_dev_ok[kMaxDevices] = {0};  // 0 unknown, 1 sm_103, -1 other
+unsigned long long g_wait_ns = 2000000000ull;
+constexpr int kSmemLimit = 232448;  // opt-in maximum per CTA on sm_103
+
+int round_up(int x, int m) { return (x + m - 1) / m * m; }
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Resolve the device-dependent handles once per device.
+int device_setup(unsigned** status) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return KINT_ERR_NO_DEVICE;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (g_dev_ok[dev] == 0) {
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) {
+      return KINT_ERR_NO_DEVICE;
+    }
+    g_dev_ok[dev] = (major == 10 && minor == 3) ? 1 : -1;
+    if (g_dev_ok[dev] == 1) {
+      void* ptr = nullptr;
+      if (cudaGetSymbolAddress(&ptr, g_status_word) != cudaSuccess) {
+        g_dev_ok[dev] = 0;
+        return KINT_ERR_NO_DEVICE;
+      }
+      g_status_ptr[dev] = static_cast<unsigned*>(ptr);
+    }
+  }
+  if (g_dev_ok[dev] != 1) return KINT_ERR_NO_DEVICE;
+  if (!g_encode) {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return KINT_ERR_NO_DEVICE;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  *status = g_status_ptr[dev];
+  return KINT_OK;
+}
+
+// Natural view of X [BH][T][d]: box (32 columns, rows).
+bool map_nat(CUtensorMap* m, const float* X, int BH, int T, int d, int rows) {
+  cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)T, (cuuint64_t)BH};
+  cuuint64_t strides[2] = {(cuuint64_t)d * 4, (cuuint64_t)T * d * 4};
+  cuuint32_t box[3] = {32, (cuuint32_t)rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(X), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+// Transposed view of X^T [BH][d][Tp] (valid columns T): box (32 keys, d rows).
+bool map_tr(CUtensorMap* m, const float* XT, int BH, int T, int Tp, int d) {
+  cuuint64_t dims[3] = {(cuuint64_t)T, (cuuint64_t)d, (cuuint64_t)BH};
+  cuuint64_t strides[2] = {(cuuint64_t)Tp * 4, (cuuint64_t)d * Tp * 4};
+  cuuint32_t box[3] = {32, (cuuint32_t)d, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(XT), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Workspace layout (floats), identical for the size query and the launches.
+struct Workspace {
+  size_t bytes = 0;
+  // forward / backward operand copies
+  float *qh = nullptr, *ql = nullptr, *kh = nullptr, *kl = nullptr, *vh = nullptr, *vl = nullptr,
+        *doh = nullptr, *dol = nullptr;
+  float *vth = nullptr, *vtl = nullptr, *kth = nullptr, *ktl = nullptr, *qth = nullptr, *qtl = nullptr,
+        *doth = nullptr, *dotl = nullptr;
+  float *Drow = nullptr, *cMn = nullptr, *cmn = nullptr, *tie = nullptr;
+};
+
+Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
+  Workspace w;
+  const int Tp = round_up(T, 32);
+  const size_t nat = (size_t)BH * T * d * 4, tr = (size_t)BH * d * Tp * 4, rows = (size_t)BH * T * 4;
+  size_t off = 0;
+  auto take = [&](size_t n) -> float* {
+    float* p = base ? reinterpret_cast<float*>(base + off) : nullptr;
+    off = align256(off + n);
+    return p;
+  };
+  if (!bwd) {
+    if (x3) {
+      w.qh = take(nat); w.ql = take(nat); w.kh = take(nat); w.kl = take(nat);
+      w.vth = take(tr); w.vtl = take(tr);
+    } else {
+      w.vth = take(tr);
+    }
+  } else {
+    if (x3) {
+      w.qh = take(nat); w.ql = take(nat); w.kh = take(nat); w.kl = take(nat);
+      w.vh = take(nat); w.vl = take(nat); w.doh = take(nat); w.dol = take(nat);
+      w.kth = take(tr); w.ktl = take(tr); w.qth = take(tr); w.qtl = take(tr); w.doth = take(tr); w.dotl = take(tr);
+    } else {
+      w.kth = take(tr); w.qth = take(tr); w.doth = take(tr);
+    }
+    w.Drow = take(rows); w.cMn = take(rows); w.cmn = take(rows);
+    w.tie = take(2 * nat);
+  }
+  w.bytes = off;
+  return w;
+}
+
+struct Common {
+  int B, H, T, d, Kint, calib, recon, ste, grad, prec;
+  float tau;
+};
+
+int validate(const Common& c, int causal) {
+  if (c.B < 1 || c.H < 1 || c.T < 1 || c.d < 1) return KINT_ERR_ARG;
+  if (causal != 1) return KINT_ERR_ARG;
+  if (c.calib < 0 || c.calib > 2 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
+      c.grad > 1 || c.prec < 0 || c.prec > 1)
+    return KINT_ERR_ARG;
+  if (c.calib != KINT_CALIB_SOFTMAX && (c.Kint < 1 || c.Kint > KMAX)) return KINT_ERR_ARG;
+  if (c.calib == KINT_CALIB_FWM && !(c.tau > 0.0f && std::isfinite(c.tau))) return KINT_ERR_ARG;
+  if (c.d != 64 && c.d != 128) return KINT_ERR_UNSUPPORTED;
+  if (c.prec == KINT_PREC_3XTF32 && c.d != 64) return KINT_ERR_UNSUPPORTED;
+  const long long BH = (long long)c.B * c.H;
+  if (BH > 65535 || (long long)c.T * BH > (1ll << 31) - 1 || c.T > (1 << 24)) return KINT_ERR_UNSUPPORTED;
+  return KINT_OK;
+}
+
+Params base_params(const Common& c, unsigned* status) {
+  Params p;
+  std::memset(&p, 0, sizeof(p));
+  p.B = c.B; p.H = c.H; p.T = c.T; p.d = c.d;
+  p.Kint = c.calib == KINT_CALIB_SOFTMAX ? 1 : c.Kint;
+  p.calib = c.calib; p.recon = c.recon; p.ste = c.ste; p.grad = c.grad;
+  p.x3 = c.prec == KINT_PREC_3XTF32;
+  p.BH = c.B * c.H;
+  p.nqb = (c.T + 127) / 128;
+  p.tau = c.tau;
+  p.scale = (float)(1.0 / std::sqrt((double)c.d));
+  if (c.calib == KINT_CALIB_FWM) {
+    p.fwm_inv_h = (float)((double)c.Kint / (double)c.tau);
+    for (int r = 0; r <= c.Kint; ++r)
+      p.fwm_e[r] = (float)std::exp(-(double)c.tau + (double)r * (double)c.tau / (double)c.Kint);
+  }
+  p.wait_ns = g_wait_ns;
+  p.status = status;
+  return p;
+}
+
+// Finish a shared-memory plan: barriers (+ TMEM slot) after `off`, + 1 KB for alignment.
+int finish_plan(Params& p, int off, int nbars) {
+  off = round_up(off, 8);
+  p.sm_bars = off;
+  off += nbars * 8 + 16;
+  return off + 1024;
+}
+// Kernels that allocate all 512 TMEM columns request more than half of an SM's
+// shared memory, so two of their CTAs are never resident on one SM at once.
+constexpr int kOneCtaPerSm = 117 * 1024;
+
+int plan_stats(Params& p) {
+  const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
+  p.sm_a = 0;
+  p.sm_stage0 = parts * tile;
+  p.sm_stage_bytes = parts * tile;
+  p.nstage = 2;
+  return finish_plan(p, p.sm_stage0 + p.nstage * p.sm_stage_bytes, 3 + p.nstage);
+}
+
+int plan_main(Params& p) {
+  const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
+  const int table = (p.Kint + 1) * 128 * 4;
+  p.sm_a = 0;
+  p.sm_stage0 = parts * tile;
+  p.sm_stage_bytes = parts * 2 * tile;
+  for (p.nstage = 2; p.nstage >= 1; --p.nstage) {
+    p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+    const int total = std::max(finish_plan(p, p.sm_table + table, 2 + p.nstage), kOneCtaPerSm);
+    if (total <= kSmemLimit || p.nstage == 1) return total;
+  }
+  return -1;
+}
+
+int plan_dq(Params& p) {
+  const int parts = p.x3 ? 2 : 1, ktile = 64 * p.d * 4;
+  const int table = (p.Kint + 1) * 128 * 4;
+  p.sm_stage0 = 0;
+  p.sm_stage_bytes = 3 * parts * ktile;
+  for (p.nstage = 2; p.nstage >= 1; --p.nstage) {
+    p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+    const int total = std::max(finish_plan(p, p.sm_table + table, 1 + p.nstage), kOneCtaPerSm);
+    if (total <= kSmemLimit || p.nstage == 1) return total;
+  }
+  return -1;
+}
+
+int plan_dkdv(Params& p) {
+  const int parts = p.x3 ? 2 : 1, qtile = 64 * p.d * 4;
+  p.sm_stage0 = 0;
+  p.sm_stage_bytes = 4 * parts * qtile;  // room for Q, dO, Q^T, dO^T
+  const int rows = 14 * 64 * 4;
+  const int table = 64 * (p.Kint + 2) * 4;
+  for (p.nstage = 2; p.nstage >= 1; --p.nstage) {
+    p.sm_rows = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+    p.sm_table = p.sm_rows + rows;
+    const int total = std::max(finish_plan(p, p.sm_table + table, 1 + p.nstage), kOneCtaPerSm);
+    if (total <= kSmemLimit || p.nstage == 1) return total;
+  }
+  return -1;
+}
+
+int launch_rc(cudaError_t e) { return e == cudaSuccess ? KINT_OK : KINT_ERR_LAUNCH; }
+
+// Forward prep + pass 1 (shared by kint_attn_fwd and kint_attn_debug_bins).
+int forward_prologue(const float* Q, const float* K, const float* V, const Params& p, const Workspace& w,
+                     Maps& maps, cudaStream_t s) {
+  const int BH = p.BH, T = p.T, d = p.d, Tp = round_up(T, 32);
+  if (p.x3) {
+    if (launch_prep(Q, w.qh, w.ql, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (launch_prep(K, w.kh, w.kl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (launch_prep(V, nullptr, nullptr, w.vth, w.vtl, BH, T, Tp, d, true, s) != cudaSuccess)
+      return KINT_ERR_LAUNCH;
+  } else {
+    if (launch_prep(V, nullptr, nullptr, w.vth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+      return KINT_ERR_LAUNCH;
+  }
+  std::memset(&maps, 0, sizeof(maps));
+  bool ok = true;
+  if (p.x3) {
+    ok = ok && map_nat(&maps.q, w.qh, BH, T, d, 128) && map_nat(&maps.q_lo, w.ql, BH, T, d, 128);
+    ok = ok && map_nat(&maps.k, w.kh, BH, T, d, 128) && map_nat(&maps.k_lo, w.kl, BH, T, d, 128);
+    ok = ok && map_tr(&maps.vt, w.vth, BH, T, Tp, d) && map_tr(&maps.vt_lo, w.vtl, BH, T, Tp, d);
+  } else {
+    ok = ok && map_nat(&maps.q, Q, BH, T, d, 128) && map_nat(&maps.k, K, BH, T, d, 128);
+    ok = ok && map_tr(&maps.vt, w.vth, BH, T, Tp, d);
+  }
+  if (!ok) return KINT_ERR_LAUNCH;
+  Params ps = p;
+  const int smem = plan_stats(ps);
+  return launch_rc(launch_fwd_stats(maps, ps, smem, s));
+}
+
+int check_stats(const kint_rowstats* st, bool prob) {
+  if (!st || !st->row_max || !st->row_min || !st->arg_max || !st->arg_min || !st->n_max || !st->n_min || !st->W)
+    return KINT_ERR_ARG;
+  if (prob && (!st->W_lerp || !st->O_lerp)) return KINT_ERR_ARG;
+  const void* ptrs[] = {st->row_max, st->row_min, st->arg_max, st->arg_min, st->n_max, st->n_min, st->W};
+  for (const void* q : ptrs)
+    if (!aligned16(q)) return KINT_ERR_ALIGN;
+  if (prob && (!aligned16(st->W_lerp) || !aligned16(st->O_lerp))) return KINT_ERR_ALIGN;
+  return KINT_OK;
+}
+
+void set_stats(Params& p, const kint_rowstats* st) {
+  p.row_max = st->row_max; p.row_min = st->row_min;
+  p.arg_max = st->arg_max; p.arg_min = st->arg_min;
+  p.n_max = st->n_max; p.n_min = st->n_min;
+  p.W = st->W; p.W_lerp = st->W_lerp; p.O_lerp = st->O_lerp;
+}
+
+bool is_prob(const Common& c) {
+  return c.calib != KINT_CALIB_SOFTMAX && c.recon == KINT_RECON_NEAREST && c.ste == KINT_STE_PROB;
+}
+
+}  // namespace
+}  // namespace kint
+
+using namespace kint;
+
+extern "C" {
+
+size_t kint_attn_workspace_bytes(int B, int H, int T, int d, kint_prec prec, int is_bwd) {
+  if (B < 1 || H < 1 || T < 1 || (d != 64 && d != 128)) return 0;
+  if ((long long)B * H * T > (1ll << 31) - 1) return 0;
+  return plan_workspace(nullptr, B * H, T, d, prec == KINT_PREC_3XTF32, is_bwd != 0).bytes;
+}
+
+int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, const kint_rowstats* st, int B, int H,
+                  int T, int d, int Kint, kint_calib calib, float tau, kint_recon recon, kint_ste ste,
+                  kint_grad grad, int causal, kint_prec prec, void* workspace, size_t workspace_bytes,
+                  void* stream) {
+  const Common c{B, H, T, d, Kint, (int)calib, (int)recon, (int)ste, (int)grad, (int)prec, tau};
+  int rc = validate(c, causal);
+  if (rc) return rc;
+  if (!Q || !K || !V || !O) return KINT_ERR_ARG;
+  const bool prob = is_prob(c);
+  if ((rc = check_stats(st, prob))) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O)) return KINT_ERR_ALIGN;
+  const size_t need = kint_attn_workspace_bytes(B, H, T, d, prec, 0);
+  if (!workspace || workspace_bytes < need) return KINT_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return KINT_ERR_ALIGN;
+  unsigned* status = nullptr;
+  if ((rc = device_setup(&status))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  Params p = base_params(c, status);
+  set_stats(p, st);
+  p.Q = Q; p.K = K; p.V = V; p.Out = O;
+  const Workspace w = plan_workspace(static_cast<char*>(workspace), p.BH, T, d, p.x3 != 0, false);
+  Maps maps;
+  if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
+
+  Params pm = p;
+  const int smem = plan_main(pm);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
+  if ((rc = launch_rc(launch_fwd_main(maps, pm, smem, s)))) return rc;
+  if (prob && p.x3) {
+    pm.pv_sel = PV_LERP;
+    if ((rc = launch_rc(launch_fwd_main(maps, pm, smem, s)))) return rc;
+  }
+  return KINT_OK;
+}
+
+int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O, const float* dO,
+                  const kint_rowstats* st, float* dQ, float* dK, float* dV, int B, int H, int T, int d, int Kint,
+                  kint_calib calib, float tau, kint_recon recon, kint_ste ste, kint_grad grad, int causal,
+                  kint_prec prec, void* workspace, size_t workspace_bytes, void* stream) {
+  const Common c{B, H, T, d, Kint, (int)calib, (int)recon, (int)ste, (int)grad, (int)prec, tau};
+  int rc = validate(c, causal);
+  if (rc) return rc;
+  if (!Q || !K || !V || !O || !dO || !dQ || !dK || !dV) return KINT_ERR_ARG;
+  const bool prob = is_prob(c);
+  if ((rc = check_stats(st, prob))) return rc;
+  const void* ptrs[] = {Q, K, V, O, dO, dQ, dK, dV};
+  for (const void* q : ptrs)
+    if (!aligned16(q)) return KINT_ERR_ALIGN;
+  const size_t need = kint_attn_workspace_bytes(B, H, T, d, prec, 1);
+  if (!workspace || workspace_bytes < need) return KINT_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return KINT_ERR_ALIGN;
+  unsigned* status = nullptr;
+  if ((rc = device_setup(&status))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  Params p = base_params(c, status);
+  set_stats(p, st);
+  p.Q = Q; p.K = K; p.V = V; p.O = O; p.dO = dO;
+  p.Ostar = prob ? st->O_lerp : O;
+  p.dQ = dQ; p.dK = dK; p.dV = dV;
+  const int BH = p.BH, Tp = round_up(T, 32);
+  const Workspace w = plan_workspace(static_cast<char*>(workspace), BH, T, d, p.x3 != 0, true);
+  p.Drow = w.Drow; p.cMn = w.cMn; p.cmn = w.cmn; p.tie_acc = w.tie;
+
+  // Operand copies: K-major transposes (and 3xTF32 splits).
+  if (p.x3) {
+    if (launch_prep(Q, w.qh, w.ql, w.qth, w.qtl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (launch_prep(K, w.kh, w.kl, w.kth, w.ktl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (launch_prep(V, w.vh, w.vl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (launch_prep(dO, w.doh, w.dol, w.doth, w.dotl, BH, T, Tp, d, true, s) != cudaSuccess)
+      return KINT_ERR_LAUNCH;
+  } else {
+    if (launch_prep(Q, nullptr, nullptr, w.qth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+      return KINT_ERR_LAUNCH;
+    if (launch_prep(K, nullptr, nullptr, w.kth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+      return KINT_ERR_LAUNCH;
+    if (launch_prep(dO, nullptr, nullptr, w.doth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+      return KINT_ERR_LAUNCH;
+  }
+  Maps maps;
+  std::memset(&maps, 0, sizeof(maps));
+  bool ok = true;
+  if (p.x3) {
+    ok = ok && map_nat(&maps.k, w.kh, BH, T, d, 64) && map_nat(&maps.k_lo, w.kl, BH, T, d, 64);
+    ok = ok && map_nat(&maps.v, w.vh, BH, T, d, 64) && map_nat(&maps.v_lo, w.vl, BH, T, d, 64);
+    ok = ok && map_nat(&maps.q, w.qh, BH, T, d, 64) && map_nat(&maps.q_lo, w.ql, BH, T, d, 64);
+    ok = ok && map_nat(&maps.dout, w.doh, BH, T, d, 64) && map_nat(&maps.dout_lo, w.dol, BH, T, d, 64);
+    ok = ok && map_tr(&maps.kt, w.kth, BH, T, Tp, d) && map_tr(&maps.kt_lo, w.ktl, BH, T, Tp, d);
+    ok = ok && map_tr(&maps.qt, w.qth, BH, T, Tp, d) && map_tr(&maps.qt_lo, w.qtl, BH, T, Tp, d);
+    ok = ok && map_tr(&maps.dot, w.doth, BH, T, Tp, d) && map_tr(&maps.dot_lo, w.dotl, BH, T, Tp, d);
+  } else {
+    ok = ok && map_nat(&maps.k, K, BH, T, d, 64) && map_nat(&maps.v, V, BH, T, d, 64);
+    ok = ok && map_nat(&maps.q, Q, BH, T, d, 64) && map_nat(&maps.dout, dO, BH, T, d, 64);
+    ok = ok && map_tr(&maps.kt, w.kth, BH, T, Tp, d) && map_tr(&maps.qt, w.qth, BH, T, Tp, d);
+    ok = ok && map_tr(&maps.dot, w.doth, BH, T, Tp, d);
+  }
+  if (!ok) return KINT_ERR_LAUNCH;
+
+  Params pq = p;
+  const int smem_dq = plan_dq(pq);
+  if (smem_dq < 0 || smem_dq > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  if ((rc = launch_rc(launch_bwd_dq(maps, pq, smem_dq, s)))) return rc;
+
+  Params pk = p;
+  const int smem_kv = plan_dkdv(pk);
+  if (smem_kv < 0 || smem_kv > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  if (!p.x3 && d == 64) {
+    pk.dkv_sel = DKV_BOTH;
+    return launch_rc(launch_bwd_dkdv(maps, pk, smem_kv, s));
+  }
+  pk.dkv_sel = DKV_DV;
+  if ((rc = launch_rc(launch_bwd_dkdv(maps, pk, smem_kv, s)))) return rc;
+  pk.dkv_sel = DKV_DK;
+  return launch_rc(launch_bwd_dkdv(maps, pk, smem_kv, s));
+}
+
+int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const kint_rowstats* st, uint8_t* bins,
+                         uint8_t* ivals, int B, int H, int T, int d, int Kint, kint_calib calib, float tau,
+                         kint_recon recon, kint_ste ste, int causal, kint_prec prec, void* workspace,
+                         size_t workspace_bytes, void* stream) {
+  const Common c{B, H, T, d, Kint, (int)calib, (int)recon, (int)ste, 0, (int)prec, tau};
+  int rc = validate(c, causal);
+  if (rc) return rc;
+  if (!Q || !K || !V || (!bins && !ivals)) return KINT_ERR_ARG;
+  if ((rc = check_stats(st, false))) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V)) return KINT_ERR_ALIGN;
+  if ((bins && !aligned16(bins)) || (ivals && !aligned16(ivals))) return KINT_ERR_ALIGN;
+  const size_t need = kint_attn_workspace_bytes(B, H, T, d, prec, 0);
+  if (!workspace || workspace_bytes < need) return KINT_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return KINT_ERR_ALIGN;
+  unsigned* status = nullptr;
+  if ((rc = device_setup(&status))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  Params p = base_params(c, status);
+  // the decisions need only the extrema; W / W_lerp / O are not written in debug mode
+  set_stats(p, st);
+  p.Q = Q; p.K = K; p.V = V;
+  const size_t n = (size_t)B * H * T * T;
+  if (bins && cudaMemsetAsync(bins, 255, n, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+  if (ivals && cudaMemsetAsync(ivals, 255, n, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+  const Workspace w = plan_workspace(static_cast<char*>(workspace), p.BH, T, d, p.x3 != 0, false);
+  Maps maps;
+  if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
+  Params pm = p;
+  const int smem = plan_main(pm);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  pm.pv_sel = PV_MAIN;
+  pm.debug = 1;
+  pm.bins = bins;
+  pm.ivals = ivals;
+  return launch_rc(launch_fwd_main(maps, pm, smem, s));
+}
+
+int kint_get_status(void* stream, unsigned* detail) {
+  unsigned* status = nullptr;
+  int rc = device_setup(&status);
+  if (rc) return rc;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return KINT_ERR_LAUNCH;
+  unsigned v = 0;
+  if (cudaMemcpy(&v, status, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return KINT_ERR_LAUNCH;
+  if (v && cudaMemset(status, 0, sizeof(unsigned)) != cudaSuccess) return KINT_ERR_LAUNCH;
+  if (detail) *detail = v;
+  return v ? KINT_ERR_DEVICE : KINT_OK;
+}
+
+const char* kint_strerror(int code) {
+  switch (code) {
+    case KINT_OK: return "ok";
+    case KINT_ERR_ARG: return "invalid argument";
+    case KINT_ERR_UNSUPPORTED: return "unsupported size or mode (d must be 64 or 128; 3xTF32 needs d = 64)";
+    case KINT_ERR_ALIGN: return "device pointer not 16-byte aligned";
+    case KINT_ERR_WORKSPACE: return "workspace missing or too small";
+    case KINT_ERR_LAUNCH: return "CUDA launch or tensor-map encoding failed";
+    case KINT_ERR_DEVICE: return "a kernel flagged a device-side fault (bounded wait timed out)";
+    case KINT_ERR_NO_DEVICE: return "no sm_103 device is current, or the driver lacks tensor maps";
+    default: return "unknown error code";
+  }
+}
+
+void kint_set_wait_timeout_ns(unsigned long long ns) { g_wait_ns = ns < 1000ull ? 1000ull : ns; }
+
+}  // extern "C"

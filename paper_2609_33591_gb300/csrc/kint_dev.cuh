@@ -1,0 +1,162 @@
+// Device building blocks of the K-interval attention kernels: the per-row grid
+// (Sec. 3 "Objects and calibration", App. A), the per-key decisions and weights
+// (App. A "LERP", "Nearest"), and the tile movement / tensor-core helpers.
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+#include "kint_params.h"
+#include "tc.cuh"
+
+namespace kint {
+
+constexpr int NT = 128;              // threads per CTA; thread t owns TMEM lane t
+constexpr int SW = 128;              // bytes of one swizzled panel row (32 fp32)
+
+__device__ __forceinline__ uint8_t* smem_base() {
+  extern __shared__ uint8_t smem_raw[];
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+}
+
+// CTA-wide "did anyone fail" barrier.  Every thread reaches it, so a thread that
+// timed out in a bounded wait never leaves another one behind.
+__device__ __forceinline__ bool cta_any(bool failed) { return __syncthreads_or(failed ? 1 : 0) != 0; }
+
+// ---------------------------------------------------------------------------
+// Row grid.  Scores s are fp32 values of acc * scale.  The position of a key in
+// grid units is u = s * inv_h + c0:
+//   MinMax: u = (s - m) / h, h = (M - m) / K       (App. A "MinMax grid")
+//   FWM:    u = (s - M + tau) / h, h = tau / K      (App. A "FWM")
+// so u in [0, K] inside the grid; FWM keys with u < 0 are the zero tail.
+// Every kernel builds it with this one function, so decisions agree bitwise
+// between the passes.
+// ---------------------------------------------------------------------------
+struct RowGrid {
+  float inv_h, c0, h, b0;
+  bool nogrid;  // degenerate MinMax row (M - m <= 1e-12) or softmax
+};
+
+__device__ __forceinline__ RowGrid row_grid(const Params& p, float M, float m) {
+  RowGrid g;
+  if (p.calib == CAL_MINMAX) {
+    const float span = __fsub_rn(M, m);
+    g.nogrid = !(span > 1e-12f);
+    const float sp = g.nogrid ? 1.0f : span;
+    g.h = __fdiv_rn(sp, (float)p.Kint);
+    g.inv_h = __fdiv_rn((float)p.Kint, sp);
+    g.c0 = -__fmul_rn(m, g.inv_h);
+    g.b0 = __fsub_rn(m, M);
+  } else if (p.calib == CAL_FWM) {
+    g.nogrid = false;
+    g.h = __fdiv_rn(p.tau, (float)p.Kint);
+    g.inv_h = p.fwm_inv_h;
+    g.c0 = __fmul_rn(__fsub_rn(p.tau, M), g.inv_h);
+    g.b0 = -p.tau;
+  } else {
+    g.nogrid = true;
+    g.h = 1.0f;
+    g.inv_h = 1.0f;
+    g.c0 = 0.0f;
+    g.b0 = 0.0f;
+  }
+  return g;
+}
+
+// Grid value e^{b_r}, r = 0..K.  MinMax: b_r = b0 + r h from the row's own
+// extrema (device expf, K + 1 calls per row).  FWM: host table.
+__device__ __forceinline__ float grid_value(const Params& p, const RowGrid& g, int r) {
+  if (p.calib == CAL_FWM) return p.fwm_e[r];
+  return expf(__fmaf_rn((float)r, g.h, g.b0));
+}
+
+// Per-key decisions of App. A from the grid position u.
+struct KeyPos {
+  int r;     // interval index, clip(floor(u), 0, K-1)
+  int l;     // Nearest index, r + [t >= 1/2]
+  float t;   // position in the interval, clip(u - r, 0, 1)
+  bool tail; // FWM zero tail (z < -tau)
+};
+
+__device__ __forceinline__ KeyPos key_pos(const Params& p, float u) {
+  KeyPos k;
+  k.tail = (p.calib == CAL_FWM) && (u < 0.0f);
+  const float uc = fminf(fmaxf(u, 0.0f), (float)p.Kint);
+  int r = __float2int_rd(uc);
+  r = min(r, p.Kint - 1);
+  k.r = r;
+  k.t = fminf(fmaxf(__fsub_rn(uc, (float)r), 0.0f), 1.0f);
+  k.l = r + (k.t >= 0.5f ? 1 : 0);
+  return k;
+}
+
+// ---------------------------------------------------------------------------
+// Tiles.  Every operand tile in shared memory is stored as 32-column panels of
+// 128-byte rows in the 128-byte swizzle that TMA writes and tcgen05 reads:
+//   natural tile    X[row0 .. row0+R) x [0, d):  d/32 panels of R*128 bytes
+//   transposed tile X^T[0 .. d) x [key0, key0+C): C/32 panels of d*128 bytes
+// In both, "rows" are the MMA's M or N index and the 32-wide panels run along K.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void load_rows_tile(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int ncols,
+                                               int nrows, int c_first, int r_first, int bh) {
+  // ncols/32 panels of nrows x 32 fp32 from coordinates (c_first + 32 p, r_first, bh)
+  for (int pnl = 0; pnl < ncols / 32; ++pnl)
+    tma_load_3d(dst + pnl * nrows * SW, map, bar, c_first + 32 * pnl, r_first, bh);
+}
+
+// D[tmem, M=128 x N] (+)= A * B^T over Ktot, A in smem (128-row panels), B in
+// smem (N-row panels).
+__device__ __forceinline__ void mma_smem_smem(uint32_t d_tmem, const uint8_t* a, const uint8_t* b, int N, int Ktot,
+                                              bool accumulate) {
+  const uint32_t idesc = idesc_tf32(128, N, 0, 0);
+  for (int kk = 0; kk < Ktot / 8; ++kk) {
+    const uint64_t ad = smem_desc_sw128(smem_u32(a + (kk >> 2) * (128 * SW) + (kk & 3) * 32), 16, 1024);
+    const uint64_t bd = smem_desc_sw128(smem_u32(b + (kk >> 2) * (N * SW) + (kk & 3) * 32), 16, 1024);
+    mma_tf32_ss(d_tmem, ad, bd, idesc, (accumulate || kk > 0) ? 1u : 0u);
+  }
+}
+// D[tmem, M=128 x N] (+)= A * B^T over Ktot, A in TMEM columns [a_col, a_col+Ktot).
+__device__ __forceinline__ void mma_tmem_smem(uint32_t d_tmem, uint32_t a_tmem, const uint8_t* b, int N, int Ktot,
+                                              bool accumulate) {
+  const uint32_t idesc = idesc_tf32(128, N, 0, 0);
+  for (int kk = 0; kk < Ktot / 8; ++kk) {
+    const uint64_t bd = smem_desc_sw128(smem_u32(b + (kk >> 2) * (N * SW) + (kk & 3) * 32), 16, 1024);
+    mma_tf32_ts(d_tmem, a_tmem + kk * 8, bd, idesc, (accumulate || kk > 0) ? 1u : 0u);
+  }
+}
+
+// The calling thread's TMEM lane (its row) at column `col`.
+__device__ __forceinline__ uint32_t lane_addr(uint32_t tmem_base, int col) {
+  const int warp = threadIdx.x >> 5;
+  return tmem_base + ((uint32_t)(warp * 32) << 16) + (uint32_t)col;
+}
+
+// Thread-owned row `row` of X (d fp32) into the thread's TMEM lane at columns
+// [col, col+d); with `split`, the tf32 hi part there and the lo part at
+// [col+d, col+2d).  Rows >= T load zeros.  Whole warps must call this.
+__device__ __forceinline__ void row_to_tmem(uint32_t tmem_base, int col, const float* X, int row, int T, int d,
+                                            bool split) {
+  const bool in = row < T;
+  const float4* src = reinterpret_cast<const float4*>(X + (size_t)row * d);
+  for (int c = 0; c < d; c += 32) {
+    float hi[32], lo[32];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      float4 v = in ? __ldg(src + (c >> 2) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+      hi[4 * q + 0] = v.x;
+      hi[4 * q + 1] = v.y;
+      hi[4 * q + 2] = v.z;
+      hi[4 * q + 3] = v.w;
+    }
+    if (split) {
+#pragma unroll
+      for (int q = 0; q < 32; ++q) {
+        const float h = tf32_rna(hi[q]);
+        lo[q] = __fsub_rn(hi[q], h);
+        hi[q] = h;
+      }
+      tmem_st32(lane_addr(tmem_base, col + d + c), lo);
+    }
+    tmem_st32(lane_addr(tmem_base, col + c), hi);
+  }
+}
+
+}  // namespace kint

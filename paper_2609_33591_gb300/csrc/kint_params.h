@@ -1,0 +1,54 @@
+// Launch parameters shared by the host launcher and the kernels of libkint.
+// Plain data only; the tensor maps travel separately as __grid_constant__.
+#pragma once
+#include <cstdint>
+#include <cuda.h>
+
+namespace kint {
+
+enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2 };
+enum Recon : int { REC_LERP = 0, REC_NEAREST = 1 };
+
+constexpr int KMAX = 64;  // largest number of intervals K
+
+// Which weights a forward main-pass launch feeds to the P V contraction.
+enum PvSel : int {
+  PV_MAIN = 0,       // forward weights (w^N, w^L or e^z) -> O, W
+  PV_MAIN_LERP = 1,  // both: forward weights -> O, w^L -> O_lerp (TF32 only)
+  PV_LERP = 2,       // w^L -> O_lerp, W_lerp (second launch of 3xTF32 Prob-STE)
+};
+// Which products a dK/dV launch computes.
+enum DkvSel : int { DKV_BOTH = 0, DKV_DV = 1, DKV_DK = 2 };
+
+// Every TMA descriptor a launch may use.  Natural maps view X as [BH][T][d]
+// (box 32 x rows); transposed maps view X^T as [BH][d][Tp] (box 32 x d).
+struct Maps {
+  CUtensorMap q, q_lo, k, k_lo, v, v_lo, dout, dout_lo;  // natural
+  CUtensorMap kt, kt_lo, vt, vt_lo, qt, qt_lo, dot, dot_lo;  // transposed
+};
+
+struct Params {
+  int B, H, T, d, Kint, calib, recon, ste, grad, x3;
+  int BH, nqb;  // number of 128-row query blocks
+  float tau, scale;       // scale = 1/sqrt(d)
+  float fwm_inv_h;        // K / tau (FWM), host-rounded
+  float fwm_e[KMAX + 2];  // FWM grid values e^{-tau + r tau/K}, r = 0..K (host fp64 -> fp32)
+  int pv_sel, dkv_sel, debug;
+  unsigned long long wait_ns;
+  unsigned* status;
+
+  // smem plan (byte offsets from the 1024-aligned base), set by the host
+  int sm_a, sm_stage0, sm_stage_bytes, nstage, sm_table, sm_rows, sm_bars;
+
+  // tensors (device pointers)
+  const float *Q, *K, *V, *O, *dO, *Ostar;
+  float* Out;
+  float *row_max, *row_min, *W, *W_lerp, *O_lerp;
+  int32_t *arg_max, *arg_min, *n_max, *n_min;
+  float *dQ, *dK, *dV;
+  float *Drow, *cMn, *cmn;  // per-row backward scalars (workspace)
+  float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
+  uint8_t *bins, *ivals;
+};
+
+}  // namespace kint

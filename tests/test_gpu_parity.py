@@ -1,0 +1,111 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on the
+same seeded inputs, element by element, for every variant of the operator."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_33591_gb300 import kint
+from paper_2609_33591_gb300.inputs import make_qkvdo
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+MM, FW, SM = kint.CALIB_MINMAX, kint.CALIB_FWM, kint.CALIB_SOFTMAX
+LE, NE = kint.RECON_LERP, kint.RECON_NEAREST
+WE, PR = kint.STE_WEIGHT, kint.STE_PROB
+FU, DE = kint.GRAD_FULL, kint.GRAD_DETACH
+X3, TF = kint.PREC_3XTF32, kint.PREC_TF32
+
+COMBOS = [(c, r, s, g) for c in (MM, FW) for r in (LE, NE) for s in (WE, PR) for g in (FU, DE)]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    kint.load()
+
+
+def _cfg(c, r, s, g, K=4, tau=8.0):
+    return kint.Config(Kint=K, calib=c, tau=tau, recon=r, ste=s, grad=g)
+
+
+def test_tiny_config_3xtf32_bit_exact_decisions():
+    """B=1, H=2, T=128, d=64, K=4, MinMax, LERP, Weight-STE, full gradient, seed 0."""
+    Q, K, V, dO = make_qkvdo(1, 2, 128, 64, seed=0)
+    rep = parity.check(Q, K, V, dO, _cfg(MM, LE, WE, FU), X3)
+    assert rep["bins_flips"] == 0 and rep["ivals_flips"] == 0
+    assert rep["arg_max_flips"] == 0 and rep["arg_min_flips"] == 0
+
+
+@pytest.mark.parametrize("c,r,s,g", COMBOS)
+@pytest.mark.parametrize("Kint", [4, 8, 16])
+def test_all_variants_3xtf32_ragged(c, r, s, g, Kint):
+    """Every combination at K in {4, 8, 16}; T = 300 spans three 128-row tiles and a ragged tail."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=2)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, g, Kint), X3)
+
+
+@pytest.mark.parametrize("c,r,s,g", COMBOS)
+def test_all_variants_tf32(c, r, s, g):
+    Q, K, V, dO = make_qkvdo(2, 2, 200, 64, seed=2)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, g, 4), TF)
+
+
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_softmax_comparator(prec):
+    Q, K, V, dO = make_qkvdo(1, 2, 260, 64, seed=5)
+    parity.check(Q, K, V, dO, _cfg(SM, LE, WE, FU), prec)
+
+
+@pytest.mark.parametrize("c,r,s", [(MM, LE, WE), (FW, NE, WE), (FW, NE, PR), (MM, NE, PR)])
+def test_head_dim_128_tf32(c, r, s):
+    Q, K, V, dO = make_qkvdo(1, 2, 200, 128, seed=6)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, FU, 4), TF)
+
+
+@pytest.mark.parametrize("T", [1, 2, 63, 64, 65, 127, 129, 257])
+def test_lengths(T):
+    Q, K, V, dO = make_qkvdo(1, 1, T, 64, seed=7)
+    for cfg in (_cfg(MM, NE, WE, FU), _cfg(FW, NE, PR, FU)):
+        parity.check(Q, K, V, dO, cfg, X3)
+
+
+def test_degenerate_and_tied_rows():
+    """Q = 0 makes every MinMax row degenerate and every FWM row all-equal; duplicate keys tie."""
+    Q, K, V, dO = make_qkvdo(1, 1, 140, 64, seed=8)
+    Qz = np.zeros_like(Q)
+    for cfg in (_cfg(MM, LE, WE, FU), _cfg(MM, NE, PR, FU), _cfg(FW, NE, WE, FU), _cfg(FW, LE, PR, FU)):
+        parity.check(Qz, K, V, dO, cfg, X3)
+    Kd = K.copy()
+    Kd[0, 0, 5] = Kd[0, 0, 2]
+    Kd[0, 0, 130] = Kd[0, 0, 2]
+    Kd[0, 0, 77] = Kd[0, 0, 40]
+    for cfg in (_cfg(MM, LE, WE, FU), _cfg(MM, NE, WE, FU), _cfg(FW, NE, PR, FU)):
+        parity.check(Q * 3, Kd, V, dO, cfg, X3)
+
+
+def test_fwm_far_tail():
+    """Scores spread far beyond tau: every key but the maximum falls in the zero tail."""
+    Q, K, V, dO = make_qkvdo(1, 1, 150, 64, seed=9)
+    for cfg in (_cfg(FW, NE, WE, FU, tau=2.0), _cfg(FW, LE, PR, FU, tau=2.0)):
+        parity.check(Q * 20, K, V, dO, cfg, X3)
+
+
+def test_large_K():
+    Q, K, V, dO = make_qkvdo(1, 2, 200, 64, seed=10)
+    for Kint in (1, 64):
+        parity.check(Q, K, V, dO, _cfg(MM, NE, WE, FU, Kint), X3)
+        parity.check(Q, K, V, dO, _cfg(FW, LE, PR, FU, Kint), X3)
+
+
+def test_value_ones_rows_sum_to_one():
+    """V = 1 gives O = 1 when the rows of P sum to one (App. A, Normalization).  O is the tensor-core sum
+    of w_j over the fp32 sum W of the same n <= T weights, so |O - 1| is bounded by the two fp32
+    summation errors, about 2 n 2^-24."""
+    T = 300
+    Q, K, _, dO = make_qkvdo(1, 2, T, 64, seed=11)
+    V = np.ones_like(Q)
+    for cfg in (_cfg(MM, NE, WE, FU), _cfg(FW, NE, PR, FU), _cfg(SM, LE, WE, FU)):
+        g = parity.run_gpu(Q, K, V, dO, cfg, X3, want_bins=False, want_bwd=False)
+        assert np.max(np.abs(g["O"] - 1.0)) <= 2 * T * 2.0 ** -24
