@@ -1,0 +1,361 @@
+#!/usr/bin/env python
+"""Throughput of K-interval attention forward + backward on GB300.
+
+One step = kint_attn_fwd + kint_attn_bwd over one batch of the GPT-2-small
+attention layer (B=8, H=12, T=1024, d=64, causal; K=4, FWM tau=8, Nearest,
+Prob-STE, full calibration gradient; TF32 tensor products), inputs resident in
+HBM.  The metric is algorithmic TFLOP/s: 6 causal T x T x d contractions per
+step (QK^T, PV, dP, dV, dQ, dK), 6 * B*H*d*T*(T+1) flops.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl cuda|reference]
+
+With N > 1 (launched by torch.distributed.run) every rank runs its own replica
+of the workload on its own GPU (the operator shards over (b, h) with no
+exchange); the value is the work of all ranks over the slowest rank's time.
+``--impl reference`` times the fp64 CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "K-interval attn fwd+bwd TFLOP/s @GPT-2-small shape; % of TF32 tensor peak"
+UNIT = "TFLOP/s"
+SHAPE = dict(B=8, H=12, T=1024, d=64)
+VARIANT = dict(Kint=4, calib=1, tau=8.0, recon=1, ste=1, grad=0)  # FWM tau=8, Nearest, Prob-STE, full
+WORKLOAD = ("GPT-2-small attention layer: B=8, H=12, T=1024, d_head=64, causal; K=4, FWM tau=8, Nearest, "
+            "Prob-STE, full calibration gradients; fwd+bwd")
+N_INPUT_SETS = 3  # rotated so that no step reads inputs the previous step left in L2
+TF32_PER_BF16 = 0.5  # nominal dense TF32 : BF16 tensor rate on GB300 (1.125 : 2.25 PFLOP/s)
+
+
+def unit_flops(B, H, T, d):
+    """One causal T x T x d contraction over all heads: 2 * B*H*d*T(T+1)/2 flops."""
+    return B * H * d * T * (T + 1)
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            m = json.load(f)
+        return {"hbm_gbs": float(m["hbm_gbs"]), "bf16": float(m["bf16_tflops"]),
+                "bf16_sustained": float(m.get("bf16_tflops_sustained", m["bf16_tflops"])), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = max(mx, float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"samples": 0}
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        import torch
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def cpu_oracle_rate(n_heads: int):
+    """Time the fp64 oracle (fwd + bwd) on the first n_heads (b, h) heads of the
+    workload at full length; return (TFLOP/s of algorithmic work, seconds, threads)."""
+    import numpy as np
+    import oracle
+    from paper_2609_33591_gb300.inputs import make_qkvdo
+    B, H, T, d = SHAPE["B"], SHAPE["H"], SHAPE["T"], SHAPE["d"]
+    Q, K, V, dO = make_qkvdo(B, H, T, d, seed=1)
+    sl = lambda X: np.ascontiguousarray(X.reshape(B * H, T, d)[:n_heads].reshape(1, n_heads, T, d))
+    q, k, v, do = sl(Q), sl(K), sl(V), sl(dO)
+    cfg = oracle.Config(**VARIANT)
+    threads = min(oracle.hardware_threads(), n_heads)
+    t0 = time.perf_counter()
+    oracle.forward(q, k, v, cfg, lerp_out=True, nthreads=threads)
+    oracle.backward(q, k, v, do, cfg, nthreads=threads)
+    dt = time.perf_counter() - t0
+    return 6 * unit_flops(1, n_heads, T, d) / dt / 1e12, dt, threads
+
+
+def run_reference(args, world, rank):
+    """The oracle as the reference arm, on a bounded sample per step."""
+    if rank != 0:
+        return 0
+    heads = 16
+    for _ in range(args.warmup):
+        cpu_oracle_rate(heads)
+    total_f, total_t, threads = 0.0, 0.0, 1
+    for _ in range(args.steps):
+        _, dt, threads = cpu_oracle_rate(heads)
+        total_t += dt
+        total_f += 6 * unit_flops(1, heads, SHAPE["T"], SHAPE["d"])
+    value = total_f / total_t / 1e12
+    sample = f"{heads} of 96 (b,h) heads at T=1024 per step (fwd+bwd, fp64 oracle)"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_t / args.steps * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": WORKLOAD, **SHAPE, "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# Algorithmic work of one launch of each kernel, in units of one causal contraction
+# (U) or in bytes for the HBM-bound preparation pass.
+KERNEL_WORK = {
+    "k_fwd_stats": ("tensor", 1),  # QK^T (the scores, computed once for the extrema)
+    "k_fwd_main": ("tensor", 1),   # PV (its QK^T is a recomputation)
+    "k_bwd_dq": ("tensor", 2),     # dP = dO V^T, dQ = dS K
+    "k_bwd_dkdv": ("tensor", 2),   # dV = P^T dO, dK = dS^T Q (S^T, dP^T are recomputations)
+    "k_prep": ("hbm", None),       # one read + one write of a [B,H,T,d] fp32 tensor
+}
+
+
+def run_cuda(args, world, rank, local):
+    import torch
+    from paper_2609_33591_gb300 import kint
+    from paper_2609_33591_gb300.inputs import make_qkvdo
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    kint.load()
+    B, H, T, d = SHAPE["B"], SHAPE["H"], SHAPE["T"], SHAPE["d"]
+    cfg = kint.Config(**VARIANT)
+    prec = kint.PREC_TF32
+    Qh, Kh, Vh, dOh = make_qkvdo(B, H, T, d, seed=1)
+    sets = []
+    for _ in range(N_INPUT_SETS):
+        sets.append(tuple(torch.from_numpy(x).to(dev) for x in (Qh, Kh, Vh, dOh)))
+    O = torch.empty_like(sets[0][0])
+    grads = tuple(torch.empty_like(sets[0][0]) for _ in range(3))
+    st = kint.alloc_rowstats(B, H, T, d, dev, cfg.prob)
+    ws_f = kint.workspace(B, H, T, d, prec, 0, dev)
+    ws_b = kint.workspace(B, H, T, d, prec, 1, dev)
+
+    def step(i, c=cfg, p=prec):
+        q, k, v, do = sets[i % N_INPUT_SETS]
+        kint.forward(q, k, v, c, p, O=O, stats=st, ws=ws_f)
+        kint.backward(q, k, v, O, do, st, c, p, grads=grads, ws=ws_b)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    def timed(n, fn):
+        barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for i in range(n):
+            fn(i)
+        e1.record()
+        torch.cuda.synchronize()
+        barrier()
+        ms = e0.elapsed_time(e1) / n
+        if world > 1:
+            t = torch.tensor([ms], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    kint.check_status()
+
+    # per-kernel events through the library's launch-trace hook, during the timed steps
+    events = {}
+    launches = [0]
+    cur_stream = torch.cuda.current_stream()
+
+    def on_launch(name, phase, stream):
+        if phase == 0:
+            launches[0] += 1
+            ev = torch.cuda.Event(enable_timing=True)
+            ev.record(cur_stream)
+            events.setdefault(name, []).append([ev, None])
+        else:
+            ev = torch.cuda.Event(enable_timing=True)
+            ev.record(cur_stream)
+            events[name][-1][1] = ev
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    kint.kint_set_launch_callback(on_launch)
+    ms = timed(args.steps, step)
+    kint.kint_set_launch_callback(None)
+    clocks = sampler.stop()
+    kint.check_status()
+
+    per_kernel = {}
+    for name, lst in events.items():
+        durs = [a.elapsed_time(b) for a, b in lst]
+        per_kernel[name] = {"launches": len(durs), "avg_us": 1e3 * sum(durs) / len(durs),
+                            "total_ms": sum(durs)}
+    flops_step = 6 * unit_flops(B, H, T, d)
+    value = world * flops_step / (ms * 1e-3) / 1e12
+
+    pk = peaks()
+    tf32_peak = pk["bf16"] * TF32_PER_BF16
+    dom = max(per_kernel, key=lambda n: per_kernel[n]["total_ms"])
+    bound, units = KERNEL_WORK[dom]
+    avg_s = per_kernel[dom]["avg_us"] * 1e-6
+    if bound == "tensor":
+        achieved = units * unit_flops(B, H, T, d) / avg_s / 1e12
+        roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": tf32_peak, "unit": "TFLOP/s",
+                "frac": achieved / tf32_peak, "traffic": None,
+                "peak_note": f"TF32 = {TF32_PER_BF16} x {pk['source']} bf16 burst {pk['bf16']} TFLOP/s"}
+    else:
+        nbytes = 2 * B * H * T * d * 4
+        achieved = nbytes / avg_s / 1e9
+        roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "traffic": None}
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "tf32", "data": "synthetic",
+            "config": {"workload": WORKLOAD, **SHAPE, **{k: v for k, v in VARIANT.items()}, "prec": "tf32",
+                       "parallelism": f"replicas x{world} (b,h)-sharded, no collective",
+                       "l2": f"{N_INPUT_SETS} rotating input sets of {4 * B * H * T * d * 4 >> 20} MiB each; "
+                             "per-step traffic (>300 MB) exceeds the 129 MB L2"},
+            "tf32_peak_frac": value / world / tf32_peak,
+            "roofline": roof, "kernels": per_kernel, "gpu_launches": launches[0], "clocks": clocks}
+
+    # plain softmax built the same way, and the 3xTF32 mode, on the same inputs
+    soft = kint.Config(Kint=4, calib=kint.CALIB_SOFTMAX, tau=8.0, recon=kint.RECON_LERP, ste=0, grad=0)
+    n_cmp = max(3, min(args.steps, 200))
+    ms_soft = timed(n_cmp, lambda i: step(i, soft, prec))
+    line["softmax_comparator"] = {"value": world * flops_step / (ms_soft * 1e-3) / 1e12, "unit": UNIT,
+                                  "ms_per_step": ms_soft}
+    ws_f3 = kint.workspace(B, H, T, d, kint.PREC_3XTF32, 0, dev)
+    ws_b3 = kint.workspace(B, H, T, d, kint.PREC_3XTF32, 1, dev)
+
+    def step3(i):
+        q, k, v, do = sets[i % N_INPUT_SETS]
+        kint.forward(q, k, v, cfg, kint.PREC_3XTF32, O=O, stats=st, ws=ws_f3)
+        kint.backward(q, k, v, O, do, st, cfg, kint.PREC_3XTF32, grads=grads, ws=ws_b3)
+
+    step3(0)
+    ms3 = timed(n_cmp, step3)
+    line["x3tf32_mode"] = {"value": world * flops_step / (ms3 * 1e-3) / 1e12, "unit": UNIT, "ms_per_step": ms3}
+    del ws_f3, ws_b3
+
+    # end to end through the public API: pinned host inputs in, results (O, dQ, dK, dV) out, every step
+    pin_in = [torch.from_numpy(x).pin_memory() for x in (Qh, Kh, Vh, dOh)]
+    pin_out = [torch.empty(B, H, T, d).pin_memory() for _ in range(4)]
+    dq, dk, dv = grads
+    q, k, v, do = sets[0]
+
+    def e2e_step(i):
+        for dst, src in zip((q, k, v, do), pin_in):
+            dst.copy_(src, non_blocking=True)
+        kint.forward(q, k, v, cfg, prec, O=O, stats=st, ws=ws_f)
+        kint.backward(q, k, v, O, do, st, cfg, prec, grads=grads, ws=ws_b)
+        for dst, src in zip(pin_out, (O, dq, dk, dv)):
+            dst.copy_(src, non_blocking=True)
+
+    e2e_step(0)
+    n_e2e = max(3, min(args.steps, 100))
+    ms_e2e = timed(n_e2e, e2e_step)
+    line["e2e"] = {"value": world * flops_step / (ms_e2e * 1e-3) / 1e12, "unit": UNIT,
+                   "h2d_bytes_per_step": sum(t.numel() * 4 for t in pin_in),
+                   "d2h_bytes_per_step": sum(t.numel() * 4 for t in pin_out), "ms_per_step": ms_e2e}
+    kint.check_status()
+
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        heads = 48
+        rate, dt, threads = cpu_oracle_rate(heads)
+        line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+                                "sample": f"{heads} of 96 (b,h) heads at T=1024, fwd+bwd, fp64 oracle, "
+                                          f"{dt:.1f} s wall"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    world, rank, local = dist_setup(args.gpus)
+    try:
+        if args.impl == "reference":
+            return run_reference(args, world, rank)
+        return run_cuda(args, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

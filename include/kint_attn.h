@@ -149,6 +149,17 @@ const char* kint_strerror(int code);
  * (default 2e9).  Values < 1000 are clamped to 1000. */
 void kint_set_wait_timeout_ns(unsigned long long ns);
 
+/*
+ * Launch tracing (a profiling aid with no counterpart in the paper).  When set,
+ * cb(kernel_name, phase, stream, user) is called on the host immediately before
+ * (phase 0) and after (phase 1) every kernel launch this library makes, with
+ * the stream the kernel is enqueued on, so a caller can record CUDA events
+ * around single kernels.  NULL disables it.  Process-wide setting; do not
+ * change it while another thread is inside an entry point.
+ */
+typedef void (*kint_launch_cb)(const char* kernel_name, int phase, void* stream, void* user);
+void kint_set_launch_callback(kint_launch_cb cb, void* user);
+
 #ifdef __cplusplus
 }
 #endif

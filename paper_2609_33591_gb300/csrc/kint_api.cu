@@ -240,17 +240,35 @@ int plan_dkdv(Params& p) {
 
 int launch_rc(cudaError_t e) { return e == cudaSuccess ? KINT_OK : KINT_ERR_LAUNCH; }
 
+kint_launch_cb g_cb = nullptr;
+void* g_cb_user = nullptr;
+
+// One kernel launch between the optional tracing callbacks.
+template <class F>
+cudaError_t traced(const char* name, cudaStream_t s, F&& launch) {
+  const kint_launch_cb cb = g_cb;
+  if (cb) cb(name, 0, s, g_cb_user);
+  const cudaError_t e = launch();
+  if (cb) cb(name, 1, s, g_cb_user);
+  return e;
+}
+
+cudaError_t prep(const float* X, float* nat_hi, float* nat_lo, float* tr_hi, float* tr_lo, int BH, int T, int Tp,
+                 int d, bool split, cudaStream_t s) {
+  return traced("k_prep", s, [&] { return launch_prep(X, nat_hi, nat_lo, tr_hi, tr_lo, BH, T, Tp, d, split, s); });
+}
+
 // Forward prep + pass 1 (shared by kint_attn_fwd and kint_attn_debug_bins).
 int forward_prologue(const float* Q, const float* K, const float* V, const Params& p, const Workspace& w,
                      Maps& maps, cudaStream_t s) {
   const int BH = p.BH, T = p.T, d = p.d, Tp = round_up(T, 32);
   if (p.x3) {
-    if (launch_prep(Q, w.qh, w.ql, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (launch_prep(K, w.kh, w.kl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (launch_prep(V, nullptr, nullptr, w.vth, w.vtl, BH, T, Tp, d, true, s) != cudaSuccess)
+    if (prep(Q, w.qh, w.ql, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (prep(K, w.kh, w.kl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (prep(V, nullptr, nullptr, w.vth, w.vtl, BH, T, Tp, d, true, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
   } else {
-    if (launch_prep(V, nullptr, nullptr, w.vth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+    if (prep(V, nullptr, nullptr, w.vth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
   }
   std::memset(&maps, 0, sizeof(maps));
@@ -266,7 +284,7 @@ int forward_prologue(const float* Q, const float* K, const float* V, const Param
   if (!ok) return KINT_ERR_LAUNCH;
   Params ps = p;
   const int smem = plan_stats(ps);
-  return launch_rc(launch_fwd_stats(maps, ps, smem, s));
+  return launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem, s); }));
 }
 
 int check_stats(const kint_rowstats* st, bool prob) {
@@ -333,10 +351,10 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
   const int smem = plan_main(pm);
   if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
-  if ((rc = launch_rc(launch_fwd_main(maps, pm, smem, s)))) return rc;
+  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
   if (prob && p.x3) {
     pm.pv_sel = PV_LERP;
-    if ((rc = launch_rc(launch_fwd_main(maps, pm, smem, s)))) return rc;
+    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
   }
   return KINT_OK;
 }
@@ -372,17 +390,17 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
 
   // Operand copies: K-major transposes (and 3xTF32 splits).
   if (p.x3) {
-    if (launch_prep(Q, w.qh, w.ql, w.qth, w.qtl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (launch_prep(K, w.kh, w.kl, w.kth, w.ktl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (launch_prep(V, w.vh, w.vl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (launch_prep(dO, w.doh, w.dol, w.doth, w.dotl, BH, T, Tp, d, true, s) != cudaSuccess)
+    if (prep(Q, w.qh, w.ql, w.qth, w.qtl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (prep(K, w.kh, w.kl, w.kth, w.ktl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (prep(V, w.vh, w.vl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    if (prep(dO, w.doh, w.dol, w.doth, w.dotl, BH, T, Tp, d, true, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
   } else {
-    if (launch_prep(Q, nullptr, nullptr, w.qth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+    if (prep(Q, nullptr, nullptr, w.qth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
-    if (launch_prep(K, nullptr, nullptr, w.kth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+    if (prep(K, nullptr, nullptr, w.kth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
-    if (launch_prep(dO, nullptr, nullptr, w.doth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+    if (prep(dO, nullptr, nullptr, w.doth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
   }
   Maps maps;
@@ -407,19 +425,19 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   Params pq = p;
   const int smem_dq = plan_dq(pq);
   if (smem_dq < 0 || smem_dq > kSmemLimit) return KINT_ERR_UNSUPPORTED;
-  if ((rc = launch_rc(launch_bwd_dq(maps, pq, smem_dq, s)))) return rc;
+  if ((rc = launch_rc(traced("k_bwd_dq", s, [&] { return launch_bwd_dq(maps, pq, smem_dq, s); })))) return rc;
 
   Params pk = p;
   const int smem_kv = plan_dkdv(pk);
   if (smem_kv < 0 || smem_kv > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   if (!p.x3 && d == 64) {
     pk.dkv_sel = DKV_BOTH;
-    return launch_rc(launch_bwd_dkdv(maps, pk, smem_kv, s));
+    return launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); }));
   }
   pk.dkv_sel = DKV_DV;
-  if ((rc = launch_rc(launch_bwd_dkdv(maps, pk, smem_kv, s)))) return rc;
+  if ((rc = launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); })))) return rc;
   pk.dkv_sel = DKV_DK;
-  return launch_rc(launch_bwd_dkdv(maps, pk, smem_kv, s));
+  return launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); }));
 }
 
 int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const kint_rowstats* st, uint8_t* bins,
@@ -457,7 +475,7 @@ int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const k
   pm.debug = 1;
   pm.bins = bins;
   pm.ivals = ivals;
-  return launch_rc(launch_fwd_main(maps, pm, smem, s));
+  return launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); }));
 }
 
 int kint_get_status(void* stream, unsigned* detail) {
@@ -487,5 +505,10 @@ const char* kint_strerror(int code) {
 }
 
 void kint_set_wait_timeout_ns(unsigned long long ns) { g_wait_ns = ns < 1000ull ? 1000ull : ns; }
+
+void kint_set_launch_callback(kint_launch_cb cb, void* user) {
+  g_cb_user = user;
+  g_cb = cb;
+}
 
 }  // extern "C"

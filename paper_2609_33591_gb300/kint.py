@@ -29,7 +29,9 @@ ERRORS = {0: "KINT_OK", -1: "KINT_ERR_ARG", -2: "KINT_ERR_UNSUPPORTED", -3: "KIN
 
 # Every symbol include/kint_attn.h declares.
 EXPORTS = ("kint_attn_workspace_bytes", "kint_attn_fwd", "kint_attn_bwd", "kint_attn_debug_bins",
-           "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns")
+           "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns", "kint_set_launch_callback")
+
+LAUNCH_CB = ctypes.CFUNCTYPE(None, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p)
 
 
 class KintError(RuntimeError):
@@ -76,6 +78,8 @@ def load(build_if_missing: bool = True):
             lib.kint_strerror.restype = ctypes.c_char_p
             lib.kint_set_wait_timeout_ns.argtypes = [ctypes.c_ulonglong]
             lib.kint_set_wait_timeout_ns.restype = None
+            lib.kint_set_launch_callback.argtypes = [LAUNCH_CB, ctypes.c_void_p]
+            lib.kint_set_launch_callback.restype = None
             _lib = lib
     return _lib
 
@@ -162,6 +166,25 @@ def kint_get_status(stream=None) -> tuple[int, int]:
 
 def kint_set_wait_timeout_ns(ns: int) -> None:
     load().kint_set_wait_timeout_ns(int(ns))
+
+
+_cb_keep = None
+
+
+def kint_set_launch_callback(fn) -> None:
+    """fn(kernel_name: str, phase: int, stream_handle: int) or None.  The C callback
+    object is kept alive here until replaced."""
+    global _cb_keep
+    if fn is None:
+        _cb_keep = None
+        load().kint_set_launch_callback(ctypes.cast(None, LAUNCH_CB), None)
+        return
+
+    def _tramp(name, phase, stream, user):
+        fn(name.decode(), int(phase), stream)
+
+    _cb_keep = LAUNCH_CB(_tramp)
+    load().kint_set_launch_callback(_cb_keep, None)
 
 
 # ---- conveniences that allocate with torch ---------------------------------------------------
