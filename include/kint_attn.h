@@ -48,6 +48,7 @@ extern "C" {
 #define KINT_ERR_LAUNCH (-5)       /* the CUDA runtime refused a launch or a tensor-map encoding */
 #define KINT_ERR_DEVICE (-6)       /* kint_get_status: a kernel flagged a device-side fault */
 #define KINT_ERR_NO_DEVICE (-7)    /* no sm_103 device current, or the driver lacks tensor maps */
+#define KINT_ERR_SCRATCH_LIMIT (-8) /* kint_attn_fwd_noalloc: problem needs more than KINT_NOALLOC_SCRATCH_BYTES */
 
 /* Calibration (Sec. 3 "Objects and calibration"; App. A "MinMax grid", "FWM";
  * App. A "Softmax" is the exact-exponential comparator). */
@@ -159,6 +160,33 @@ void kint_set_wait_timeout_ns(unsigned long long ns);
  */
 typedef void (*kint_launch_cb)(const char* kernel_name, int phase, void* stream, void* user);
 void kint_set_launch_callback(kint_launch_cb cb, void* user);
+
+/*
+ * Forward without a caller-supplied workspace (the paper has no counterpart).
+ *
+ * Some callers cannot hand the library scratch memory: code that runs while a
+ * stream is being captured into a CUDA graph (where cudaMalloc is not allowed),
+ * serving loops that forbid any device allocation after start-up, and plug-in
+ * hosts that pass only input and output buffers.  This entry point behaves like
+ * kint_attn_fwd but takes its scratch from a fixed array of
+ * KINT_NOALLOC_SCRATCH_BYTES that the library keeps in device memory (every GPU
+ * that loads the library holds it until the process exits).  It allocates
+ * nothing.  The caller still provides Q, K, V, O and the row statistics.
+ *   - The first call on a device (with that device current) looks up the
+ *     array's device address; make that first call before any stream capture.
+ *   - Problems whose forward workspace, kint_attn_workspace_bytes(..., 0),
+ *     exceeds KINT_NOALLOC_SCRATCH_BYTES return KINT_ERR_SCRATCH_LIMIT before
+ *     any work is enqueued (TF32 at d = 64 fits B*H*T up to 131072).
+ *   - All calls share the one array: calls whose work overlaps on the GPU
+ *     (different streams, or concurrent host threads) race and must be
+ *     serialised by the caller.  The array keeps the previous call's contents;
+ *     nothing in it needs to start at zero, because every forward writes the
+ *     whole region it later reads.
+ */
+#define KINT_NOALLOC_SCRATCH_BYTES (32u << 20)
+int kint_attn_fwd_noalloc(const float* Q, const float* K, const float* V, float* O, const kint_rowstats* st, int B,
+                          int H, int T, int d, int Kint, kint_calib calib, float tau, kint_recon recon,
+                          kint_ste ste, kint_grad grad, int causal, kint_prec prec, void* stream);
 
 #ifdef __cplusplus
 }

@@ -500,6 +500,7 @@ const char* kint_strerror(int code) {
     case KINT_ERR_LAUNCH: return "CUDA launch or tensor-map encoding failed";
     case KINT_ERR_DEVICE: return "a kernel flagged a device-side fault (bounded wait timed out)";
     case KINT_ERR_NO_DEVICE: return "no sm_103 device is current, or the driver lacks tensor maps";
+    case KINT_ERR_SCRATCH_LIMIT: return "problem too large for the library's fixed scratch (kint_attn_fwd_noalloc)";
     default: return "unknown error code";
   }
 }
@@ -509,6 +510,75 @@ void kint_set_wait_timeout_ns(unsigned long long ns) { g_wait_ns = ns < 1000ull 
 void kint_set_launch_callback(kint_launch_cb cb, void* user) {
   g_cb_user = user;
   g_cb = cb;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Forward with library-owned scratch, for callers that cannot allocate device
+// memory or pass a workspace (see kint_attn_fwd_noalloc in kint_attn.h).  The
+// scratch is this fixed device array; host code never hands its symbol to a
+// kernel, only the device address looked up per device below.
+// ---------------------------------------------------------------------------
+namespace kint {
+namespace {
+static __device__ __align__(256) unsigned char g_noalloc_scratch[KINT_NOALLOC_SCRATCH_BYTES];
+void* g_noalloc_ptr[kMaxDevices] = {nullptr};
+
+// Device address of the scratch array on the current device, looked up once per
+// device with that device current.
+int noalloc_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return KINT_ERR_NO_DEVICE;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return KINT_ERR_NO_DEVICE;
+    g_noalloc_ptr[dev] = ptr;
+  }
+  *out = g_noalloc_ptr[dev];
+  return KINT_OK;
+}
+}  // namespace
+}  // namespace kint
+
+extern "C" {
+
+int kint_attn_fwd_noalloc(const float* Q, const float* K, const float* V, float* O, const kint_rowstats* st, int B,
+                          int H, int T, int d, int Kint, kint_calib calib, float tau, kint_recon recon,
+                          kint_ste ste, kint_grad grad, int causal, kint_prec prec, void* stream) {
+  const Common c{B, H, T, d, Kint, (int)calib, (int)recon, (int)ste, (int)grad, (int)prec, tau};
+  int rc = validate(c, causal);
+  if (rc) return rc;
+  if (!Q || !K || !V || !O) return KINT_ERR_ARG;
+  const bool prob = is_prob(c);
+  if ((rc = check_stats(st, prob))) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(V) || !aligned16(O)) return KINT_ERR_ALIGN;
+  const size_t need = kint_attn_workspace_bytes(B, H, T, d, prec, 0);
+  if (need == 0) return KINT_ERR_UNSUPPORTED;
+  if (need > (size_t)KINT_NOALLOC_SCRATCH_BYTES) return KINT_ERR_SCRATCH_LIMIT;
+  unsigned* status = nullptr;
+  if ((rc = device_setup(&status))) return rc;
+  void* scratch = nullptr;
+  if ((rc = noalloc_scratch(&scratch))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  Params p = base_params(c, status);
+  set_stats(p, st);
+  p.Q = Q; p.K = K; p.V = V; p.Out = O;
+  const Workspace w = plan_workspace(static_cast<char*>(scratch), p.BH, T, d, p.x3 != 0, false);
+  Maps maps;
+  if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
+  Params pm = p;
+  const int smem = plan_main(pm);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
+  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
+  if (prob && p.x3) {
+    pm.pv_sel = PV_LERP;
+    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
+  }
+  return KINT_OK;
 }
 
 }  // extern "C"

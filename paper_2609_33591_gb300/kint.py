@@ -25,11 +25,14 @@ PREC_TF32, PREC_3XTF32 = 0, 1
 CODE_NOGRID, CODE_TAIL, CODE_MASKED = 253, 254, 255
 
 ERRORS = {0: "KINT_OK", -1: "KINT_ERR_ARG", -2: "KINT_ERR_UNSUPPORTED", -3: "KINT_ERR_ALIGN",
-          -4: "KINT_ERR_WORKSPACE", -5: "KINT_ERR_LAUNCH", -6: "KINT_ERR_DEVICE", -7: "KINT_ERR_NO_DEVICE"}
+          -4: "KINT_ERR_WORKSPACE", -5: "KINT_ERR_LAUNCH", -6: "KINT_ERR_DEVICE", -7: "KINT_ERR_NO_DEVICE",
+          -8: "KINT_ERR_SCRATCH_LIMIT"}
+NOALLOC_SCRATCH_BYTES = 32 << 20
 
 # Every symbol include/kint_attn.h declares.
 EXPORTS = ("kint_attn_workspace_bytes", "kint_attn_fwd", "kint_attn_bwd", "kint_attn_debug_bins",
-           "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns", "kint_set_launch_callback")
+           "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns", "kint_set_launch_callback",
+           "kint_attn_fwd_noalloc")
 
 LAUNCH_CB = ctypes.CFUNCTYPE(None, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p)
 
@@ -80,6 +83,9 @@ def load(build_if_missing: bool = True):
             lib.kint_set_wait_timeout_ns.restype = None
             lib.kint_set_launch_callback.argtypes = [LAUNCH_CB, ctypes.c_void_p]
             lib.kint_set_launch_callback.restype = None
+            lib.kint_attn_fwd_noalloc.argtypes = [vp, vp, vp, vp, ctypes.POINTER(kint_rowstats), i, i, i, i, i, i,
+                                                  f, i, i, i, i, i, vp]
+            lib.kint_attn_fwd_noalloc.restype = i
             _lib = lib
     return _lib
 
@@ -147,6 +153,15 @@ def kint_attn_bwd(Q, K, V, O, dO, st: dict, dQ, dK, dV, B, H, T, d, Kint, calib,
                                 T, d, Kint, calib, float(tau), recon, ste, grad, causal, prec, _p(workspace),
                                 0 if workspace is None else workspace.numel() * workspace.element_size(),
                                 _stream(stream))
+
+
+def kint_attn_fwd_noalloc(Q, K, V, O, st: dict, B, H, T, d, Kint, calib, tau, recon, ste, grad, causal, prec,
+                          stream=None) -> int:
+    """Forward with the library's fixed device scratch instead of a workspace: for callers
+    that cannot allocate device memory (e.g. inside stream capture)."""
+    s = _stats_struct(st)
+    return load().kint_attn_fwd_noalloc(_p(Q), _p(K), _p(V), _p(O), ctypes.byref(s), B, H, T, d, Kint, calib,
+                                        float(tau), recon, ste, grad, causal, prec, _stream(stream))
 
 
 def kint_attn_debug_bins(Q, K, V, st: dict, bins, ivals, B, H, T, d, Kint, calib, tau, recon, ste, causal, prec,
