@@ -42,7 +42,8 @@ extern "C" {
 /* Return codes. */
 #define KINT_OK 0
 #define KINT_ERR_ARG (-1)          /* null pointer, size < 1, K out of [1, 64], tau <= 0, bad enum, causal != 1 */
-#define KINT_ERR_UNSUPPORTED (-2)  /* d not in {64, 128}; sizes beyond the limits above */
+#define KINT_ERR_UNSUPPORTED (-2)  /* d not in {64, 128}; 3xTF32 with d != 64; MinMax with K > 32 unless
+                                      TF32 at d = 64; sizes beyond the limits above */
 #define KINT_ERR_ALIGN (-3)        /* a device pointer is not 16-byte aligned */
 #define KINT_ERR_WORKSPACE (-4)    /* workspace NULL or smaller than kint_attn_workspace_bytes() */
 #define KINT_ERR_LAUNCH (-5)       /* the CUDA runtime refused a launch or a tensor-map encoding */

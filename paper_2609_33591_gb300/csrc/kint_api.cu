@@ -150,6 +150,10 @@ int validate(const Common& c, int causal) {
   if (c.calib == KINT_CALIB_FWM && !(c.tau > 0.0f && std::isfinite(c.tau))) return KINT_ERR_ARG;
   if (c.d != 64 && c.d != 128) return KINT_ERR_UNSUPPORTED;
   if (c.prec == KINT_PREC_3XTF32 && c.d != 64) return KINT_ERR_UNSUPPORTED;
+  // MinMax keeps a (K x 128)-pair grid table per query block in shared memory;
+  // above K = 32 it fits only beside the TF32, d = 64 operand tiles.
+  if (c.calib == KINT_CALIB_MINMAX && c.Kint > 32 && (c.prec == KINT_PREC_3XTF32 || c.d != 64))
+    return KINT_ERR_UNSUPPORTED;
   const long long BH = (long long)c.B * c.H;
   if (BH > 65535 || (long long)c.T * BH > (1ll << 31) - 1 || c.T > (1 << 24)) return KINT_ERR_UNSUPPORTED;
   return KINT_OK;
@@ -193,19 +197,33 @@ int plan_stats(Params& p) {
   p.sm_stage0 = parts * tile;
   p.sm_stage_bytes = parts * tile;
   p.nstage = 2;
-  return finish_plan(p, p.sm_stage0 + p.nstage * p.sm_stage_bytes, 3 + p.nstage);
+  p.sm_rows = p.sm_a;  // the 6 x 128 exchange words reuse the Q tile after the last product
+  return finish_plan(p, p.sm_stage0 + p.nstage * p.sm_stage_bytes, 3 + 2 * p.nstage);
 }
 
-int plan_main(Params& p) {
+// mode: PV_MAIN / PV_MAIN_LERP / PV_LERP.  Picks the TMEM score double-buffering
+// and the deepest K/V ring that fit.
+int plan_main(Params& p, int mode) {
   const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
-  const int table = (p.Kint + 1) * 128 * 4;
+  // (e_r, e_{r+1}) pairs: per row for MinMax ([K][128]), one shared [K] for FWM
+  const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : (p.calib == KINT_CALIB_FWM ? 1024 : 0);
+  const bool useA2 = mode == PV_MAIN_LERP || p.x3;
+  const int cols1 = 128 + (useA2 ? 128 : 0) + p.d + (mode == PV_MAIN_LERP ? p.d : 0);
+  p.nbuf = (cols1 + 128 <= 512) ? 2 : 1;
   p.sm_a = 0;
   p.sm_stage0 = parts * tile;
   p.sm_stage_bytes = parts * 2 * tile;
-  for (p.nstage = 2; p.nstage >= 1; --p.nstage) {
+  for (p.nstage = 3; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    const int total = std::max(finish_plan(p, p.sm_table + table, 2 + p.nstage), kOneCtaPerSm);
-    if (total <= kSmemLimit || p.nstage == 1) return total;
+    p.sm_rows = p.sm_a;  // the 4 x 128 exchange words reuse the Q tile after the last product
+    const int total = std::max(finish_plan(p, p.sm_table + table, 4 + 2 * p.nstage), kOneCtaPerSm);
+    if (total <= kSmemLimit) {
+      // Issuing S(kb+1) before P V(kb) needs tile kb+1 in a second stage while
+      // tile kb's V^T is still being read; with one stage the two would wait on
+      // each other, so a single stage means a single score buffer.
+      if (p.nstage == 1) p.nbuf = 1;
+      return total;
+    }
   }
   return -1;
 }
@@ -348,13 +366,16 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
   if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
 
   Params pm = p;
-  const int smem = plan_main(pm);
-  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
+  const int smem = plan_main(pm, pm.pv_sel);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
   if (prob && p.x3) {
-    pm.pv_sel = PV_LERP;
-    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
+    Params pl = p;
+    pl.pv_sel = PV_LERP;
+    const int smem2 = plan_main(pl, PV_LERP);
+    if (smem2 < 0) return KINT_ERR_UNSUPPORTED;
+    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s); })))) return rc;
   }
   return KINT_OK;
 }
@@ -469,9 +490,9 @@ int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const k
   Maps maps;
   if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
   Params pm = p;
-  const int smem = plan_main(pm);
-  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   pm.pv_sel = PV_MAIN;
+  const int smem = plan_main(pm, PV_MAIN);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   pm.debug = 1;
   pm.bins = bins;
   pm.ivals = ivals;
@@ -494,7 +515,9 @@ const char* kint_strerror(int code) {
   switch (code) {
     case KINT_OK: return "ok";
     case KINT_ERR_ARG: return "invalid argument";
-    case KINT_ERR_UNSUPPORTED: return "unsupported size or mode (d must be 64 or 128; 3xTF32 needs d = 64)";
+    case KINT_ERR_UNSUPPORTED:
+      return "unsupported size or mode (d must be 64 or 128; 3xTF32 needs d = 64; MinMax with K > 32 needs TF32 "
+             "at d = 64)";
     case KINT_ERR_ALIGN: return "device pointer not 16-byte aligned";
     case KINT_ERR_WORKSPACE: return "workspace missing or too small";
     case KINT_ERR_LAUNCH: return "CUDA launch or tensor-map encoding failed";
@@ -570,13 +593,16 @@ int kint_attn_fwd_noalloc(const float* Q, const float* K, const float* V, float*
   Maps maps;
   if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
   Params pm = p;
-  const int smem = plan_main(pm);
-  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
+  const int smem = plan_main(pm, pm.pv_sel);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
   if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
   if (prob && p.x3) {
-    pm.pv_sel = PV_LERP;
-    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
+    Params pl = p;
+    pl.pv_sel = PV_LERP;
+    const int smem2 = plan_main(pl, PV_LERP);
+    if (smem2 < 0) return KINT_ERR_UNSUPPORTED;
+    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s); })))) return rc;
   }
   return KINT_OK;
 }

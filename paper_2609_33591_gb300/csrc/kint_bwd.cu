@@ -221,7 +221,7 @@ __global__ void __launch_bounds__(NT, 1) k_bwd_dq(const __grid_constant__ Maps m
           KeyPos kp{0, 0, 0.f, false};
           float er = 0.f, er1 = 0.f, el = 0.f;
           if (p.calib != CAL_SOFTMAX && !R.g.nogrid) {
-            kp = key_pos(p, __fmaf_rn(s, R.g.inv_h, R.g.c0));
+            kp = key_pos(p, __fmaf_rn(sv[jj], R.g.k1, R.g.c0));
             if (!kp.tail) {
               er = tab[kp.r * NT + tid];
               er1 = tab[(kp.r + 1) * NT + tid];
@@ -493,6 +493,7 @@ __global__ void __launch_bounds__(NT, 1) k_bwd_dkdv(const __grid_constant__ Maps
           R.M = qr->M[r_];
           R.m = qr->m[r_];
           R.g.inv_h = qr->inv_h[r_];
+          R.g.k1 = __fmul_rn(p.scale, R.g.inv_h);
           R.g.c0 = qr->c0[r_];
           R.g.nogrid = qr->nogrid[r_] != 0;
           R.invWf = qr->invWf[r_];
@@ -502,7 +503,7 @@ __global__ void __launch_bounds__(NT, 1) k_bwd_dkdv(const __grid_constant__ Maps
           KeyPos kp{0, 0, 0.f, false};
           float er = 0.f, er1 = 0.f, el = 0.f;
           if (p.calib != CAL_SOFTMAX && !R.g.nogrid) {
-            kp = key_pos(p, __fmaf_rn(s, R.g.inv_h, R.g.c0));
+            kp = key_pos(p, __fmaf_rn(sv[ii], R.g.k1, R.g.c0));
             if (!kp.tail) {
               const float* t_ = tab + r_ * tstride;
               er = t_[kp.r];

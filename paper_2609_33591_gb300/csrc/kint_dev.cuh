@@ -21,6 +21,33 @@ __device__ __forceinline__ uint8_t* smem_base() {
 // timed out in a bounded wait never leaves another one behind.
 __device__ __forceinline__ bool cta_any(bool failed) { return __syncthreads_or(failed ? 1 : 0) != 0; }
 
+// Named barrier over the `n` compute threads only (the producer warp never takes
+// part), and its "did anyone fail" reduction.
+__device__ __forceinline__ void group_sync(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ bool group_any(int id, int n, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
+}
+
+// Thread roles of the warp-specialised kernels: NCG column groups of 128
+// compute threads (thread t owns TMEM lane t % 128, columns by group t / 128;
+// thread 0 also issues the tensor-core instructions) and one TMA producer warp.
+constexpr int NCG = 2;
+constexpr int NCOMP = 128 * NCG;
+constexpr int NTHR = NCOMP + 32;
+constexpr int PRODUCER_WARP = NCOMP / 32;
+constexpr int BAR_COMPUTE = 1;  // named barrier id of the compute group
+
 // ---------------------------------------------------------------------------
 // Row grid.  Scores s are fp32 values of acc * scale.  The position of a key in
 // grid units is u = s * inv_h + c0:
@@ -32,6 +59,7 @@ __device__ __forceinline__ bool cta_any(bool failed) { return __syncthreads_or(f
 // ---------------------------------------------------------------------------
 struct RowGrid {
   float inv_h, c0, h, b0;
+  float k1;     // scale * inv_h: u = acc * k1 + c0 straight from the raw accumulator
   bool nogrid;  // degenerate MinMax row (M - m <= 1e-12) or softmax
 };
 
@@ -45,20 +73,59 @@ __device__ __forceinline__ RowGrid row_grid(const Params& p, float M, float m) {
     g.inv_h = __fdiv_rn((float)p.Kint, sp);
     g.c0 = -__fmul_rn(m, g.inv_h);
     g.b0 = __fsub_rn(m, M);
+    g.k1 = __fmul_rn(p.scale, g.inv_h);
   } else if (p.calib == CAL_FWM) {
     g.nogrid = false;
     g.h = __fdiv_rn(p.tau, (float)p.Kint);
     g.inv_h = p.fwm_inv_h;
     g.c0 = __fmul_rn(__fsub_rn(p.tau, M), g.inv_h);
     g.b0 = -p.tau;
+    g.k1 = __fmul_rn(p.scale, g.inv_h);
   } else {
     g.nogrid = true;
     g.h = 1.0f;
     g.inv_h = 1.0f;
     g.c0 = 0.0f;
     g.b0 = 0.0f;
+    g.k1 = 1.0f;
   }
   return g;
+}
+
+// ---------------------------------------------------------------------------
+// Branch-free per-key decisions from the grid position u (App. A):
+//   uc = clip(u, 0, K); r = min(floor(uc), K-1); t = uc - r in [0, 1];
+//   Nearest takes e_{r+1} when t >= 1/2 (l = r + [t >= 1/2], midpoint up).
+// floor uses the float-to-int magic-number method: adding 2^23 with rounding
+// toward -inf leaves 2^23 + floor(uc) exactly for 0 <= uc < 2^23, so the float's
+// bit pattern is 0x4B000000 + r.  `rb` is that bit pattern; a table whose rows
+// are 1024 bytes apart is addressed as base + rb * 1024 (mod 2^32), since
+// 0x4B000000 * 1024 = 0 mod 2^32.
+// ---------------------------------------------------------------------------
+constexpr float kMagic = 8388608.0f;  // 2^23
+
+__device__ __forceinline__ void decode_u(float u, float Kf, float& t, uint32_t& rb, float& rf) {
+  const float uc = fminf(fmaxf(u, 0.0f), Kf);
+  const float fr = fminf(__fadd_rd(uc, kMagic), kMagic + (Kf - 1.0f));
+  rf = __fsub_rn(fr, kMagic);
+  t = __fsub_rn(uc, rf);
+  rb = __float_as_uint(fr);
+}
+
+__device__ __forceinline__ float2 lds_f2(uint32_t addr) {
+  float2 v;
+  asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ float4 lds_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 // Grid value e^{b_r}, r = 0..K.  MinMax: b_r = b0 + r h from the row's own
@@ -123,10 +190,11 @@ __device__ __forceinline__ void mma_tmem_smem(uint32_t d_tmem, uint32_t a_tmem, 
   }
 }
 
-// The calling thread's TMEM lane (its row) at column `col`.
+// The calling thread's TMEM lane (its row) at column `col`.  Warp w may only
+// touch lane quarter w % 4.
 __device__ __forceinline__ uint32_t lane_addr(uint32_t tmem_base, int col) {
   const int warp = threadIdx.x >> 5;
-  return tmem_base + ((uint32_t)(warp * 32) << 16) + (uint32_t)col;
+  return tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)col;
 }
 
 // Thread-owned row `row` of X (d fp32) into the thread's TMEM lane at columns

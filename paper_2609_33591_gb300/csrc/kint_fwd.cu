@@ -58,32 +58,36 @@ cudaError_t launch_prep(const float* X, float* nat_hi, float* nat_lo, float* tr_
 // ---------------------------------------------------------------------------
 // Pass 1: row extrema (App. A: M = max_j s_j, m = min_j s_j over valid keys,
 // lowest index among ties and the tie counts of Table "Edge cases").
-// CTA = one 128-row query block of one head; thread t owns query row
-// qb*128 + t, which is TMEM lane t of the score tile S = Q K^T (M = N = 128).
-// Thread 0 issues TMA and MMA; S is double-buffered in TMEM so the product of
+// CTA = one 128-row query block of one head.  Threads [0, NCOMP) compute:
+// thread t owns query row qb*128 + t%128 (TMEM lane t%128) and the column half
+// t/128 of every 128-key score tile S = Q K^T.  Thread 0 issues the MMAs; the
+// last warp streams K tiles through an nstage-deep TMA ring.  S is
+// double-buffered in TMEM (columns [0,128) and [128,256)), so the product of
 // key tile kb+1 runs while tile kb is reduced.
-// smem: Q tile (hi[, lo]) at sm_a; nstage key stages (K hi[, lo]).
-// TMEM: S buffers at columns [0,128) and [128,256).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(NT, 1) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
-  const int D = p.d, tile = D * 512, parts = p.x3 ? 2 : 1;
+  const int D = p.d, tile = D * 512, parts = p.x3 ? 2 : 1, NS = p.nstage;
   uint8_t* sQ = sm + p.sm_a;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.sm_bars);
   uint64_t* bar_q = bars;
-  uint64_t* bar_st = bars + 1;               // [nstage]
-  uint64_t* bar_mma = bars + 1 + p.nstage;   // [2], one per S buffer
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 + p.nstage);
+  uint64_t* bar_full = bars + 1;
+  uint64_t* bar_empty = bars + 1 + NS;
+  uint64_t* bar_s = bars + 1 + 2 * NS;  // [2]
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 + 2 * NS);
+  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [6][128], aliases Q once all products are done
   const int tid = threadIdx.x, warp = tid >> 5;
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
-  const int i = qb * 128 + tid;
   const int nkb = qb + 1;
 
   if (tid == 0) {
     mbar_init(bar_q, 1);
-    for (int s = 0; s < p.nstage; ++s) mbar_init(&bar_st[s], 1);
-    mbar_init(&bar_mma[0], 1);
-    mbar_init(&bar_mma[1], 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_empty[s], 1);
+    }
+    mbar_init(&bar_s[0], 1);
+    mbar_init(&bar_s[1], 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -95,107 +99,138 @@ __global__ void __launch_bounds__(NT, 1) k_fwd_stats(const __grid_constant__ Map
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  auto stage_ptr = [&](int kb) { return sm + p.sm_stage0 + (kb % p.nstage) * p.sm_stage_bytes; };
-  auto load_k = [&](int kb) {
-    uint64_t* b = &bar_st[kb % p.nstage];
-    uint8_t* dst = stage_ptr(kb);
-    mbar_arrive_expect_tx(b, parts * tile);
-    load_rows_tile(dst, &maps.k, b, D, 128, 0, kb * 128, bh);
-    if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, b, D, 128, 0, kb * 128, bh);
-  };
-  // Thread 0: wait for key tile kb and issue S[kb & 1] = Q K_kb^T.
-  auto issue_s = [&](int kb) -> bool {
-    if (kb == 0 && !mbar_wait(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
-    if (!mbar_wait(&bar_st[kb % p.nstage], (kb / p.nstage) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-      return false;
-    tc_fence_after();
-    const uint8_t* sk = stage_ptr(kb);
-    const uint32_t dcol = tmem + (kb & 1) * 128;
-    if (p.x3) {
-      mma_smem_smem(dcol, sQ + tile, sk, 128, D, false);  // Q_lo K_hi
-      mma_smem_smem(dcol, sQ, sk + tile, 128, D, true);   // Q_hi K_lo
-      mma_smem_smem(dcol, sQ, sk, 128, D, true);          // Q_hi K_hi
-    } else {
-      mma_smem_smem(dcol, sQ, sk, 128, D, false);
-    }
-    mma_commit(&bar_mma[kb & 1]);
-    return true;
-  };
-
-  if (tid == 0) {
-    mbar_arrive_expect_tx(bar_q, parts * tile);
-    load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
-    if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-    for (int kb = 0; kb < min(p.nstage, nkb); ++kb) load_k(kb);
-    issue_s(0);
-  }
-
-  float M = -FLT_MAX, m = FLT_MAX;
-  int amax = 0, amin = 0, nmax = 0, nmin = 0;
-  bool failed = false;
-  for (int kb = 0; kb < nkb; ++kb) {
-    if (tid == 0 && kb + 1 < nkb) {
-      // S[(kb+1)&1] was last read in iteration kb-1 (closed by a CTA barrier).
-      // Its key tile sits in stage (kb+1)%nstage; with one stage that stage is
-      // refilled below only after S[kb] completed, so wait for it here first.
-      if (p.nstage == 1) {
-        // single stage: tile kb+1 is loaded after MMA kb completes (below)
-      } else {
-        issue_s(kb + 1);
+  if (warp == PRODUCER_WARP) {
+    if ((tid & 31) == 0) {
+      mbar_arrive_expect_tx(bar_q, parts * tile);
+      load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
+      if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
+      for (int kb = 0; kb < nkb; ++kb) {
+        const int s = kb % NS;
+        if (kb >= NS &&
+            !mbar_wait(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+          break;
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        mbar_arrive_expect_tx(&bar_full[s], parts * tile);
+        load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
+        if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
       }
     }
-    const bool ok = mbar_wait(&bar_mma[kb & 1], (kb >> 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0) {
-      if (kb + p.nstage < nkb) load_k(kb + p.nstage);  // this stage's product has completed
-      if (p.nstage == 1 && kb + 1 < nkb) issue_s(kb + 1);
-    }
-    const uint32_t scol = (kb & 1) * 128;
+  } else {
+    const int row = tid & 127, cg = tid >> 7;
+    const int i = qb * 128 + row;
+    // Thread 0: wait for key tile kb, issue S[kb & 1] = Q K_kb^T, release the stage.
+    auto issue_s = [&](int kb) {
+      if (kb == 0 && !mbar_wait(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
+      const int s = kb % NS;
+      if (!mbar_wait(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
+      tc_fence_after();
+      const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      const uint32_t dcol = tmem + (kb & 1) * 128;
+      if (p.x3) {
+        mma_smem_smem(dcol, sQ + tile, sk, 128, D, false);  // Q_lo K_hi
+        mma_smem_smem(dcol, sQ, sk + tile, 128, D, true);   // Q_hi K_lo
+        mma_smem_smem(dcol, sQ, sk, 128, D, true);          // Q_hi K_hi
+      } else {
+        mma_smem_smem(dcol, sQ, sk, 128, D, false);
+      }
+      mma_commit(&bar_s[kb & 1]);
+      mma_commit(&bar_empty[s]);
+    };
+    if (tid == 0) issue_s(0);
+
+    float M = -FLT_MAX, m = FLT_MAX;
+    int amax = 0, amin = 0, nmax = 0, nmin = 0;
+    bool failed = false;
+    for (int kb = 0; kb < nkb; ++kb) {
+      if (tid == 0 && kb + 1 < nkb) issue_s(kb + 1);  // S[(kb+1)&1] was last read in iteration kb-1
+      const bool ok = mbar_wait(&bar_s[kb & 1], (kb >> 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      if (group_any(BAR_COMPUTE, NCOMP, !ok)) {
+        failed = true;
+        break;
+      }
+      tc_fence_after();
+      const bool diag = kb == qb;
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
-      float v[32];
-      tmem_ld32(lane_addr(tmem, scol + c * 32), v);
-      tmem_ld_wait();
-      const int j0 = kb * 128 + c * 32;
+      for (int cc = 0; cc < 2; ++cc) {
+        const int c = cg * 2 + cc;
+        float v[32];
+        tmem_ld32(lane_addr(tmem, (kb & 1) * 128 + c * 32), v);
+        tmem_ld_wait();
+        const int j0 = kb * 128 + c * 32;
+        float cmax = -FLT_MAX, cmin = FLT_MAX;
 #pragma unroll
-      for (int jj = 0; jj < 32; ++jj) {
-        const int j = j0 + jj;
-        if (j <= i) {
+        for (int jj = 0; jj < 32; ++jj) {
           const float sc = __fmul_rn(v[jj], p.scale);
-          if (sc > M) {
-            M = sc;
-            amax = j;
-            nmax = 1;
-          } else if (sc == M) {
-            ++nmax;
-          }
-          if (sc < m) {
-            m = sc;
-            amin = j;
-            nmin = 1;
-          } else if (sc == m) {
-            ++nmin;
+          v[jj] = sc;
+          const bool okj = !diag || (j0 + jj <= i);
+          cmax = fmaxf(cmax, okj ? sc : -FLT_MAX);
+          cmin = fminf(cmin, okj ? sc : FLT_MAX);
+        }
+        if (cmax >= M || cmin <= m) {  // rare after the first chunks: exact scan with indices and ties
+          for (int jj = 0; jj < 32; ++jj) {
+            const int j = j0 + jj;
+            if (diag && j > i) break;
+            const float sc = v[jj];
+            if (sc > M) {
+              M = sc;
+              amax = j;
+              nmax = 1;
+            } else if (sc == M) {
+              ++nmax;
+            }
+            if (sc < m) {
+              m = sc;
+              amin = j;
+              nmin = 1;
+            } else if (sc == m) {
+              ++nmin;
+            }
           }
         }
       }
+      tc_fence_before();
+      group_sync(BAR_COMPUTE, NCOMP);
+    }
+    if (!failed) {
+      // combine the two column halves of each row
+      if (cg == 1) {
+        xch[0 * 128 + row] = M;
+        xch[1 * 128 + row] = m;
+        xch[2 * 128 + row] = __int_as_float(amax);
+        xch[3 * 128 + row] = __int_as_float(amin);
+        xch[4 * 128 + row] = __int_as_float(nmax);
+        xch[5 * 128 + row] = __int_as_float(nmin);
+      }
+      group_sync(BAR_COMPUTE, NCOMP);
+      if (cg == 0 && i < p.T) {
+        const float M1 = xch[row], m1 = xch[128 + row];
+        const int amax1 = __float_as_int(xch[256 + row]), amin1 = __float_as_int(xch[384 + row]);
+        const int nmax1 = __float_as_int(xch[512 + row]), nmin1 = __float_as_int(xch[640 + row]);
+        if (M1 > M || (M1 == M && nmax1 > 0 && amax1 < amax)) amax = (M1 > M || nmax == 0) ? amax1 : min(amax, amax1);
+        if (M1 > M) {
+          nmax = nmax1;
+          M = M1;
+        } else if (M1 == M) {
+          nmax += nmax1;
+        }
+        if (m1 < m || (m1 == m && nmin1 > 0 && amin1 < amin)) amin = (m1 < m || nmin == 0) ? amin1 : min(amin, amin1);
+        if (m1 < m) {
+          nmin = nmin1;
+          m = m1;
+        } else if (m1 == m) {
+          nmin += nmin1;
+        }
+        const size_t rw = (size_t)bh * p.T + i;
+        p.row_max[rw] = M;
+        p.row_min[rw] = m;
+        p.arg_max[rw] = amax;
+        p.arg_min[rw] = amin;
+        p.n_max[rw] = nmax;
+        p.n_min[rw] = nmin;
+      }
     }
     tc_fence_before();
-    __syncthreads();
   }
-  if (!failed && i < p.T) {
-    const size_t row = (size_t)bh * p.T + i;
-    p.row_max[row] = M;
-    p.row_min[row] = m;
-    p.arg_max[row] = amax;
-    p.arg_min[row] = amin;
-    p.n_max[row] = nmax;
-    p.n_min[row] = nmin;
-  }
-  tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 256);
 }
@@ -203,45 +238,128 @@ __global__ void __launch_bounds__(NT, 1) k_fwd_stats(const __grid_constant__ Map
 cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(k_fwd_stats, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  k_fwd_stats<<<dim3(p.nqb, p.BH), NT, smem_bytes, s>>>(maps, p);
+  k_fwd_stats<<<dim3(p.nqb, p.BH), NTHR, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------------------
-// Pass 2: per key, the grid position u, the decisions (r, t, l, tail) and the
-// reconstructed weight (App. A "LERP": w^L = (1-t) e_r + t e_{r+1};
-// "Nearest": w^N = e_l; FWM tail: 0), by shared-memory table lookup and FMA in
-// place of the exponential; W = sum w; O = (sum_j w_j V_j) / W.
-// TMEM: S / A (weights as MMA operand A) at [0,128); A2 (second weights, or
-// the lo part of A under 3xTF32) at [128,256); O at [256, 256+d); O_lerp at
-// [256+d, 256+2d).
-// smem: Q (hi[, lo]) at sm_a; stages {K tile, V^T tile} (hi[, lo] each);
-// per-thread grid table [K+1][128] fp32 at sm_table.
+// Pass 2 element work on one 32-key chunk of one row (App. A): the grid
+// position u = acc * k1 + c0, the decisions (r, t, Nearest, FWM tail) and the
+// weights w^L = e_r + t (e_{r+1} - e_r), w^N = (t >= 1/2 ? e_{r+1} : e_r), by a
+// lookup of the pair (e_r, e_{r+1}) in the row's table and one FMA in place of
+// the exponential.  MODE 0: a = forward weight; 1: also w^L for O_lerp; 2: a = w^L.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(NT, 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p) {
+template <int CAL, int REC, int MODE, bool DIAG>
+__device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32], float (&a2)[32], int j0, int i,
+                                          const RowGrid& g, float Kf, uint32_t tab, float sk1, float sc0,
+                                          float& wm_sum, float& wl_sum) {
+  float wm_acc = 0.f, wl_acc = 0.f;
+#pragma unroll
+  for (int jj = 0; jj < 32; ++jj) {
+    float wm, wl = 0.f;
+    if constexpr (CAL == CAL_SOFTMAX) {
+      wm = ex2_approx(__fmaf_rn(v[jj], sk1, sc0));  // e^{s - M} (App. A, Softmax)
+    } else {
+      const float u = __fmaf_rn(v[jj], g.k1, g.c0);
+      float t, rf;
+      uint32_t rb;
+      decode_u(u, Kf, t, rb, rf);
+      // MinMax: this row's table, rows 1024 bytes apart; FWM: one shared table, entries 8 bytes apart
+      const float2 e = lds_f2(CAL == CAL_FWM ? tab + rb * 8u : tab + rb * 1024u);
+      wl = __fmaf_rn(t, __fsub_rn(e.y, e.x), e.x);
+      float wn = (t >= 0.5f) ? e.y : e.x;
+      if constexpr (CAL == CAL_FWM) {
+        const bool tail = u < 0.0f;
+        wl = tail ? 0.f : wl;
+        wn = tail ? 0.f : wn;
+      }
+      if constexpr (CAL == CAL_MINMAX) {
+        wl = g.nogrid ? 1.f : wl;
+        wn = g.nogrid ? 1.f : wn;
+      }
+      wm = (REC == REC_NEAREST) ? wn : wl;
+    }
+    if constexpr (DIAG) {
+      const bool ok = (j0 + jj) <= i;
+      wm = ok ? wm : 0.f;
+      wl = ok ? wl : 0.f;
+    }
+    wm_acc += wm;
+    if constexpr (MODE != 0) wl_acc += wl;
+    a1[jj] = (MODE == 2) ? wl : wm;
+    if constexpr (MODE == 1) a2[jj] = wl;
+  }
+  wm_sum += wm_acc;
+  wl_sum += wl_acc;
+}
+
+// Decision codes of one chunk for kint_attn_debug_bins (not on the timed path).
+__device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, int i, int bh, const RowGrid& g) {
+  if (i >= p.T) return;
+  for (int jj = 0; jj < 32; ++jj) {
+    const int j = j0 + jj;
+    if (j >= p.T) break;
+    uint8_t cb = 255, ci = 255;
+    if (j <= i) {
+      if (p.calib == CAL_SOFTMAX || g.nogrid) {
+        cb = ci = 253;
+      } else {
+        const float u = __fmaf_rn(v[jj], g.k1, g.c0);
+        float t, rf;
+        uint32_t rb;
+        decode_u(u, (float)p.Kint, t, rb, rf);
+        if (p.calib == CAL_FWM && u < 0.0f) {
+          cb = ci = 254;
+        } else {
+          const int r = (int)rf;
+          ci = (uint8_t)r;
+          cb = (uint8_t)(r + (t >= 0.5f ? 1 : 0));
+        }
+      }
+    }
+    const size_t idx = ((size_t)bh * p.T + i) * p.T + j;
+    if (p.bins) p.bins[idx] = cb;
+    if (p.ivals) p.ivals[idx] = ci;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Pass 2: reconstruction, normalization and P V (App. A).
+// TMEM: score buffers S_b at [128 b, 128 b + 128), b < nbuf (the weights
+// overwrite their scores as MMA operand A); A2 (w^L for O_lerp, or the tf32 lo
+// part of A under 3xTF32) at [128 nbuf, +128); O at cO, O_lerp at cO + d.
+// smem: Q (hi[, lo]) at sm_a; stages {K tile, V^T tile} (hi[, lo] each) fed by
+// the producer warp; per-row pair tables (e_r, e_{r+1}) [K][128] at sm_table.
+// ---------------------------------------------------------------------------
+template <int CAL, int REC, int MODE>
+__global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
-  const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1;
-  const int qtile = D * 512;       // [128 x D]
-  const int vtile = D * 512;       // [D x 128] transposed
+  const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
+  const int qtile = D * 512, vtile = D * 512;
   uint8_t* sQ = sm + p.sm_a;
-  float* tab = reinterpret_cast<float*>(sm + p.sm_table);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.sm_bars);
   uint64_t* bar_q = bars;
-  uint64_t* bar_st = bars + 1;
-  uint64_t* bar_mma = bars + 1 + p.nstage;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 + p.nstage);
+  uint64_t* bar_full = bars + 1;
+  uint64_t* bar_empty = bars + 1 + NS;
+  uint64_t* bar_s = bars + 1 + 2 * NS;  // [2]
+  uint64_t* bar_pv = bars + 3 + 2 * NS;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * NS);
+  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [4][128], aliases Q once all products are done
   const int tid = threadIdx.x, warp = tid >> 5;
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
-  const int i = qb * 128 + tid;
-  const bool row_ok = i < p.T;
   const int nkb = qb + 1;
-  const bool nearest = p.recon == REC_NEAREST;
-  const int sel = p.pv_sel;
+  const bool useA2 = (MODE == 1) || p.x3;
+  const int cA2 = 128 * nbuf, cO = cA2 + (useA2 ? 128 : 0), cOL = cO + D;
 
   if (tid == 0) {
     mbar_init(bar_q, 1);
-    for (int s = 0; s < p.nstage; ++s) mbar_init(&bar_st[s], 1);
-    mbar_init(bar_mma, 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_empty[s], 1);
+    }
+    mbar_init(&bar_s[0], 1);
+    mbar_init(&bar_s[1], 1);
+    mbar_init(bar_pv, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -253,192 +371,213 @@ __global__ void __launch_bounds__(NT, 1) k_fwd_main(const __grid_constant__ Maps
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  auto stage_ptr = [&](int kb) { return sm + p.sm_stage0 + (kb % p.nstage) * p.sm_stage_bytes; };
-  auto load_kv = [&](int kb) {
-    uint64_t* b = &bar_st[kb % p.nstage];
-    uint8_t* dst = stage_ptr(kb);
-    mbar_arrive_expect_tx(b, parts * (qtile + vtile));
-    load_rows_tile(dst, &maps.k, b, D, 128, 0, kb * 128, bh);
-    load_rows_tile(dst + parts * qtile, &maps.vt, b, 128, D, kb * 128, 0, bh);
-    if (p.x3) {
-      load_rows_tile(dst + qtile, &maps.k_lo, b, D, 128, 0, kb * 128, bh);
-      load_rows_tile(dst + parts * qtile + vtile, &maps.vt_lo, b, 128, D, kb * 128, 0, bh);
-    }
-  };
-  if (tid == 0) {
-    mbar_arrive_expect_tx(bar_q, parts * qtile);
-    load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
-    if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-    for (int kb = 0; kb < min(p.nstage, nkb); ++kb) load_kv(kb);
-  }
-
-  // Row set-up: extrema from pass 1, grid, per-thread table of e_r.
-  const size_t row = (size_t)bh * p.T + (row_ok ? i : 0);
-  const float M = row_ok ? p.row_max[row] : 0.0f;
-  const float m = row_ok ? p.row_min[row] : 0.0f;
-  const RowGrid g = row_grid(p, M, m);
-  if (p.calib != CAL_SOFTMAX)
-    for (int r = 0; r <= Kq; ++r) tab[r * NT + tid] = grid_value(p, g, r);
-
-  float Wm = 0.0f, Wl = 0.0f;
-  bool failed = false;
-  uint32_t mph = 0;
-  for (int kb = 0; kb < nkb; ++kb) {
-    const uint8_t* st = stage_ptr(kb);
-    if (tid == 0) {
-      bool ok = (kb > 0 || mbar_wait(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) &&
-                mbar_wait(&bar_st[kb % p.nstage], (kb / p.nstage) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-      if (ok) {
-        tc_fence_after();
+  if (warp == PRODUCER_WARP) {
+    if ((tid & 31) == 0) {
+      mbar_arrive_expect_tx(bar_q, parts * qtile);
+      load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
+      if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
+      for (int kb = 0; kb < nkb; ++kb) {
+        const int s = kb % NS;
+        if (kb >= NS &&
+            !mbar_wait(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+          break;
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        mbar_arrive_expect_tx(&bar_full[s], parts * (qtile + vtile));
+        load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
+        load_rows_tile(dst + parts * qtile, &maps.vt, &bar_full[s], 128, D, kb * 128, 0, bh);
         if (p.x3) {
-          mma_smem_smem(tmem, sQ + qtile, st, 128, D, false);
-          mma_smem_smem(tmem, sQ, st + qtile, 128, D, true);
-          mma_smem_smem(tmem, sQ, st, 128, D, true);
-        } else {
-          mma_smem_smem(tmem, sQ, st, 128, D, false);
+          load_rows_tile(dst + qtile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
+          load_rows_tile(dst + parts * qtile + vtile, &maps.vt_lo, &bar_full[s], 128, D, kb * 128, 0, bh);
         }
-        mma_commit(bar_mma);
       }
     }
-    bool ok = mbar_wait(bar_mma, mph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    mph ^= 1;
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
+  } else {
+    const int row = tid & 127, cg = tid >> 7;
+    const int i = qb * 128 + row;
+    const bool row_ok = i < p.T;
+    const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
+    const float M = row_ok ? p.row_max[rw] : 0.0f;
+    const float m = row_ok ? p.row_min[rw] : 0.0f;
+    const RowGrid g = row_grid(p, M, m);
+    const float Kf = (float)Kq;
+    const float sk1 = p.scale * 1.4426950408889634f, sc0 = -M * 1.4426950408889634f;  // softmax, base 2
+    // Pair tables, entry r = (e_r, e_{r+1}), r = 0..K-1, addressed by the float bits
+    // rb = 0x4B000000 + r of the floored position: MinMax keeps one table per row
+    // ([K][128], 1024 bytes per r: rb * 1024 wraps to r * 1024); FWM's grid is the
+    // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r).
+    uint32_t tab;
+    if constexpr (CAL == CAL_FWM) {
+      tab = smem_u32(sm + p.sm_table) - 0x58000000u;
+      if (tid < Kq) *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+    } else {
+      tab = smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
+      if constexpr (CAL == CAL_MINMAX) {
+        for (int r = cg; r < Kq; r += NCG) {
+          const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
+          *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
+        }
+      }
     }
-    tc_fence_after();
+    group_sync(BAR_COMPUTE, NCOMP);
 
+    auto issue_s = [&](int kb) {
+      if (kb == 0 && !mbar_wait(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
+      const int s = kb % NS;
+      if (!mbar_wait(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
+      tc_fence_after();
+      const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      const uint32_t dcol = tmem + (kb % nbuf) * 128;
+      if (p.x3) {
+        mma_smem_smem(dcol, sQ + qtile, sk, 128, D, false);
+        mma_smem_smem(dcol, sQ, sk + qtile, 128, D, true);
+        mma_smem_smem(dcol, sQ, sk, 128, D, true);
+      } else {
+        mma_smem_smem(dcol, sQ, sk, 128, D, false);
+      }
+      mma_commit(&bar_s[kb % nbuf]);
+    };
+    if (tid == 0) issue_s(0);
+
+    float Wm = 0.f, Wl = 0.f;
+    bool failed = false;
+    for (int kb = 0; kb < nkb; ++kb) {
+      if (nbuf == 2 && tid == 0 && kb + 1 < nkb) issue_s(kb + 1);
+      const int b = kb % nbuf;
+      const uint32_t sparity = (nbuf == 2) ? ((kb >> 1) & 1) : (kb & 1);
+      bool ok = mbar_wait(&bar_s[b], sparity, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      if (group_any(BAR_COMPUTE, NCOMP, !ok)) {
+        failed = true;
+        break;
+      }
+      tc_fence_after();
+      const bool diag = kb == qb;
+      bool pv_ok = true;
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
-      float v[32], a1[32], a2[32];
-      tmem_ld32(lane_addr(tmem, c * 32), v);
-      tmem_ld_wait();
-      const int j0 = kb * 128 + c * 32;
-      float wm_part = 0.0f, wl_part = 0.0f;
+      for (int cc = 0; cc < 2; ++cc) {
+        const int c = cg * 2 + cc;
+        float v[32], a1[32], a2[32];
+        tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
+        tmem_ld_wait();
+        const int j0 = kb * 128 + c * 32;
+        if (p.debug) fwd_debug_codes(p, v, j0, i, bh, g);
+        if (diag)
+          fwd_chunk<CAL, REC, MODE, true>(v, a1, a2, j0, i, g, Kf, tab, sk1, sc0, Wm, Wl);
+        else
+          fwd_chunk<CAL, REC, MODE, false>(v, a1, a2, j0, i, g, Kf, tab, sk1, sc0, Wm, Wl);
+        if (p.x3) {
 #pragma unroll
-      for (int jj = 0; jj < 32; ++jj) {
-        const int j = j0 + jj;
-        const bool valid = row_ok && j <= i;
-        const float s = __fmul_rn(v[jj], p.scale);
-        float wmain = 0.0f, wlerp = 0.0f;
-        uint8_t cb = 255, ci = 255;
-        if (valid) {
-          if (p.calib == CAL_SOFTMAX) {
-            wmain = expf(__fsub_rn(s, M));
-            cb = ci = 253;
-          } else if (g.nogrid) {
-            wmain = wlerp = 1.0f;
-            cb = ci = 253;
-          } else {
-            const KeyPos kp = key_pos(p, __fmaf_rn(s, g.inv_h, g.c0));
-            if (kp.tail) {
-              cb = ci = 254;
-            } else {
-              const float er = tab[kp.r * NT + tid];
-              const float er1 = tab[(kp.r + 1) * NT + tid];
-              wlerp = __fmaf_rn(kp.t, __fsub_rn(er1, er), er);
-              wmain = nearest ? tab[kp.l * NT + tid] : wlerp;
-              cb = (uint8_t)kp.l;
-              ci = (uint8_t)kp.r;
+          for (int q = 0; q < 32; ++q) {
+            const float h = tf32_rna(a1[q]);
+            a2[q] = __fsub_rn(a1[q], h);
+            a1[q] = h;
+          }
+        }
+        // A2 is still the operand of the previous tile's products until they complete
+        if (cc == 0 && useA2 && kb > 0)
+          pv_ok = mbar_wait(bar_pv, (kb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+        tmem_st32(lane_addr(tmem, b * 128 + c * 32), a1);
+        if (useA2) tmem_st32(lane_addr(tmem, cA2 + c * 32), a2);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      if (group_any(BAR_COMPUTE, NCOMP, !pv_ok)) {
+        failed = true;
+        break;
+      }
+      if (tid == 0) {
+        tc_fence_after();
+        const uint8_t* vt = sm + p.sm_stage0 + (kb % NS) * p.sm_stage_bytes + parts * qtile;
+        const bool acc = kb > 0;
+        const uint32_t a = tmem + b * 128;
+        if (p.x3) {
+          mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);                // A_hi V_hi
+          mma_tmem_smem(tmem + cO, a, vt + vtile, D, 128, true);       // A_hi V_lo
+          mma_tmem_smem(tmem + cO, tmem + cA2, vt, D, 128, true);      // A_lo V_hi
+        } else {
+          mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);
+          if (MODE == 1) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);
+        }
+        mma_commit(bar_pv);
+        mma_commit(&bar_empty[kb % NS]);
+        if (nbuf == 1 && kb + 1 < nkb) issue_s(kb + 1);  // in-order after the products that read S_0
+      }
+    }
+    if (!failed) {
+      const bool ok = mbar_wait(bar_pv, (nkb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      failed = group_any(BAR_COMPUTE, NCOMP, !ok);
+    }
+    if (!failed) {
+      tc_fence_after();
+      xch[cg * 128 + row] = Wm;
+      xch[(2 + cg) * 128 + row] = Wl;
+      group_sync(BAR_COMPUTE, NCOMP);
+      const float Wmt = xch[row] + xch[128 + row];
+      const float Wlt = xch[256 + row] + xch[384 + row];
+      if (!p.debug) {
+        // O = (sum_j w_j V_j) / W; each column group stores half of the d columns
+        const float Wout = (MODE == 2) ? Wlt : Wmt;
+        const float inv = row_ok ? 1.0f / Wout : 0.0f;
+        float* dst = ((MODE == 2) ? p.O_lerp : p.Out) + rw * D;
+        for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
+          float v[32];
+          tmem_ld32(lane_addr(tmem, cO + c), v);
+          tmem_ld_wait();
+          if (row_ok) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              reinterpret_cast<float4*>(dst + c)[q] =
+                  make_float4(v[4 * q] * inv, v[4 * q + 1] * inv, v[4 * q + 2] * inv, v[4 * q + 3] * inv);
+          }
+        }
+        if constexpr (MODE == 1) {
+          const float invl = row_ok ? 1.0f / Wlt : 0.0f;
+          float* dl = p.O_lerp + rw * D;
+          for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
+            float v[32];
+            tmem_ld32(lane_addr(tmem, cOL + c), v);
+            tmem_ld_wait();
+            if (row_ok) {
+#pragma unroll
+              for (int q = 0; q < 8; ++q)
+                reinterpret_cast<float4*>(dl + c)[q] =
+                    make_float4(v[4 * q] * invl, v[4 * q + 1] * invl, v[4 * q + 2] * invl, v[4 * q + 3] * invl);
             }
           }
         }
-        wm_part += wmain;
-        wl_part += wlerp;
-        const float a = (sel == PV_LERP) ? wlerp : wmain;
-        if (p.x3) {
-          const float h = tf32_rna(a);
-          a1[jj] = h;
-          a2[jj] = __fsub_rn(a, h);
-        } else {
-          a1[jj] = a;
-          a2[jj] = wlerp;
-        }
-        if (p.debug && row_ok && j < p.T) {
-          const size_t idx = ((size_t)bh * p.T + i) * p.T + j;
-          if (p.bins) p.bins[idx] = cb;
-          if (p.ivals) p.ivals[idx] = ci;
+        if (row_ok && cg == 0) {
+          if (MODE != 2) p.W[rw] = Wmt;
+          if (MODE != 0 && p.W_lerp) p.W_lerp[rw] = Wlt;
         }
       }
-      Wm += wm_part;
-      Wl += wl_part;
-      tmem_st32(lane_addr(tmem, c * 32), a1);
-      if (p.x3 || sel == PV_MAIN_LERP) tmem_st32(lane_addr(tmem, 128 + c * 32), a2);
     }
-    tmem_st_wait();
     tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint8_t* vt = st + parts * qtile;
-      const bool acc = kb > 0;
-      if (p.x3) {
-        mma_tmem_smem(tmem + 256, tmem + 0, vt, D, 128, acc);            // A_hi V_hi
-        mma_tmem_smem(tmem + 256, tmem + 0, vt + vtile, D, 128, true);   // A_hi V_lo
-        mma_tmem_smem(tmem + 256, tmem + 128, vt, D, 128, true);         // A_lo V_hi
-      } else {
-        mma_tmem_smem(tmem + 256, tmem + 0, vt, D, 128, acc);
-        if (sel == PV_MAIN_LERP) mma_tmem_smem(tmem + 256 + D, tmem + 128, vt, D, 128, acc);
-      }
-      mma_commit(bar_mma);
-    }
-    ok = mbar_wait(bar_mma, mph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    mph ^= 1;
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && kb + p.nstage < nkb) load_kv(kb + p.nstage);
   }
-
-  if (!failed && !p.debug) {
-    // Normalization (App. A): O = (sum_j w_j V_j) / W.  Every lane runs the
-    // warp-collective TMEM loads; only rows < T store.
-    const float Wout = (sel == PV_LERP) ? Wl : Wm;
-    const float inv = row_ok ? 1.0f / Wout : 0.0f;
-    float* dst = (sel == PV_LERP ? p.O_lerp : p.Out) + row * D;
-    for (int c = 0; c < D; c += 32) {
-      float v[32];
-      tmem_ld32(lane_addr(tmem, 256 + c), v);
-      tmem_ld_wait();
-      if (row_ok) {
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          reinterpret_cast<float4*>(dst + c)[q] =
-              make_float4(v[4 * q] * inv, v[4 * q + 1] * inv, v[4 * q + 2] * inv, v[4 * q + 3] * inv);
-      }
-    }
-    if (sel == PV_MAIN_LERP) {
-      const float invl = row_ok ? 1.0f / Wl : 0.0f;
-      float* dl = p.O_lerp + row * D;
-      for (int c = 0; c < D; c += 32) {
-        float v[32];
-        tmem_ld32(lane_addr(tmem, 256 + D + c), v);
-        tmem_ld_wait();
-        if (row_ok) {
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            reinterpret_cast<float4*>(dl + c)[q] =
-                make_float4(v[4 * q] * invl, v[4 * q + 1] * invl, v[4 * q + 2] * invl, v[4 * q + 3] * invl);
-        }
-      }
-    }
-    if (row_ok) {
-      if (sel != PV_LERP) p.W[row] = Wm;
-      if (sel != PV_MAIN && p.W_lerp) p.W_lerp[row] = Wl;
-    }
-  }
-  tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
-cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(k_fwd_main, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+template <int CAL, int REC, int MODE>
+static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+  auto kern = k_fwd_main<CAL, REC, MODE>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  k_fwd_main<<<dim3(p.nqb, p.BH), NT, smem_bytes, s>>>(maps, p);
+  kern<<<dim3(p.nqb, p.BH), NTHR, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+  const int mode = p.pv_sel;
+  if (p.calib == CAL_SOFTMAX) return launch_main_t<CAL_SOFTMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
+  if (p.calib == CAL_MINMAX) {
+    if (p.recon == REC_LERP) return launch_main_t<CAL_MINMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
+    if (mode == PV_MAIN) return launch_main_t<CAL_MINMAX, REC_NEAREST, 0>(maps, p, smem_bytes, s);
+    if (mode == PV_MAIN_LERP) return launch_main_t<CAL_MINMAX, REC_NEAREST, 1>(maps, p, smem_bytes, s);
+    return launch_main_t<CAL_MINMAX, REC_NEAREST, 2>(maps, p, smem_bytes, s);
+  }
+  if (p.recon == REC_LERP) return launch_main_t<CAL_FWM, REC_LERP, 0>(maps, p, smem_bytes, s);
+  if (mode == PV_MAIN) return launch_main_t<CAL_FWM, REC_NEAREST, 0>(maps, p, smem_bytes, s);
+  if (mode == PV_MAIN_LERP) return launch_main_t<CAL_FWM, REC_NEAREST, 1>(maps, p, smem_bytes, s);
+  return launch_main_t<CAL_FWM, REC_NEAREST, 2>(maps, p, smem_bytes, s);
 }
 
 }  // namespace kint

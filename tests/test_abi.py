@@ -43,7 +43,7 @@ def test_workspace_sizes():
 @pytest.mark.parametrize("kw,code", [
     (dict(B=0), -1), (dict(T=0), -1), (dict(Kint=0), -1), (dict(Kint=65), -1),
     (dict(calib=1, tau=0.0), -1), (dict(calib=7), -1), (dict(causal=0), -1), (dict(d=96), -2),
-    (dict(d=128, prec=1), -2),
+    (dict(d=128, prec=1), -2), (dict(Kint=33, prec=1), -2), (dict(Kint=33, d=128), -2),
 ])
 def test_argument_errors_are_returned_before_any_launch(kw, code):
     args = dict(B=1, H=1, T=8, d=64, Kint=4, calib=0, tau=8.0, recon=0, ste=0, grad=0, causal=1, prec=0)

@@ -92,11 +92,15 @@ def test_fwm_far_tail():
         parity.check(Q * 20, K, V, dO, cfg, X3)
 
 
-def test_large_K():
+def test_extreme_K():
+    """K = 1 and the largest K each configuration supports (MinMax K = 64 only in TF32 at d = 64)."""
     Q, K, V, dO = make_qkvdo(1, 2, 200, 64, seed=10)
-    for Kint in (1, 64):
-        parity.check(Q, K, V, dO, _cfg(MM, NE, WE, FU, Kint), X3)
-        parity.check(Q, K, V, dO, _cfg(FW, LE, PR, FU, Kint), X3)
+    parity.check(Q, K, V, dO, _cfg(MM, NE, WE, FU, 1), X3)
+    parity.check(Q, K, V, dO, _cfg(FW, LE, PR, FU, 1), X3)
+    parity.check(Q, K, V, dO, _cfg(MM, NE, WE, FU, 32), X3)
+    parity.check(Q, K, V, dO, _cfg(FW, LE, PR, FU, 64), X3)
+    parity.check(Q, K, V, dO, _cfg(MM, LE, PR, FU, 64), TF)
+    parity.check(Q, K, V, dO, _cfg(FW, NE, PR, DE, 64), TF)
 
 
 def test_value_ones_rows_sum_to_one():
