@@ -100,7 +100,9 @@ struct Workspace {
         *doh = nullptr, *dol = nullptr;
   float *vth = nullptr, *vtl = nullptr, *kth = nullptr, *ktl = nullptr, *qth = nullptr, *qtl = nullptr,
         *doth = nullptr, *dotl = nullptr;
-  float *Drow = nullptr, *cMn = nullptr, *cmn = nullptr, *tie = nullptr;
+  void* rec = nullptr;    // [BHT] 64-byte per-row records (dQ kernel -> dK/dV kernel)
+  float* rtab = nullptr;  // [BHT][KMAX] (e_r, e_{r+1}) MinMax grid pairs
+  float* tie = nullptr;   // [2][BHT][d] sums of tied arg-extremum keys
 };
 
 Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
@@ -128,7 +130,8 @@ Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
     } else {
       w.kth = take(tr); w.qth = take(tr); w.doth = take(tr);
     }
-    w.Drow = take(rows); w.cMn = take(rows); w.cmn = take(rows);
+    w.rec = take(rows * 16);
+    w.rtab = take(rows * 2 * KMAX);
     w.tie = take(2 * nat);
   }
   w.bytes = off;
@@ -228,30 +231,44 @@ int plan_main(Params& p, int mode) {
   return -1;
 }
 
+// Backward kernels: compute warps + MMA warp + producer warp.  A second score
+// buffer (S/g of tile t+1 computed under the element work of tile t) needs TMEM
+// room and at least two stages.
 int plan_dq(Params& p) {
-  const int parts = p.x3 ? 2 : 1, ktile = 64 * p.d * 4;
-  const int table = (p.Kint + 1) * 128 * 4;
+  const int parts = p.x3 ? 2 : 1, ktile = 64 * p.d * 4, dp = p.d * parts;
+  const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : 1024;
+  p.nbuf = (2 * dp + 256 + p.d <= 512) ? 2 : 1;
   p.sm_stage0 = 0;
   p.sm_stage_bytes = 3 * parts * ktile;
-  for (p.nstage = 2; p.nstage >= 1; --p.nstage) {
+  for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    const int total = std::max(finish_plan(p, p.sm_table + table, 1 + p.nstage), kOneCtaPerSm);
-    if (total <= kSmemLimit || p.nstage == 1) return total;
+    p.sm_rows = p.sm_table + table;
+    const int total = std::max(finish_plan(p, p.sm_rows + 4 * 128 * 4, 2 * p.nstage + 5), kOneCtaPerSm);
+    if (total <= kSmemLimit) {
+      if (p.nstage == 1) p.nbuf = 1;
+      return total;
+    }
   }
   return -1;
 }
 
-int plan_dkdv(Params& p) {
-  const int parts = p.x3 ? 2 : 1, qtile = 64 * p.d * 4;
+int plan_dkdv(Params& p, int sel) {
+  const int parts = p.x3 ? 2 : 1, qtile = 64 * p.d * 4, dp = p.d * parts;
+  const bool doDV = sel != DKV_DK, doDK = sel != DKV_DV;
+  const int base = doDK ? 2 * dp : dp;
+  const int acc = (doDV ? p.d : 0) + (doDK ? p.d : 0);
+  if (base + 128 + acc > 512) return -1;
+  p.dkv_sel = sel;
+  p.nbuf = (base + 256 + acc <= 512) ? 2 : 1;
   p.sm_stage0 = 0;
-  p.sm_stage_bytes = 4 * parts * qtile;  // room for Q, dO, Q^T, dO^T
-  const int rows = 14 * 64 * 4;
-  const int table = 64 * (p.Kint + 2) * 4;
-  for (p.nstage = 2; p.nstage >= 1; --p.nstage) {
-    p.sm_rows = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    p.sm_table = p.sm_rows + rows;
-    const int total = std::max(finish_plan(p, p.sm_table + table, 1 + p.nstage), kOneCtaPerSm);
-    if (total <= kSmemLimit || p.nstage == 1) return total;
+  p.sm_stage_bytes = 4 * parts * qtile + 64 * 64 + (p.calib == KINT_CALIB_MINMAX ? 64 * p.Kp * 8 : 0);
+  for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
+    p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+    const int total = std::max(finish_plan(p, p.sm_table + 1024, 2 * p.nstage + 5), kOneCtaPerSm);
+    if (total <= kSmemLimit) {
+      if (p.nstage == 1) p.nbuf = 1;
+      return total;
+    }
   }
   return -1;
 }
@@ -407,7 +424,8 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   p.dQ = dQ; p.dK = dK; p.dV = dV;
   const int BH = p.BH, Tp = round_up(T, 32);
   const Workspace w = plan_workspace(static_cast<char*>(workspace), BH, T, d, p.x3 != 0, true);
-  p.Drow = w.Drow; p.cMn = w.cMn; p.cmn = w.cmn; p.tie_acc = w.tie;
+  p.rec = w.rec; p.rtab = w.rtab; p.tie_acc = w.tie;
+  p.Kp = (p.Kint + 1) & ~1;
 
   // Operand copies: K-major transposes (and 3xTF32 splits).
   if (p.x3) {
@@ -449,16 +467,16 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   if ((rc = launch_rc(traced("k_bwd_dq", s, [&] { return launch_bwd_dq(maps, pq, smem_dq, s); })))) return rc;
 
   Params pk = p;
-  const int smem_kv = plan_dkdv(pk);
-  if (smem_kv < 0 || smem_kv > kSmemLimit) return KINT_ERR_UNSUPPORTED;
-  if (!p.x3 && d == 64) {
-    pk.dkv_sel = DKV_BOTH;
-    return launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); }));
-  }
-  pk.dkv_sel = DKV_DV;
+  int smem_kv = plan_dkdv(pk, DKV_BOTH);
+  if (!p.x3 && smem_kv > 0) return launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); }));
+  // one product per launch (3xTF32 hi/lo operands, or d = 128): dV, then dK
+  smem_kv = plan_dkdv(pk, DKV_DV);
+  if (smem_kv < 0) return KINT_ERR_UNSUPPORTED;
   if ((rc = launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); })))) return rc;
-  pk.dkv_sel = DKV_DK;
-  return launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk, smem_kv, s); }));
+  Params pk2 = p;
+  const int smem_kv2 = plan_dkdv(pk2, DKV_DK);
+  if (smem_kv2 < 0) return KINT_ERR_UNSUPPORTED;
+  return launch_rc(traced("k_bwd_dkdv", s, [&] { return launch_bwd_dkdv(maps, pk2, smem_kv2, s); }));
 }
 
 int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const kint_rowstats* st, uint8_t* bins,

@@ -1,98 +1,117 @@
 // Backward of K-interval attention on sm_103a (App. B).
 //
-// k_bwd_dq   (one CTA per 128-row query block, thread = query row): recomputes
-//   S = Q K^T and g = dO V^T per 64-key tile, forms the own-score term
-//   dS_own = gamma Delta, accumulates the row's calibration sums, and
-//   dQ = dS_own K.  At the end of the row it knows c_M and c_m (Eq. full) and
-//   adds their contribution at the arg-max / arg-min keys; it also leaves the
-//   row scalars <g>_{P*}, c_M / n_max, c_m / n_min for the second kernel.
-// k_bwd_dkdv (one CTA per 128-key block, thread = key): recomputes S^T and
-//   g^T per 64-query tile, forms the full dS (calibration terms included, now
-//   that c_M, c_m are known) and the forward P, and accumulates
-//   dV = P^T dO, dK = dS^T Q.
+// k_bwd_dq   (one CTA per 128-row query block, a thread per query row and
+//   column half): per 64-key tile, S = Q K^T and g = dO V^T on the tensor
+//   cores, then the own-score term dS_own = gamma Delta with
+//   gamma = (g - <g>_{P*}) / W* (normalization Jacobian) and Delta the LERP
+//   secant (e_{r+1} - e_r) / h, and dQ += dS_own K.  The row's calibration sums
+//   complete at the end of the row; it then adds c_M / n_max (and c_m / n_min)
+//   times the arg-extremum keys to dQ (Eq. full) and writes a 64-byte record of
+//   the row's constants for the second kernel.
+// k_bwd_dkdv (one CTA per 128-key block, a thread per key and column half): per
+//   64-query tile, S^T and g^T, the forward P and the full dS (extremum terms
+//   now known), and dV += P^T dO, dK += dS^T Q.
+// Both: compute warps 0-7, an MMA-issuing warp 8, a TMA/bulk-copy producer warp
+// 9; tiles change hands through mbarriers only.
 #include <cfloat>
 #include "kint_dev.cuh"
 #include "kint_launch.h"
 
 namespace kint {
 
-constexpr int BKEY = 64;  // keys per tile in k_bwd_dq
-constexpr int BQRY = 64;  // queries per tile in k_bwd_dkdv
+constexpr int BT = 64;  // keys per tile (k_bwd_dq), queries per tile (k_bwd_dkdv)
+constexpr float kLog2e = 1.4426950408889634f;
 
-// Quantities of one score element needed by the backward.
-struct BwdElem {
-  float p;    // forward probability P_ij
-  float ds;   // dL/ds_ij without the extremum terms
-  float dm;   // gamma * dw/dm (MinMax calibration sum term)
-};
-
-// Row-level constants of query row i.
-struct RowB {
-  RowGrid g;
-  float M, m, invWf, invWs, D;
-};
-
-// Own-score gradient and forward probability of one valid key (App. B):
-//   gamma = (g - <g>_{P*}) / W*, Delta = (e_{r+1} - e_r) / h, dS_own = gamma Delta,
-//   dw/dm = A_r + t B_r with A_r = (1 - r/K)(e_r - Delta), B_r = (1-(r+1)/K) e_{r+1} - (1 - r/K) e_r + Delta/K
-//   (Eq. calgrad rewritten per interval; dw/dM = -Delta - dw/dm).
-__device__ __forceinline__ BwdElem bwd_elem(const Params& p, const RowB& R, float s, float gval, float er_tab_r,
-                                            float er_tab_r1, float el_tab, const KeyPos& kp) {
-  BwdElem e{0.f, 0.f, 0.f};
-  if (p.calib == CAL_SOFTMAX) {
-    e.p = expf(__fsub_rn(s, R.M)) * R.invWf;
-    e.ds = e.p * (gval - R.D);  // P (g - <g>_P)  (App. B, Softmax)
-    return e;
+// ---------------------------------------------------------------------------
+// dQ kernel element work on one 32-key chunk of one row.
+// Returns dS_own in out[]; accumulates sum dS_own and sum gamma dw/dm.
+//   dw/dm = A_r + t B_r, A_r = (1 - r/K)(e_r - Delta),
+//   B_r = (1 - r/K)(e_{r+1} - e_r) - (e_{r+1} - Delta)/K   (Eq. calgrad per interval)
+// ---------------------------------------------------------------------------
+template <int CAL, bool FULLG, bool DIAG>
+__device__ __forceinline__ void dq_chunk(const float (&sv)[32], const float (&gv)[32], float (&out)[32], int j0,
+                                         int i, float k1, float c0, float inv_h, float ga, float gb, bool nogrid,
+                                         float Kf, float fk, uint32_t tab, float sk1, float sc0, float invWf,
+                                         float& own, float& cm) {
+#pragma unroll
+  for (int jj = 0; jj < 32; ++jj) {
+    float ds, dm = 0.f;
+    if constexpr (CAL == CAL_SOFTMAX) {
+      const float pr = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * invWf;
+      ds = pr * __fmaf_rn(gv[jj], ga, gb);  // P (g - <g>_P)
+    } else {
+      const float u = __fmaf_rn(sv[jj], k1, c0);
+      float t, rf;
+      uint32_t rb;
+      decode_u(u, Kf, t, rb, rf);
+      const float2 e = lds_f2(CAL == CAL_FWM ? tab + rb * 8u : tab + rb * 1024u);
+      const float de = __fsub_rn(e.y, e.x);
+      const float dlt = de * inv_h;
+      const float gam = __fmaf_rn(gv[jj], ga, gb);
+      ds = gam * dlt;
+      if constexpr (CAL == CAL_FWM) ds = (u < 0.0f) ? 0.f : ds;
+      if constexpr (CAL == CAL_MINMAX) {
+        if constexpr (FULLG) {
+          const float ar = __fmaf_rn(rf, -fk, 1.0f);
+          const float A = ar * __fsub_rn(e.x, dlt);
+          const float Bc = __fmaf_rn(ar, de, -fk * __fsub_rn(e.y, dlt));
+          dm = gam * __fmaf_rn(t, Bc, A);
+          dm = nogrid ? 0.f : dm;
+        }
+        ds = nogrid ? 0.f : ds;
+      }
+    }
+    if constexpr (DIAG) {
+      const bool ok = (j0 + jj) <= i;
+      ds = ok ? ds : 0.f;
+      dm = ok ? dm : 0.f;
+    }
+    if constexpr (FULLG && CAL != CAL_SOFTMAX) {
+      own += ds;
+      if constexpr (CAL == CAL_MINMAX) cm += dm;
+    }
+    out[jj] = ds;
   }
-  if (R.g.nogrid) {  // degenerate MinMax row: uniform P, zero gradient
-    e.p = R.invWf;
-    return e;
-  }
-  if (kp.tail) return e;  // FWM zero tail: weight and gradient 0
-  const float wl = __fmaf_rn(kp.t, __fsub_rn(er_tab_r1, er_tab_r), er_tab_r);
-  const float wf = (p.recon == REC_NEAREST) ? el_tab : wl;
-  e.p = wf * R.invWf;
-  const float gam = (gval - R.D) * R.invWs;
-  const float dlt = __fsub_rn(er_tab_r1, er_tab_r) * R.g.inv_h;
-  e.ds = gam * dlt;
-  if (p.calib == CAL_MINMAX && p.grad == 0) {
-    const float fk = 1.0f / (float)p.Kint;
-    const float ar = 1.0f - (float)kp.r * fk;
-    const float ar1 = ar - fk;
-    const float A = ar * (er_tab_r - dlt);
-    const float Bc = ar1 * er_tab_r1 - ar * er_tab_r + dlt * fk;
-    e.dm = gam * (A + kp.t * Bc);
-  }
-  return e;
 }
 
 // ---------------------------------------------------------------------------
-// k_bwd_dq.  TMEM columns: Q [0, dp), dO [dp, 2dp), S [2dp, 2dp+64),
-// g [2dp+64, 2dp+128), dQ [2dp+128, 2dp+128+d), dp = d (TF32) or 2d (3xTF32:
-// hi then lo).  dS overwrites S (and, as the lo part under 3xTF32, g).
-// smem: stages {K [64 x d], V [64 x d], K^T [d x 64]} (hi[, lo] each);
-// per-thread grid table [K+1][128] at sm_table.
+// k_bwd_dq.
+// TMEM: Q [0, dp), dO [dp, 2dp) (dp = d, or 2d for 3xTF32 hi|lo; loaded by the
+// compute threads), then per score buffer b: S_b at 2dp + 128 b (64 columns), g_b
+// right after it (64 columns); dQ at 2dp + 128 nbuf.  dS overwrites S_b (its tf32
+// lo part, under 3xTF32, overwrites g_b).
+// smem: stages {K [64 x d], V [64 x d], K^T [d x 64]} (hi[, lo] each) at
+// sm_stage0; the grid pair table at sm_table; exchange words at sm_rows.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(NT, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
+template <int CAL, bool FULLG>
+__global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
-  const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1;
-  const int ktile = BKEY * D * 4;  // [64 x D] natural or [D x 64] transposed
-  float* tab = reinterpret_cast<float*>(sm + p.sm_table);
+  const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
+  const int ktile = BT * D * 4;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.sm_bars);
-  uint64_t* bar_st = bars;
-  uint64_t* bar_mma = bars + p.nstage;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 1 + p.nstage);
+  uint64_t* bar_full = bars;               // [NS]
+  uint64_t* bar_empty = bars + NS;         // [NS]
+  uint64_t* bar_sfull = bars + 2 * NS;     // [2]
+  uint64_t* bar_pready = bars + 2 * NS + 2;  // [2]
+  uint64_t* bar_done = bars + 2 * NS + 4;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
+  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [4][128]
   const int tid = threadIdx.x, warp = tid >> 5;
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
-  const int i = qb * 128 + tid;
-  const bool row_ok = i < p.T;
-  const int nkt = min(2 * qb + 2, (p.T + BKEY - 1) / BKEY);
+  const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
   const int dp = D * parts;
-  const int cQ = 0, cdO = dp, cS = 2 * dp, cG = 2 * dp + 64, cdQ = 2 * dp + 128;
+  const int cQ = 0, cdO = dp, cdQ = 2 * dp + 128 * nbuf;
 
   if (tid == 0) {
-    for (int s = 0; s < p.nstage; ++s) mbar_init(&bar_st[s], 1);
-    mbar_init(bar_mma, 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bar_sfull[b], 1);
+      mbar_init(&bar_pready[b], NCOMP / 32);
+    }
+    mbar_init(bar_done, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -104,45 +123,35 @@ __global__ void __launch_bounds__(NT, 1) k_bwd_dq(const __grid_constant__ Maps m
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  auto stage_ptr = [&](int kt) { return sm + p.sm_stage0 + (kt % p.nstage) * p.sm_stage_bytes; };
-  auto load_stage = [&](int kt) {
-    uint64_t* b = &bar_st[kt % p.nstage];
-    uint8_t* dst = stage_ptr(kt);
-    mbar_arrive_expect_tx(b, 3 * parts * ktile);
-    load_rows_tile(dst, &maps.k, b, D, BKEY, 0, kt * BKEY, bh);
-    load_rows_tile(dst + parts * ktile, &maps.v, b, D, BKEY, 0, kt * BKEY, bh);
-    load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BKEY, D, kt * BKEY, 0, bh);
-    if (p.x3) {
-      load_rows_tile(dst + ktile, &maps.k_lo, b, D, BKEY, 0, kt * BKEY, bh);
-      load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BKEY, 0, kt * BKEY, bh);
-      load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BKEY, D, kt * BKEY, 0, bh);
+  // ---- compute-thread set-up: operands Q / dO into TMEM, row constants, grid table ----
+  const int row = tid & 127, cg = (tid >> 7) & 1;
+  const int i = qb * 128 + row;
+  const bool row_ok = i < p.T;
+  const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
+  float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
+  int nmax = 1, nmin = 1, amax = 0, amin = 0;
+  RowGrid g{};
+  if (warp < NCOMP / 32) {
+    const float* src = cg == 0 ? p.Q : p.dO;
+    row_to_tmem(tmem, cg == 0 ? cQ : cdO, src, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    if (row_ok) {
+      M = p.row_max[rw];
+      m = p.row_min[rw];
+      Wf = p.W[rw];
+      nmax = p.n_max[rw];
+      nmin = p.n_min[rw];
+      amax = p.arg_max[rw];
+      amin = p.arg_min[rw];
     }
-  };
-  if (tid == 0)
-    for (int kt = 0; kt < min(p.nstage, nkt); ++kt) load_stage(kt);
-
-  // Operands A = Q and dO of this thread's row into TMEM.
-  row_to_tmem(tmem, cQ, p.Q, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-  row_to_tmem(tmem, cdO, p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-
-  // Row constants.
-  const size_t row = (size_t)bh * p.T + (row_ok ? i : 0);
-  RowB R;
-  R.M = row_ok ? p.row_max[row] : 0.f;
-  R.m = row_ok ? p.row_min[row] : 0.f;
-  R.g = row_grid(p, R.M, R.m);
-  const float Wf = row_ok ? p.W[row] : 1.f;
-  const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && p.calib != CAL_SOFTMAX);
-  const float Ws = prob ? (row_ok ? p.W_lerp[row] : 1.f) : Wf;
-  R.invWf = 1.0f / Wf;
-  R.invWs = 1.0f / Ws;
-  // <g>_{P*} = dO_i . O*_i  with O* = P* V (P* = P^L for Prob-STE, else the forward P)
-  {
+    g = row_grid(p, M, m);
+    const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
+    Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
+    // <g>_{P*} = dO_i . O*_i, the two column groups each take half of the d columns
     float acc = 0.f;
     if (row_ok) {
-      const float4* a = reinterpret_cast<const float4*>(p.dO + row * D);
-      const float4* b = reinterpret_cast<const float4*>(p.Ostar + row * D);
-      for (int q = 0; q < D / 4; ++q) {
+      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / 8);
+      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / 8);
+      for (int q = 0; q < D / 8; ++q) {
         const float4 x = __ldg(a + q), y = __ldg(b + q);
         acc = __fmaf_rn(x.x, y.x, acc);
         acc = __fmaf_rn(x.y, y.y, acc);
@@ -150,218 +159,326 @@ __global__ void __launch_bounds__(NT, 1) k_bwd_dq(const __grid_constant__ Maps m
         acc = __fmaf_rn(x.w, y.w, acc);
       }
     }
-    R.D = acc;
-  }
-  const int nmax = row_ok ? p.n_max[row] : 1, nmin = row_ok ? p.n_min[row] : 1;
-  const int amax = row_ok ? p.arg_max[row] : 0, amin = row_ok ? p.arg_min[row] : 0;
-  const bool full = p.grad == 0 && p.calib != CAL_SOFTMAX && !R.g.nogrid;
-  const bool minmax = p.calib == CAL_MINMAX;
-  if (p.calib != CAL_SOFTMAX)
-    for (int r = 0; r <= Kq; ++r) tab[r * NT + tid] = grid_value(p, R.g, r);
-  float* tie_max = p.tie_acc + row * D;
-  float* tie_min = p.tie_acc + ((size_t)p.BH * p.T + row) * D;
-  const bool track_ties = row_ok && full && (nmax > 1 || (minmax && nmin > 1));
-  if (track_ties)
-    for (int k = 0; k < D; ++k) {
-      tie_max[k] = 0.f;
-      tie_min[k] = 0.f;
-    }
-
-  tmem_st_wait();
-  tc_fence_before();
-  __syncthreads();
-
-  float own_acc = 0.f, cm_acc = 0.f;
-  bool failed = false;
-  uint32_t mph = 0;
-  for (int kt = 0; kt < nkt; ++kt) {
-    const uint8_t* st = stage_ptr(kt);
-    if (tid == 0) {
-      const bool ok =
-          mbar_wait(&bar_st[kt % p.nstage], (kt / p.nstage) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-      if (ok) {
-        tc_fence_after();
-        const uint8_t* sk = st;
-        const uint8_t* sv = st + parts * ktile;
-        if (p.x3) {
-          mma_tmem_smem(tmem + cS, tmem + cQ + D, sk, BKEY, D, false);   // Q_lo K_hi
-          mma_tmem_smem(tmem + cS, tmem + cQ, sk + ktile, BKEY, D, true); // Q_hi K_lo
-          mma_tmem_smem(tmem + cS, tmem + cQ, sk, BKEY, D, true);         // Q_hi K_hi
-          mma_tmem_smem(tmem + cG, tmem + cdO + D, sv, BKEY, D, false);
-          mma_tmem_smem(tmem + cG, tmem + cdO, sv + ktile, BKEY, D, true);
-          mma_tmem_smem(tmem + cG, tmem + cdO, sv, BKEY, D, true);
-        } else {
-          mma_tmem_smem(tmem + cS, tmem + cQ, sk, BKEY, D, false);
-          mma_tmem_smem(tmem + cG, tmem + cdO, sv, BKEY, D, false);
-        }
-        mma_commit(bar_mma);
+    xch[cg * 128 + row] = acc;
+    if constexpr (CAL == CAL_FWM) {
+      if (tid < Kq)
+        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+    } else if constexpr (CAL == CAL_MINMAX) {
+      for (int r = cg; r < Kq; r += NCG) {
+        const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
+        *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
+        if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
       }
-    }
-    bool ok = mbar_wait(bar_mma, mph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    mph ^= 1;
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
-    }
-    tc_fence_after();
-#pragma unroll 1
-    for (int c = 0; c < BKEY / 32; ++c) {
-      float sv[32], gv[32], a1[32], a2[32];
-      tmem_ld32(lane_addr(tmem, cS + c * 32), sv);
-      tmem_ld32(lane_addr(tmem, cG + c * 32), gv);
-      tmem_ld_wait();
-      const int j0 = kt * BKEY + c * 32;
-#pragma unroll
-      for (int jj = 0; jj < 32; ++jj) {
-        const int j = j0 + jj;
-        const bool valid = row_ok && j <= i;
-        float ds = 0.f;
-        if (valid) {
-          const float s = __fmul_rn(sv[jj], p.scale);
-          KeyPos kp{0, 0, 0.f, false};
-          float er = 0.f, er1 = 0.f, el = 0.f;
-          if (p.calib != CAL_SOFTMAX && !R.g.nogrid) {
-            kp = key_pos(p, __fmaf_rn(sv[jj], R.g.k1, R.g.c0));
-            if (!kp.tail) {
-              er = tab[kp.r * NT + tid];
-              er1 = tab[(kp.r + 1) * NT + tid];
-              el = tab[kp.l * NT + tid];
-            }
-          }
-          const BwdElem e = bwd_elem(p, R, s, gv[jj], er, er1, el, kp);
-          ds = e.ds;
-          if (full) {
-            own_acc += e.ds;
-            cm_acc += e.dm;
-            if (track_ties) {
-              if (nmax > 1 && s == R.M)
-                for (int k = 0; k < D; ++k) tie_max[k] += p.K[((size_t)bh * p.T + j) * D + k];
-              if (minmax && nmin > 1 && s == R.m)
-                for (int k = 0; k < D; ++k) tie_min[k] += p.K[((size_t)bh * p.T + j) * D + k];
-            }
-          }
-        }
-        if (p.x3) {
-          const float h = tf32_rna(ds);
-          a1[jj] = h;
-          a2[jj] = __fsub_rn(ds, h);
-        } else {
-          a1[jj] = ds;
-        }
-      }
-      tmem_st32(lane_addr(tmem, cS + c * 32), a1);
-      if (p.x3) tmem_st32(lane_addr(tmem, cG + c * 32), a2);
     }
     tmem_st_wait();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const uint8_t* skt = st + 2 * parts * ktile;
-      const bool acc = kt > 0;
-      if (p.x3) {
-        mma_tmem_smem(tmem + cdQ, tmem + cS, skt, D, BKEY, acc);           // dS_hi K_hi
-        mma_tmem_smem(tmem + cdQ, tmem + cS, skt + ktile, D, BKEY, true);  // dS_hi K_lo
-        mma_tmem_smem(tmem + cdQ, tmem + cG, skt, D, BKEY, true);          // dS_lo K_hi
-      } else {
-        mma_tmem_smem(tmem + cdQ, tmem + cS, skt, D, BKEY, acc);
-      }
-      mma_commit(bar_mma);
-    }
-    ok = mbar_wait(bar_mma, mph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    mph ^= 1;
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && kt + p.nstage < nkt) load_stage(kt + p.nstage);
   }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
 
-  if (!failed) {
-    // Extremum terms of Eq. (full): c_m = sum_j gamma_j dw_j/dm; c_M = -sum_j gamma_j Delta_j - c_m
-    // (App. B: Delta + dw/dM + dw/dm = 0); FWM: c_M = -sum_window gamma Delta, no m term.
-    const float cm = (full && minmax) ? cm_acc : 0.f;
-    const float cM = full ? (-own_acc - cm) : 0.f;
-    const float cMn = cM / (float)nmax, cmn = cm / (float)nmin;
-    const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
-    const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
-    float* dst = p.dQ + row * D;
-    for (int c = 0; c < D; c += 32) {
-      float v[32];
-      tmem_ld32(lane_addr(tmem, cdQ + c), v);
-      tmem_ld_wait();
-      if (row_ok) {
-#pragma unroll 4
-        for (int q = 0; q < 32; ++q) {
-          float x = v[q];
-          if (full) {
-            x = __fmaf_rn(cMn, kmax[c + q], x);
-            if (minmax) x = __fmaf_rn(cmn, kmin[c + q], x);
-          }
-          dst[c + q] = x * p.scale;
+  if (warp == PRODUCER_WARP3) {
+    if ((tid & 31) == 0) {
+      for (int kt = 0; kt < nkt; ++kt) {
+        const int s = kt % NS;
+        if (kt >= NS &&
+            !mbar_wait(&bar_empty[s], ((kt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+          break;
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        uint64_t* b = &bar_full[s];
+        mbar_arrive_expect_tx(b, 3 * parts * ktile);
+        load_rows_tile(dst, &maps.k, b, D, BT, 0, kt * BT, bh);
+        load_rows_tile(dst + parts * ktile, &maps.v, b, D, BT, 0, kt * BT, bh);
+        load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
+        if (p.x3) {
+          load_rows_tile(dst + ktile, &maps.k_lo, b, D, BT, 0, kt * BT, bh);
+          load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BT, 0, kt * BT, bh);
+          load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
         }
       }
     }
-    if (row_ok) {
-      p.Drow[row] = R.D;
-      p.cMn[row] = cMn;
-      p.cmn[row] = cmn;
+  } else if (warp == MMA_WARP3) {
+    if ((tid & 31) == 0) {
+      auto issue_sg = [&](int kt) -> bool {
+        const int s = kt % NS, b = kt % nbuf;
+        if (!mbar_wait(&bar_full[s], (kt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+        tc_fence_after();
+        const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        const uint8_t* sv = sk + parts * ktile;
+        const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
+        if (p.x3) {
+          mma_tmem_smem(cS, tmem + cQ + D, sk, BT, D, false);     // Q_lo K_hi
+          mma_tmem_smem(cS, tmem + cQ, sk + ktile, BT, D, true);  // Q_hi K_lo
+          mma_tmem_smem(cS, tmem + cQ, sk, BT, D, true);          // Q_hi K_hi
+          mma_tmem_smem(cG, tmem + cdO + D, sv, BT, D, false);
+          mma_tmem_smem(cG, tmem + cdO, sv + ktile, BT, D, true);
+          mma_tmem_smem(cG, tmem + cdO, sv, BT, D, true);
+        } else {
+          mma_tmem_smem(cS, tmem + cQ, sk, BT, D, false);
+          mma_tmem_smem(cG, tmem + cdO, sv, BT, D, false);
+        }
+        mma_commit(&bar_sfull[b]);
+        return true;
+      };
+      bool ok = issue_sg(0);
+      for (int kt = 0; kt < nkt && ok; ++kt) {
+        const int b = kt % nbuf, s = kt % NS;
+        if (nbuf == 2 && kt + 1 < nkt) ok = issue_sg(kt + 1);
+        if (!ok) break;
+        if (!mbar_wait(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        tc_fence_after();
+        const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
+        const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
+        const bool acc = kt > 0;
+        if (p.x3) {
+          mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);           // dS_hi K_hi
+          mma_tmem_smem(tmem + cdQ, cS, skt + ktile, D, BT, true);  // dS_hi K_lo
+          mma_tmem_smem(tmem + cdQ, cG, skt, D, BT, true);          // dS_lo K_hi
+        } else {
+          mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
+        }
+        mma_commit(&bar_empty[s]);
+        if (nbuf == 1 && kt + 1 < nkt) ok = issue_sg(kt + 1);  // in order after the product reading S_0
+      }
+      mma_commit(bar_done);
     }
+  } else {
+    // ---- compute warps ----
+    group_sync(BAR_COMPUTE, NCOMP);
+    Dg = xch[row] + xch[128 + row];
+    const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
+    const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
+    const float invWf = 1.0f / Wf;
+    const float sk1 = p.scale * kLog2e, sc0 = -M * kLog2e;
+    const float Kf = (float)Kq, fk = 1.0f / Kf;
+    const uint32_t tab = (CAL == CAL_FWM) ? smem_u32(sm + p.sm_table) - 0x58000000u
+                                          : smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
+    const bool minmax = CAL == CAL_MINMAX;
+    const bool track = FULLG && CAL != CAL_SOFTMAX && row_ok && !g.nogrid && (nmax > 1 || (minmax && nmin > 1));
+    float* tie_max = p.tie_acc + rw * D;
+    float* tie_min = p.tie_acc + ((size_t)p.BH * p.T + rw) * D;
+    if (track && cg == 0)
+      for (int k = 0; k < D; ++k) tie_max[k] = tie_min[k] = 0.f;
+    group_sync(BAR_COMPUTE, NCOMP);  // the two halves of a row may both add to its tie sums
+    float own = 0.f, cm = 0.f;
+    bool failed = false;
+    for (int kt = 0; kt < nkt; ++kt) {
+      const int b = kt % nbuf;
+      const bool ok = mbar_wait(&bar_sfull[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      if (!ok) {
+        failed = true;
+        break;
+      }
+      tc_fence_after();
+      const int cS = 2 * dp + 128 * b + cg * 32, cG = cS + 64;
+      float sv[32], gv[32], out[32];
+      tmem_ld32(lane_addr(tmem, cS), sv);
+      tmem_ld32(lane_addr(tmem, cG), gv);
+      tmem_ld_wait();
+      const int j0 = kt * BT + cg * 32;
+      if (j0 + 31 > qb * 128)
+        dq_chunk<CAL, FULLG, true>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
+                                   sc0, invWf, own, cm);
+      else
+        dq_chunk<CAL, FULLG, false>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
+                                    sc0, invWf, own, cm);
+      if (__any_sync(0xffffffffu, track)) {
+        // rare: tied extrema, the tie set is found by equality on the recomputed scores
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) {
+          const int j = j0 + jj;
+          const float s = __fmul_rn(sv[jj], p.scale);
+          const bool okj = track && j <= i;
+          if (okj && nmax > 1 && s == M)
+            for (int k = 0; k < D; ++k) atomicAdd(&tie_max[k], p.K[((size_t)bh * p.T + j) * D + k]);
+          if (okj && minmax && nmin > 1 && s == m)
+            for (int k = 0; k < D; ++k) atomicAdd(&tie_min[k], p.K[((size_t)bh * p.T + j) * D + k]);
+        }
+      }
+      if (p.x3) {
+        float lo[32];
+#pragma unroll
+        for (int q = 0; q < 32; ++q) {
+          const float h = tf32_rna(out[q]);
+          lo[q] = __fsub_rn(out[q], h);
+          out[q] = h;
+        }
+        tmem_st32(lane_addr(tmem, cG), lo);
+      }
+      tmem_st32(lane_addr(tmem, cS), out);
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
+    }
+    const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+    if (!failed) {
+      tc_fence_after();
+      xch[(cg)*128 + row] = own;
+      xch[(2 + cg) * 128 + row] = cm;
+      group_sync(BAR_COMPUTE, NCOMP);
+      const float own_t = xch[row] + xch[128 + row];
+      const float cm_t = xch[256 + row] + xch[384 + row];
+      // Eq. (full): c_m = sum gamma dw/dm; c_M = -sum gamma Delta - c_m (Delta + dw/dM + dw/dm = 0);
+      // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys.
+      const bool full = FULLG && CAL != CAL_SOFTMAX && !g.nogrid;
+      const float cmv = (full && minmax) ? cm_t : 0.f;
+      const float cMv = full ? (-own_t - cmv) : 0.f;
+      const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
+      const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
+      const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
+      float* dst = p.dQ + rw * D;
+      for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
+        float v[32];
+        tmem_ld32(lane_addr(tmem, cdQ + c), v);
+        tmem_ld_wait();
+        if (row_ok) {
+#pragma unroll 8
+          for (int q = 0; q < 32; ++q) {
+            float x = v[q];
+            if (full) {
+              x = __fmaf_rn(cMn, __ldg(kmax + c + q), x);
+              if (minmax) x = __fmaf_rn(cmn, __ldg(kmin + c + q), x);
+            }
+            dst[c + q] = x * p.scale;
+          }
+        }
+      }
+      if (row_ok && cg == 0) {
+        RowRec r;
+        r.c0 = g.c0;
+        r.k1 = g.k1;
+        r.inv_h = g.inv_h;
+        r.invWf = invWf;
+        r.ga = ga;
+        r.gb = gb;
+        r.cMn = full ? cMn : 0.f;
+        r.cmn = (full && minmax) ? cmn : 0.f;
+        r.amax = (nmax == 1) ? amax : -1;
+        r.amin = (nmin == 1) ? amin : -1;
+        r.flags = (g.nogrid ? REC_NOGRID : 0) | (nmax > 1 ? REC_TIEMAX : 0) | (nmin > 1 ? REC_TIEMIN : 0);
+        r.pad = 0;
+        r.M = M;
+        r.m = m;
+        r.sk1 = sk1;
+        r.sc0 = sc0;
+        reinterpret_cast<RowRec*>(p.rec)[rw] = r;
+      }
+    }
+    tc_fence_before();
   }
-  tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
-cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(k_bwd_dq, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
-  if (e != cudaSuccess) return e;
-  k_bwd_dq<<<dim3(p.nqb, p.BH), NT, smem_bytes, s>>>(maps, p);
-  return cudaGetLastError();
+// ---------------------------------------------------------------------------
+// dK/dV kernel element work on one 32-query chunk of one key j: the forward
+// probability P_ij and dS_ij = gamma_ij Delta_ij plus, at the arg-max / arg-min
+// key of row i, c_M / n_max and c_m / n_min (Eq. full).  Row constants come
+// from the RowRec array of the tile in shared memory (broadcast loads).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int4 lds_i4(uint32_t addr) {
+  int4 v;
+  asm volatile("ld.shared.v4.s32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+  return v;
+}
+
+template <int CAL, int REC, bool FULLG, bool MASKED>
+__device__ __forceinline__ void kv_chunk(const float (&sv)[32], const float (&gv)[32], float (&pa)[32],
+                                         float (&da)[32], int j, int i0, int T, uint32_t recs, uint32_t tabs,
+                                         uint32_t fwtab, uint32_t tstride, float Kf) {
+#pragma unroll
+  for (int ii = 0; ii < 32; ++ii) {
+    const uint32_t ra = recs + ii * 64u;  // RowRec of query row i0 + ii
+    const float4 r0 = lds_f4(ra);          // c0, k1, inv_h, invWf
+    const float4 r1 = lds_f4(ra + 16);     // ga, gb, cMn, cmn
+    float pv, ds;
+    if constexpr (CAL == CAL_SOFTMAX) {
+      const float4 r3 = lds_f4(ra + 48);  // M, m, sk1, sc0
+      pv = ex2_approx(__fmaf_rn(sv[ii], r3.z, r3.w)) * r0.w;
+      ds = pv * __fmaf_rn(gv[ii], r1.x, r1.y);
+    } else {
+      const int4 r2 = lds_i4(ra + 32);  // amax, amin, flags, -
+      const float u = __fmaf_rn(sv[ii], r0.y, r0.x);
+      float t, rf;
+      uint32_t rb;
+      decode_u(u, Kf, t, rb, rf);
+      const float2 e = lds_f2(CAL == CAL_FWM ? fwtab + rb * 8u : tabs + ii * tstride + rb * 8u);
+      const float de = __fsub_rn(e.y, e.x);
+      const float wl = __fmaf_rn(t, de, e.x);
+      const float wn = (t >= 0.5f) ? e.y : e.x;
+      float w = (REC == REC_NEAREST) ? wn : wl;
+      const float gam = __fmaf_rn(gv[ii], r1.x, r1.y);
+      ds = gam * (de * r0.z);
+      if constexpr (CAL == CAL_FWM) {
+        const bool tail = u < 0.0f;
+        w = tail ? 0.f : w;
+        ds = tail ? 0.f : ds;
+      }
+      if constexpr (CAL == CAL_MINMAX) {
+        const bool ng = (r2.z & REC_NOGRID) != 0;
+        w = ng ? 1.f : w;
+        ds = ng ? 0.f : ds;
+      }
+      pv = w * r0.w;
+      if constexpr (FULLG) {
+        ds += (j == r2.x) ? r1.z : 0.f;
+        if constexpr (CAL == CAL_MINMAX) ds += (j == r2.y) ? r1.w : 0.f;
+      }
+    }
+    if constexpr (MASKED) {
+      const int iq = i0 + ii;
+      const bool ok = iq >= j && iq < T;
+      pv = ok ? pv : 0.f;
+      ds = ok ? ds : 0.f;
+    }
+    pa[ii] = pv;
+    da[ii] = ds;
+  }
 }
 
 // ---------------------------------------------------------------------------
-// k_bwd_dkdv.  Thread t owns key j = kb*128 + t (TMEM lane t).  TMEM columns:
-// K [0, dp), V [dp, 2dp) (dK launches), then S^T (64), g^T (64), dV (d), dK (d).
-// P^T overwrites S^T and dS^T overwrites g^T; under 3xTF32 (one product per
-// launch) the hi part goes to the first and the lo part to the second.
-// smem: stages {Q [64 x d], dO [64 x d], Q^T [d x 64], dO^T [d x 64]} (hi[, lo]);
-// per-query-row constants and grid tables of the current query tile.
+// k_bwd_dkdv.  Thread t (< 256) owns key j = kb*128 + t%128 and the query half
+// t/128 of each 64-query tile.  TMEM: K [0, dp), V [dp, 2dp) (dK launches),
+// then per buffer b: S^T_b (64 columns) and g^T_b (64 columns) from `base`,
+// dV, dK.  P^T overwrites S^T_b and dS^T overwrites g^T_b (3xTF32: the single
+// product's hi part goes to S^T_b, its lo part to g^T_b).
+// smem stage: Q | dO | Q^T | dO^T tiles (hi[, lo]), the 64 RowRecs of the tile,
+// and (MinMax) their grid pair tables; FWM's shared table at sm_table.
 // ---------------------------------------------------------------------------
-struct QRows {  // per query row of the current tile, in shared memory
-  float M[BQRY], m[BQRY], inv_h[BQRY], c0[BQRY], invWf[BQRY], invWs[BQRY], D[BQRY], cMn[BQRY], cmn[BQRY];
-  int amax[BQRY], amin[BQRY], nmax[BQRY], nmin[BQRY], nogrid[BQRY];
-};
-
-__global__ void __launch_bounds__(NT, 1) k_bwd_dkdv(const __grid_constant__ Maps maps, const Params p) {
+template <int CAL, int REC, bool FULLG>
+__global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
-  const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1;
-  const int qtile = BQRY * D * 4;
-  const bool do_dv = p.dkv_sel != DKV_DK, do_dk = p.dkv_sel != DKV_DV;
-  QRows* qr = reinterpret_cast<QRows*>(sm + p.sm_rows);
-  float* tab = reinterpret_cast<float*>(sm + p.sm_table);  // [BQRY][K+2]
+  const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
+  const int qtile = BT * D * 4;
+  const bool doDV = p.dkv_sel != DKV_DK, doDK = p.dkv_sel != DKV_DV, needV = doDK;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.sm_bars);
-  uint64_t* bar_st = bars;
-  uint64_t* bar_mma = bars + p.nstage;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 1 + p.nstage);
+  uint64_t* bar_full = bars;
+  uint64_t* bar_empty = bars + NS;
+  uint64_t* bar_sfull = bars + 2 * NS;
+  uint64_t* bar_pready = bars + 2 * NS + 2;
+  uint64_t* bar_done = bars + 2 * NS + 4;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
   const int tid = threadIdx.x, warp = tid >> 5;
   const int bh = blockIdx.y, kb = blockIdx.x;
-  const int j = kb * 128 + tid;
   const int dp = D * parts;
-  const int cK = 0, cV = dp;
-  const int cS = do_dk ? 2 * dp : dp;
-  const int cG = cS + 64, cdV = cS + 128, cdK = cdV + (do_dv ? D : 0);
-  const int qt0 = (kb * 128) / BQRY;
-  const int nqt = (p.T + BQRY - 1) / BQRY;
-  const int tstride = Kq + 2;
-  // Stage layout: Q | dO | Q^T | dO^T, each `parts` tiles; only the needed ones are loaded.
+  const int cK = 0, cV = dp, base = needV ? 2 * dp : dp;
+  const int cdV = base + 128 * nbuf, cdK = cdV + (doDV ? D : 0);
+  const int qt0 = (kb * 128) / BT, nqt = (p.T + BT - 1) / BT, nit = nqt - qt0;
   const int oQ = 0, odO = parts * qtile, oQT = 2 * parts * qtile, odOT = 3 * parts * qtile;
-  const bool need_dO = do_dk, need_QT = do_dk, need_dOT = do_dv;
+  const int oRec = 4 * parts * qtile, oTab = oRec + BT * 64;
+  const uint32_t tstride = (uint32_t)p.Kp * 8u;
 
   if (tid == 0) {
-    for (int s = 0; s < p.nstage; ++s) mbar_init(&bar_st[s], 1);
-    mbar_init(bar_mma, 1);
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bar_sfull[b], 1);
+      mbar_init(&bar_pready[b], NCOMP / 32);
+    }
+    mbar_init(bar_done, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -372,230 +489,237 @@ __global__ void __launch_bounds__(NT, 1) k_bwd_dkdv(const __grid_constant__ Maps
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-
-  auto stage_ptr = [&](int it) { return sm + p.sm_stage0 + (it % p.nstage) * p.sm_stage_bytes; };
-  auto load_stage = [&](int it) {
-    const int q0 = (qt0 + it) * BQRY;
-    uint64_t* b = &bar_st[it % p.nstage];
-    uint8_t* dst = stage_ptr(it);
-    const int ntiles = 1 + (need_dO ? 1 : 0) + (need_QT ? 1 : 0) + (need_dOT ? 1 : 0);
-    mbar_arrive_expect_tx(b, ntiles * parts * qtile);
-    load_rows_tile(dst + oQ, &maps.q, b, D, BQRY, 0, q0, bh);
-    if (p.x3) load_rows_tile(dst + oQ + qtile, &maps.q_lo, b, D, BQRY, 0, q0, bh);
-    if (need_dO) {
-      load_rows_tile(dst + odO, &maps.dout, b, D, BQRY, 0, q0, bh);
-      if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BQRY, 0, q0, bh);
-    }
-    if (need_QT) {
-      load_rows_tile(dst + oQT, &maps.qt, b, BQRY, D, q0, 0, bh);
-      if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BQRY, D, q0, 0, bh);
-    }
-    if (need_dOT) {
-      load_rows_tile(dst + odOT, &maps.dot, b, BQRY, D, q0, 0, bh);
-      if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BQRY, D, q0, 0, bh);
-    }
-  };
-  const int nit = nqt - qt0;
-  if (tid == 0)
-    for (int it = 0; it < min(p.nstage, nit); ++it) load_stage(it);
-
+  const int row = tid & 127, cg = (tid >> 7) & 1;
+  const int j = kb * 128 + row;
   const bool key_ok = j < p.T;
-  row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-  if (do_dk) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-  tmem_st_wait();
-
-  const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && p.calib != CAL_SOFTMAX);
-  const bool minmax = p.calib == CAL_MINMAX;
-  const bool fullg = p.grad == 0 && p.calib != CAL_SOFTMAX;
-  bool failed = false;
-  uint32_t mph = 0;
-  for (int it = 0; it < nit; ++it) {
-    const int q0 = (qt0 + it) * BQRY;
-    // Per-query-row constants of this tile (the previous tile's readers have
-    // passed the CTA barrier that closed their iteration).
-    if (tid < BQRY) {
-      const int iq = q0 + tid;
-      const bool ok = iq < p.T;
-      const size_t rw = (size_t)bh * p.T + (ok ? iq : 0);
-      const float M = ok ? p.row_max[rw] : 0.f, m = ok ? p.row_min[rw] : 0.f;
-      const RowGrid g = row_grid(p, M, m);
-      const float Wf = ok ? p.W[rw] : 1.f;
-      const float Ws = prob ? (ok ? p.W_lerp[rw] : 1.f) : Wf;
-      qr->M[tid] = M;
-      qr->m[tid] = m;
-      qr->inv_h[tid] = g.inv_h;
-      qr->c0[tid] = g.c0;
-      qr->invWf[tid] = 1.0f / Wf;
-      qr->invWs[tid] = 1.0f / Ws;
-      qr->D[tid] = ok ? p.Drow[rw] : 0.f;
-      qr->cMn[tid] = ok ? p.cMn[rw] : 0.f;
-      qr->cmn[tid] = ok ? p.cmn[rw] : 0.f;
-      qr->amax[tid] = ok ? p.arg_max[rw] : -1;
-      qr->amin[tid] = ok ? p.arg_min[rw] : -1;
-      qr->nmax[tid] = ok ? p.n_max[rw] : 1;
-      qr->nmin[tid] = ok ? p.n_min[rw] : 1;
-      qr->nogrid[tid] = g.nogrid ? 1 : 0;
-    }
-    if (p.calib != CAL_SOFTMAX) {
-      // grid tables: row (tid % 64), entries r = tid/64, tid/64 + 2, ...
-      const int rr = tid % BQRY, iq = q0 + rr;
-      const bool ok = iq < p.T;
-      const size_t rw = (size_t)bh * p.T + (ok ? iq : 0);
-      const float M = ok ? p.row_max[rw] : 0.f, m = ok ? p.row_min[rw] : 0.f;
-      const RowGrid g = row_grid(p, M, m);
-      for (int r = tid / BQRY; r <= Kq; r += NT / BQRY) tab[rr * tstride + r] = grid_value(p, g, r);
-    }
-    __syncthreads();
-
-    const uint8_t* st = stage_ptr(it);
-    if (tid == 0) {
-      const bool ok =
-          mbar_wait(&bar_st[it % p.nstage], (it / p.nstage) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-      if (ok) {
-        tc_fence_after();
-        if (p.x3) {
-          mma_tmem_smem(tmem + cS, tmem + cK + D, st + oQ, BQRY, D, false);
-          mma_tmem_smem(tmem + cS, tmem + cK, st + oQ + qtile, BQRY, D, true);
-          mma_tmem_smem(tmem + cS, tmem + cK, st + oQ, BQRY, D, true);
-          if (do_dk) {
-            mma_tmem_smem(tmem + cG, tmem + cV + D, st + odO, BQRY, D, false);
-            mma_tmem_smem(tmem + cG, tmem + cV, st + odO + qtile, BQRY, D, true);
-            mma_tmem_smem(tmem + cG, tmem + cV, st + odO, BQRY, D, true);
-          }
-        } else {
-          mma_tmem_smem(tmem + cS, tmem + cK, st + oQ, BQRY, D, false);
-          if (do_dk) mma_tmem_smem(tmem + cG, tmem + cV, st + odO, BQRY, D, false);
-        }
-        mma_commit(bar_mma);
-      }
-    }
-    bool ok = mbar_wait(bar_mma, mph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    mph ^= 1;
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
-    }
-    tc_fence_after();
-#pragma unroll 1
-    for (int c = 0; c < BQRY / 32; ++c) {
-      float sv[32], gv[32], pa[32], da[32];
-      tmem_ld32(lane_addr(tmem, cS + c * 32), sv);
-      if (do_dk) tmem_ld32(lane_addr(tmem, cG + c * 32), gv);
-      tmem_ld_wait();
-#pragma unroll
-      for (int ii = 0; ii < 32; ++ii) {
-        const int r_ = c * 32 + ii;  // query row within the tile
-        const int iq = q0 + r_;
-        const bool valid = key_ok && iq < p.T && iq >= j;
-        float pv = 0.f, ds = 0.f;
-        if (valid) {
-          RowB R;
-          R.M = qr->M[r_];
-          R.m = qr->m[r_];
-          R.g.inv_h = qr->inv_h[r_];
-          R.g.k1 = __fmul_rn(p.scale, R.g.inv_h);
-          R.g.c0 = qr->c0[r_];
-          R.g.nogrid = qr->nogrid[r_] != 0;
-          R.invWf = qr->invWf[r_];
-          R.invWs = qr->invWs[r_];
-          R.D = qr->D[r_];
-          const float s = __fmul_rn(sv[ii], p.scale);
-          KeyPos kp{0, 0, 0.f, false};
-          float er = 0.f, er1 = 0.f, el = 0.f;
-          if (p.calib != CAL_SOFTMAX && !R.g.nogrid) {
-            kp = key_pos(p, __fmaf_rn(sv[ii], R.g.k1, R.g.c0));
-            if (!kp.tail) {
-              const float* t_ = tab + r_ * tstride;
-              er = t_[kp.r];
-              er1 = t_[kp.r + 1];
-              el = t_[kp.l];
-            }
-          }
-          const BwdElem e = bwd_elem(p, R, s, do_dk ? gv[ii] : 0.f, er, er1, el, kp);
-          pv = e.p;
-          ds = e.ds;
-          if (fullg && !R.g.nogrid) {
-            const int nM = qr->nmax[r_];
-            if (nM == 1 ? (j == qr->amax[r_]) : (s == R.M)) ds += qr->cMn[r_];
-            if (minmax) {
-              const int nm = qr->nmin[r_];
-              if (nm == 1 ? (j == qr->amin[r_]) : (s == R.m)) ds += qr->cmn[r_];
-            }
-          }
-        }
-        if (p.x3) {
-          const float x = do_dv ? pv : ds;
-          const float h = tf32_rna(x);
-          pa[ii] = h;
-          da[ii] = __fsub_rn(x, h);
-        } else {
-          pa[ii] = pv;
-          da[ii] = ds;
-        }
-      }
-      if (p.x3 || do_dv) tmem_st32(lane_addr(tmem, cS + c * 32), pa);
-      if (p.x3 || do_dk) tmem_st32(lane_addr(tmem, cG + c * 32), da);
-    }
+  if (warp < NCOMP / 32) {
+    if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    if (CAL == CAL_FWM && tid < Kq)
+      *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
     tmem_st_wait();
-    tc_fence_before();
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-      const bool acc = it > 0;
-      if (p.x3) {
-        // one product per launch: A_hi at cS, A_lo at cG
-        const int cacc = do_dv ? cdV : cdK;
-        const uint8_t* b = st + (do_dv ? odOT : oQT);
-        mma_tmem_smem(tmem + cacc, tmem + cS, b, D, BQRY, acc);
-        mma_tmem_smem(tmem + cacc, tmem + cS, b + qtile, D, BQRY, true);
-        mma_tmem_smem(tmem + cacc, tmem + cG, b, D, BQRY, true);
-      } else {
-        if (do_dv) mma_tmem_smem(tmem + cdV, tmem + cS, st + odOT, D, BQRY, acc);
-        if (do_dk) mma_tmem_smem(tmem + cdK, tmem + cG, st + oQT, D, BQRY, acc);
-      }
-      mma_commit(bar_mma);
-    }
-    ok = mbar_wait(bar_mma, mph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    mph ^= 1;
-    if (cta_any(!ok)) {
-      failed = true;
-      break;
-    }
-    tc_fence_after();
-    if (tid == 0 && it + p.nstage < nit) load_stage(it + p.nstage);
-  }
-
-  if (!failed) {
-    const size_t krow = (size_t)bh * p.T + (key_ok ? j : 0);
-    for (int pass = 0; pass < 2; ++pass) {
-      const bool want = pass == 0 ? do_dv : do_dk;
-      if (!want) continue;
-      const int col = pass == 0 ? cdV : cdK;
-      const float mul = pass == 0 ? 1.0f : p.scale;
-      float* dst = (pass == 0 ? p.dV : p.dK) + krow * D;
-      for (int c = 0; c < D; c += 32) {
-        float v[32];
-        tmem_ld32(lane_addr(tmem, col + c), v);
-        tmem_ld_wait();
-        if (key_ok) {
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            reinterpret_cast<float4*>(dst + c)[q] =
-                make_float4(v[4 * q] * mul, v[4 * q + 1] * mul, v[4 * q + 2] * mul, v[4 * q + 3] * mul);
-        }
-      }
-    }
   }
   tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+
+  if (warp == PRODUCER_WARP3) {
+    if ((tid & 31) == 0) {
+      for (int it = 0; it < nit; ++it) {
+        const int s = it % NS, q0 = (qt0 + it) * BT;
+        if (it >= NS &&
+            !mbar_wait(&bar_empty[s], ((it / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+          break;
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        uint64_t* b = &bar_full[s];
+        const int nrows = min(BT, p.T - q0);
+        const int ntiles = 1 + (needV ? 1 : 0) + (doDK ? 1 : 0) + (doDV ? 1 : 0);
+        uint32_t bytes = ntiles * parts * qtile + nrows * 64;
+        if (CAL == CAL_MINMAX) bytes += nrows * tstride;
+        mbar_arrive_expect_tx(b, bytes);
+        load_rows_tile(dst + oQ, &maps.q, b, D, BT, 0, q0, bh);
+        if (p.x3) load_rows_tile(dst + oQ + qtile, &maps.q_lo, b, D, BT, 0, q0, bh);
+        if (needV) {
+          load_rows_tile(dst + odO, &maps.dout, b, D, BT, 0, q0, bh);
+          if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BT, 0, q0, bh);
+        }
+        if (doDK) {
+          load_rows_tile(dst + oQT, &maps.qt, b, BT, D, q0, 0, bh);
+          if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BT, D, q0, 0, bh);
+        }
+        if (doDV) {
+          load_rows_tile(dst + odOT, &maps.dot, b, BT, D, q0, 0, bh);
+          if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BT, D, q0, 0, bh);
+        }
+        const size_t r0 = (size_t)bh * p.T + q0;
+        bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
+        if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
+      }
+    }
+  } else if (warp == MMA_WARP3) {
+    if ((tid & 31) == 0) {
+      auto issue_sg = [&](int it) -> bool {
+        const int s = it % NS, b = it % nbuf;
+        if (!mbar_wait(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+        tc_fence_after();
+        const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
+        if (p.x3) {
+          mma_tmem_smem(cS, tmem + cK + D, st + oQ, BT, D, false);
+          mma_tmem_smem(cS, tmem + cK, st + oQ + qtile, BT, D, true);
+          mma_tmem_smem(cS, tmem + cK, st + oQ, BT, D, true);
+          if (needV) {
+            mma_tmem_smem(cG, tmem + cV + D, st + odO, BT, D, false);
+            mma_tmem_smem(cG, tmem + cV, st + odO + qtile, BT, D, true);
+            mma_tmem_smem(cG, tmem + cV, st + odO, BT, D, true);
+          }
+        } else {
+          mma_tmem_smem(cS, tmem + cK, st + oQ, BT, D, false);
+          if (needV) mma_tmem_smem(cG, tmem + cV, st + odO, BT, D, false);
+        }
+        mma_commit(&bar_sfull[b]);
+        return true;
+      };
+      bool ok = issue_sg(0);
+      for (int it = 0; it < nit && ok; ++it) {
+        const int b = it % nbuf, s = it % NS;
+        if (nbuf == 2 && it + 1 < nit) ok = issue_sg(it + 1);
+        if (!ok) break;
+        if (!mbar_wait(&bar_pready[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        tc_fence_after();
+        const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
+        const bool acc = it > 0;
+        if (p.x3) {
+          const uint32_t cacc = tmem + (doDV ? cdV : cdK);
+          const uint8_t* bt = st + (doDV ? odOT : oQT);
+          mma_tmem_smem(cacc, cS, bt, D, BT, acc);
+          mma_tmem_smem(cacc, cS, bt + qtile, D, BT, true);
+          mma_tmem_smem(cacc, cG, bt, D, BT, true);
+        } else {
+          if (doDV) mma_tmem_smem(tmem + cdV, cS, st + odOT, D, BT, acc);
+          if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
+        }
+        mma_commit(&bar_empty[s]);
+        if (nbuf == 1 && it + 1 < nit) ok = issue_sg(it + 1);
+      }
+      mma_commit(bar_done);
+    }
+  } else {
+    const float Kf = (float)Kq;
+    const uint32_t fwtab = smem_u32(sm + p.sm_table) - 0x58000000u;
+    bool failed = false;
+    for (int it = 0; it < nit; ++it) {
+      const int b = it % nbuf, s = it % NS;
+      const int q0 = (qt0 + it) * BT, i0 = q0 + cg * 32;
+      const bool ok1 = mbar_wait(&bar_sfull[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      // the stage's row records arrived with its tiles (bar_full), before the products were issued
+      const bool ok2 = ok1 && mbar_wait(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+      if (!ok2) {
+        failed = true;
+        break;
+      }
+      tc_fence_after();
+      const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      const uint32_t recs = smem_u32(st + oRec) + cg * 32 * 64;
+      const uint32_t tabs = smem_u32(st + oTab) + cg * 32 * tstride - 0x58000000u;
+      const int cS = base + 128 * b + cg * 32, cG = cS + 64;
+      float sv[32], gv[32], pa[32], da[32];
+      tmem_ld32(lane_addr(tmem, cS), sv);
+      if (needV) {
+        tmem_ld32(lane_addr(tmem, cG), gv);
+      } else {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) gv[q] = 0.f;
+      }
+      tmem_ld_wait();
+      const bool masked = (i0 < kb * 128 + 128) || (i0 + 32 > p.T);
+      if (masked)
+        kv_chunk<CAL, REC, FULLG, true>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
+      else
+        kv_chunk<CAL, REC, FULLG, false>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
+      if constexpr (FULLG && CAL != CAL_SOFTMAX) {
+        // rows with tied extrema: the tie set is found by equality on the recomputed scores
+        const int nr = min(32, p.T - i0);
+        bool any = false;
+        for (int ii = 0; ii < nr; ++ii) any |= (reinterpret_cast<const RowRec*>(st + oRec)[cg * 32 + ii].flags &
+                                                 (REC_TIEMAX | REC_TIEMIN)) != 0;
+        if (any) {
+#pragma unroll
+          for (int ii = 0; ii < 32; ++ii) {
+            const RowRec& r = reinterpret_cast<const RowRec*>(st + oRec)[cg * 32 + ii];
+            const bool okr = ii < nr && i0 + ii >= j && (r.flags & (REC_TIEMAX | REC_TIEMIN)) &&
+                             !(r.flags & REC_NOGRID);
+            const float sc = __fmul_rn(sv[ii], p.scale);
+            if (okr && (r.flags & REC_TIEMAX) && sc == r.M) da[ii] += r.cMn;
+            if (CAL == CAL_MINMAX && okr && (r.flags & REC_TIEMIN) && sc == r.m) da[ii] += r.cmn;
+          }
+        }
+      }
+      if (p.x3) {
+#pragma unroll
+        for (int q = 0; q < 32; ++q) {
+          const float x = doDV ? pa[q] : da[q];
+          const float h = tf32_rna(x);
+          pa[q] = h;
+          da[q] = __fsub_rn(x, h);
+        }
+        tmem_st32(lane_addr(tmem, cS), pa);
+        tmem_st32(lane_addr(tmem, cG), da);
+      } else {
+        if (doDV) tmem_st32(lane_addr(tmem, cS), pa);
+        if (doDK) tmem_st32(lane_addr(tmem, cG), da);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
+    }
+    const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+    if (!failed) {
+      tc_fence_after();
+      const size_t krow = (size_t)bh * p.T + (key_ok ? j : 0);
+      for (int pass = 0; pass < 2; ++pass) {
+        if (pass == 0 ? !doDV : !doDK) continue;
+        const int col = pass == 0 ? cdV : cdK;
+        const float mul = pass == 0 ? 1.0f : p.scale;
+        float* dst = (pass == 0 ? p.dV : p.dK) + krow * D;
+        for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
+          float v[32];
+          tmem_ld32(lane_addr(tmem, col + c), v);
+          tmem_ld_wait();
+          if (key_ok) {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              reinterpret_cast<float4*>(dst + c)[q] =
+                  make_float4(v[4 * q] * mul, v[4 * q + 1] * mul, v[4 * q + 2] * mul, v[4 * q + 3] * mul);
+          }
+        }
+      }
+    }
+    tc_fence_before();
+  }
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
 
-cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(k_bwd_dkdv, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+// ---------------------------------------------------------------------------
+template <class K>
+static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  k_bwd_dkdv<<<dim3((p.T + 127) / 128, p.BH), NT, smem_bytes, s>>>(maps, p);
+  kern<<<grid, NTHR3, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
+}
+
+cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+  const dim3 grid(p.nqb, p.BH);
+  const bool full = p.grad == 0;
+  if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s);
+  if (p.calib == CAL_MINMAX)
+    return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s)
+                : launch3(k_bwd_dq<CAL_MINMAX, false>, grid, maps, p, smem_bytes, s);
+  return full ? launch3(k_bwd_dq<CAL_FWM, true>, grid, maps, p, smem_bytes, s)
+              : launch3(k_bwd_dq<CAL_FWM, false>, grid, maps, p, smem_bytes, s);
+}
+
+cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+  const dim3 grid((p.T + 127) / 128, p.BH);
+  const bool full = p.grad == 0, near = p.recon == REC_NEAREST;
+  if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dkdv<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+  if (p.calib == CAL_MINMAX) {
+    if (near)
+      return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)
+                  : launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
+    return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, true>, grid, maps, p, smem_bytes, s)
+                : launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+  }
+  if (near)
+    return full ? launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)
+                : launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
+  return full ? launch3(k_bwd_dkdv<CAL_FWM, REC_LERP, true>, grid, maps, p, smem_bytes, s)
+              : launch3(k_bwd_dkdv<CAL_FWM, REC_LERP, false>, grid, maps, p, smem_bytes, s);
 }
 
 }  // namespace kint

@@ -48,6 +48,22 @@ constexpr int NTHR = NCOMP + 32;
 constexpr int PRODUCER_WARP = NCOMP / 32;
 constexpr int BAR_COMPUTE = 1;  // named barrier id of the compute group
 
+// Kernels with a dedicated MMA warp: compute warps [0, 8), MMA warp 8, producer
+// warp 9.  The compute warps meet no CTA-wide barrier inside the tile loop; they
+// hand tiles to the MMA warp through mbarriers.
+constexpr int NTHR3 = NCOMP + 64;
+constexpr int MMA_WARP3 = NCOMP / 32;
+constexpr int PRODUCER_WARP3 = NCOMP / 32 + 1;
+
+// Per-query-row record written by the dQ kernel for the dK/dV kernel (64 bytes).
+struct RowRec {
+  float c0, k1, inv_h, invWf;  // grid position u = acc * k1 + c0; forward 1/W
+  float ga, gb, cMn, cmn;      // gamma = g * ga + gb; extremum terms c_M / n_max, c_m / n_min
+  int amax, amin, flags, pad;  // arg-extrema; flags: 1 no grid, 2 tied maxima, 4 tied minima
+  float M, m, sk1, sc0;        // extrema; softmax e^{s-M} = 2^(acc * sk1 + sc0)
+};
+constexpr int REC_NOGRID = 1, REC_TIEMAX = 2, REC_TIEMIN = 4;
+
 // ---------------------------------------------------------------------------
 // Row grid.  Scores s are fp32 values of acc * scale.  The position of a key in
 // grid units is u = s * inv_h + c0:

@@ -47,7 +47,9 @@ struct Params {
   float *row_max, *row_min, *W, *W_lerp, *O_lerp;
   int32_t *arg_max, *arg_min, *n_max, *n_min;
   float *dQ, *dK, *dV;
-  float *Drow, *cMn, *cmn;  // per-row backward scalars (workspace)
+  void* rec;                // [B*H*T] per-query-row records (RowRec) written by the dQ kernel
+  float* rtab;              // [B*H*T][Kp] (e_r, e_{r+1}) MinMax grid pairs per row (workspace)
+  int Kp;                   // K rounded up to even (pair-table row stride in pairs)
   float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
   uint8_t *bins, *ivals;
 };
