@@ -103,6 +103,7 @@ struct Workspace {
   void* rec = nullptr;    // [BHT] 64-byte per-row records (dQ kernel -> dK/dV kernel)
   float* rtab = nullptr;  // [BHT][KMAX] (e_r, e_{r+1}) MinMax grid pairs
   float* tie = nullptr;   // [2][BHT][d] sums of tied arg-extremum keys
+  int* tileflags = nullptr;  // [BH][ceil(T/64)]
 };
 
 Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
@@ -133,6 +134,7 @@ Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
     w.rec = take(rows * 16);
     w.rtab = take(rows * 2 * KMAX);
     w.tie = take(2 * nat);
+    w.tileflags = reinterpret_cast<int*>(take((size_t)BH * ((T + 63) / 64) * 4));
   }
   w.bytes = off;
   return w;
@@ -243,7 +245,7 @@ int plan_dq(Params& p) {
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
-    const int total = std::max(finish_plan(p, p.sm_rows + 4 * 128 * 4, 2 * p.nstage + 5), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 5), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       return total;
@@ -426,6 +428,9 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   const Workspace w = plan_workspace(static_cast<char*>(workspace), BH, T, d, p.x3 != 0, true);
   p.rec = w.rec; p.rtab = w.rtab; p.tie_acc = w.tie;
   p.Kp = (p.Kint + 1) & ~1;
+  p.tileflags = w.tileflags;
+  p.nqt = (T + 63) / 64;
+  if (cudaMemsetAsync(p.tileflags, 0, (size_t)BH * p.nqt * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
 
   // Operand copies: K-major transposes (and 3xTF32 splits).
   if (p.x3) {

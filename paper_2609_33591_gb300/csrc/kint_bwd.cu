@@ -28,13 +28,13 @@ constexpr float kLog2e = 1.4426950408889634f;
 //   dw/dm = A_r + t B_r, A_r = (1 - r/K)(e_r - Delta),
 //   B_r = (1 - r/K)(e_{r+1} - e_r) - (e_{r+1} - Delta)/K   (Eq. calgrad per interval)
 // ---------------------------------------------------------------------------
-template <int CAL, bool FULLG, bool DIAG>
-__device__ __forceinline__ void dq_chunk(const float (&sv)[32], const float (&gv)[32], float (&out)[32], int j0,
+template <int CAL, bool FULLG, bool DIAG, int W>
+__device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)[W], float (&out)[W], int j0,
                                          int i, float k1, float c0, float inv_h, float ga, float gb, bool nogrid,
                                          float Kf, float fk, uint32_t tab, float sk1, float sc0, float invWf,
                                          float& own, float& cm) {
 #pragma unroll
-  for (int jj = 0; jj < 32; ++jj) {
+  for (int jj = 0; jj < W; ++jj) {
     float ds, dm = 0.f;
     if constexpr (CAL == CAL_SOFTMAX) {
       const float pr = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * invWf;
@@ -95,10 +95,11 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
   uint64_t* bar_pready = bars + 2 * NS + 2;  // [2]
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
-  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [4][128]
+  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = tid >> 5;
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
   const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
+  constexpr int W = BT / NCG3;  // key columns per thread per tile
   const int dp = D * parts;
   const int cQ = 0, cdO = dp, cdQ = 2 * dp + 128 * nbuf;
 
@@ -109,7 +110,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
-      mbar_init(&bar_pready[b], NCOMP / 32);
+      mbar_init(&bar_pready[b], NCOMP3 / 32);
     }
     mbar_init(bar_done, 1);
     fence_mbar_init();
@@ -124,16 +125,17 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
   const uint32_t tmem = *tslot;
 
   // ---- compute-thread set-up: operands Q / dO into TMEM, row constants, grid table ----
-  const int row = tid & 127, cg = (tid >> 7) & 1;
+  const int row = tid & 127, cg = (tid >> 7) & (NCG3 - 1);
   const int i = qb * 128 + row;
   const bool row_ok = i < p.T;
   const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
   float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
   int nmax = 1, nmin = 1, amax = 0, amin = 0;
   RowGrid g{};
-  if (warp < NCOMP / 32) {
-    const float* src = cg == 0 ? p.Q : p.dO;
-    row_to_tmem(tmem, cg == 0 ? cQ : cdO, src, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+  if (warp < NCOMP3 / 32) {
+    if (cg < 2)
+      row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
+                  p.x3 != 0);
     if (row_ok) {
       M = p.row_max[rw];
       m = p.row_min[rw];
@@ -146,12 +148,12 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     g = row_grid(p, M, m);
     const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
     Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
-    // <g>_{P*} = dO_i . O*_i, the two column groups each take half of the d columns
+    // <g>_{P*} = dO_i . O*_i, each column group takes a quarter of the d columns
     float acc = 0.f;
     if (row_ok) {
-      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / 8);
-      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / 8);
-      for (int q = 0; q < D / 8; ++q) {
+      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / 16);
+      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / 16);
+      for (int q = 0; q < D / 16; ++q) {
         const float4 x = __ldg(a + q), y = __ldg(b + q);
         acc = __fmaf_rn(x.x, y.x, acc);
         acc = __fmaf_rn(x.y, y.y, acc);
@@ -164,7 +166,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       if (tid < Kq)
         *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
     } else if constexpr (CAL == CAL_MINMAX) {
-      for (int r = cg; r < Kq; r += NCG) {
+      for (int r = cg; r < Kq; r += NCG3) {
         const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
         *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
         if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
@@ -243,8 +245,8 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     }
   } else {
     // ---- compute warps ----
-    group_sync(BAR_COMPUTE, NCOMP);
-    Dg = xch[row] + xch[128 + row];
+    group_sync(BAR_COMPUTE, NCOMP3);
+    Dg = xch[row] + xch[128 + row] + xch[256 + row] + xch[384 + row];
     const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
     const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
     const float invWf = 1.0f / Wf;
@@ -256,9 +258,11 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     const bool track = FULLG && CAL != CAL_SOFTMAX && row_ok && !g.nogrid && (nmax > 1 || (minmax && nmin > 1));
     float* tie_max = p.tie_acc + rw * D;
     float* tie_min = p.tie_acc + ((size_t)p.BH * p.T + rw) * D;
-    if (track && cg == 0)
+    if (track && cg == 0) {
       for (int k = 0; k < D; ++k) tie_max[k] = tie_min[k] = 0.f;
-    group_sync(BAR_COMPUTE, NCOMP);  // the two halves of a row may both add to its tie sums
+      atomicOr(p.tileflags + (size_t)bh * p.nqt + i / BT, 1);
+    }
+    group_sync(BAR_COMPUTE, NCOMP3);  // every column group of a row may add to its tie sums
     float own = 0.f, cm = 0.f;
     bool failed = false;
     for (int kt = 0; kt < nkt; ++kt) {
@@ -269,22 +273,22 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
         break;
       }
       tc_fence_after();
-      const int cS = 2 * dp + 128 * b + cg * 32, cG = cS + 64;
-      float sv[32], gv[32], out[32];
-      tmem_ld32(lane_addr(tmem, cS), sv);
-      tmem_ld32(lane_addr(tmem, cG), gv);
+      const int cS = 2 * dp + 128 * b + cg * W, cG = cS + 64;
+      float sv[W], gv[W], out[W];
+      tmem_ld16(lane_addr(tmem, cS), sv);
+      tmem_ld16(lane_addr(tmem, cG), gv);
       tmem_ld_wait();
-      const int j0 = kt * BT + cg * 32;
-      if (j0 + 31 > qb * 128)
-        dq_chunk<CAL, FULLG, true>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
-                                   sc0, invWf, own, cm);
+      const int j0 = kt * BT + cg * W;
+      if (j0 + W - 1 > qb * 128)
+        dq_chunk<CAL, FULLG, true, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
+                                      sc0, invWf, own, cm);
       else
-        dq_chunk<CAL, FULLG, false>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
-                                    sc0, invWf, own, cm);
+        dq_chunk<CAL, FULLG, false, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab,
+                                       sk1, sc0, invWf, own, cm);
       if (__any_sync(0xffffffffu, track)) {
         // rare: tied extrema, the tie set is found by equality on the recomputed scores
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
+        for (int jj = 0; jj < W; ++jj) {
           const int j = j0 + jj;
           const float s = __fmul_rn(sv[jj], p.scale);
           const bool okj = track && j <= i;
@@ -295,30 +299,34 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
         }
       }
       if (p.x3) {
-        float lo[32];
+        float lo[W];
 #pragma unroll
-        for (int q = 0; q < 32; ++q) {
+        for (int q = 0; q < W; ++q) {
           const float h = tf32_rna(out[q]);
           lo[q] = __fsub_rn(out[q], h);
           out[q] = h;
         }
-        tmem_st32(lane_addr(tmem, cG), lo);
+        tmem_st16(lane_addr(tmem, cG), lo);
       }
-      tmem_st32(lane_addr(tmem, cS), out);
+      tmem_st16(lane_addr(tmem, cS), out);
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
       if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
     }
     const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+    failed = group_any(BAR_COMPUTE, NCOMP3, !dok);
     if (!failed) {
       tc_fence_after();
-      xch[(cg)*128 + row] = own;
-      xch[(2 + cg) * 128 + row] = cm;
-      group_sync(BAR_COMPUTE, NCOMP);
-      const float own_t = xch[row] + xch[128 + row];
-      const float cm_t = xch[256 + row] + xch[384 + row];
+      xch[cg * 128 + row] = own;
+      xch[(NCG3 + cg) * 128 + row] = cm;
+      group_sync(BAR_COMPUTE, NCOMP3);
+      float own_t = 0.f, cm_t = 0.f;
+#pragma unroll
+      for (int q = 0; q < NCG3; ++q) {
+        own_t += xch[q * 128 + row];
+        cm_t += xch[(NCG3 + q) * 128 + row];
+      }
       // Eq. (full): c_m = sum gamma dw/dm; c_M = -sum gamma Delta - c_m (Delta + dw/dM + dw/dm = 0);
       // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys.
       const bool full = FULLG && CAL != CAL_SOFTMAX && !g.nogrid;
@@ -328,13 +336,13 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
       const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
       float* dst = p.dQ + rw * D;
-      for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
-        float v[32];
-        tmem_ld32(lane_addr(tmem, cdQ + c), v);
+      for (int c = cg * (D / NCG3); c < (cg + 1) * (D / NCG3); c += 16) {
+        float v[16];
+        tmem_ld16(lane_addr(tmem, cdQ + c), v);
         tmem_ld_wait();
         if (row_ok) {
-#pragma unroll 8
-          for (int q = 0; q < 32; ++q) {
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
             float x = v[q];
             if (full) {
               x = __fmaf_rn(cMn, __ldg(kmax + c + q), x);
@@ -383,12 +391,12 @@ __device__ __forceinline__ int4 lds_i4(uint32_t addr) {
   return v;
 }
 
-template <int CAL, int REC, bool FULLG, bool MASKED>
-__device__ __forceinline__ void kv_chunk(const float (&sv)[32], const float (&gv)[32], float (&pa)[32],
-                                         float (&da)[32], int j, int i0, int T, uint32_t recs, uint32_t tabs,
+template <int CAL, int REC, bool FULLG, bool MASKED, int W>
+__device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)[W], float (&pa)[W],
+                                         float (&da)[W], int j, int i0, int T, uint32_t recs, uint32_t tabs,
                                          uint32_t fwtab, uint32_t tstride, float Kf) {
 #pragma unroll
-  for (int ii = 0; ii < 32; ++ii) {
+  for (int ii = 0; ii < W; ++ii) {
     const uint32_t ra = recs + ii * 64u;  // RowRec of query row i0 + ii
     const float4 r0 = lds_f4(ra);          // c0, k1, inv_h, invWf
     const float4 r1 = lds_f4(ra + 16);     // ga, gb, cMn, cmn
@@ -468,6 +476,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   const int oQ = 0, odO = parts * qtile, oQT = 2 * parts * qtile, odOT = 3 * parts * qtile;
   const int oRec = 4 * parts * qtile, oTab = oRec + BT * 64;
   const uint32_t tstride = (uint32_t)p.Kp * 8u;
+  constexpr int W = BT / NCG3;  // query columns per thread per tile
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -476,7 +485,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
-      mbar_init(&bar_pready[b], NCOMP / 32);
+      mbar_init(&bar_pready[b], NCOMP3 / 32);
     }
     mbar_init(bar_done, 1);
     fence_mbar_init();
@@ -489,12 +498,12 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-  const int row = tid & 127, cg = (tid >> 7) & 1;
+  const int row = tid & 127, cg = (tid >> 7) & (NCG3 - 1);
   const int j = kb * 128 + row;
   const bool key_ok = j < p.T;
-  if (warp < NCOMP / 32) {
+  if (warp < NCOMP3 / 32) {
     if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-    else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    else if (cg == 1 && needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
     if (CAL == CAL_FWM && tid < Kq)
       *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
     tmem_st_wait();
@@ -591,7 +600,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
     bool failed = false;
     for (int it = 0; it < nit; ++it) {
       const int b = it % nbuf, s = it % NS;
-      const int q0 = (qt0 + it) * BT, i0 = q0 + cg * 32;
+      const int q0 = (qt0 + it) * BT, i0 = q0 + cg * W;
       const bool ok1 = mbar_wait(&bar_sfull[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       // the stage's row records arrived with its tiles (bar_full), before the products were issued
       const bool ok2 = ok1 && mbar_wait(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
@@ -601,33 +610,31 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
       }
       tc_fence_after();
       const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      const uint32_t recs = smem_u32(st + oRec) + cg * 32 * 64;
-      const uint32_t tabs = smem_u32(st + oTab) + cg * 32 * tstride - 0x58000000u;
-      const int cS = base + 128 * b + cg * 32, cG = cS + 64;
-      float sv[32], gv[32], pa[32], da[32];
-      tmem_ld32(lane_addr(tmem, cS), sv);
+      const uint32_t recs = smem_u32(st + oRec) + cg * W * 64;
+      const uint32_t tabs = smem_u32(st + oTab) + cg * W * tstride - 0x58000000u;
+      const int cS = base + 128 * b + cg * W, cG = cS + 64;
+      float sv[W], gv[W], pa[W], da[W];
+      tmem_ld16(lane_addr(tmem, cS), sv);
       if (needV) {
-        tmem_ld32(lane_addr(tmem, cG), gv);
+        tmem_ld16(lane_addr(tmem, cG), gv);
       } else {
 #pragma unroll
-        for (int q = 0; q < 32; ++q) gv[q] = 0.f;
+        for (int q = 0; q < W; ++q) gv[q] = 0.f;
       }
       tmem_ld_wait();
-      const bool masked = (i0 < kb * 128 + 128) || (i0 + 32 > p.T);
+      const bool masked = (i0 < kb * 128 + 128) || (i0 + W > p.T);
       if (masked)
-        kv_chunk<CAL, REC, FULLG, true>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
+        kv_chunk<CAL, REC, FULLG, true, W>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
       else
-        kv_chunk<CAL, REC, FULLG, false>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
+        kv_chunk<CAL, REC, FULLG, false, W>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
       if constexpr (FULLG && CAL != CAL_SOFTMAX) {
-        // rows with tied extrema: the tie set is found by equality on the recomputed scores
-        const int nr = min(32, p.T - i0);
-        bool any = false;
-        for (int ii = 0; ii < nr; ++ii) any |= (reinterpret_cast<const RowRec*>(st + oRec)[cg * 32 + ii].flags &
-                                                 (REC_TIEMAX | REC_TIEMIN)) != 0;
-        if (any) {
+        // rows with tied extrema (flagged per 64-row tile by the dQ kernel): the tie set is
+        // found by equality on the recomputed scores
+        if (__ldg(p.tileflags + (size_t)bh * p.nqt + qt0 + it)) {
+          const int nr = min(W, p.T - i0);
 #pragma unroll
-          for (int ii = 0; ii < 32; ++ii) {
-            const RowRec& r = reinterpret_cast<const RowRec*>(st + oRec)[cg * 32 + ii];
+          for (int ii = 0; ii < W; ++ii) {
+            const RowRec& r = reinterpret_cast<const RowRec*>(st + oRec)[cg * W + ii];
             const bool okr = ii < nr && i0 + ii >= j && (r.flags & (REC_TIEMAX | REC_TIEMIN)) &&
                              !(r.flags & REC_NOGRID);
             const float sc = __fmul_rn(sv[ii], p.scale);
@@ -638,17 +645,17 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
       }
       if (p.x3) {
 #pragma unroll
-        for (int q = 0; q < 32; ++q) {
+        for (int q = 0; q < W; ++q) {
           const float x = doDV ? pa[q] : da[q];
           const float h = tf32_rna(x);
           pa[q] = h;
           da[q] = __fsub_rn(x, h);
         }
-        tmem_st32(lane_addr(tmem, cS), pa);
-        tmem_st32(lane_addr(tmem, cG), da);
+        tmem_st16(lane_addr(tmem, cS), pa);
+        tmem_st16(lane_addr(tmem, cG), da);
       } else {
-        if (doDV) tmem_st32(lane_addr(tmem, cS), pa);
-        if (doDK) tmem_st32(lane_addr(tmem, cG), da);
+        if (doDV) tmem_st16(lane_addr(tmem, cS), pa);
+        if (doDK) tmem_st16(lane_addr(tmem, cG), da);
       }
       tmem_st_wait();
       tc_fence_before();
@@ -656,7 +663,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
       if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
     }
     const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+    failed = group_any(BAR_COMPUTE, NCOMP3, !dok);
     if (!failed) {
       tc_fence_after();
       const size_t krow = (size_t)bh * p.T + (key_ok ? j : 0);
@@ -665,13 +672,13 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
         const int col = pass == 0 ? cdV : cdK;
         const float mul = pass == 0 ? 1.0f : p.scale;
         float* dst = (pass == 0 ? p.dV : p.dK) + krow * D;
-        for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
-          float v[32];
-          tmem_ld32(lane_addr(tmem, col + c), v);
+        for (int c = cg * (D / NCG3); c < (cg + 1) * (D / NCG3); c += 16) {
+          float v[16];
+          tmem_ld16(lane_addr(tmem, col + c), v);
           tmem_ld_wait();
           if (key_ok) {
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
+            for (int q = 0; q < 4; ++q)
               reinterpret_cast<float4*>(dst + c)[q] =
                   make_float4(v[4 * q] * mul, v[4 * q + 1] * mul, v[4 * q + 2] * mul, v[4 * q + 3] * mul);
           }

@@ -48,12 +48,15 @@ constexpr int NTHR = NCOMP + 32;
 constexpr int PRODUCER_WARP = NCOMP / 32;
 constexpr int BAR_COMPUTE = 1;  // named barrier id of the compute group
 
-// Kernels with a dedicated MMA warp: compute warps [0, 8), MMA warp 8, producer
-// warp 9.  The compute warps meet no CTA-wide barrier inside the tile loop; they
-// hand tiles to the MMA warp through mbarriers.
-constexpr int NTHR3 = NCOMP + 64;
-constexpr int MMA_WARP3 = NCOMP / 32;
-constexpr int PRODUCER_WARP3 = NCOMP / 32 + 1;
+// Kernels with a dedicated MMA warp: NCG3 column groups of 128 compute threads
+// (warps [0, 4 NCG3)), then the MMA warp and the producer warp.  The compute
+// warps meet no CTA-wide barrier inside the tile loop; they hand tiles to the
+// MMA warp through mbarriers.
+constexpr int NCG3 = 4;
+constexpr int NCOMP3 = 128 * NCG3;
+constexpr int NTHR3 = NCOMP3 + 64;
+constexpr int MMA_WARP3 = NCOMP3 / 32;
+constexpr int PRODUCER_WARP3 = NCOMP3 / 32 + 1;
 
 // Per-query-row record written by the dQ kernel for the dK/dV kernel (64 bytes).
 struct RowRec {

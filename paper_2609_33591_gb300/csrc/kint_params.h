@@ -50,6 +50,8 @@ struct Params {
   void* rec;                // [B*H*T] per-query-row records (RowRec) written by the dQ kernel
   float* rtab;              // [B*H*T][Kp] (e_r, e_{r+1}) MinMax grid pairs per row (workspace)
   int Kp;                   // K rounded up to even (pair-table row stride in pairs)
+  int* tileflags;           // [B*H][nqt] 1 where a 64-row query tile holds a row with tied extrema
+  int nqt;                  // ceil(T / 64)
   float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
   uint8_t *bins, *ivals;
 };
