@@ -74,6 +74,32 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
   }
 }
 
+// MMA thread of k_bwd_dq: wait for key tile kt, then S_b = Q K^T and g_b = dO V^T
+// into score buffer b = kt % nbuf.
+__device__ __forceinline__ bool dq_issue_sg(const Params& p, int kt, uint64_t* bar_full, uint64_t* bar_sfull,
+                                            const uint8_t* st0, uint32_t cQa, uint32_t cdOa, uint32_t cSG,
+                                            int ktile) {
+  const int D = p.d, NS = p.nstage, s = kt % NS, b = kt % p.nbuf, parts = p.x3 ? 2 : 1;
+  if (!mbar_wait_spin(&bar_full[s], (kt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+  tc_fence_after();
+  const uint8_t* sk = st0 + s * p.sm_stage_bytes;
+  const uint8_t* sv = sk + parts * ktile;
+  const uint32_t cS = cSG + 128 * b, cG = cS + 64;
+  if (p.x3) {
+    mma_tmem_smem(cS, cQa + D, sk, BT, D, false);     // Q_lo K_hi
+    mma_tmem_smem(cS, cQa, sk + ktile, BT, D, true);  // Q_hi K_lo
+    mma_tmem_smem(cS, cQa, sk, BT, D, true);          // Q_hi K_hi
+    mma_tmem_smem(cG, cdOa + D, sv, BT, D, false);
+    mma_tmem_smem(cG, cdOa, sv + ktile, BT, D, true);
+    mma_tmem_smem(cG, cdOa, sv, BT, D, true);
+  } else {
+    mma_tmem_smem(cS, cQa, sk, BT, D, false);
+    mma_tmem_smem(cG, cdOa, sv, BT, D, false);
+  }
+  mma_commit(&bar_sfull[b]);
+  return true;
+}
+
 // ---------------------------------------------------------------------------
 // k_bwd_dq.
 // TMEM: Q [0, dp), dO [dp, 2dp) (dp = d, or 2d for 3xTF32 hi|lo; loaded by the
@@ -133,9 +159,9 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
   int nmax = 1, nmin = 1, amax = 0, amin = 0;
   RowGrid g{};
   if (warp < NCOMP3 / 32) {
-    if (cg < 2)
-      row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
-                  p.x3 != 0);
+    // operand rows into TMEM: column group 0 takes Q, group 1 takes dO
+    row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
+                p.x3 != 0);
     if (row_ok) {
       M = p.row_max[rw];
       m = p.row_min[rw];
@@ -148,12 +174,12 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     g = row_grid(p, M, m);
     const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
     Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
-    // <g>_{P*} = dO_i . O*_i, each column group takes a quarter of the d columns
+    // <g>_{P*} = dO_i . O*_i, each column group takes its share of the d columns
     float acc = 0.f;
     if (row_ok) {
-      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / 16);
-      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / 16);
-      for (int q = 0; q < D / 16; ++q) {
+      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / (4 * NCG3));
+      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / (4 * NCG3));
+      for (int q = 0; q < D / (4 * NCG3); ++q) {
         const float4 x = __ldg(a + q), y = __ldg(b + q);
         acc = __fmaf_rn(x.x, y.x, acc);
         acc = __fmaf_rn(x.y, y.y, acc);
@@ -183,7 +209,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       for (int kt = 0; kt < nkt; ++kt) {
         const int s = kt % NS;
         if (kt >= NS &&
-            !mbar_wait(&bar_empty[s], ((kt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+            !mbar_wait_spin(&bar_empty[s], ((kt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
           break;
         uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
         uint64_t* b = &bar_full[s];
@@ -200,33 +226,14 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     }
   } else if (warp == MMA_WARP3) {
     if ((tid & 31) == 0) {
-      auto issue_sg = [&](int kt) -> bool {
-        const int s = kt % NS, b = kt % nbuf;
-        if (!mbar_wait(&bar_full[s], (kt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
-        tc_fence_after();
-        const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        const uint8_t* sv = sk + parts * ktile;
-        const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
-        if (p.x3) {
-          mma_tmem_smem(cS, tmem + cQ + D, sk, BT, D, false);     // Q_lo K_hi
-          mma_tmem_smem(cS, tmem + cQ, sk + ktile, BT, D, true);  // Q_hi K_lo
-          mma_tmem_smem(cS, tmem + cQ, sk, BT, D, true);          // Q_hi K_hi
-          mma_tmem_smem(cG, tmem + cdO + D, sv, BT, D, false);
-          mma_tmem_smem(cG, tmem + cdO, sv + ktile, BT, D, true);
-          mma_tmem_smem(cG, tmem + cdO, sv, BT, D, true);
-        } else {
-          mma_tmem_smem(cS, tmem + cQ, sk, BT, D, false);
-          mma_tmem_smem(cG, tmem + cdO, sv, BT, D, false);
-        }
-        mma_commit(&bar_sfull[b]);
-        return true;
-      };
-      bool ok = issue_sg(0);
+      const uint8_t* st0 = sm + p.sm_stage0;
+      const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + 2 * dp;
+      bool ok = dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
       for (int kt = 0; kt < nkt && ok; ++kt) {
         const int b = kt % nbuf, s = kt % NS;
-        if (nbuf == 2 && kt + 1 < nkt) ok = issue_sg(kt + 1);
+        if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
         if (!ok) break;
-        if (!mbar_wait(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        if (!mbar_wait_spin(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
         tc_fence_after();
         const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
         const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
@@ -239,14 +246,17 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
           mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
         }
         mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && kt + 1 < nkt) ok = issue_sg(kt + 1);  // in order after the product reading S_0
+        if (nbuf == 1 && kt + 1 < nkt)  // in order after the product reading S_0
+          ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
       }
       mma_commit(bar_done);
     }
   } else {
     // ---- compute warps ----
     group_sync(BAR_COMPUTE, NCOMP3);
-    Dg = xch[row] + xch[128 + row] + xch[256 + row] + xch[384 + row];
+    Dg = 0.f;
+#pragma unroll
+    for (int q = 0; q < NCG3; ++q) Dg += xch[q * 128 + row];
     const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
     const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
     const float invWf = 1.0f / Wf;
@@ -275,8 +285,8 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       tc_fence_after();
       const int cS = 2 * dp + 128 * b + cg * W, cG = cS + 64;
       float sv[W], gv[W], out[W];
-      tmem_ld16(lane_addr(tmem, cS), sv);
-      tmem_ld16(lane_addr(tmem, cG), gv);
+      tmem_ldw<W>(lane_addr(tmem, cS), sv);
+      tmem_ldw<W>(lane_addr(tmem, cG), gv);
       tmem_ld_wait();
       const int j0 = kt * BT + cg * W;
       if (j0 + W - 1 > qb * 128)
@@ -306,9 +316,9 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
           lo[q] = __fsub_rn(out[q], h);
           out[q] = h;
         }
-        tmem_st16(lane_addr(tmem, cG), lo);
+        tmem_stw<W>(lane_addr(tmem, cG), lo);
       }
-      tmem_st16(lane_addr(tmem, cS), out);
+      tmem_stw<W>(lane_addr(tmem, cS), out);
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
@@ -337,19 +347,26 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
       float* dst = p.dQ + rw * D;
       for (int c = cg * (D / NCG3); c < (cg + 1) * (D / NCG3); c += 16) {
+        // the arg-extremum key rows first (all loads in flight before any store)
+        float km[16], kn[16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float4 a = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
+          const float4 b2 = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
+                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+          km[4 * q] = a.x; km[4 * q + 1] = a.y; km[4 * q + 2] = a.z; km[4 * q + 3] = a.w;
+          kn[4 * q] = b2.x; kn[4 * q + 1] = b2.y; kn[4 * q + 2] = b2.z; kn[4 * q + 3] = b2.w;
+        }
         float v[16];
         tmem_ld16(lane_addr(tmem, cdQ + c), v);
         tmem_ld_wait();
         if (row_ok) {
 #pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            float x = v[q];
-            if (full) {
-              x = __fmaf_rn(cMn, __ldg(kmax + c + q), x);
-              if (minmax) x = __fmaf_rn(cmn, __ldg(kmin + c + q), x);
-            }
-            dst[c + q] = x * p.scale;
-          }
+          for (int q = 0; q < 16; ++q) v[q] = __fmaf_rn(cmn, kn[q], __fmaf_rn(cMn, km[q], v[q])) * p.scale;
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            reinterpret_cast<float4*>(dst + c)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
         }
       }
       if (row_ok && cg == 0) {
@@ -445,6 +462,33 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
   }
 }
 
+// MMA thread of k_bwd_dkdv: wait for query tile it, then S^T_b = K Q^T and (dK launches)
+// g^T_b = V dO^T into score buffer b = it % nbuf.
+__device__ __forceinline__ bool kv_issue_sg(const Params& p, int it, uint64_t* bar_full, uint64_t* bar_sfull,
+                                            const uint8_t* st0, uint32_t cKa, uint32_t cVa, uint32_t cSG,
+                                            int qtile, bool needV, int oQ, int odO) {
+  const int D = p.d, NS = p.nstage, s = it % NS, b = it % p.nbuf;
+  if (!mbar_wait_spin(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+  tc_fence_after();
+  const uint8_t* st = st0 + s * p.sm_stage_bytes;
+  const uint32_t cS = cSG + 128 * b, cG = cS + 64;
+  if (p.x3) {
+    mma_tmem_smem(cS, cKa + D, st + oQ, BT, D, false);
+    mma_tmem_smem(cS, cKa, st + oQ + qtile, BT, D, true);
+    mma_tmem_smem(cS, cKa, st + oQ, BT, D, true);
+    if (needV) {
+      mma_tmem_smem(cG, cVa + D, st + odO, BT, D, false);
+      mma_tmem_smem(cG, cVa, st + odO + qtile, BT, D, true);
+      mma_tmem_smem(cG, cVa, st + odO, BT, D, true);
+    }
+  } else {
+    mma_tmem_smem(cS, cKa, st + oQ, BT, D, false);
+    if (needV) mma_tmem_smem(cG, cVa, st + odO, BT, D, false);
+  }
+  mma_commit(&bar_sfull[b]);
+  return true;
+}
+
 // ---------------------------------------------------------------------------
 // k_bwd_dkdv.  Thread t (< 256) owns key j = kb*128 + t%128 and the query half
 // t/128 of each 64-query tile.  TMEM: K [0, dp), V [dp, 2dp) (dK launches),
@@ -502,8 +546,9 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   const int j = kb * 128 + row;
   const bool key_ok = j < p.T;
   if (warp < NCOMP3 / 32) {
+    // operand rows into TMEM: column group 0 takes K, group 1 takes V
     if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-    else if (cg == 1 && needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
     if (CAL == CAL_FWM && tid < Kq)
       *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
     tmem_st_wait();
@@ -517,7 +562,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
       for (int it = 0; it < nit; ++it) {
         const int s = it % NS, q0 = (qt0 + it) * BT;
         if (it >= NS &&
-            !mbar_wait(&bar_empty[s], ((it / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+            !mbar_wait_spin(&bar_empty[s], ((it / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
           break;
         uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
         uint64_t* b = &bar_full[s];
@@ -547,34 +592,15 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
     }
   } else if (warp == MMA_WARP3) {
     if ((tid & 31) == 0) {
-      auto issue_sg = [&](int it) -> bool {
-        const int s = it % NS, b = it % nbuf;
-        if (!mbar_wait(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
-        tc_fence_after();
-        const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
-        if (p.x3) {
-          mma_tmem_smem(cS, tmem + cK + D, st + oQ, BT, D, false);
-          mma_tmem_smem(cS, tmem + cK, st + oQ + qtile, BT, D, true);
-          mma_tmem_smem(cS, tmem + cK, st + oQ, BT, D, true);
-          if (needV) {
-            mma_tmem_smem(cG, tmem + cV + D, st + odO, BT, D, false);
-            mma_tmem_smem(cG, tmem + cV, st + odO + qtile, BT, D, true);
-            mma_tmem_smem(cG, tmem + cV, st + odO, BT, D, true);
-          }
-        } else {
-          mma_tmem_smem(cS, tmem + cK, st + oQ, BT, D, false);
-          if (needV) mma_tmem_smem(cG, tmem + cV, st + odO, BT, D, false);
-        }
-        mma_commit(&bar_sfull[b]);
-        return true;
-      };
-      bool ok = issue_sg(0);
+      const uint8_t* st0 = sm + p.sm_stage0;
+      const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;
+      bool ok = kv_issue_sg(p, 0, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
       for (int it = 0; it < nit && ok; ++it) {
         const int b = it % nbuf, s = it % NS;
-        if (nbuf == 2 && it + 1 < nit) ok = issue_sg(it + 1);
+        if (nbuf == 2 && it + 1 < nit)
+          ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
         if (!ok) break;
-        if (!mbar_wait(&bar_pready[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        if (!mbar_wait_spin(&bar_pready[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
         tc_fence_after();
         const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
         const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
@@ -590,7 +616,8 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
           if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
         }
         mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && it + 1 < nit) ok = issue_sg(it + 1);
+        if (nbuf == 1 && it + 1 < nit)
+          ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
       }
       mma_commit(bar_done);
     }
@@ -614,9 +641,9 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
       const uint32_t tabs = smem_u32(st + oTab) + cg * W * tstride - 0x58000000u;
       const int cS = base + 128 * b + cg * W, cG = cS + 64;
       float sv[W], gv[W], pa[W], da[W];
-      tmem_ld16(lane_addr(tmem, cS), sv);
+      tmem_ldw<W>(lane_addr(tmem, cS), sv);
       if (needV) {
-        tmem_ld16(lane_addr(tmem, cG), gv);
+        tmem_ldw<W>(lane_addr(tmem, cG), gv);
       } else {
 #pragma unroll
         for (int q = 0; q < W; ++q) gv[q] = 0.f;
@@ -651,11 +678,11 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
           pa[q] = h;
           da[q] = __fsub_rn(x, h);
         }
-        tmem_st16(lane_addr(tmem, cS), pa);
-        tmem_st16(lane_addr(tmem, cG), da);
+        tmem_stw<W>(lane_addr(tmem, cS), pa);
+        tmem_stw<W>(lane_addr(tmem, cG), da);
       } else {
-        if (doDV) tmem_st16(lane_addr(tmem, cS), pa);
-        if (doDK) tmem_st16(lane_addr(tmem, cG), da);
+        if (doDV) tmem_stw<W>(lane_addr(tmem, cS), pa);
+        if (doDK) tmem_stw<W>(lane_addr(tmem, cG), da);
       }
       tmem_st_wait();
       tc_fence_before();

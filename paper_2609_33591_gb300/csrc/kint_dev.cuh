@@ -52,11 +52,29 @@ constexpr int BAR_COMPUTE = 1;  // named barrier id of the compute group
 // (warps [0, 4 NCG3)), then the MMA warp and the producer warp.  The compute
 // warps meet no CTA-wide barrier inside the tile loop; they hand tiles to the
 // MMA warp through mbarriers.
-constexpr int NCG3 = 4;
+constexpr int NCG3 = 2;
 constexpr int NCOMP3 = 128 * NCG3;
 constexpr int NTHR3 = NCOMP3 + 64;
 constexpr int MMA_WARP3 = NCOMP3 / 32;
 constexpr int PRODUCER_WARP3 = NCOMP3 / 32 + 1;
+
+// W-column TMEM row access (W = 16 or 32).
+template <int W>
+__device__ __forceinline__ void tmem_ldw(uint32_t taddr, float (&v)[W]) {
+  if constexpr (W == 32) {
+    tmem_ld32(taddr, v);
+  } else {
+    tmem_ld16(taddr, v);
+  }
+}
+template <int W>
+__device__ __forceinline__ void tmem_stw(uint32_t taddr, const float (&v)[W]) {
+  if constexpr (W == 32) {
+    tmem_st32(taddr, v);
+  } else {
+    tmem_st16(taddr, v);
+  }
+}
 
 // Per-query-row record written by the dQ kernel for the dK/dV kernel (64 bytes).
 struct RowRec {
@@ -188,25 +206,62 @@ __device__ __forceinline__ void load_rows_tile(uint8_t* dst, const CUtensorMap* 
     tma_load_3d(dst + pnl * nrows * SW, map, bar, c_first + 32 * pnl, r_first, bh);
 }
 
-// D[tmem, M=128 x N] (+)= A * B^T over Ktot, A in smem (128-row panels), B in
-// smem (N-row panels).
+// ---------------------------------------------------------------------------
+// Tensor-core products.  The issuing thread's own instruction stream bounds the
+// MMA rate (measured on GB300: an M=128, N=128 tf32 MMA every ~33 ns with
+// constant descriptors, ~43 ns when each descriptor is rebuilt), so descriptors
+// are built once per operand and advanced with one 32-bit add per k-step: the
+// start-address field holds (address >> 4) in 14 bits and shared addresses
+// stay below 256 KB, so the add never carries out of the field.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t desc_add(uint64_t d, uint32_t off16) {
+  uint32_t lo = (uint32_t)d + off16, hi = (uint32_t)(d >> 32);
+  return ((uint64_t)hi << 32) | lo;
+}
+
+// D[tmem, M=128 x N] (+)= A * B^T over KSTEPS x 8, A and B in smem (panels of
+// 32 K-columns, 128 B per row; A panels a_pnl bytes apart, B panels b_pnl).
+template <int KSTEPS>
+__device__ __forceinline__ void mma_ss_k(uint32_t d_tmem, const uint8_t* a, const uint8_t* b, int a_pnl, int b_pnl,
+                                         uint32_t idesc, bool accumulate) {
+  const uint64_t a0 = smem_desc_sw128(smem_u32(a), 16, 1024);
+  const uint64_t b0 = smem_desc_sw128(smem_u32(b), 16, 1024);
+  const uint32_t ap = (uint32_t)a_pnl >> 4, bp = (uint32_t)b_pnl >> 4;
+#pragma unroll
+  for (int kk = 0; kk < KSTEPS; ++kk) {
+    const uint32_t sub = (uint32_t)(kk & 3) * 2u;  // 32 bytes per k-step inside a panel
+    mma_tf32_ss(d_tmem, desc_add(a0, (uint32_t)(kk >> 2) * ap + sub), desc_add(b0, (uint32_t)(kk >> 2) * bp + sub),
+                idesc, (accumulate || kk > 0) ? 1u : 0u);
+  }
+}
+// D[tmem, M=128 x N] (+)= A * B^T over KSTEPS x 8, A in TMEM columns.
+template <int KSTEPS>
+__device__ __forceinline__ void mma_ts_k(uint32_t d_tmem, uint32_t a_tmem, const uint8_t* b, int b_pnl,
+                                         uint32_t idesc, bool accumulate) {
+  const uint64_t b0 = smem_desc_sw128(smem_u32(b), 16, 1024);
+  const uint32_t bp = (uint32_t)b_pnl >> 4;
+#pragma unroll
+  for (int kk = 0; kk < KSTEPS; ++kk)
+    mma_tf32_ts(d_tmem, a_tmem + kk * 8, desc_add(b0, (uint32_t)(kk >> 2) * bp + (uint32_t)(kk & 3) * 2u), idesc,
+                (accumulate || kk > 0) ? 1u : 0u);
+}
+
+// Runtime-K wrappers (K = 64 or 128 columns, or 128 / 256 for the key products).
 __device__ __forceinline__ void mma_smem_smem(uint32_t d_tmem, const uint8_t* a, const uint8_t* b, int N, int Ktot,
                                               bool accumulate) {
   const uint32_t idesc = idesc_tf32(128, N, 0, 0);
-  for (int kk = 0; kk < Ktot / 8; ++kk) {
-    const uint64_t ad = smem_desc_sw128(smem_u32(a + (kk >> 2) * (128 * SW) + (kk & 3) * 32), 16, 1024);
-    const uint64_t bd = smem_desc_sw128(smem_u32(b + (kk >> 2) * (N * SW) + (kk & 3) * 32), 16, 1024);
-    mma_tf32_ss(d_tmem, ad, bd, idesc, (accumulate || kk > 0) ? 1u : 0u);
-  }
+  if (Ktot == 64)
+    mma_ss_k<8>(d_tmem, a, b, 128 * SW, N * SW, idesc, accumulate);
+  else
+    mma_ss_k<16>(d_tmem, a, b, 128 * SW, N * SW, idesc, accumulate);
 }
-// D[tmem, M=128 x N] (+)= A * B^T over Ktot, A in TMEM columns [a_col, a_col+Ktot).
 __device__ __forceinline__ void mma_tmem_smem(uint32_t d_tmem, uint32_t a_tmem, const uint8_t* b, int N, int Ktot,
                                               bool accumulate) {
   const uint32_t idesc = idesc_tf32(128, N, 0, 0);
-  for (int kk = 0; kk < Ktot / 8; ++kk) {
-    const uint64_t bd = smem_desc_sw128(smem_u32(b + (kk >> 2) * (N * SW) + (kk & 3) * 32), 16, 1024);
-    mma_tf32_ts(d_tmem, a_tmem + kk * 8, bd, idesc, (accumulate || kk > 0) ? 1u : 0u);
-  }
+  if (Ktot == 64)
+    mma_ts_k<8>(d_tmem, a_tmem, b, N * SW, idesc, accumulate);
+  else
+    mma_ts_k<16>(d_tmem, a_tmem, b, N * SW, idesc, accumulate);
 }
 
 // The calling thread's TMEM lane (its row) at column `col`.  Warp w may only
@@ -216,33 +271,51 @@ __device__ __forceinline__ uint32_t lane_addr(uint32_t tmem_base, int col) {
   return tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + (uint32_t)col;
 }
 
-// Thread-owned row `row` of X (d fp32) into the thread's TMEM lane at columns
-// [col, col+d); with `split`, the tf32 hi part there and the lo part at
-// [col+d, col+2d).  Rows >= T load zeros.  Whole warps must call this.
-__device__ __forceinline__ void row_to_tmem(uint32_t tmem_base, int col, const float* X, int row, int T, int d,
-                                            bool split) {
+// Columns [c0, c0 + n) of row `row` of X (d fp32 per row) into the calling
+// thread's TMEM lane at columns [col + c0, col + c0 + n); with `split`, the tf32 hi
+// part there and the lo part d columns further.  All global loads are issued
+// before the first TMEM store.  Rows >= T load zeros.  n is 32 or 64; whole
+// warps must call this with the same c0, n.
+template <int N>
+__device__ __forceinline__ void row_to_tmem_part(uint32_t tmem_base, int col, const float* X, int row, int T, int d,
+                                                 int c0, bool split) {
   const bool in = row < T;
-  const float4* src = reinterpret_cast<const float4*>(X + (size_t)row * d);
-  for (int c = 0; c < d; c += 32) {
+  const float4* src = reinterpret_cast<const float4*>(X + (size_t)row * d + c0);
+  float v[N];
+#pragma unroll
+  for (int q = 0; q < N / 4; ++q) {
+    const float4 x = in ? __ldg(src + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+    v[4 * q] = x.x;
+    v[4 * q + 1] = x.y;
+    v[4 * q + 2] = x.z;
+    v[4 * q + 3] = x.w;
+  }
+#pragma unroll
+  for (int c = 0; c < N; c += 32) {
     float hi[32], lo[32];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      float4 v = in ? __ldg(src + (c >> 2) + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-      hi[4 * q + 0] = v.x;
-      hi[4 * q + 1] = v.y;
-      hi[4 * q + 2] = v.z;
-      hi[4 * q + 3] = v.w;
-    }
-    if (split) {
-#pragma unroll
-      for (int q = 0; q < 32; ++q) {
+    for (int q = 0; q < 32; ++q) {
+      hi[q] = v[c + q];
+      if (split) {
         const float h = tf32_rna(hi[q]);
         lo[q] = __fsub_rn(hi[q], h);
         hi[q] = h;
       }
-      tmem_st32(lane_addr(tmem_base, col + d + c), lo);
     }
-    tmem_st32(lane_addr(tmem_base, col + c), hi);
+    if (split) tmem_st32(lane_addr(tmem_base, col + d + c0 + c), lo);
+    tmem_st32(lane_addr(tmem_base, col + c0 + c), hi);
+  }
+}
+
+// Thread-owned row `row` of X (d fp32) into the thread's TMEM lane at columns
+// [col, col+d) (hi/lo with `split`, lo at [col+d, col+2d)).
+__device__ __forceinline__ void row_to_tmem(uint32_t tmem_base, int col, const float* X, int row, int T, int d,
+                                            bool split) {
+  if (d == 64) {
+    row_to_tmem_part<64>(tmem_base, col, X, row, T, d, 0, split);
+  } else {
+    row_to_tmem_part<64>(tmem_base, col, X, row, T, d, 0, split);
+    row_to_tmem_part<64>(tmem_base, col, X, row, T, d, 64, split);
   }
 }
 
