@@ -80,7 +80,7 @@ __device__ __forceinline__ bool dq_issue_sg(const Params& p, int kt, uint64_t* b
                                             const uint8_t* st0, uint32_t cQa, uint32_t cdOa, uint32_t cSG,
                                             int ktile) {
   const int D = p.d, NS = p.nstage, s = kt % NS, b = kt % p.nbuf, parts = p.x3 ? 2 : 1;
-  if (!mbar_wait_spin(&bar_full[s], (kt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+  if (!mbar_wait_warp(&bar_full[s], (kt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
   tc_fence_after();
   const uint8_t* sk = st0 + s * p.sm_stage_bytes;
   const uint8_t* sv = sk + parts * ktile;
@@ -110,7 +110,7 @@ __device__ __forceinline__ bool dq_issue_sg(const Params& p, int kt, uint64_t* b
 // sm_stage0; the grid pair table at sm_table; exchange words at sm_rows.
 // ---------------------------------------------------------------------------
 template <int CAL, bool FULLG>
-__global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int ktile = BT * D * 4;
@@ -122,10 +122,10 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
   const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
-  constexpr int W = BT / NCG3;  // key columns per thread per tile
+  constexpr int W = BT / NCG;  // key columns per thread per tile
   const int dp = D * parts;
   const int cQ = 0, cdO = dp, cdQ = 2 * dp + 128 * nbuf;
 
@@ -136,7 +136,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
-      mbar_init(&bar_pready[b], NCOMP3 / 32);
+      mbar_init(&bar_pready[b], NCOMP / 32);
     }
     mbar_init(bar_done, 1);
     fence_mbar_init();
@@ -151,14 +151,14 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
   const uint32_t tmem = *tslot;
 
   // ---- compute-thread set-up: operands Q / dO into TMEM, row constants, grid table ----
-  const int row = tid & 127, cg = (tid >> 7) & (NCG3 - 1);
+  const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
   const int i = qb * 128 + row;
   const bool row_ok = i < p.T;
   const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
   float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
   int nmax = 1, nmin = 1, amax = 0, amin = 0;
   RowGrid g{};
-  if (warp < NCOMP3 / 32) {
+  if (warp < NCOMP / 32) {
     // operand rows into TMEM: column group 0 takes Q, group 1 takes dO
     row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
                 p.x3 != 0);
@@ -177,9 +177,9 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
     // <g>_{P*} = dO_i . O*_i, each column group takes its share of the d columns
     float acc = 0.f;
     if (row_ok) {
-      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / (4 * NCG3));
-      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / (4 * NCG3));
-      for (int q = 0; q < D / (4 * NCG3); ++q) {
+      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / (4 * NCG));
+      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / (4 * NCG));
+      for (int q = 0; q < D / (4 * NCG); ++q) {
         const float4 x = __ldg(a + q), y = __ldg(b + q);
         acc = __fmaf_rn(x.x, y.x, acc);
         acc = __fmaf_rn(x.y, y.y, acc);
@@ -192,7 +192,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       if (tid < Kq)
         *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
     } else if constexpr (CAL == CAL_MINMAX) {
-      for (int r = cg; r < Kq; r += NCG3) {
+      for (int r = cg; r < Kq; r += NCG) {
         const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
         *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
         if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
@@ -204,59 +204,55 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
   __syncthreads();
   tc_fence_after();
 
-  if (warp == PRODUCER_WARP3) {
-    if ((tid & 31) == 0) {
-      for (int kt = 0; kt < nkt; ++kt) {
-        const int s = kt % NS;
-        if (kt >= NS &&
-            !mbar_wait_spin(&bar_empty[s], ((kt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-          break;
-        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        uint64_t* b = &bar_full[s];
-        mbar_arrive_expect_tx(b, 3 * parts * ktile);
-        load_rows_tile(dst, &maps.k, b, D, BT, 0, kt * BT, bh);
-        load_rows_tile(dst + parts * ktile, &maps.v, b, D, BT, 0, kt * BT, bh);
-        load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
-        if (p.x3) {
-          load_rows_tile(dst + ktile, &maps.k_lo, b, D, BT, 0, kt * BT, bh);
-          load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BT, 0, kt * BT, bh);
-          load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
-        }
+  if (warp == PRODUCER_WARP) {
+    for (int kt = 0; kt < nkt; ++kt) {
+      const int s = kt % NS;
+      if (kt >= NS &&
+          !mbar_wait_warp(&bar_empty[s], ((kt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+        break;
+      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      uint64_t* b = &bar_full[s];
+      mbar_arrive_expect_tx(b, 3 * parts * ktile);
+      load_rows_tile(dst, &maps.k, b, D, BT, 0, kt * BT, bh);
+      load_rows_tile(dst + parts * ktile, &maps.v, b, D, BT, 0, kt * BT, bh);
+      load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
+      if (p.x3) {
+        load_rows_tile(dst + ktile, &maps.k_lo, b, D, BT, 0, kt * BT, bh);
+        load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BT, 0, kt * BT, bh);
+        load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
       }
     }
-  } else if (warp == MMA_WARP3) {
-    if ((tid & 31) == 0) {
-      const uint8_t* st0 = sm + p.sm_stage0;
-      const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + 2 * dp;
-      bool ok = dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-      for (int kt = 0; kt < nkt && ok; ++kt) {
-        const int b = kt % nbuf, s = kt % NS;
-        if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-        if (!ok) break;
-        if (!mbar_wait_spin(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-        tc_fence_after();
-        const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
-        const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
-        const bool acc = kt > 0;
-        if (p.x3) {
-          mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);           // dS_hi K_hi
-          mma_tmem_smem(tmem + cdQ, cS, skt + ktile, D, BT, true);  // dS_hi K_lo
-          mma_tmem_smem(tmem + cdQ, cG, skt, D, BT, true);          // dS_lo K_hi
-        } else {
-          mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
-        }
-        mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && kt + 1 < nkt)  // in order after the product reading S_0
-          ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+  } else if (warp == MMA_WARP) {
+    const uint8_t* st0 = sm + p.sm_stage0;
+    const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + 2 * dp;
+    bool ok = dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+    for (int kt = 0; kt < nkt && ok; ++kt) {
+      const int b = kt % nbuf, s = kt % NS;
+      if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+      if (!ok) break;
+      if (!mbar_wait_warp(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+      tc_fence_after();
+      const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
+      const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
+      const bool acc = kt > 0;
+      if (p.x3) {
+        mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);           // dS_hi K_hi
+        mma_tmem_smem(tmem + cdQ, cS, skt + ktile, D, BT, true);  // dS_hi K_lo
+        mma_tmem_smem(tmem + cdQ, cG, skt, D, BT, true);          // dS_lo K_hi
+      } else {
+        mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
       }
-      mma_commit(bar_done);
+      mma_commit(&bar_empty[s]);
+      if (nbuf == 1 && kt + 1 < nkt)  // in order after the product reading S_0
+        ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
     }
+    mma_commit(bar_done);
   } else {
     // ---- compute warps ----
-    group_sync(BAR_COMPUTE, NCOMP3);
+    group_sync(BAR_COMPUTE, NCOMP);
     Dg = 0.f;
 #pragma unroll
-    for (int q = 0; q < NCG3; ++q) Dg += xch[q * 128 + row];
+    for (int q = 0; q < NCG; ++q) Dg += xch[q * 128 + row];
     const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
     const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
     const float invWf = 1.0f / Wf;
@@ -272,7 +268,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       for (int k = 0; k < D; ++k) tie_max[k] = tie_min[k] = 0.f;
       atomicOr(p.tileflags + (size_t)bh * p.nqt + i / BT, 1);
     }
-    group_sync(BAR_COMPUTE, NCOMP3);  // every column group of a row may add to its tie sums
+    group_sync(BAR_COMPUTE, NCOMP);  // every column group of a row may add to its tie sums
     float own = 0.f, cm = 0.f;
     bool failed = false;
     for (int kt = 0; kt < nkt; ++kt) {
@@ -325,17 +321,17 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
     }
     const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP3, !dok);
+    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
     if (!failed) {
       tc_fence_after();
       xch[cg * 128 + row] = own;
-      xch[(NCG3 + cg) * 128 + row] = cm;
-      group_sync(BAR_COMPUTE, NCOMP3);
+      xch[(NCG + cg) * 128 + row] = cm;
+      group_sync(BAR_COMPUTE, NCOMP);
       float own_t = 0.f, cm_t = 0.f;
 #pragma unroll
-      for (int q = 0; q < NCG3; ++q) {
+      for (int q = 0; q < NCG; ++q) {
         own_t += xch[q * 128 + row];
-        cm_t += xch[(NCG3 + q) * 128 + row];
+        cm_t += xch[(NCG + q) * 128 + row];
       }
       // Eq. (full): c_m = sum gamma dw/dm; c_M = -sum gamma Delta - c_m (Delta + dw/dM + dw/dm = 0);
       // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys.
@@ -346,7 +342,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dq(const __grid_constant__ Map
       const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
       const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
       float* dst = p.dQ + rw * D;
-      for (int c = cg * (D / NCG3); c < (cg + 1) * (D / NCG3); c += 16) {
+      for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 16) {
         // the arg-extremum key rows first (all loads in flight before any store)
         float km[16], kn[16];
 #pragma unroll
@@ -468,7 +464,7 @@ __device__ __forceinline__ bool kv_issue_sg(const Params& p, int it, uint64_t* b
                                             const uint8_t* st0, uint32_t cKa, uint32_t cVa, uint32_t cSG,
                                             int qtile, bool needV, int oQ, int odO) {
   const int D = p.d, NS = p.nstage, s = it % NS, b = it % p.nbuf;
-  if (!mbar_wait_spin(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+  if (!mbar_wait_warp(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
   tc_fence_after();
   const uint8_t* st = st0 + s * p.sm_stage_bytes;
   const uint32_t cS = cSG + 128 * b, cG = cS + 64;
@@ -499,7 +495,7 @@ __device__ __forceinline__ bool kv_issue_sg(const Params& p, int it, uint64_t* b
 // and (MinMax) their grid pair tables; FWM's shared table at sm_table.
 // ---------------------------------------------------------------------------
 template <int CAL, int REC, bool FULLG>
-__global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int qtile = BT * D * 4;
@@ -511,7 +507,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   uint64_t* bar_pready = bars + 2 * NS + 2;
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, kb = blockIdx.x;
   const int dp = D * parts;
   const int cK = 0, cV = dp, base = needV ? 2 * dp : dp;
@@ -520,7 +516,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   const int oQ = 0, odO = parts * qtile, oQT = 2 * parts * qtile, odOT = 3 * parts * qtile;
   const int oRec = 4 * parts * qtile, oTab = oRec + BT * 64;
   const uint32_t tstride = (uint32_t)p.Kp * 8u;
-  constexpr int W = BT / NCG3;  // query columns per thread per tile
+  constexpr int W = BT / NCG;  // query columns per thread per tile
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -529,7 +525,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
-      mbar_init(&bar_pready[b], NCOMP3 / 32);
+      mbar_init(&bar_pready[b], NCOMP / 32);
     }
     mbar_init(bar_done, 1);
     fence_mbar_init();
@@ -542,10 +538,10 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-  const int row = tid & 127, cg = (tid >> 7) & (NCG3 - 1);
+  const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
   const int j = kb * 128 + row;
   const bool key_ok = j < p.T;
-  if (warp < NCOMP3 / 32) {
+  if (warp < NCOMP / 32) {
     // operand rows into TMEM: column group 0 takes K, group 1 takes V
     if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
     else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
@@ -557,70 +553,66 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
   __syncthreads();
   tc_fence_after();
 
-  if (warp == PRODUCER_WARP3) {
-    if ((tid & 31) == 0) {
-      for (int it = 0; it < nit; ++it) {
-        const int s = it % NS, q0 = (qt0 + it) * BT;
-        if (it >= NS &&
-            !mbar_wait_spin(&bar_empty[s], ((it / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-          break;
-        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        uint64_t* b = &bar_full[s];
-        const int nrows = min(BT, p.T - q0);
-        const int ntiles = 1 + (needV ? 1 : 0) + (doDK ? 1 : 0) + (doDV ? 1 : 0);
-        uint32_t bytes = ntiles * parts * qtile + nrows * 64;
-        if (CAL == CAL_MINMAX) bytes += nrows * tstride;
-        mbar_arrive_expect_tx(b, bytes);
-        load_rows_tile(dst + oQ, &maps.q, b, D, BT, 0, q0, bh);
-        if (p.x3) load_rows_tile(dst + oQ + qtile, &maps.q_lo, b, D, BT, 0, q0, bh);
-        if (needV) {
-          load_rows_tile(dst + odO, &maps.dout, b, D, BT, 0, q0, bh);
-          if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BT, 0, q0, bh);
-        }
-        if (doDK) {
-          load_rows_tile(dst + oQT, &maps.qt, b, BT, D, q0, 0, bh);
-          if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BT, D, q0, 0, bh);
-        }
-        if (doDV) {
-          load_rows_tile(dst + odOT, &maps.dot, b, BT, D, q0, 0, bh);
-          if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BT, D, q0, 0, bh);
-        }
-        const size_t r0 = (size_t)bh * p.T + q0;
-        bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
-        if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
+  if (warp == PRODUCER_WARP) {
+    for (int it = 0; it < nit; ++it) {
+      const int s = it % NS, q0 = (qt0 + it) * BT;
+      if (it >= NS &&
+          !mbar_wait_warp(&bar_empty[s], ((it / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+        break;
+      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      uint64_t* b = &bar_full[s];
+      const int nrows = min(BT, p.T - q0);
+      const int ntiles = 1 + (needV ? 1 : 0) + (doDK ? 1 : 0) + (doDV ? 1 : 0);
+      uint32_t bytes = ntiles * parts * qtile + nrows * 64;
+      if (CAL == CAL_MINMAX) bytes += nrows * tstride;
+      mbar_arrive_expect_tx(b, bytes);
+      load_rows_tile(dst + oQ, &maps.q, b, D, BT, 0, q0, bh);
+      if (p.x3) load_rows_tile(dst + oQ + qtile, &maps.q_lo, b, D, BT, 0, q0, bh);
+      if (needV) {
+        load_rows_tile(dst + odO, &maps.dout, b, D, BT, 0, q0, bh);
+        if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BT, 0, q0, bh);
       }
-    }
-  } else if (warp == MMA_WARP3) {
-    if ((tid & 31) == 0) {
-      const uint8_t* st0 = sm + p.sm_stage0;
-      const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;
-      bool ok = kv_issue_sg(p, 0, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
-      for (int it = 0; it < nit && ok; ++it) {
-        const int b = it % nbuf, s = it % NS;
-        if (nbuf == 2 && it + 1 < nit)
-          ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
-        if (!ok) break;
-        if (!mbar_wait_spin(&bar_pready[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-        tc_fence_after();
-        const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
-        const bool acc = it > 0;
-        if (p.x3) {
-          const uint32_t cacc = tmem + (doDV ? cdV : cdK);
-          const uint8_t* bt = st + (doDV ? odOT : oQT);
-          mma_tmem_smem(cacc, cS, bt, D, BT, acc);
-          mma_tmem_smem(cacc, cS, bt + qtile, D, BT, true);
-          mma_tmem_smem(cacc, cG, bt, D, BT, true);
-        } else {
-          if (doDV) mma_tmem_smem(tmem + cdV, cS, st + odOT, D, BT, acc);
-          if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
-        }
-        mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && it + 1 < nit)
-          ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+      if (doDK) {
+        load_rows_tile(dst + oQT, &maps.qt, b, BT, D, q0, 0, bh);
+        if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BT, D, q0, 0, bh);
       }
-      mma_commit(bar_done);
+      if (doDV) {
+        load_rows_tile(dst + odOT, &maps.dot, b, BT, D, q0, 0, bh);
+        if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BT, D, q0, 0, bh);
+      }
+      const size_t r0 = (size_t)bh * p.T + q0;
+      bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
+      if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
     }
+  } else if (warp == MMA_WARP) {
+    const uint8_t* st0 = sm + p.sm_stage0;
+    const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;
+    bool ok = kv_issue_sg(p, 0, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+    for (int it = 0; it < nit && ok; ++it) {
+      const int b = it % nbuf, s = it % NS;
+      if (nbuf == 2 && it + 1 < nit)
+        ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+      if (!ok) break;
+      if (!mbar_wait_warp(&bar_pready[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+      tc_fence_after();
+      const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
+      const bool acc = it > 0;
+      if (p.x3) {
+        const uint32_t cacc = tmem + (doDV ? cdV : cdK);
+        const uint8_t* bt = st + (doDV ? odOT : oQT);
+        mma_tmem_smem(cacc, cS, bt, D, BT, acc);
+        mma_tmem_smem(cacc, cS, bt + qtile, D, BT, true);
+        mma_tmem_smem(cacc, cG, bt, D, BT, true);
+      } else {
+        if (doDV) mma_tmem_smem(tmem + cdV, cS, st + odOT, D, BT, acc);
+        if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
+      }
+      mma_commit(&bar_empty[s]);
+      if (nbuf == 1 && it + 1 < nit)
+        ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+    }
+    mma_commit(bar_done);
   } else {
     const float Kf = (float)Kq;
     const uint32_t fwtab = smem_u32(sm + p.sm_table) - 0x58000000u;
@@ -690,7 +682,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
       if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
     }
     const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP3, !dok);
+    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
     if (!failed) {
       tc_fence_after();
       const size_t krow = (size_t)bh * p.T + (key_ok ? j : 0);
@@ -699,7 +691,7 @@ __global__ void __launch_bounds__(NTHR3, 1) k_bwd_dkdv(const __grid_constant__ M
         const int col = pass == 0 ? cdV : cdK;
         const float mul = pass == 0 ? 1.0f : p.scale;
         float* dst = (pass == 0 ? p.dV : p.dK) + krow * D;
-        for (int c = cg * (D / NCG3); c < (cg + 1) * (D / NCG3); c += 16) {
+        for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 16) {
           float v[16];
           tmem_ld16(lane_addr(tmem, col + c), v);
           tmem_ld_wait();
@@ -723,7 +715,7 @@ template <class K>
 static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<grid, NTHR3, smem_bytes, s>>>(maps, p);
+  kern<<<grid, NTHR, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
 }
 

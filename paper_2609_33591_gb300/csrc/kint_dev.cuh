@@ -40,23 +40,16 @@ __device__ __forceinline__ bool group_any(int id, int n, bool pred) {
 }
 
 // Thread roles of the warp-specialised kernels: NCG column groups of 128
-// compute threads (thread t owns TMEM lane t % 128, columns by group t / 128;
-// thread 0 also issues the tensor-core instructions) and one TMA producer warp.
+// compute threads (warps [0, 4 NCG); thread t owns TMEM lane t % 128 and the
+// column group t / 128 of every score tile), then one MMA warp and one TMA
+// producer warp.  The compute warps meet no CTA-wide barrier inside the tile
+// loops: tiles change hands through mbarriers only.
 constexpr int NCG = 2;
 constexpr int NCOMP = 128 * NCG;
-constexpr int NTHR = NCOMP + 32;
-constexpr int PRODUCER_WARP = NCOMP / 32;
+constexpr int NTHR = NCOMP + 64;
+constexpr int MMA_WARP = NCOMP / 32;
+constexpr int PRODUCER_WARP = NCOMP / 32 + 1;
 constexpr int BAR_COMPUTE = 1;  // named barrier id of the compute group
-
-// Kernels with a dedicated MMA warp: NCG3 column groups of 128 compute threads
-// (warps [0, 4 NCG3)), then the MMA warp and the producer warp.  The compute
-// warps meet no CTA-wide barrier inside the tile loop; they hand tiles to the
-// MMA warp through mbarriers.
-constexpr int NCG3 = 2;
-constexpr int NCOMP3 = 128 * NCG3;
-constexpr int NTHR3 = NCOMP3 + 64;
-constexpr int MMA_WARP3 = NCOMP3 / 32;
-constexpr int PRODUCER_WARP3 = NCOMP3 / 32 + 1;
 
 // W-column TMEM row access (W = 16 or 32).
 template <int W>

@@ -58,14 +58,82 @@ cudaError_t launch_prep(const float* X, float* nat_hi, float* nat_lo, float* tr_
 // ---------------------------------------------------------------------------
 // Pass 1: row extrema (App. A: M = max_j s_j, m = min_j s_j over valid keys,
 // lowest index among ties and the tie counts of Table "Edge cases").
-// CTA = one 128-row query block of one head.  Threads [0, NCOMP) compute:
-// thread t owns query row qb*128 + t%128 (TMEM lane t%128) and the column half
-// t/128 of every 128-key score tile S = Q K^T.  Thread 0 issues the MMAs; the
-// last warp streams K tiles through an nstage-deep TMA ring.  S is
-// double-buffered in TMEM (columns [0,128) and [128,256)), so the product of
-// key tile kb+1 runs while tile kb is reduced.
+// CTA = one 128-row query block of one head.  Compute thread t owns query row
+// qb*128 + t%128 (TMEM lane t%128) and the column half t/128 of every 128-key
+// score tile S = Q K^T.  The MMA warp computes S into two TMEM buffers
+// (columns [0,128) and [128,256)), so the product of tile kb+1 runs while tile
+// kb is reduced; the producer warp streams K tiles through a TMA ring.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
+
+// One 32-key chunk: chunk extrema by a max/min tree, then (warp-uniform branch,
+// taken while a lane's running extremum can still move) the lanes whose chunk
+// reaches their running extremum count the chunk's equal keys with a bit mask;
+// its lowest set bit is the lowest index.  Masked keys (j > i) take -inf / +inf.
+template <bool DIAG>
+__device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float scale, float& M, float& m,
+                                            int& amax, int& amin, int& nmax, int& nmin) {
+  float hi[16], lo[16];
+#pragma unroll
+  for (int jj = 0; jj < 32; ++jj) v[jj] = __fmul_rn(v[jj], scale);
+#pragma unroll
+  for (int jj = 0; jj < 16; ++jj) {
+    float a = v[jj], b = v[jj + 16], a2 = a, b2 = b;
+    if constexpr (DIAG) {
+      const bool oa = j0 + jj <= i, ob = j0 + jj + 16 <= i;
+      a = oa ? a : -INFINITY;
+      b = ob ? b : -INFINITY;
+      a2 = oa ? a2 : INFINITY;
+      b2 = ob ? b2 : INFINITY;
+    }
+    hi[jj] = fmaxf(a, b);
+    lo[jj] = fminf(a2, b2);
+  }
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+    for (int jj = 0; jj < w; ++jj) {
+      hi[jj] = fmaxf(hi[jj], hi[jj + w]);
+      lo[jj] = fminf(lo[jj], lo[jj + w]);
+    }
+  const float cmax = hi[0], cmin = lo[0];
+  const bool um = cmax >= M, un = cmin <= m;
+  if (__any_sync(0xffffffffu, um)) {
+    uint32_t mk = 0;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+      const bool e = (v[jj] == cmax) && (!DIAG || j0 + jj <= i);
+      mk |= e ? (1u << jj) : 0u;
+    }
+    if (um) {
+      if (cmax > M) {
+        M = cmax;
+        amax = j0 + __ffs(mk) - 1;
+        nmax = __popc(mk);
+      } else {
+        nmax += __popc(mk);
+      }
+    }
+  }
+  if (__any_sync(0xffffffffu, un)) {
+    uint32_t mk = 0;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+      const bool e = (v[jj] == cmin) && (!DIAG || j0 + jj <= i);
+      mk |= e ? (1u << jj) : 0u;
+    }
+    if (un) {
+      if (cmin < m) {
+        m = cmin;
+        amin = j0 + __ffs(mk) - 1;
+        nmin = __popc(mk);
+      } else {
+        nmin += __popc(mk);
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, tile = D * 512, parts = p.x3 ? 2 : 1, NS = p.nstage;
   uint8_t* sQ = sm + p.sm_a;
@@ -73,10 +141,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ M
   uint64_t* bar_q = bars;
   uint64_t* bar_full = bars + 1;
   uint64_t* bar_empty = bars + 1 + NS;
-  uint64_t* bar_s = bars + 1 + 2 * NS;  // [2]
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 + 2 * NS);
+  uint64_t* bar_s = bars + 1 + 2 * NS;      // [2] S_b computed
+  uint64_t* bar_sfree = bars + 3 + 2 * NS;  // [2] S_b read by every compute warp
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 5 + 2 * NS);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [6][128], aliases Q once all products are done
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
   const int nkb = qb + 1;
 
@@ -86,8 +155,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ M
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_empty[s], 1);
     }
-    mbar_init(&bar_s[0], 1);
-    mbar_init(&bar_s[1], 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bar_s[b], 1);
+      mbar_init(&bar_sfree[b], NCOMP / 32);
+    }
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -100,32 +171,29 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ M
   const uint32_t tmem = *tslot;
 
   if (warp == PRODUCER_WARP) {
-    if ((tid & 31) == 0) {
-      mbar_arrive_expect_tx(bar_q, parts * tile);
-      load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
-      if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-      for (int kb = 0; kb < nkb; ++kb) {
-        const int s = kb % NS;
-        if (kb >= NS &&
-            !mbar_wait(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-          break;
-        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        mbar_arrive_expect_tx(&bar_full[s], parts * tile);
-        load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
-        if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
-      }
-    }
-  } else {
-    const int row = tid & 127, cg = tid >> 7;
-    const int i = qb * 128 + row;
-    // Thread 0: wait for key tile kb, issue S[kb & 1] = Q K_kb^T, release the stage.
-    auto issue_s = [&](int kb) {
-      if (kb == 0 && !mbar_wait(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
+    mbar_arrive_expect_tx(bar_q, parts * tile);
+    load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
+    if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
+    for (int kb = 0; kb < nkb; ++kb) {
       const int s = kb % NS;
-      if (!mbar_wait(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
+      if (kb >= NS && !mbar_wait_warp(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+        break;
+      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      mbar_arrive_expect_tx(&bar_full[s], parts * tile);
+      load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
+      if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
+    }
+  } else if (warp == MMA_WARP) {
+    bool ok = mbar_wait_warp(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+    for (int kb = 0; kb < nkb && ok; ++kb) {
+      const int s = kb % NS, b = kb & 1;
+      // S_b was last read in tile kb - 2
+      if (kb >= 2 && !mbar_wait_warp(&bar_sfree[b], ((kb >> 1) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC))
+        break;
+      if (!mbar_wait_warp(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) break;
       tc_fence_after();
       const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      const uint32_t dcol = tmem + (kb & 1) * 128;
+      const uint32_t dcol = tmem + b * 128;
       if (p.x3) {
         mma_smem_smem(dcol, sQ + tile, sk, 128, D, false);  // Q_lo K_hi
         mma_smem_smem(dcol, sQ, sk + tile, 128, D, true);   // Q_hi K_lo
@@ -133,18 +201,18 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ M
       } else {
         mma_smem_smem(dcol, sQ, sk, 128, D, false);
       }
-      mma_commit(&bar_s[kb & 1]);
+      mma_commit(&bar_s[b]);
       mma_commit(&bar_empty[s]);
-    };
-    if (tid == 0) issue_s(0);
-
+    }
+  } else {
+    const int row = tid & 127, cg = tid >> 7;
+    const int i = qb * 128 + row;
     float M = -FLT_MAX, m = FLT_MAX;
     int amax = 0, amin = 0, nmax = 0, nmin = 0;
     bool failed = false;
     for (int kb = 0; kb < nkb; ++kb) {
-      if (tid == 0 && kb + 1 < nkb) issue_s(kb + 1);  // S[(kb+1)&1] was last read in iteration kb-1
-      const bool ok = mbar_wait(&bar_s[kb & 1], (kb >> 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-      if (group_any(BAR_COMPUTE, NCOMP, !ok)) {
+      const int b = kb & 1;
+      if (!mbar_wait(&bar_s[b], (kb >> 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
         failed = true;
         break;
       }
@@ -154,43 +222,19 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ M
       for (int cc = 0; cc < 2; ++cc) {
         const int c = cg * 2 + cc;
         float v[32];
-        tmem_ld32(lane_addr(tmem, (kb & 1) * 128 + c * 32), v);
+        tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
         tmem_ld_wait();
         const int j0 = kb * 128 + c * 32;
-        float cmax = -FLT_MAX, cmin = FLT_MAX;
-#pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-          const float sc = __fmul_rn(v[jj], p.scale);
-          v[jj] = sc;
-          const bool okj = !diag || (j0 + jj <= i);
-          cmax = fmaxf(cmax, okj ? sc : -FLT_MAX);
-          cmin = fminf(cmin, okj ? sc : FLT_MAX);
-        }
-        if (cmax >= M || cmin <= m) {  // rare after the first chunks: exact scan with indices and ties
-          for (int jj = 0; jj < 32; ++jj) {
-            const int j = j0 + jj;
-            if (diag && j > i) break;
-            const float sc = v[jj];
-            if (sc > M) {
-              M = sc;
-              amax = j;
-              nmax = 1;
-            } else if (sc == M) {
-              ++nmax;
-            }
-            if (sc < m) {
-              m = sc;
-              amin = j;
-              nmin = 1;
-            } else if (sc == m) {
-              ++nmin;
-            }
-          }
-        }
+        if (diag)
+          stats_chunk<true>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+        else
+          stats_chunk<false>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
       }
       tc_fence_before();
-      group_sync(BAR_COMPUTE, NCOMP);
+      __syncwarp();
+      if ((tid & 31) == 0) mbar_arrive(&bar_sfree[b]);
     }
+    failed = group_any(BAR_COMPUTE, NCOMP, failed);
     if (!failed) {
       // combine the two column halves of each row
       if (cg == 1) {
@@ -229,8 +273,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_stats(const __grid_constant__ M
         p.n_min[rw] = nmin;
       }
     }
-    tc_fence_before();
   }
+  tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 256);
 }
@@ -331,6 +375,26 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
 // smem: Q (hi[, lo]) at sm_a; stages {K tile, V^T tile} (hi[, lo] each) fed by
 // the producer warp; per-row pair tables (e_r, e_{r+1}) [K][128] at sm_table.
 // ---------------------------------------------------------------------------
+// MMA warp of k_fwd_main: wait for K/V stage of tile kb, S_b = Q K_kb^T into
+// score buffer b = kb % nbuf, commit to bar_s[b].
+__device__ __forceinline__ bool main_issue_s(const Params& p, int kb, uint64_t* bar_full, uint64_t* bar_s,
+                                             const uint8_t* st0, const uint8_t* sQ, uint32_t tmem, int qtile) {
+  const int NS = p.nstage, s = kb % NS, b = kb % p.nbuf, D = p.d;
+  if (!mbar_wait_warp(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+  tc_fence_after();
+  const uint8_t* sk = st0 + s * p.sm_stage_bytes;
+  const uint32_t dcol = tmem + b * 128;
+  if (p.x3) {
+    mma_smem_smem(dcol, sQ + qtile, sk, 128, D, false);  // Q_lo K_hi
+    mma_smem_smem(dcol, sQ, sk + qtile, 128, D, true);   // Q_hi K_lo
+    mma_smem_smem(dcol, sQ, sk, 128, D, true);           // Q_hi K_hi
+  } else {
+    mma_smem_smem(dcol, sQ, sk, 128, D, false);
+  }
+  mma_commit(&bar_s[b]);
+  return true;
+}
+
 template <int CAL, int REC, int MODE>
 __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
@@ -341,11 +405,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   uint64_t* bar_q = bars;
   uint64_t* bar_full = bars + 1;
   uint64_t* bar_empty = bars + 1 + NS;
-  uint64_t* bar_s = bars + 1 + 2 * NS;  // [2]
-  uint64_t* bar_pv = bars + 3 + 2 * NS;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4 + 2 * NS);
+  uint64_t* bar_s = bars + 1 + 2 * NS;       // [2] S_b computed
+  uint64_t* bar_pready = bars + 3 + 2 * NS;  // [2] weights of buffer b stored by every compute warp
+  uint64_t* bar_pv = bars + 5 + 2 * NS;      // P V of a tile complete
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 6 + 2 * NS);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [4][128], aliases Q once all products are done
-  const int tid = threadIdx.x, warp = tid >> 5;
+  const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
   const int nkb = qb + 1;
   const bool useA2 = (MODE == 1) || p.x3;
@@ -357,8 +422,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_empty[s], 1);
     }
-    mbar_init(&bar_s[0], 1);
-    mbar_init(&bar_s[1], 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bar_s[b], 1);
+      mbar_init(&bar_pready[b], NCOMP / 32);
+    }
     mbar_init(bar_pv, 1);
     fence_mbar_init();
   }
@@ -372,24 +439,47 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   const uint32_t tmem = *tslot;
 
   if (warp == PRODUCER_WARP) {
-    if ((tid & 31) == 0) {
-      mbar_arrive_expect_tx(bar_q, parts * qtile);
-      load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
-      if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-      for (int kb = 0; kb < nkb; ++kb) {
-        const int s = kb % NS;
-        if (kb >= NS &&
-            !mbar_wait(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-          break;
-        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-        mbar_arrive_expect_tx(&bar_full[s], parts * (qtile + vtile));
-        load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
-        load_rows_tile(dst + parts * qtile, &maps.vt, &bar_full[s], 128, D, kb * 128, 0, bh);
-        if (p.x3) {
-          load_rows_tile(dst + qtile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
-          load_rows_tile(dst + parts * qtile + vtile, &maps.vt_lo, &bar_full[s], 128, D, kb * 128, 0, bh);
-        }
+    mbar_arrive_expect_tx(bar_q, parts * qtile);
+    load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
+    if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
+    for (int kb = 0; kb < nkb; ++kb) {
+      const int s = kb % NS;
+      if (kb >= NS && !mbar_wait_warp(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+        break;
+      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+      mbar_arrive_expect_tx(&bar_full[s], parts * (qtile + vtile));
+      load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
+      load_rows_tile(dst + parts * qtile, &maps.vt, &bar_full[s], 128, D, kb * 128, 0, bh);
+      if (p.x3) {
+        load_rows_tile(dst + qtile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
+        load_rows_tile(dst + parts * qtile + vtile, &maps.vt_lo, &bar_full[s], 128, D, kb * 128, 0, bh);
       }
+    }
+  } else if (warp == MMA_WARP) {
+    const uint8_t* st0 = sm + p.sm_stage0;
+    bool ok = mbar_wait_warp(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) &&
+              main_issue_s(p, 0, bar_full, bar_s, st0, sQ, tmem, qtile);
+    for (int kb = 0; kb < nkb && ok; ++kb) {
+      const int b = kb % nbuf, s = kb % NS;
+      // S(kb+1) goes to the other buffer, whose last reader P V(kb-1) precedes it in issue order
+      if (nbuf == 2 && kb + 1 < nkb && !main_issue_s(p, kb + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+      if (!mbar_wait_warp(&bar_pready[b], (kb / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+      tc_fence_after();
+      const uint8_t* vt = st0 + s * p.sm_stage_bytes + parts * qtile;
+      const bool acc = kb > 0;
+      const uint32_t a = tmem + b * 128;
+      if (p.x3) {
+        mma_tmem_smem(tmem + cO, tmem + cA2, vt, D, 128, acc);  // A_lo V_hi (frees A2 first)
+        mma_tmem_smem(tmem + cO, a, vt + vtile, D, 128, true);   // A_hi V_lo
+        mma_tmem_smem(tmem + cO, a, vt, D, 128, true);           // A_hi V_hi
+      } else {
+        if (MODE == 1) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);  // frees A2 first
+        mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);
+      }
+      mma_commit(bar_pv);
+      mma_commit(&bar_empty[s]);
+      // one buffer: S(kb+1) overwrites the weights P V(kb) reads, in issue order after it
+      if (nbuf == 1 && kb + 1 < nkb && !main_issue_s(p, kb + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
     }
   } else {
     const int row = tid & 127, cg = tid >> 7;
@@ -420,38 +510,16 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     }
     group_sync(BAR_COMPUTE, NCOMP);
 
-    auto issue_s = [&](int kb) {
-      if (kb == 0 && !mbar_wait(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
-      const int s = kb % NS;
-      if (!mbar_wait(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return;
-      tc_fence_after();
-      const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      const uint32_t dcol = tmem + (kb % nbuf) * 128;
-      if (p.x3) {
-        mma_smem_smem(dcol, sQ + qtile, sk, 128, D, false);
-        mma_smem_smem(dcol, sQ, sk + qtile, 128, D, true);
-        mma_smem_smem(dcol, sQ, sk, 128, D, true);
-      } else {
-        mma_smem_smem(dcol, sQ, sk, 128, D, false);
-      }
-      mma_commit(&bar_s[kb % nbuf]);
-    };
-    if (tid == 0) issue_s(0);
-
     float Wm = 0.f, Wl = 0.f;
     bool failed = false;
-    for (int kb = 0; kb < nkb; ++kb) {
-      if (nbuf == 2 && tid == 0 && kb + 1 < nkb) issue_s(kb + 1);
+    for (int kb = 0; kb < nkb && !failed; ++kb) {
       const int b = kb % nbuf;
-      const uint32_t sparity = (nbuf == 2) ? ((kb >> 1) & 1) : (kb & 1);
-      bool ok = mbar_wait(&bar_s[b], sparity, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-      if (group_any(BAR_COMPUTE, NCOMP, !ok)) {
+      if (!mbar_wait(&bar_s[b], (kb / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
         failed = true;
         break;
       }
       tc_fence_after();
       const bool diag = kb == qb;
-      bool pv_ok = true;
 #pragma unroll 1
       for (int cc = 0; cc < 2; ++cc) {
         const int c = cg * 2 + cc;
@@ -472,40 +540,23 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
             a1[q] = h;
           }
         }
-        // A2 is still the operand of the previous tile's products until they complete
-        if (cc == 0 && useA2 && kb > 0)
-          pv_ok = mbar_wait(bar_pv, (kb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+        // A2 is still an operand of the previous tile's products until they complete
+        if (cc == 0 && useA2 && kb > 0 &&
+            !mbar_wait(bar_pv, (kb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
+          failed = true;
+          break;
+        }
         tmem_st32(lane_addr(tmem, b * 128 + c * 32), a1);
         if (useA2) tmem_st32(lane_addr(tmem, cA2 + c * 32), a2);
       }
+      if (failed) break;
       tmem_st_wait();
       tc_fence_before();
-      if (group_any(BAR_COMPUTE, NCOMP, !pv_ok)) {
-        failed = true;
-        break;
-      }
-      if (tid == 0) {
-        tc_fence_after();
-        const uint8_t* vt = sm + p.sm_stage0 + (kb % NS) * p.sm_stage_bytes + parts * qtile;
-        const bool acc = kb > 0;
-        const uint32_t a = tmem + b * 128;
-        if (p.x3) {
-          mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);                // A_hi V_hi
-          mma_tmem_smem(tmem + cO, a, vt + vtile, D, 128, true);       // A_hi V_lo
-          mma_tmem_smem(tmem + cO, tmem + cA2, vt, D, 128, true);      // A_lo V_hi
-        } else {
-          mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);
-          if (MODE == 1) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);
-        }
-        mma_commit(bar_pv);
-        mma_commit(&bar_empty[kb % NS]);
-        if (nbuf == 1 && kb + 1 < nkb) issue_s(kb + 1);  // in-order after the products that read S_0
-      }
+      __syncwarp();
+      if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
     }
-    if (!failed) {
-      const bool ok = mbar_wait(bar_pv, (nkb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-      failed = group_any(BAR_COMPUTE, NCOMP, !ok);
-    }
+    if (!failed) failed = !mbar_wait(bar_pv, (nkb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+    failed = group_any(BAR_COMPUTE, NCOMP, failed);
     if (!failed) {
       tc_fence_after();
       xch[cg * 128 + row] = Wm;
@@ -550,8 +601,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
         }
       }
     }
-    tc_fence_before();
   }
+  tc_fence_before();
   __syncthreads();
   if (warp == 0) tmem_dealloc(tmem, 512);
 }
