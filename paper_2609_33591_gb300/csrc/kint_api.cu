@@ -245,7 +245,7 @@ int plan_dq(Params& p) {
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
-    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 5), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 6), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       return total;
@@ -266,7 +266,7 @@ int plan_dkdv(Params& p, int sel) {
   p.sm_stage_bytes = 4 * parts * qtile + 64 * 64 + (p.calib == KINT_CALIB_MINMAX ? 64 * p.Kp * 8 : 0);
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    const int total = std::max(finish_plan(p, p.sm_table + 1024, 2 * p.nstage + 5), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_table + 1024, 2 * p.nstage + 6), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       return total;

@@ -120,7 +120,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   uint64_t* bar_sfull = bars + 2 * NS;     // [2]
   uint64_t* bar_pready = bars + 2 * NS + 2;  // [2]
   uint64_t* bar_done = bars + 2 * NS + 4;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
+  uint64_t* bar_ops = bars + 2 * NS + 5;  // Q / dO rows stored in TMEM by every compute warp
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 6);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
@@ -139,6 +140,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       mbar_init(&bar_pready[b], NCOMP / 32);
     }
     mbar_init(bar_done, 1);
+    mbar_init(bar_ops, NCOMP / 32);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -159,9 +161,28 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   int nmax = 1, nmin = 1, amax = 0, amin = 0;
   RowGrid g{};
   if (warp < NCOMP / 32) {
-    // operand rows into TMEM: column group 0 takes Q, group 1 takes dO
+    // operand rows into TMEM (column group 0 takes Q, group 1 takes dO), handed to
+    // the MMA warp through bar_ops; the rest of the set-up runs under the first products
     row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
                 p.x3 != 0);
+    tmem_st_wait();
+    tc_fence_before();
+    __syncwarp();
+    if ((tid & 31) == 0) mbar_arrive(bar_ops);
+    // <g>_{P*} = dO_i . O*_i, each column group takes its share of the d columns (all loads first)
+    constexpr int kMaxQ = 128 / (4 * NCG);
+    const int nq = D / (4 * NCG);
+    float4 xa[kMaxQ], ya[kMaxQ];
+    {
+      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * nq;
+      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * nq;
+#pragma unroll
+      for (int q = 0; q < kMaxQ; ++q) {
+        const bool in = row_ok && q < nq;
+        xa[q] = in ? __ldg(a + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+        ya[q] = in ? __ldg(b + q) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
     if (row_ok) {
       M = p.row_max[rw];
       m = p.row_min[rw];
@@ -171,23 +192,18 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       amax = p.arg_max[rw];
       amin = p.arg_min[rw];
     }
-    g = row_grid(p, M, m);
     const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
     Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
-    // <g>_{P*} = dO_i . O*_i, each column group takes its share of the d columns
     float acc = 0.f;
-    if (row_ok) {
-      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * (D / (4 * NCG));
-      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * (D / (4 * NCG));
-      for (int q = 0; q < D / (4 * NCG); ++q) {
-        const float4 x = __ldg(a + q), y = __ldg(b + q);
-        acc = __fmaf_rn(x.x, y.x, acc);
-        acc = __fmaf_rn(x.y, y.y, acc);
-        acc = __fmaf_rn(x.z, y.z, acc);
-        acc = __fmaf_rn(x.w, y.w, acc);
-      }
+#pragma unroll
+    for (int q = 0; q < kMaxQ; ++q) {
+      acc = __fmaf_rn(xa[q].x, ya[q].x, acc);
+      acc = __fmaf_rn(xa[q].y, ya[q].y, acc);
+      acc = __fmaf_rn(xa[q].z, ya[q].z, acc);
+      acc = __fmaf_rn(xa[q].w, ya[q].w, acc);
     }
     xch[cg * 128 + row] = acc;
+    g = row_grid(p, M, m);
     if constexpr (CAL == CAL_FWM) {
       if (tid < Kq)
         *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
@@ -198,11 +214,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
       }
     }
-    tmem_st_wait();
   }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
 
   if (warp == PRODUCER_WARP) {
     for (int kt = 0; kt < nkt; ++kt) {
@@ -225,7 +237,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + 2 * dp;
-    bool ok = dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+    bool ok = mbar_wait_warp(bar_ops, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
+    if (ok) tc_fence_after();
+    ok = ok && dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
     for (int kt = 0; kt < nkt && ok; ++kt) {
       const int b = kt % nbuf, s = kt % NS;
       if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
@@ -342,27 +356,29 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
       const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
       float* dst = p.dQ + rw * D;
-      for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 16) {
+      for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
         // the arg-extremum key rows first (all loads in flight before any store)
-        float km[16], kn[16];
+        float4 km[8], kn[8];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float4 a = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
-                                            : make_float4(0.f, 0.f, 0.f, 0.f);
-          const float4 b2 = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
-                                                       : make_float4(0.f, 0.f, 0.f, 0.f);
-          km[4 * q] = a.x; km[4 * q + 1] = a.y; km[4 * q + 2] = a.z; km[4 * q + 3] = a.w;
-          kn[4 * q] = b2.x; kn[4 * q + 1] = b2.y; kn[4 * q + 2] = b2.z; kn[4 * q + 3] = b2.w;
+        for (int q = 0; q < 8; ++q) {
+          km[q] = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+          kn[q] = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
+                                             : make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        float v[16];
-        tmem_ld16(lane_addr(tmem, cdQ + c), v);
+        float v[32];
+        tmem_ld32(lane_addr(tmem, cdQ + c), v);
         tmem_ld_wait();
         if (row_ok) {
 #pragma unroll
-          for (int q = 0; q < 16; ++q) v[q] = __fmaf_rn(cmn, kn[q], __fmaf_rn(cMn, km[q], v[q])) * p.scale;
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            reinterpret_cast<float4*>(dst + c)[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          for (int q = 0; q < 8; ++q) {
+            float4 o;
+            o.x = __fmaf_rn(cmn, kn[q].x, __fmaf_rn(cMn, km[q].x, v[4 * q])) * p.scale;
+            o.y = __fmaf_rn(cmn, kn[q].y, __fmaf_rn(cMn, km[q].y, v[4 * q + 1])) * p.scale;
+            o.z = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
+            o.w = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
+            reinterpret_cast<float4*>(dst + c)[q] = o;
+          }
         }
       }
       if (row_ok && cg == 0) {
@@ -506,7 +522,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   uint64_t* bar_sfull = bars + 2 * NS;
   uint64_t* bar_pready = bars + 2 * NS + 2;
   uint64_t* bar_done = bars + 2 * NS + 4;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 5);
+  uint64_t* bar_ops = bars + 2 * NS + 5;  // K / V rows stored in TMEM by every compute warp
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 6);
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, kb = blockIdx.x;
   const int dp = D * parts;
@@ -517,6 +534,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   const int oRec = 4 * parts * qtile, oTab = oRec + BT * 64;
   const uint32_t tstride = (uint32_t)p.Kp * 8u;
   constexpr int W = BT / NCG;  // query columns per thread per tile
+  constexpr int WS = 16;       // columns per register chunk
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -528,6 +546,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
       mbar_init(&bar_pready[b], NCOMP / 32);
     }
     mbar_init(bar_done, 1);
+    mbar_init(bar_ops, NCOMP / 32);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -545,13 +564,13 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     // operand rows into TMEM: column group 0 takes K, group 1 takes V
     if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
     else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    tmem_st_wait();
+    tc_fence_before();
+    __syncwarp();
+    if ((tid & 31) == 0) mbar_arrive(bar_ops);
     if (CAL == CAL_FWM && tid < Kq)
       *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
-    tmem_st_wait();
   }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
 
   if (warp == PRODUCER_WARP) {
     for (int it = 0; it < nit; ++it) {
@@ -587,7 +606,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;
-    bool ok = kv_issue_sg(p, 0, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+    bool ok = mbar_wait_warp(bar_ops, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
+    if (ok) tc_fence_after();
+    ok = ok && kv_issue_sg(p, 0, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
     for (int it = 0; it < nit && ok; ++it) {
       const int b = it % nbuf, s = it % NS;
       if (nbuf == 2 && it + 1 < nit)
@@ -616,8 +637,14 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   } else {
     const float Kf = (float)Kq;
     const uint32_t fwtab = smem_u32(sm + p.sm_table) - 0x58000000u;
+    group_sync(BAR_COMPUTE, NCOMP);  // the FWM table
     bool failed = false;
+    const int* tflags = p.tileflags + (size_t)bh * p.nqt + qt0;
+    int tie_next = (FULLG && CAL != CAL_SOFTMAX) ? __ldg(tflags) : 0;
     for (int it = 0; it < nit; ++it) {
+      // the tie flag of this 64-row query tile, loaded one tile ahead
+      const int tie_here = tie_next;
+      if (FULLG && CAL != CAL_SOFTMAX && it + 1 < nit) tie_next = __ldg(tflags + it + 1);
       const int b = it % nbuf, s = it % NS;
       const int q0 = (qt0 + it) * BT, i0 = q0 + cg * W;
       const bool ok1 = mbar_wait(&bar_sfull[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
@@ -629,52 +656,57 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
       }
       tc_fence_after();
       const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      const uint32_t recs = smem_u32(st + oRec) + cg * W * 64;
-      const uint32_t tabs = smem_u32(st + oTab) + cg * W * tstride - 0x58000000u;
-      const int cS = base + 128 * b + cg * W, cG = cS + 64;
-      float sv[W], gv[W], pa[W], da[W];
-      tmem_ldw<W>(lane_addr(tmem, cS), sv);
-      if (needV) {
-        tmem_ldw<W>(lane_addr(tmem, cG), gv);
-      } else {
+      // two 16-column halves of the thread's W columns (bounds the live registers)
+#pragma unroll 1
+      for (int h = 0; h < W / WS; ++h) {
+        const int c0 = cg * W + h * WS, i0h = q0 + c0;
+        const uint32_t recs = smem_u32(st + oRec) + c0 * 64;
+        const uint32_t tabs = smem_u32(st + oTab) + c0 * tstride - 0x58000000u;
+        const int cS = base + 128 * b + c0, cG = cS + 64;
+        float sv[WS], gv[WS], pa[WS], da[WS];
+        tmem_ldw<WS>(lane_addr(tmem, cS), sv);
+        if (needV) {
+          tmem_ldw<WS>(lane_addr(tmem, cG), gv);
+        } else {
 #pragma unroll
-        for (int q = 0; q < W; ++q) gv[q] = 0.f;
-      }
-      tmem_ld_wait();
-      const bool masked = (i0 < kb * 128 + 128) || (i0 + W > p.T);
-      if (masked)
-        kv_chunk<CAL, REC, FULLG, true, W>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
-      else
-        kv_chunk<CAL, REC, FULLG, false, W>(sv, gv, pa, da, j, i0, p.T, recs, tabs, fwtab, tstride, Kf);
-      if constexpr (FULLG && CAL != CAL_SOFTMAX) {
-        // rows with tied extrema (flagged per 64-row tile by the dQ kernel): the tie set is
-        // found by equality on the recomputed scores
-        if (__ldg(p.tileflags + (size_t)bh * p.nqt + qt0 + it)) {
-          const int nr = min(W, p.T - i0);
+          for (int q = 0; q < WS; ++q) gv[q] = 0.f;
+        }
+        tmem_ld_wait();
+        const bool masked = (i0h < kb * 128 + 128) || (i0h + WS > p.T);
+        if (masked)
+          kv_chunk<CAL, REC, FULLG, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf);
+        else
+          kv_chunk<CAL, REC, FULLG, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf);
+        if constexpr (FULLG && CAL != CAL_SOFTMAX) {
+          // rows with tied extrema (flagged per 64-row tile by the dQ kernel): the tie set is
+          // found by equality on the recomputed scores
+          if (tie_here) {
+            const int nr = min(WS, p.T - i0h);
 #pragma unroll
-          for (int ii = 0; ii < W; ++ii) {
-            const RowRec& r = reinterpret_cast<const RowRec*>(st + oRec)[cg * W + ii];
-            const bool okr = ii < nr && i0 + ii >= j && (r.flags & (REC_TIEMAX | REC_TIEMIN)) &&
-                             !(r.flags & REC_NOGRID);
-            const float sc = __fmul_rn(sv[ii], p.scale);
-            if (okr && (r.flags & REC_TIEMAX) && sc == r.M) da[ii] += r.cMn;
-            if (CAL == CAL_MINMAX && okr && (r.flags & REC_TIEMIN) && sc == r.m) da[ii] += r.cmn;
+            for (int ii = 0; ii < WS; ++ii) {
+              const RowRec& r = reinterpret_cast<const RowRec*>(st + oRec)[c0 + ii];
+              const bool okr = ii < nr && i0h + ii >= j && (r.flags & (REC_TIEMAX | REC_TIEMIN)) &&
+                               !(r.flags & REC_NOGRID);
+              const float sc = __fmul_rn(sv[ii], p.scale);
+              if (okr && (r.flags & REC_TIEMAX) && sc == r.M) da[ii] += r.cMn;
+              if (CAL == CAL_MINMAX && okr && (r.flags & REC_TIEMIN) && sc == r.m) da[ii] += r.cmn;
+            }
           }
         }
-      }
-      if (p.x3) {
+        if (p.x3) {
 #pragma unroll
-        for (int q = 0; q < W; ++q) {
-          const float x = doDV ? pa[q] : da[q];
-          const float h = tf32_rna(x);
-          pa[q] = h;
-          da[q] = __fsub_rn(x, h);
+          for (int q = 0; q < WS; ++q) {
+            const float x = doDV ? pa[q] : da[q];
+            const float hh = tf32_rna(x);
+            pa[q] = hh;
+            da[q] = __fsub_rn(x, hh);
+          }
+          tmem_stw<WS>(lane_addr(tmem, cS), pa);
+          tmem_stw<WS>(lane_addr(tmem, cG), da);
+        } else {
+          if (doDV) tmem_stw<WS>(lane_addr(tmem, cS), pa);
+          if (doDK) tmem_stw<WS>(lane_addr(tmem, cG), da);
         }
-        tmem_stw<W>(lane_addr(tmem, cS), pa);
-        tmem_stw<W>(lane_addr(tmem, cG), da);
-      } else {
-        if (doDV) tmem_stw<W>(lane_addr(tmem, cS), pa);
-        if (doDK) tmem_stw<W>(lane_addr(tmem, cG), da);
       }
       tmem_st_wait();
       tc_fence_before();
