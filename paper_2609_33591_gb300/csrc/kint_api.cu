@@ -104,6 +104,7 @@ struct Workspace {
   float* rtab = nullptr;  // [BHT][KMAX] (e_r, e_{r+1}) MinMax grid pairs
   float* tie = nullptr;   // [2][BHT][d] sums of tied arg-extremum keys
   int* tileflags = nullptr;  // [BH][ceil(T/64)]
+  float* gbar = nullptr;     // [BHT] <g>_{P*} = dO_i . O*_i
 };
 
 Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
@@ -135,6 +136,7 @@ Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
     w.rtab = take(rows * 2 * KMAX);
     w.tie = take(2 * nat);
     w.tileflags = reinterpret_cast<int*>(take((size_t)BH * ((T + 63) / 64) * 4));
+    w.gbar = take(rows);
   }
   w.bytes = off;
   return w;
@@ -291,8 +293,9 @@ cudaError_t traced(const char* name, cudaStream_t s, F&& launch) {
 }
 
 cudaError_t prep(const float* X, float* nat_hi, float* nat_lo, float* tr_hi, float* tr_lo, int BH, int T, int Tp,
-                 int d, bool split, cudaStream_t s) {
-  return traced("k_prep", s, [&] { return launch_prep(X, nat_hi, nat_lo, tr_hi, tr_lo, BH, T, Tp, d, split, s); });
+                 int d, bool split, cudaStream_t s, const float* Y = nullptr, float* dot = nullptr) {
+  return traced("k_prep", s,
+                [&] { return launch_prep(X, nat_hi, nat_lo, tr_hi, tr_lo, BH, T, Tp, d, split, s, Y, dot); });
 }
 
 // Forward prep + pass 1 (shared by kint_attn_fwd and kint_attn_debug_bins).
@@ -429,6 +432,7 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   p.rec = w.rec; p.rtab = w.rtab; p.tie_acc = w.tie;
   p.Kp = (p.Kint + 1) & ~1;
   p.tileflags = w.tileflags;
+  p.gbar = w.gbar;
   p.nqt = (T + 63) / 64;
   if (cudaMemsetAsync(p.tileflags, 0, (size_t)BH * p.nqt * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
 
@@ -437,14 +441,14 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     if (prep(Q, w.qh, w.ql, w.qth, w.qtl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
     if (prep(K, w.kh, w.kl, w.kth, w.ktl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
     if (prep(V, w.vh, w.vl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (prep(dO, w.doh, w.dol, w.doth, w.dotl, BH, T, Tp, d, true, s) != cudaSuccess)
+    if (prep(dO, w.doh, w.dol, w.doth, w.dotl, BH, T, Tp, d, true, s, p.Ostar, w.gbar) != cudaSuccess)
       return KINT_ERR_LAUNCH;
   } else {
     if (prep(Q, nullptr, nullptr, w.qth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
     if (prep(K, nullptr, nullptr, w.kth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
       return KINT_ERR_LAUNCH;
-    if (prep(dO, nullptr, nullptr, w.doth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
+    if (prep(dO, nullptr, nullptr, w.doth, nullptr, BH, T, Tp, d, false, s, p.Ostar, w.gbar) != cudaSuccess)
       return KINT_ERR_LAUNCH;
   }
   Maps maps;

@@ -169,20 +169,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     tc_fence_before();
     __syncwarp();
     if ((tid & 31) == 0) mbar_arrive(bar_ops);
-    // <g>_{P*} = dO_i . O*_i, each column group takes its share of the d columns (all loads first)
-    constexpr int kMaxQ = 128 / (4 * NCG);
-    const int nq = D / (4 * NCG);
-    float4 xa[kMaxQ], ya[kMaxQ];
-    {
-      const float4* a = reinterpret_cast<const float4*>(p.dO + rw * D) + cg * nq;
-      const float4* b = reinterpret_cast<const float4*>(p.Ostar + rw * D) + cg * nq;
-#pragma unroll
-      for (int q = 0; q < kMaxQ; ++q) {
-        const bool in = row_ok && q < nq;
-        xa[q] = in ? __ldg(a + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-        ya[q] = in ? __ldg(b + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-    }
     if (row_ok) {
       M = p.row_max[rw];
       m = p.row_min[rw];
@@ -191,18 +177,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       nmin = p.n_min[rw];
       amax = p.arg_max[rw];
       amin = p.arg_min[rw];
+      Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
     }
     const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
     Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
-    float acc = 0.f;
-#pragma unroll
-    for (int q = 0; q < kMaxQ; ++q) {
-      acc = __fmaf_rn(xa[q].x, ya[q].x, acc);
-      acc = __fmaf_rn(xa[q].y, ya[q].y, acc);
-      acc = __fmaf_rn(xa[q].z, ya[q].z, acc);
-      acc = __fmaf_rn(xa[q].w, ya[q].w, acc);
-    }
-    xch[cg * 128 + row] = acc;
     g = row_grid(p, M, m);
     if constexpr (CAL == CAL_FWM) {
       if (tid < Kq)
@@ -263,10 +241,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     mma_commit(bar_done);
   } else {
     // ---- compute warps ----
-    group_sync(BAR_COMPUTE, NCOMP);
-    Dg = 0.f;
-#pragma unroll
-    for (int q = 0; q < NCG; ++q) Dg += xch[q * 128 + row];
+    group_sync(BAR_COMPUTE, NCOMP);  // the grid table
     const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
     const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
     const float invWf = 1.0f / Wf;

@@ -13,45 +13,100 @@ namespace kint {
 // ---------------------------------------------------------------------------
 // Operand preparation (HBM-bound).  tcgen05.mma kind::tf32 reads both operands
 // K-major, so every second-stage product (P V, dS K, P^T dO, dS^T Q) reads a
-// transposed copy X^T [BH][d][Tp].  3xTF32 also needs tf32 hi/lo splits.
+// transposed copy X^T [BH][d][Tp].  3xTF32 also needs tf32 hi/lo splits.  With
+// DOT the block also forms the row dot products dot[t] = X_t . Y_t (the
+// backward's <g>_{P*} = dO_i . O*_i, App. B) from the rows it already holds.
+// CTA = 64 rows of one head, all d columns in 64-column steps; float4 loads and
+// stores, a padded 64 x 65 shared tile per step.
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_prep(const float* __restrict__ X, float* __restrict__ nat_hi,
-                                              float* __restrict__ nat_lo, float* __restrict__ tr_hi,
-                                              float* __restrict__ tr_lo, int T, int Tp, int d, int split) {
-  __shared__ float hi_s[32][33];
-  __shared__ float lo_s[32][33];
-  const int t0 = blockIdx.x * 32, k0 = blockIdx.y * 32, bh = blockIdx.z;
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  const size_t nat = (size_t)bh * T * d;
-  for (int r = ty; r < 32; r += 8) {
-    const int t = t0 + r;
-    float x = (t < T) ? X[nat + (size_t)t * d + k0 + tx] : 0.0f;
-    float lo = 0.0f;
-    if (split) {
-      const float h = tf32_rna(x);
-      lo = __fsub_rn(x, h);
-      x = h;
-      if (t < T && nat_hi) {
-        nat_hi[nat + (size_t)t * d + k0 + tx] = x;
-        nat_lo[nat + (size_t)t * d + k0 + tx] = lo;
+template <bool SPLIT, bool DOT>
+__global__ void __launch_bounds__(256) k_prep(const float* __restrict__ X, const float* __restrict__ Y,
+                                              float* __restrict__ nat_hi, float* __restrict__ nat_lo,
+                                              float* __restrict__ tr_hi, float* __restrict__ tr_lo,
+                                              float* __restrict__ dot, int T, int Tp, int d) {
+  __shared__ float hs[64][65];
+  __shared__ float ls[SPLIT ? 64 : 1][65];
+  const int t0 = blockIdx.x * 64, bh = blockIdx.y, tid = threadIdx.x;
+  const int r = tid >> 4, c4 = tid & 15;  // load phase: rows r + 16 q, columns 4 c4 .. 4 c4 + 3
+  const int k = tid >> 4, tq = tid & 15;  // store phase: output rows k + 16 q, keys 4 tq .. 4 tq + 3
+  const size_t nat = (size_t)bh * T * d, tr = (size_t)bh * d * Tp;
+  float dacc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int k0 = 0; k0 < d; k0 += 64) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int rr = r + 16 * q, t = t0 + rr;
+      const size_t off = nat + (size_t)t * d + k0 + 4 * c4;
+      float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (t < T) x = __ldg(reinterpret_cast<const float4*>(X + off));
+      if constexpr (DOT) {
+        if (t < T) {
+          const float4 y = __ldg(reinterpret_cast<const float4*>(Y + off));
+          dacc[q] = __fmaf_rn(x.x, y.x, dacc[q]);
+          dacc[q] = __fmaf_rn(x.y, y.y, dacc[q]);
+          dacc[q] = __fmaf_rn(x.z, y.z, dacc[q]);
+          dacc[q] = __fmaf_rn(x.w, y.w, dacc[q]);
+        }
+      }
+      if constexpr (SPLIT) {
+        float4 h, l;
+        h.x = tf32_rna(x.x); l.x = __fsub_rn(x.x, h.x);
+        h.y = tf32_rna(x.y); l.y = __fsub_rn(x.y, h.y);
+        h.z = tf32_rna(x.z); l.z = __fsub_rn(x.z, h.z);
+        h.w = tf32_rna(x.w); l.w = __fsub_rn(x.w, h.w);
+        if (t < T && nat_hi) {
+          *reinterpret_cast<float4*>(nat_hi + off) = h;
+          *reinterpret_cast<float4*>(nat_lo + off) = l;
+        }
+        x = h;
+        ls[rr][4 * c4] = l.x; ls[rr][4 * c4 + 1] = l.y; ls[rr][4 * c4 + 2] = l.z; ls[rr][4 * c4 + 3] = l.w;
+      }
+      hs[rr][4 * c4] = x.x; hs[rr][4 * c4 + 1] = x.y; hs[rr][4 * c4 + 2] = x.z; hs[rr][4 * c4 + 3] = x.w;
+    }
+    __syncthreads();
+    if (tr_hi) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int kk = k + 16 * q, t = t0 + 4 * tq;
+        if (t < Tp) {
+          const size_t off = tr + (size_t)(k0 + kk) * Tp + t;
+          *reinterpret_cast<float4*>(tr_hi + off) =
+              make_float4(hs[4 * tq][kk], hs[4 * tq + 1][kk], hs[4 * tq + 2][kk], hs[4 * tq + 3][kk]);
+          if constexpr (SPLIT) {
+            if (tr_lo)
+              *reinterpret_cast<float4*>(tr_lo + off) =
+                  make_float4(ls[4 * tq][kk], ls[4 * tq + 1][kk], ls[4 * tq + 2][kk], ls[4 * tq + 3][kk]);
+          }
+        }
       }
     }
-    hi_s[r][tx] = x;
-    lo_s[r][tx] = lo;
+    __syncthreads();
   }
-  __syncthreads();
-  const size_t tr = (size_t)bh * d * Tp;
-  for (int r = ty; r < 32; r += 8) {
-    const int k = k0 + r, t = t0 + tx;  // t < Tp by construction of the grid
-    if (tr_hi) tr_hi[tr + (size_t)k * Tp + t] = hi_s[tx][r];
-    if (split && tr_lo) tr_lo[tr + (size_t)k * Tp + t] = lo_s[tx][r];
+  if constexpr (DOT) {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float v = dacc[q];
+#pragma unroll
+      for (int o = 8; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      const int t = t0 + r + 16 * q;
+      if (c4 == 0 && t < T) dot[(size_t)bh * T + t] = v;
+    }
   }
 }
 
 cudaError_t launch_prep(const float* X, float* nat_hi, float* nat_lo, float* tr_hi, float* tr_lo, int BH, int T,
-                        int Tp, int d, bool split, cudaStream_t s) {
-  dim3 grid(Tp / 32, d / 32, BH), block(32, 8);
-  k_prep<<<grid, block, 0, s>>>(X, nat_hi, nat_lo, tr_hi, tr_lo, T, Tp, d, split ? 1 : 0);
+                        int Tp, int d, bool split, cudaStream_t s, const float* Y, float* dot) {
+  dim3 grid((Tp + 63) / 64, BH), block(256);
+  if (dot) {
+    if (split)
+      k_prep<true, true><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
+    else
+      k_prep<false, true><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
+  } else {
+    if (split)
+      k_prep<true, false><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
+    else
+      k_prep<false, false><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
+  }
   return cudaGetLastError();
 }
 

@@ -53,6 +53,7 @@ struct Params {
   int* tileflags;           // [B*H][nqt] 1 where a 64-row query tile holds a row with tied extrema
   int nqt;                  // ceil(T / 64)
   float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
+  const float* gbar;        // [BH*T] <g>_{P*} = dO_i . O*_i (workspace, written by the dO prep)
   uint8_t *bins, *ivals;
 };
 
