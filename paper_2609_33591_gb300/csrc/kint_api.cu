@@ -241,13 +241,18 @@ int plan_main(Params& p, int mode) {
 int plan_dq(Params& p) {
   const int parts = p.x3 ? 2 : 1, ktile = 64 * p.d * 4, dp = p.d * parts;
   const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : 1024;
+  // TF32 at d = 64: Q and dO arrive as TMA tiles staged in smem (64 KB) and are copied
+  // to TMEM from there; otherwise (3xTF32 hi/lo, d = 128) the staging area would not fit
+  // next to the K/V stages and the rows are read from global memory.
+  p.ops_smem = (!p.x3 && p.d == 64) ? 1 : 0;
   p.nbuf = (2 * dp + 256 + p.d <= 512) ? 2 : 1;
-  p.sm_stage0 = 0;
+  p.sm_a = 0;
+  p.sm_stage0 = p.ops_smem ? 2 * 128 * p.d * 4 : 0;
   p.sm_stage_bytes = 3 * parts * ktile;
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
-    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 6), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 7), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       return total;
@@ -259,16 +264,19 @@ int plan_dq(Params& p) {
 int plan_dkdv(Params& p, int sel) {
   const int parts = p.x3 ? 2 : 1, qtile = 64 * p.d * 4, dp = p.d * parts;
   const bool doDV = sel != DKV_DK, doDK = sel != DKV_DV;
+  // TF32 at d = 64, both products: K and V staged in smem by TMA (see plan_dq)
+  p.ops_smem = (!p.x3 && p.d == 64 && doDV && doDK) ? 1 : 0;
   const int base = doDK ? 2 * dp : dp;
   const int acc = (doDV ? p.d : 0) + (doDK ? p.d : 0);
   if (base + 128 + acc > 512) return -1;
   p.dkv_sel = sel;
   p.nbuf = (base + 256 + acc <= 512) ? 2 : 1;
-  p.sm_stage0 = 0;
+  p.sm_a = 0;
+  p.sm_stage0 = p.ops_smem ? 2 * 128 * p.d * 4 : 0;
   p.sm_stage_bytes = 4 * parts * qtile + 64 * 64 + (p.calib == KINT_CALIB_MINMAX ? 64 * p.Kp * 8 : 0);
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    const int total = std::max(finish_plan(p, p.sm_table + 1024, 2 * p.nstage + 6), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_table + 1024, 2 * p.nstage + 7), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       return total;

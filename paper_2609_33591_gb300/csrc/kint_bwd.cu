@@ -121,14 +121,15 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   uint64_t* bar_pready = bars + 2 * NS + 2;  // [2]
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint64_t* bar_ops = bars + 2 * NS + 5;  // Q / dO rows stored in TMEM by every compute warp
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 6);
+  uint64_t* bar_stg = bars + 2 * NS + 6;  // Q / dO tiles staged in smem by TMA
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 7);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
   const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
   constexpr int W = BT / NCG;  // key columns per thread per tile
   const int dp = D * parts;
-  const int cQ = 0, cdO = dp, cdQ = 2 * dp + 128 * nbuf;
+  const int cQ = 0, cdO = dp, cSG0 = 2 * dp, cdQ = cSG0 + 128 * nbuf;
 
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
@@ -141,6 +142,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     }
     mbar_init(bar_done, 1);
     mbar_init(bar_ops, NCOMP / 32);
+    mbar_init(bar_stg, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -161,10 +163,16 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   int nmax = 1, nmin = 1, amax = 0, amin = 0;
   RowGrid g{};
   if (warp < NCOMP / 32) {
-    // operand rows into TMEM (column group 0 takes Q, group 1 takes dO), handed to
-    // the MMA warp through bar_ops; the rest of the set-up runs under the first products
-    row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
-                p.x3 != 0);
+    // operand rows into TMEM (column group 0 takes Q, group 1 takes dO), handed to the
+    // MMA warp through bar_ops; the rest of the set-up runs under the first products.
+    // TF32 at d = 64: from tiles the producer staged in smem; otherwise from global rows.
+    if (p.ops_smem) {
+      if (mbar_wait(bar_stg, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+        staged_row_to_tmem(tmem, cg == 0 ? cQ : cdO, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
+    } else {
+      row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
+                  p.x3 != 0);
+    }
     tmem_st_wait();
     tc_fence_before();
     __syncwarp();
@@ -195,6 +203,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   }
 
   if (warp == PRODUCER_WARP) {
+    if (p.ops_smem) {
+      mbar_arrive_expect_tx(bar_stg, 2 * 128 * D * 4);
+      load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb * 128, bh);
+      load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb * 128, bh);
+    }
     for (int kt = 0; kt < nkt; ++kt) {
       const int s = kt % NS;
       if (kt >= NS &&
@@ -214,7 +227,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     }
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
-    const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + 2 * dp;
+    const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + cSG0;
     bool ok = mbar_wait_warp(bar_ops, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
     if (ok) tc_fence_after();
     ok = ok && dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
@@ -225,7 +238,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       if (!mbar_wait_warp(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
       tc_fence_after();
       const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
-      const uint32_t cS = tmem + 2 * dp + 128 * b, cG = cS + 64;
+      const uint32_t cS = tmem + cSG0 + 128 * b, cG = cS + 64;
       const bool acc = kt > 0;
       if (p.x3) {
         mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);           // dS_hi K_hi
@@ -268,7 +281,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         break;
       }
       tc_fence_after();
-      const int cS = 2 * dp + 128 * b + cg * W, cG = cS + 64;
+      const int cS = cSG0 + 128 * b + cg * W, cG = cS + 64;
       float sv[W], gv[W], out[W];
       tmem_ldw<W>(lane_addr(tmem, cS), sv);
       tmem_ldw<W>(lane_addr(tmem, cG), gv);
@@ -498,7 +511,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   uint64_t* bar_pready = bars + 2 * NS + 2;
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint64_t* bar_ops = bars + 2 * NS + 5;  // K / V rows stored in TMEM by every compute warp
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 6);
+  uint64_t* bar_stg = bars + 2 * NS + 6;  // K / V tiles staged in smem by TMA
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 7);
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, kb = blockIdx.x;
   const int dp = D * parts;
@@ -522,6 +536,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     }
     mbar_init(bar_done, 1);
     mbar_init(bar_ops, NCOMP / 32);
+    mbar_init(bar_stg, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -536,9 +551,15 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   const int j = kb * 128 + row;
   const bool key_ok = j < p.T;
   if (warp < NCOMP / 32) {
-    // operand rows into TMEM: column group 0 takes K, group 1 takes V
-    if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-    else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    // operand rows into TMEM: column group 0 takes K, group 1 takes V (staged tiles at
+    // TF32 d = 64, global rows otherwise)
+    if (p.ops_smem) {
+      if (mbar_wait(bar_stg, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) && (cg == 0 || needV))
+        staged_row_to_tmem(tmem, cg == 0 ? cK : cV, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
+    } else {
+      if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+      else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
+    }
     tmem_st_wait();
     tc_fence_before();
     __syncwarp();
@@ -548,6 +569,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   }
 
   if (warp == PRODUCER_WARP) {
+    if (p.ops_smem) {
+      mbar_arrive_expect_tx(bar_stg, (needV ? 2 : 1) * 128 * D * 4);
+      load_rows_tile_boxed(sm + p.sm_a, &maps.k, bar_stg, D, 128, BT, 0, kb * 128, bh);
+      if (needV) load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.v, bar_stg, D, 128, BT, 0, kb * 128, bh);
+    }
     for (int it = 0; it < nit; ++it) {
       const int s = it % NS, q0 = (qt0 + it) * BT;
       if (it >= NS &&

@@ -198,6 +198,14 @@ __device__ __forceinline__ void load_rows_tile(uint8_t* dst, const CUtensorMap* 
   for (int pnl = 0; pnl < ncols / 32; ++pnl)
     tma_load_3d(dst + pnl * nrows * SW, map, bar, c_first + 32 * pnl, r_first, bh);
 }
+// A tile of nrows rows fetched as nrows / box row boxes per panel (a map whose box is
+// `box` rows); box * 128 bytes is a multiple of the 1024-byte swizzle atom.
+__device__ __forceinline__ void load_rows_tile_boxed(uint8_t* dst, const CUtensorMap* map, uint64_t* bar, int ncols,
+                                                     int nrows, int box, int c_first, int r_first, int bh) {
+  for (int pnl = 0; pnl < ncols / 32; ++pnl)
+    for (int r = 0; r < nrows; r += box)
+      tma_load_3d(dst + pnl * nrows * SW + r * SW, map, bar, c_first + 32 * pnl, r_first + r, bh);
+}
 
 // ---------------------------------------------------------------------------
 // Tensor-core products.  The issuing thread's own instruction stream bounds the
@@ -297,6 +305,25 @@ __device__ __forceinline__ void row_to_tmem_part(uint32_t tmem_base, int col, co
     }
     if (split) tmem_st32(lane_addr(tmem_base, col + d + c0 + c), lo);
     tmem_st32(lane_addr(tmem_base, col + c0 + c), hi);
+  }
+}
+
+// Row `row` of a 128-row K-major tile staged in smem by TMA (128-byte swizzle,
+// 32-column panels 128 x 128 bytes apart) into the calling thread's TMEM lane at
+// columns [col, col + d).  Chunk c (16 bytes) of a row sits at chunk c ^ (row % 8).
+__device__ __forceinline__ void staged_row_to_tmem(uint32_t tmem_base, int col, const uint8_t* tile, int row, int d) {
+  const uint32_t base = smem_u32(tile) + (uint32_t)row * SW;
+  for (int pnl = 0; pnl < d / 32; ++pnl) {
+    float v[32];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const float4 x = lds_f4(base + (uint32_t)pnl * 128u * SW + (uint32_t)((c ^ (row & 7)) << 4));
+      v[4 * c] = x.x;
+      v[4 * c + 1] = x.y;
+      v[4 * c + 2] = x.z;
+      v[4 * c + 3] = x.w;
+    }
+    tmem_st32(lane_addr(tmem_base, col + 32 * pnl), v);
   }
 }
 

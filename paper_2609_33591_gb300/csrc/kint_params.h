@@ -40,6 +40,7 @@ struct Params {
   // smem plan (byte offsets from the 1024-aligned base), set by the host
   int sm_a, sm_stage0, sm_stage_bytes, nstage, sm_table, sm_rows, sm_bars;
   int nbuf;  // score buffers in TMEM (2: the next tile's product runs under this tile's element work)
+  int ops_smem;  // backward: the 128-row TMEM operands (Q, dO / K, V) are staged in smem by TMA first
 
   // tensors (device pointers)
   const float *Q, *K, *V, *O, *dO, *Ostar;
