@@ -223,7 +223,7 @@ int plan_main(Params& p, int mode) {
   for (p.nstage = 3; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_a;  // the 4 x 128 exchange words reuse the Q tile after the last product
-    const int total = std::max(finish_plan(p, p.sm_table + table, 6 + 2 * p.nstage), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_table + table, 7 + 2 * p.nstage), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       // Issuing S(kb+1) before P V(kb) needs tile kb+1 in a second stage while
       // tile kb's V^T is still being read; with one stage the two would wait on

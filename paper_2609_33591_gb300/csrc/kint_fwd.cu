@@ -462,8 +462,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   uint64_t* bar_empty = bars + 1 + NS;
   uint64_t* bar_s = bars + 1 + 2 * NS;       // [2] S_b computed
   uint64_t* bar_pready = bars + 3 + 2 * NS;  // [2] weights of buffer b stored by every compute warp
-  uint64_t* bar_pv = bars + 5 + 2 * NS;      // P V of a tile complete
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 6 + 2 * NS);
+  uint64_t* bar_pv = bars + 5 + 2 * NS;      // P V of a tile complete (A2 free again)
+  uint64_t* bar_done = bars + 6 + 2 * NS;    // every product of the CTA complete (one phase)
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 7 + 2 * NS);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [4][128], aliases Q once all products are done
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
@@ -482,6 +483,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       mbar_init(&bar_pready[b], NCOMP / 32);
     }
     mbar_init(bar_pv, 1);
+    mbar_init(bar_done, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -536,6 +538,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       // one buffer: S(kb+1) overwrites the weights P V(kb) reads, in issue order after it
       if (nbuf == 1 && kb + 1 < nkb && !main_issue_s(p, kb + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
     }
+    mma_commit(bar_done);
   } else {
     const int row = tid & 127, cg = tid >> 7;
     const int i = qb * 128 + row;
@@ -610,7 +613,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       __syncwarp();
       if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
     }
-    if (!failed) failed = !mbar_wait(bar_pv, (nkb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+    // bar_done, not bar_pv: without A2 the compute warps may run more than one tile
+    // ahead of P V, and a parity wait cannot tell phase nkb - 1 from phase nkb - 3
+    if (!failed) failed = !mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
     failed = group_any(BAR_COMPUTE, NCOMP, failed);
     if (!failed) {
       tc_fence_after();

@@ -105,8 +105,7 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint64_t* bar, uint32_t parit
       : "memory");
   return ok != 0;
 }
-// Bounded spin for single-thread roles (MMA issuer, producer): a suspended
-// try_wait was measured to resume up to ~1 us after the phase completed.
+// Bounded spin on test_wait (the time limit is checked every 64 polls).
 __device__ __forceinline__ bool mbar_wait_spin(uint64_t* bar, uint32_t parity, uint64_t timeout_ns, unsigned* status,
                                                unsigned err) {
   if (mbar_test_wait(bar, parity)) return true;
@@ -131,18 +130,12 @@ __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, u
 }
 
 // Bounded wait on the phase with the given parity.  Returns false (and flags
-// `err`) once `timeout_ns` of wall time has passed without completion.
+// `err`) once `timeout_ns` of wall time has passed without completion.  It polls
+// with test_wait: a suspended try_wait was measured to resume up to ~1 us after
+// the phase completed, which put that latency on every tile hand-off.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t timeout_ns, unsigned* status,
                                           unsigned err) {
-  if (mbar_test_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (true) {
-    if (mbar_try_wait_hint(bar, parity, 40)) return true;
-    if (globaltimer_ns() - t0 > timeout_ns) {
-      dev_flag(status, err);
-      return false;
-    }
-  }
+  return mbar_wait_spin(bar, parity, timeout_ns, status, err);
 }
 
 // ----------------------------------------------------------------------------
