@@ -74,6 +74,19 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
   }
 }
 
+// Adds key rows j0 + b (b a set bit of `mask`) of K (rows of d floats from `k0`) to
+// the tie sum `acc` (rare path, kept rolled).
+__device__ __forceinline__ void add_tied_keys(uint32_t mask, float* acc, const float* k0, int d) {
+#pragma unroll 1
+  while (mask) {
+    const int b = __ffs(mask) - 1;
+    mask &= mask - 1;
+    const float* kr = k0 + (size_t)b * d;
+#pragma unroll 1
+    for (int k = 0; k < d; ++k) atomicAdd(&acc[k], kr[k]);
+  }
+}
+
 // MMA thread of k_bwd_dq: wait for key tile kt, then S_b = Q K^T and g_b = dO V^T
 // into score buffer b = kt % nbuf.
 __device__ __forceinline__ bool dq_issue_sg(const Params& p, int kt, uint64_t* bar_full, uint64_t* bar_sfull,
@@ -295,16 +308,16 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
                                        sk1, sc0, invWf, own, cm);
       if (__any_sync(0xffffffffu, track)) {
         // rare: tied extrema, the tie set is found by equality on the recomputed scores
+        uint32_t mk_max = 0, mk_min = 0;
 #pragma unroll
         for (int jj = 0; jj < W; ++jj) {
-          const int j = j0 + jj;
           const float s = __fmul_rn(sv[jj], p.scale);
-          const bool okj = track && j <= i;
-          if (okj && nmax > 1 && s == M)
-            for (int k = 0; k < D; ++k) atomicAdd(&tie_max[k], p.K[((size_t)bh * p.T + j) * D + k]);
-          if (okj && minmax && nmin > 1 && s == m)
-            for (int k = 0; k < D; ++k) atomicAdd(&tie_min[k], p.K[((size_t)bh * p.T + j) * D + k]);
+          const bool okj = track && j0 + jj <= i;
+          mk_max |= (okj && nmax > 1 && s == M) ? (1u << jj) : 0u;
+          mk_min |= (okj && minmax && nmin > 1 && s == m) ? (1u << jj) : 0u;
         }
+        add_tied_keys(mk_max, tie_max, p.K + ((size_t)bh * p.T + j0) * D, D);
+        add_tied_keys(mk_min, tie_min, p.K + ((size_t)bh * p.T + j0) * D, D);
       }
       if (p.x3) {
         float lo[W];

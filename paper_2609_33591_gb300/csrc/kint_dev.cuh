@@ -247,22 +247,22 @@ __device__ __forceinline__ void mma_ts_k(uint32_t d_tmem, uint32_t a_tmem, const
                 (accumulate || kk > 0) ? 1u : 0u);
 }
 
-// Runtime-K wrappers (K = 64 or 128 columns, or 128 / 256 for the key products).
+// Runtime-K wrappers: K = Ktot columns (a multiple of 64) as a rolled loop over
+// blocks of eight unrolled steps, which keeps the issuing code small.
 __device__ __forceinline__ void mma_smem_smem(uint32_t d_tmem, const uint8_t* a, const uint8_t* b, int N, int Ktot,
                                               bool accumulate) {
   const uint32_t idesc = idesc_tf32(128, N, 0, 0);
-  if (Ktot == 64)
-    mma_ss_k<8>(d_tmem, a, b, 128 * SW, N * SW, idesc, accumulate);
-  else
-    mma_ss_k<16>(d_tmem, a, b, 128 * SW, N * SW, idesc, accumulate);
+#pragma unroll 1
+  for (int k0 = 0; k0 < Ktot; k0 += 64)
+    mma_ss_k<8>(d_tmem, a + (k0 / 32) * 128 * SW, b + (k0 / 32) * N * SW, 128 * SW, N * SW, idesc,
+                accumulate || k0 > 0);
 }
 __device__ __forceinline__ void mma_tmem_smem(uint32_t d_tmem, uint32_t a_tmem, const uint8_t* b, int N, int Ktot,
                                               bool accumulate) {
   const uint32_t idesc = idesc_tf32(128, N, 0, 0);
-  if (Ktot == 64)
-    mma_ts_k<8>(d_tmem, a_tmem, b, N * SW, idesc, accumulate);
-  else
-    mma_ts_k<16>(d_tmem, a_tmem, b, N * SW, idesc, accumulate);
+#pragma unroll 1
+  for (int k0 = 0; k0 < Ktot; k0 += 64)
+    mma_ts_k<8>(d_tmem, a_tmem + k0, b + (k0 / 32) * N * SW, N * SW, idesc, accumulate || k0 > 0);
 }
 
 // The calling thread's TMEM lane (its row) at column `col`.  Warp w may only
