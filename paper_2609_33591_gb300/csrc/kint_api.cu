@@ -346,6 +346,13 @@ int check_stats(const kint_rowstats* st, bool prob) {
   return KINT_OK;
 }
 
+// Output maps of pass 2 (O, and O_lerp when the stats carry it) for its TMA stores.
+bool map_fwd_outputs(Maps& maps, const Params& p) {
+  bool ok = map_nat(&maps.out, p.Out, p.BH, p.T, p.d, 64);
+  if (p.O_lerp) ok = ok && map_nat(&maps.out_lerp, p.O_lerp, p.BH, p.T, p.d, 64);
+  return ok;
+}
+
 void set_stats(Params& p, const kint_rowstats* st) {
   p.row_max = st->row_max; p.row_min = st->row_min;
   p.arg_max = st->arg_max; p.arg_min = st->arg_min;
@@ -394,6 +401,7 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
   const Workspace w = plan_workspace(static_cast<char*>(workspace), p.BH, T, d, p.x3 != 0, false);
   Maps maps;
   if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
+  if (!map_fwd_outputs(maps, p)) return KINT_ERR_LAUNCH;
 
   Params pm = p;
   pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
@@ -476,6 +484,8 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     ok = ok && map_tr(&maps.kt, w.kth, BH, T, Tp, d) && map_tr(&maps.qt, w.qth, BH, T, Tp, d);
     ok = ok && map_tr(&maps.dot, w.doth, BH, T, Tp, d);
   }
+  ok = ok && map_nat(&maps.dq, dQ, BH, T, d, 64) && map_nat(&maps.dk, dK, BH, T, d, 64) &&
+       map_nat(&maps.dv, dV, BH, T, d, 64);
   if (!ok) return KINT_ERR_LAUNCH;
 
   Params pq = p;
@@ -627,6 +637,7 @@ int kint_attn_fwd_noalloc(const float* Q, const float* K, const float* V, float*
   const Workspace w = plan_workspace(static_cast<char*>(scratch), p.BH, T, d, p.x3 != 0, false);
   Maps maps;
   if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
+  if (!map_fwd_outputs(maps, p)) return KINT_ERR_LAUNCH;
   Params pm = p;
   pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
   const int smem = plan_main(pm, pm.pv_sel);

@@ -356,9 +356,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
       const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
       const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
-      float* dst = p.dQ + rw * D;
+      // dQ rows into a swizzled tile in the idle stage ring, then one TMA store
+      uint8_t* stg = sm + p.sm_stage0;
       for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
-        // the arg-extremum key rows first (all loads in flight before any store)
+        // the arg-extremum key rows first (all loads in flight before the TMEM read)
         float4 km[8], kn[8];
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
@@ -370,18 +371,18 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         float v[32];
         tmem_ld32(lane_addr(tmem, cdQ + c), v);
         tmem_ld_wait();
-        if (row_ok) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            float4 o;
-            o.x = __fmaf_rn(cmn, kn[q].x, __fmaf_rn(cMn, km[q].x, v[4 * q])) * p.scale;
-            o.y = __fmaf_rn(cmn, kn[q].y, __fmaf_rn(cMn, km[q].y, v[4 * q + 1])) * p.scale;
-            o.z = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
-            o.w = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
-            reinterpret_cast<float4*>(dst + c)[q] = o;
-          }
+        for (int q = 0; q < 8; ++q) {
+          v[4 * q] = __fmaf_rn(cmn, kn[q].x, __fmaf_rn(cMn, km[q].x, v[4 * q])) * p.scale;
+          v[4 * q + 1] = __fmaf_rn(cmn, kn[q].y, __fmaf_rn(cMn, km[q].y, v[4 * q + 1])) * p.scale;
+          v[4 * q + 2] = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
+          v[4 * q + 3] = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
         }
+        row_to_staged(stg, row, c / 32, v);
       }
+      fence_async_smem();
+      group_sync(BAR_COMPUTE, NCOMP);
+      if (warp == 0) store_rows_tile_boxed(stg, &maps.dq, D, 64, qb * 128, bh);
       if (row_ok && cg == 0) {
         RowRec r;
         r.c0 = g.c0;
@@ -731,24 +732,26 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     failed = group_any(BAR_COMPUTE, NCOMP, !dok);
     if (!failed) {
       tc_fence_after();
-      const size_t krow = (size_t)bh * p.T + (key_ok ? j : 0);
+      // dV, dK rows into swizzled tiles in the idle stage ring, then one TMA store each
+      uint8_t* stg = sm + p.sm_stage0;
       for (int pass = 0; pass < 2; ++pass) {
         if (pass == 0 ? !doDV : !doDK) continue;
         const int col = pass == 0 ? cdV : cdK;
         const float mul = pass == 0 ? 1.0f : p.scale;
-        float* dst = (pass == 0 ? p.dV : p.dK) + krow * D;
-        for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 16) {
-          float v[16];
-          tmem_ld16(lane_addr(tmem, col + c), v);
+        uint8_t* tile = stg + pass * 128 * D * 4;
+        for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
+          float v[32];
+          tmem_ld32(lane_addr(tmem, col + c), v);
           tmem_ld_wait();
-          if (key_ok) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-              reinterpret_cast<float4*>(dst + c)[q] =
-                  make_float4(v[4 * q] * mul, v[4 * q + 1] * mul, v[4 * q + 2] * mul, v[4 * q + 3] * mul);
-          }
+          for (int q = 0; q < 32; ++q) v[q] *= mul;
+          row_to_staged(tile, row, c / 32, v);
         }
       }
+      fence_async_smem();
+      group_sync(BAR_COMPUTE, NCOMP);
+      if (warp == 0 && doDV) store_rows_tile_boxed(stg, &maps.dv, D, 64, kb * 128, bh);
+      if (warp == 1 && doDK) store_rows_tile_boxed(stg + 128 * D * 4, &maps.dk, D, 64, kb * 128, bh);
     }
     tc_fence_before();
   }

@@ -207,6 +207,28 @@ __device__ __forceinline__ void load_rows_tile_boxed(uint8_t* dst, const CUtenso
       tma_load_3d(dst + pnl * nrows * SW + r * SW, map, bar, c_first + 32 * pnl, r_first + r, bh);
 }
 
+// The calling thread's row `row` (values v[0..31], columns [32 pnl, 32 pnl + 32))
+// into a 128-row tile in smem laid out like the TMA tiles (128-byte swizzle, panels
+// of 32 columns 128 x 128 bytes apart), for a TMA store.
+__device__ __forceinline__ void row_to_staged(uint8_t* tile, int row, int pnl, const float (&v)[32]) {
+  const uint32_t base = smem_u32(tile) + (uint32_t)pnl * 128u * SW + (uint32_t)row * SW;
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    const uint32_t a = base + (uint32_t)((c ^ (row & 7)) << 4);
+    asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(a), "f"(v[4 * c]), "f"(v[4 * c + 1]),
+                 "f"(v[4 * c + 2]), "f"(v[4 * c + 3])
+                 : "memory");
+  }
+}
+// A staged 128-row tile (ncols columns) to rows [r_first, r_first + 128) of head bh
+// through a map whose box is `box` rows (warp-collective; waits until it was read).
+__device__ __forceinline__ void store_rows_tile_boxed(const uint8_t* tile, const CUtensorMap* map, int ncols, int box,
+                                                      int r_first, int bh) {
+  for (int pnl = 0; pnl < ncols / 32; ++pnl)
+    for (int r = 0; r < 128; r += box) tma_store_3d(map, tile + pnl * 128 * SW + r * SW, 32 * pnl, r_first + r, bh);
+  tma_store_commit_and_wait_read();
+}
+
 // ---------------------------------------------------------------------------
 // Tensor-core products.  The issuing thread's own instruction stream bounds the
 // MMA rate (measured on GB300: an M=128, N=128 tf32 MMA every ~33 ns with

@@ -625,36 +625,35 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       const float Wmt = xch[row] + xch[128 + row];
       const float Wlt = xch[256 + row] + xch[384 + row];
       if (!p.debug) {
-        // O = (sum_j w_j V_j) / W; each column group stores half of the d columns
+        // O = (sum_j w_j V_j) / W (and O_lerp): each column group scales half of the d
+        // columns into a swizzled tile in the idle stage ring, one TMA store per tile
         const float Wout = (MODE == 2) ? Wlt : Wmt;
         const float inv = row_ok ? 1.0f / Wout : 0.0f;
-        float* dst = ((MODE == 2) ? p.O_lerp : p.Out) + rw * D;
+        uint8_t* stg = sm + p.sm_stage0;
+        uint8_t* stgl = stg + 128 * D * 4;
         for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
           float v[32];
           tmem_ld32(lane_addr(tmem, cO + c), v);
           tmem_ld_wait();
-          if (row_ok) {
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-              reinterpret_cast<float4*>(dst + c)[q] =
-                  make_float4(v[4 * q] * inv, v[4 * q + 1] * inv, v[4 * q + 2] * inv, v[4 * q + 3] * inv);
-          }
+          for (int q = 0; q < 32; ++q) v[q] *= inv;
+          row_to_staged(stg, row, c / 32, v);
         }
         if constexpr (MODE == 1) {
           const float invl = row_ok ? 1.0f / Wlt : 0.0f;
-          float* dl = p.O_lerp + rw * D;
           for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
             float v[32];
             tmem_ld32(lane_addr(tmem, cOL + c), v);
             tmem_ld_wait();
-            if (row_ok) {
 #pragma unroll
-              for (int q = 0; q < 8; ++q)
-                reinterpret_cast<float4*>(dl + c)[q] =
-                    make_float4(v[4 * q] * invl, v[4 * q + 1] * invl, v[4 * q + 2] * invl, v[4 * q + 3] * invl);
-            }
+            for (int q = 0; q < 32; ++q) v[q] *= invl;
+            row_to_staged(stgl, row, c / 32, v);
           }
         }
+        fence_async_smem();
+        group_sync(BAR_COMPUTE, NCOMP);
+        if (warp == 0) store_rows_tile_boxed(stg, (MODE == 2) ? &maps.out_lerp : &maps.out, D, 64, qb * 128, bh);
+        if (MODE == 1 && warp == 1) store_rows_tile_boxed(stgl, &maps.out_lerp, D, 64, qb * 128, bh);
         if (row_ok && cg == 0) {
           if (MODE != 2) p.W[rw] = Wmt;
           if (MODE != 0 && p.W_lerp) p.W_lerp[rw] = Wlt;

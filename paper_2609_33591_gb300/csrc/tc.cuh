@@ -147,6 +147,26 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
       : "memory");
 }
+// TMA: 3-D tiled store shared -> global of a tile written by this CTA's threads
+// (they fence the async proxy and synchronize first).  Elements outside the
+// tensor are not written.  Warp-collective; the elected lane also commits the
+// bulk group and waits until the tile has been read out of shared memory.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1, int c2) {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];\n\t}" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void tma_store_commit_and_wait_read() {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e cp.async.bulk.commit_group;\n\t"
+      "@e cp.async.bulk.wait_group.read 0;\n\t}" ::
+          : "memory");
+  __syncwarp();
+}
 // 1-D bulk copy global -> shared (both addresses 16-byte aligned, bytes a
 // multiple of 16), completion counted on an mbarrier (warp-collective).
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
