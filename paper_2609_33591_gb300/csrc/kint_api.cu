@@ -28,6 +28,7 @@ std::mutex g_mu;
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 unsigned* g_status_ptr[kMaxDevices] = {nullptr};
 int g_dev_ok[kMaxDevices] = {0};  // 0 unknown, 1 sm_103, -1 other
+int g_num_sms[kMaxDevices] = {0};
 unsigned long long g_wait_ns = 2000000000ull;
 constexpr int kSmemLimit = 232448;  // opt-in maximum per CTA on sm_103
 
@@ -35,6 +36,12 @@ int round_up(int x, int m) { return (x + m - 1) / m * m; }
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Resolve the device-dependent handles once per device.
+int num_sms() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 1;
+  return g_num_sms[dev] > 0 ? g_num_sms[dev] : 1;
+}
+
 int device_setup(unsigned** status) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return KINT_ERR_NO_DEVICE;
@@ -53,6 +60,11 @@ int device_setup(unsigned** status) {
         return KINT_ERR_NO_DEVICE;
       }
       g_status_ptr[dev] = static_cast<unsigned*>(ptr);
+      if (cudaDeviceGetAttribute(&g_num_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+          g_num_sms[dev] < 1) {
+        g_dev_ok[dev] = 0;
+        return KINT_ERR_NO_DEVICE;
+      }
     }
   }
   if (g_dev_ok[dev] != 1) return KINT_ERR_NO_DEVICE;
@@ -216,20 +228,29 @@ int plan_main(Params& p, int mode) {
   const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : (p.calib == KINT_CALIB_FWM ? 1024 : 0);
   const bool useA2 = mode == PV_MAIN_LERP || p.x3;
   const int cols1 = 128 + (useA2 ? 128 : 0) + p.d + (mode == PV_MAIN_LERP ? p.d : 0);
-  p.nbuf = (cols1 + 128 <= 512) ? 2 : 1;
+  const int ostage = (mode == PV_MAIN_LERP ? 2 : 1) * 128 * p.d * 4;  // O (and O_lerp) staging tiles
+  p.nitems = p.nqb * p.BH;
   p.sm_a = 0;
   p.sm_stage0 = parts * tile;
   p.sm_stage_bytes = parts * 2 * tile;
-  for (p.nstage = 3; p.nstage >= 1; --p.nstage) {
-    p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    p.sm_rows = p.sm_a;  // the 4 x 128 exchange words reuse the Q tile after the last product
-    const int total = std::max(finish_plan(p, p.sm_table + table, 7 + 2 * p.nstage), kOneCtaPerSm);
-    if (total <= kSmemLimit) {
-      // Issuing S(kb+1) before P V(kb) needs tile kb+1 in a second stage while
-      // tile kb's V^T is still being read; with one stage the two would wait on
-      // each other, so a single stage means a single score buffer.
-      if (p.nstage == 1) p.nbuf = 1;
-      return total;
+  // One CTA per SM looping over the items needs its own output staging area (the
+  // stage ring keeps loading the next item); at least two stages.  Otherwise one item
+  // per CTA, staging in the ring, which is idle by the epilogue.
+  for (int persist = 1; persist >= 0; --persist) {
+    for (p.nstage = 3; p.nstage >= (persist ? 2 : 1); --p.nstage) {
+      p.nbuf = (cols1 + 128 <= 512) ? 2 : 1;
+      p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+      p.sm_ostage = persist ? round_up(p.sm_table + table, 1024) : p.sm_stage0;
+      const int end = persist ? p.sm_ostage + ostage : p.sm_table + table;
+      const int total = std::max(finish_plan(p, end, 9 + 2 * p.nstage), kOneCtaPerSm);
+      if (total <= kSmemLimit) {
+        // Issuing S(kb+1) before P V(kb) needs tile kb+1 in a second stage while
+        // tile kb's V^T is still being read; with one stage the two would wait on
+        // each other, so a single stage means a single score buffer.
+        if (p.nstage == 1) p.nbuf = 1;
+        p.ngrid = persist ? std::min(p.nitems, num_sms()) : p.nitems;
+        return total;
+      }
     }
   }
   return -1;

@@ -221,12 +221,15 @@ __device__ __forceinline__ void row_to_staged(uint8_t* tile, int row, int pnl, c
   }
 }
 // A staged 128-row tile (ncols columns) to rows [r_first, r_first + 128) of head bh
-// through a map whose box is `box` rows (warp-collective; waits until it was read).
+// through a map whose box is `box` rows (warp-collective).  With `wait`, returns once
+// the tile has been read out of shared memory; otherwise the caller waits later
+// (tma_store_wait_read) before it writes the tile again.
 __device__ __forceinline__ void store_rows_tile_boxed(const uint8_t* tile, const CUtensorMap* map, int ncols, int box,
-                                                      int r_first, int bh) {
+                                                      int r_first, int bh, bool wait = true) {
   for (int pnl = 0; pnl < ncols / 32; ++pnl)
     for (int r = 0; r < 128; r += box) tma_store_3d(map, tile + pnl * 128 * SW + r * SW, 32 * pnl, r_first + r, bh);
-  tma_store_commit_and_wait_read();
+  tma_store_commit();
+  if (wait) tma_store_wait_read();
 }
 
 // ---------------------------------------------------------------------------

@@ -334,6 +334,8 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
+static dim3 launch_grid(const Params& p) { return dim3((unsigned)p.ngrid); }
+
 cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(k_fwd_stats, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
@@ -424,18 +426,25 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
 
 // ---------------------------------------------------------------------------
 // Pass 2: reconstruction, normalization and P V (App. A).
+// Work items are (128-row query block, head) pairs, longest blocks first; a CTA
+// takes items blockIdx.x, blockIdx.x + gridDim.x, ... (one item per CTA when the
+// grid covers them all).  Tile counters run on across items, so the next item's Q
+// and first K/V tiles load while the current one finishes.
 // TMEM: score buffers S_b at [128 b, 128 b + 128), b < nbuf (the weights
 // overwrite their scores as MMA operand A); A2 (w^L for O_lerp, or the tf32 lo
 // part of A under 3xTF32) at [128 nbuf, +128); O at cO, O_lerp at cO + d.
 // smem: Q (hi[, lo]) at sm_a; stages {K tile, V^T tile} (hi[, lo] each) fed by
-// the producer warp; per-row pair tables (e_r, e_{r+1}) [K][128] at sm_table.
+// the producer warp; per-row pair tables (e_r, e_{r+1}) [K][128] at sm_table; the
+// output staging tile(s) at sm_ostage (also the W exchange words).
 // ---------------------------------------------------------------------------
-// MMA warp of k_fwd_main: wait for K/V stage of tile kb, S_b = Q K_kb^T into
-// score buffer b = kb % nbuf, commit to bar_s[b].
-__device__ __forceinline__ bool main_issue_s(const Params& p, int kb, uint64_t* bar_full, uint64_t* bar_s,
+__device__ __forceinline__ const uint8_t* stgl_of(const uint8_t* ostg, int d) { return ostg + 128 * d * 4; }
+
+// MMA warp of k_fwd_main: wait for the K/V stage of global tile gt, S_b = Q K^T into
+// score buffer b = gt % nbuf, commit to bar_s[b].
+__device__ __forceinline__ bool main_issue_s(const Params& p, int gt, uint64_t* bar_full, uint64_t* bar_s,
                                              const uint8_t* st0, const uint8_t* sQ, uint32_t tmem, int qtile) {
-  const int NS = p.nstage, s = kb % NS, b = kb % p.nbuf, D = p.d;
-  if (!mbar_wait_warp(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+  const int NS = p.nstage, s = gt % NS, b = gt % p.nbuf, D = p.d;
+  if (!mbar_wait_warp(&bar_full[s], (gt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
   tc_fence_after();
   const uint8_t* sk = st0 + s * p.sm_stage_bytes;
   const uint32_t dcol = tmem + b * 128;
@@ -457,18 +466,19 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   const int qtile = D * 512, vtile = D * 512;
   uint8_t* sQ = sm + p.sm_a;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.sm_bars);
-  uint64_t* bar_q = bars;
-  uint64_t* bar_full = bars + 1;
-  uint64_t* bar_empty = bars + 1 + NS;
-  uint64_t* bar_s = bars + 1 + 2 * NS;       // [2] S_b computed
-  uint64_t* bar_pready = bars + 3 + 2 * NS;  // [2] weights of buffer b stored by every compute warp
-  uint64_t* bar_pv = bars + 5 + 2 * NS;      // P V of a tile complete (A2 free again)
-  uint64_t* bar_done = bars + 6 + 2 * NS;    // every product of the CTA complete (one phase)
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 7 + 2 * NS);
-  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [4][128], aliases Q once all products are done
+  uint64_t* bar_q = bars;                     // Q of the item landed
+  uint64_t* bar_full = bars + 1;              // [NS]
+  uint64_t* bar_empty = bars + 1 + NS;        // [NS]
+  uint64_t* bar_s = bars + 1 + 2 * NS;        // [2] S_b computed
+  uint64_t* bar_pready = bars + 3 + 2 * NS;   // [2] weights of buffer b stored by every compute warp
+  uint64_t* bar_pv = bars + 5 + 2 * NS;       // P V of a tile complete (A2 free again)
+  uint64_t* bar_done = bars + 6 + 2 * NS;     // every product of the item complete
+  uint64_t* bar_qfree = bars + 7 + 2 * NS;    // the item's last S product complete: Q may be reloaded
+  uint64_t* bar_ofree = bars + 8 + 2 * NS;    // O / O_lerp read out of TMEM by every compute warp
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 9 + 2 * NS);
+  uint8_t* ostg = sm + p.sm_ostage;
+  float* xch = reinterpret_cast<float*>(ostg);  // [4][128], written before the staging tiles each item
   const int tid = threadIdx.x, warp = warp_id_uniform();
-  const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
-  const int nkb = qb + 1;
   const bool useA2 = (MODE == 1) || p.x3;
   const int cA2 = 128 * nbuf, cO = cA2 + (useA2 ? 128 : 0), cOL = cO + D;
 
@@ -484,6 +494,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     }
     mbar_init(bar_pv, 1);
     mbar_init(bar_done, 1);
+    mbar_init(bar_qfree, 1);
+    mbar_init(bar_ofree, NCOMP / 32);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -496,153 +508,181 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   const uint32_t tmem = *tslot;
 
   if (warp == PRODUCER_WARP) {
-    mbar_arrive_expect_tx(bar_q, parts * qtile);
-    load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
-    if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int s = kb % NS;
-      if (kb >= NS && !mbar_wait_warp(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-        break;
-      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      mbar_arrive_expect_tx(&bar_full[s], parts * (qtile + vtile));
-      load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
-      load_rows_tile(dst + parts * qtile, &maps.vt, &bar_full[s], 128, D, kb * 128, 0, bh);
-      if (p.x3) {
-        load_rows_tile(dst + qtile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
-        load_rows_tile(dst + parts * qtile + vtile, &maps.vt_lo, &bar_full[s], 128, D, kb * 128, 0, bh);
+    int g = 0, n = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
+      // Q of the previous item is an operand until its last S product completes
+      if (n > 0 && !mbar_wait_warp(bar_qfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+      mbar_arrive_expect_tx(bar_q, parts * qtile);
+      load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
+      if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
+      for (int kb = 0; kb < nkb; ++kb, ++g) {
+        const int s = g % NS;
+        if (g >= NS && !mbar_wait_warp(&bar_empty[s], ((g / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        mbar_arrive_expect_tx(&bar_full[s], parts * (qtile + vtile));
+        load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
+        load_rows_tile(dst + parts * qtile, &maps.vt, &bar_full[s], 128, D, kb * 128, 0, bh);
+        if (p.x3) {
+          load_rows_tile(dst + qtile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
+          load_rows_tile(dst + parts * qtile + vtile, &maps.vt_lo, &bar_full[s], 128, D, kb * 128, 0, bh);
+        }
       }
     }
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
-    bool ok = mbar_wait_warp(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) &&
-              main_issue_s(p, 0, bar_full, bar_s, st0, sQ, tmem, qtile);
-    for (int kb = 0; kb < nkb && ok; ++kb) {
-      const int b = kb % nbuf, s = kb % NS;
-      // S(kb+1) goes to the other buffer, whose last reader P V(kb-1) precedes it in issue order
-      if (nbuf == 2 && kb + 1 < nkb && !main_issue_s(p, kb + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
-      if (!mbar_wait_warp(&bar_pready[b], (kb / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-      tc_fence_after();
-      const uint8_t* vt = st0 + s * p.sm_stage_bytes + parts * qtile;
-      const bool acc = kb > 0;
-      const uint32_t a = tmem + b * 128;
-      if (p.x3) {
-        mma_tmem_smem(tmem + cO, tmem + cA2, vt, D, 128, acc);  // A_lo V_hi (frees A2 first)
-        mma_tmem_smem(tmem + cO, a, vt + vtile, D, 128, true);   // A_hi V_lo
-        mma_tmem_smem(tmem + cO, a, vt, D, 128, true);           // A_hi V_hi
-      } else {
-        if (MODE == 1) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);  // frees A2 first
-        mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);
+    int g = 0, n = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
+      ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) &&
+           main_issue_s(p, g, bar_full, bar_s, st0, sQ, tmem, qtile);
+      if (ok && nkb == 1) mma_commit(bar_qfree);
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+        const int gk = g + kb, b = gk % nbuf, s = gk % NS;
+        // S(kb+1) goes to the other buffer, whose last reader P V(kb-1) precedes it in issue order
+        if (nbuf == 2 && kb + 1 < nkb) {
+          if (!main_issue_s(p, gk + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+          if (kb + 2 == nkb) mma_commit(bar_qfree);
+        }
+        if (!mbar_wait_warp(&bar_pready[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        // the item's first P V overwrites O: the previous item's epilogue must have read it
+        if (kb == 0 && n > 0 && !mbar_wait_warp(bar_ofree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC))
+          break;
+        tc_fence_after();
+        const uint8_t* vt = st0 + s * p.sm_stage_bytes + parts * qtile;
+        const bool acc = kb > 0;
+        const uint32_t a = tmem + b * 128;
+        if (p.x3) {
+          mma_tmem_smem(tmem + cO, tmem + cA2, vt, D, 128, acc);  // A_lo V_hi (frees A2 first)
+          mma_tmem_smem(tmem + cO, a, vt + vtile, D, 128, true);   // A_hi V_lo
+          mma_tmem_smem(tmem + cO, a, vt, D, 128, true);           // A_hi V_hi
+        } else {
+          if (MODE == 1) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);  // frees A2 first
+          mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);
+        }
+        mma_commit(bar_pv);
+        mma_commit(&bar_empty[s]);
+        // one buffer: S(kb+1) overwrites the weights P V(kb) reads, in issue order after it
+        if (nbuf == 1 && kb + 1 < nkb) {
+          if (!main_issue_s(p, gk + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+          if (kb + 2 == nkb) mma_commit(bar_qfree);
+        }
       }
-      mma_commit(bar_pv);
-      mma_commit(&bar_empty[s]);
-      // one buffer: S(kb+1) overwrites the weights P V(kb) reads, in issue order after it
-      if (nbuf == 1 && kb + 1 < nkb && !main_issue_s(p, kb + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+      g += nkb;
+      mma_commit(bar_done);
     }
-    mma_commit(bar_done);
   } else {
     const int row = tid & 127, cg = tid >> 7;
-    const int i = qb * 128 + row;
-    const bool row_ok = i < p.T;
-    const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
-    const float M = row_ok ? p.row_max[rw] : 0.0f;
-    const float m = row_ok ? p.row_min[rw] : 0.0f;
-    const RowGrid g = row_grid(p, M, m);
     const float Kf = (float)Kq;
-    const float sk1 = p.scale * 1.4426950408889634f, sc0 = -M * 1.4426950408889634f;  // softmax, base 2
-    // Pair tables, entry r = (e_r, e_{r+1}), r = 0..K-1, addressed by the float bits
-    // rb = 0x4B000000 + r of the floored position: MinMax keeps one table per row
-    // ([K][128], 1024 bytes per r: rb * 1024 wraps to r * 1024); FWM's grid is the
-    // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r).
-    uint32_t tab;
-    if constexpr (CAL == CAL_FWM) {
-      tab = smem_u32(sm + p.sm_table) - 0x58000000u;
-      if (tid < Kq) *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
-    } else {
-      tab = smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
-      if constexpr (CAL == CAL_MINMAX) {
-        for (int r = cg; r < Kq; r += NCG) {
-          const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
-          *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
-        }
-      }
-    }
-    group_sync(BAR_COMPUTE, NCOMP);
-
-    float Wm = 0.f, Wl = 0.f;
+    int g = 0, n = 0;
     bool failed = false;
-    for (int kb = 0; kb < nkb && !failed; ++kb) {
-      const int b = kb % nbuf;
-      if (!mbar_wait(&bar_s[b], (kb / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
-        failed = true;
-        break;
-      }
-      tc_fence_after();
-      const bool diag = kb == qb;
-#pragma unroll 1
-      for (int cc = 0; cc < 2; ++cc) {
-        const int c = cg * 2 + cc;
-        float v[32], a1[32], a2[32];
-        tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
-        tmem_ld_wait();
-        const int j0 = kb * 128 + c * 32;
-        if (p.debug) fwd_debug_codes(p, v, j0, i, bh, g);
-        if (diag)
-          fwd_chunk<CAL, REC, MODE, true>(v, a1, a2, j0, i, g, Kf, tab, sk1, sc0, Wm, Wl);
-        else
-          fwd_chunk<CAL, REC, MODE, false>(v, a1, a2, j0, i, g, Kf, tab, sk1, sc0, Wm, Wl);
-        if (p.x3) {
-#pragma unroll
-          for (int q = 0; q < 32; ++q) {
-            const float h = tf32_rna(a1[q]);
-            a2[q] = __fsub_rn(a1[q], h);
-            a1[q] = h;
+    for (int item = blockIdx.x; item < p.nitems && !failed; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
+      const int i = qb * 128 + row;
+      const bool row_ok = i < p.T;
+      const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
+      const float M = row_ok ? p.row_max[rw] : 0.0f;
+      const float m = row_ok ? p.row_min[rw] : 0.0f;
+      const RowGrid gr = row_grid(p, M, m);
+      const float sk1 = p.scale * 1.4426950408889634f, sc0 = -M * 1.4426950408889634f;  // softmax, base 2
+      // Pair tables, entry r = (e_r, e_{r+1}), r = 0..K-1, addressed by the float bits
+      // rb = 0x4B000000 + r of the floored position: MinMax keeps one table per row
+      // ([K][128], 1024 bytes per r: rb * 1024 wraps to r * 1024); FWM's grid is the
+      // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r).
+      uint32_t tab;
+      if constexpr (CAL == CAL_FWM) {
+        tab = smem_u32(sm + p.sm_table) - 0x58000000u;
+        if (n == 0 && tid < Kq)
+          *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+      } else {
+        tab = smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
+        if constexpr (CAL == CAL_MINMAX) {
+          for (int r = cg; r < Kq; r += NCG) {
+            const float2 e = make_float2(grid_value(p, gr, r), grid_value(p, gr, r + 1));
+            *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
           }
         }
-        // A2 is still an operand of the previous tile's products until they complete
-        if (cc == 0 && useA2 && kb > 0 &&
-            !mbar_wait(bar_pv, (kb - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
+      }
+      group_sync(BAR_COMPUTE, NCOMP);
+
+      float Wm = 0.f, Wl = 0.f;
+      for (int kb = 0; kb < nkb && !failed; ++kb) {
+        const int gk = g + kb, b = gk % nbuf;
+        if (!mbar_wait(&bar_s[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
           failed = true;
           break;
         }
-        tmem_st32(lane_addr(tmem, b * 128 + c * 32), a1);
-        if (useA2) tmem_st32(lane_addr(tmem, cA2 + c * 32), a2);
+        tc_fence_after();
+        const bool diag = kb == qb;
+#pragma unroll 1
+        for (int cc = 0; cc < 2; ++cc) {
+          const int c = cg * 2 + cc;
+          float v[32], a1[32], a2[32];
+          tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
+          tmem_ld_wait();
+          const int j0 = kb * 128 + c * 32;
+          if (p.debug) fwd_debug_codes(p, v, j0, i, bh, gr);
+          if (diag)
+            fwd_chunk<CAL, REC, MODE, true>(v, a1, a2, j0, i, gr, Kf, tab, sk1, sc0, Wm, Wl);
+          else
+            fwd_chunk<CAL, REC, MODE, false>(v, a1, a2, j0, i, gr, Kf, tab, sk1, sc0, Wm, Wl);
+          if (p.x3) {
+#pragma unroll
+            for (int q = 0; q < 32; ++q) {
+              const float h = tf32_rna(a1[q]);
+              a2[q] = __fsub_rn(a1[q], h);
+              a1[q] = h;
+            }
+          }
+          // A2 is still an operand of the previous tile's products until they complete
+          if (cc == 0 && useA2 && gk > 0 &&
+              !mbar_wait(bar_pv, (gk - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
+            failed = true;
+            break;
+          }
+          tmem_st32(lane_addr(tmem, b * 128 + c * 32), a1);
+          if (useA2) tmem_st32(lane_addr(tmem, cA2 + c * 32), a2);
+        }
+        if (failed) break;
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
+      g += nkb;
+      if (!failed) failed = !mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      failed = group_any(BAR_COMPUTE, NCOMP, failed);
       if (failed) break;
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
-    }
-    // bar_done, not bar_pv: without A2 the compute warps may run more than one tile
-    // ahead of P V, and a parity wait cannot tell phase nkb - 1 from phase nkb - 3
-    if (!failed) failed = !mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP, failed);
-    if (!failed) {
       tc_fence_after();
+      // the previous item's stores have left the staging area before it is written again
+      if (warp < 2) tma_store_wait_read();
+      group_sync(BAR_COMPUTE, NCOMP);
       xch[cg * 128 + row] = Wm;
       xch[(2 + cg) * 128 + row] = Wl;
       group_sync(BAR_COMPUTE, NCOMP);
       const float Wmt = xch[row] + xch[128 + row];
       const float Wlt = xch[256 + row] + xch[384 + row];
+      group_sync(BAR_COMPUTE, NCOMP);  // the exchange words are read before the tiles overwrite them
       if (!p.debug) {
         // O = (sum_j w_j V_j) / W (and O_lerp): each column group scales half of the d
-        // columns into a swizzled tile in the idle stage ring, one TMA store per tile
+        // columns into a swizzled tile, one TMA store per tile
         const float Wout = (MODE == 2) ? Wlt : Wmt;
         const float inv = row_ok ? 1.0f / Wout : 0.0f;
-        uint8_t* stg = sm + p.sm_stage0;
-        uint8_t* stgl = stg + 128 * D * 4;
+        const float invl = row_ok ? 1.0f / Wlt : 0.0f;
+        uint8_t* stgl = ostg + 128 * D * 4;
         for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
           float v[32];
           tmem_ld32(lane_addr(tmem, cO + c), v);
           tmem_ld_wait();
 #pragma unroll
           for (int q = 0; q < 32; ++q) v[q] *= inv;
-          row_to_staged(stg, row, c / 32, v);
-        }
-        if constexpr (MODE == 1) {
-          const float invl = row_ok ? 1.0f / Wlt : 0.0f;
-          for (int c = cg * (D / 2); c < (cg + 1) * (D / 2); c += 32) {
-            float v[32];
+          row_to_staged(ostg, row, c / 32, v);
+          if constexpr (MODE == 1) {
             tmem_ld32(lane_addr(tmem, cOL + c), v);
             tmem_ld_wait();
 #pragma unroll
@@ -650,16 +690,24 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
             row_to_staged(stgl, row, c / 32, v);
           }
         }
+      }
+      // the accumulators go back to the MMA warp for the next item
+      tc_fence_before();
+      __syncwarp();
+      if ((tid & 31) == 0) mbar_arrive(bar_ofree);
+      if (!p.debug) {
         fence_async_smem();
         group_sync(BAR_COMPUTE, NCOMP);
-        if (warp == 0) store_rows_tile_boxed(stg, (MODE == 2) ? &maps.out_lerp : &maps.out, D, 64, qb * 128, bh);
-        if (MODE == 1 && warp == 1) store_rows_tile_boxed(stgl, &maps.out_lerp, D, 64, qb * 128, bh);
+        if (warp == 0)
+          store_rows_tile_boxed(ostg, (MODE == 2) ? &maps.out_lerp : &maps.out, D, 64, qb * 128, bh, false);
+        if (MODE == 1 && warp == 1) store_rows_tile_boxed(stgl_of(ostg, D), &maps.out_lerp, D, 64, qb * 128, bh, false);
         if (row_ok && cg == 0) {
           if (MODE != 2) p.W[rw] = Wmt;
           if (MODE != 0 && p.W_lerp) p.W_lerp[rw] = Wlt;
         }
       }
     }
+    if (warp < 2) tma_store_wait_all();
   }
   tc_fence_before();
   __syncthreads();
@@ -671,7 +719,7 @@ static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_byt
   auto kern = k_fwd_main<CAL, REC, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<dim3(p.nqb, p.BH), NTHR, smem_bytes, s>>>(maps, p);
+  kern<<<launch_grid(p), NTHR, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
 }
 

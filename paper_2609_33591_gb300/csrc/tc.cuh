@@ -159,13 +159,31 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void*
       "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
       : "memory");
 }
-__device__ __forceinline__ void tma_store_commit_and_wait_read() {
+__device__ __forceinline__ void tma_store_commit() {
   asm volatile(
       "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
-      "@e cp.async.bulk.commit_group;\n\t"
+      "@e cp.async.bulk.commit_group;\n\t}" ::
+          : "memory");
+}
+// Waits until this warp's committed stores have read their shared-memory source.
+__device__ __forceinline__ void tma_store_wait_read() {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
       "@e cp.async.bulk.wait_group.read 0;\n\t}" ::
           : "memory");
   __syncwarp();
+}
+// Waits until this warp's committed stores are complete.
+__device__ __forceinline__ void tma_store_wait_all() {
+  asm volatile(
+      "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+      "@e cp.async.bulk.wait_group 0;\n\t}" ::
+          : "memory");
+  __syncwarp();
+}
+__device__ __forceinline__ void tma_store_commit_and_wait_read() {
+  tma_store_commit();
+  tma_store_wait_read();
 }
 // 1-D bulk copy global -> shared (both addresses 16-byte aligned, bytes a
 // multiple of 16), completion counted on an mbarrier (warp-collective).

@@ -113,3 +113,11 @@ def test_value_ones_rows_sum_to_one():
     for cfg in (_cfg(MM, NE, WE, FU), _cfg(FW, NE, PR, FU), _cfg(SM, LE, WE, FU)):
         g = parity.run_gpu(Q, K, V, dO, cfg, X3, want_bins=False, want_bwd=False)
         assert np.max(np.abs(g["O"] - 1.0)) <= 2 * T * 2.0 ** -24
+
+
+@pytest.mark.parametrize("c,r,s", [(FW, NE, PR), (MM, LE, WE), (SM, LE, WE)])
+def test_many_items_per_cta(c, r, s):
+    """More (block, head) items than SMs, so CTAs that loop over items (tile counters
+    and barrier phases running on across items) are exercised; ragged T."""
+    Q, K, V, dO = make_qkvdo(4, 40, 200, 64, seed=11)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, FU, 4), TF)
