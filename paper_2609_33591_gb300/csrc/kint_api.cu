@@ -212,12 +212,17 @@ constexpr int kOneCtaPerSm = 117 * 1024;
 
 int plan_stats(Params& p) {
   const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
+  p.nitems = p.nqb * p.BH;
   p.sm_a = 0;
   p.sm_stage0 = parts * tile;
   p.sm_stage_bytes = parts * tile;
   p.nstage = 2;
-  p.sm_rows = p.sm_a;  // the 6 x 128 exchange words reuse the Q tile after the last product
-  return finish_plan(p, p.sm_stage0 + p.nstage * p.sm_stage_bytes, 5 + 2 * p.nstage);
+  p.sm_rows = p.sm_stage0 + p.nstage * p.sm_stage_bytes;  // the 6 x 128 exchange words
+  const int total = finish_plan(p, p.sm_rows + 6 * 128 * 4, 6 + 2 * p.nstage);
+  // CTAs loop over the items, as many as are resident at once (two per SM when they fit)
+  const int per_sm = (2 * total <= 228 * 1024) ? 2 : 1;
+  p.ngrid = std::min(p.nitems, per_sm * num_sms());
+  return total;
 }
 
 // mode: PV_MAIN / PV_MAIN_LERP / PV_LERP.  Picks the TMEM score double-buffering

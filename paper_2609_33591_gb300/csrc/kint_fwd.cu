@@ -188,6 +188,8 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
   }
 }
 
+static dim3 launch_grid(const Params& p) { return dim3((unsigned)p.ngrid); }
+
 __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, tile = D * 512, parts = p.x3 ? 2 : 1, NS = p.nstage;
@@ -198,11 +200,10 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   uint64_t* bar_empty = bars + 1 + NS;
   uint64_t* bar_s = bars + 1 + 2 * NS;      // [2] S_b computed
   uint64_t* bar_sfree = bars + 3 + 2 * NS;  // [2] S_b read by every compute warp
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 5 + 2 * NS);
-  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [6][128], aliases Q once all products are done
+  uint64_t* bar_qfree = bars + 5 + 2 * NS;  // the item's last product complete: Q may be reloaded
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 6 + 2 * NS);
+  float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [6][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
-  const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
-  const int nkb = qb + 1;
 
   if (tid == 0) {
     mbar_init(bar_q, 1);
@@ -214,6 +215,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
       mbar_init(&bar_s[b], 1);
       mbar_init(&bar_sfree[b], NCOMP / 32);
     }
+    mbar_init(bar_qfree, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -225,72 +227,97 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
+  // Work items as in pass 2: (query block, head), longest first, strided over the grid.
   if (warp == PRODUCER_WARP) {
-    mbar_arrive_expect_tx(bar_q, parts * tile);
-    load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
-    if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int s = kb % NS;
-      if (kb >= NS && !mbar_wait_warp(&bar_empty[s], ((kb / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-        break;
-      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      mbar_arrive_expect_tx(&bar_full[s], parts * tile);
-      load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
-      if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
+    int g = 0, n = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
+      if (n > 0 && !mbar_wait_warp(bar_qfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+      mbar_arrive_expect_tx(bar_q, parts * tile);
+      load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
+      if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
+      for (int kb = 0; kb < nkb; ++kb, ++g) {
+        const int s = g % NS;
+        if (g >= NS && !mbar_wait_warp(&bar_empty[s], ((g / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        mbar_arrive_expect_tx(&bar_full[s], parts * tile);
+        load_rows_tile(dst, &maps.k, &bar_full[s], D, 128, 0, kb * 128, bh);
+        if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
+      }
     }
   } else if (warp == MMA_WARP) {
-    bool ok = mbar_wait_warp(bar_q, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-    for (int kb = 0; kb < nkb && ok; ++kb) {
-      const int s = kb % NS, b = kb & 1;
-      // S_b was last read in tile kb - 2
-      if (kb >= 2 && !mbar_wait_warp(&bar_sfree[b], ((kb >> 1) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC))
-        break;
-      if (!mbar_wait_warp(&bar_full[s], (kb / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) break;
-      tc_fence_after();
-      const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      const uint32_t dcol = tmem + b * 128;
-      if (p.x3) {
-        mma_smem_smem(dcol, sQ + tile, sk, 128, D, false);  // Q_lo K_hi
-        mma_smem_smem(dcol, sQ, sk + tile, 128, D, true);   // Q_hi K_lo
-        mma_smem_smem(dcol, sQ, sk, 128, D, true);          // Q_hi K_hi
-      } else {
-        mma_smem_smem(dcol, sQ, sk, 128, D, false);
+    int g = 0, n = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
+      ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+      for (int kb = 0; kb < nkb && ok; ++kb) {
+        const int gk = g + kb, s = gk % NS, b = gk & 1;
+        // S_b was last read two tiles ago
+        if (gk >= 2 && !mbar_wait_warp(&bar_sfree[b], ((gk >> 1) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
+          ok = false;
+          break;
+        }
+        if (!mbar_wait_warp(&bar_full[s], (gk / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint8_t* sk = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        const uint32_t dcol = tmem + b * 128;
+        if (p.x3) {
+          mma_smem_smem(dcol, sQ + tile, sk, 128, D, false);  // Q_lo K_hi
+          mma_smem_smem(dcol, sQ, sk + tile, 128, D, true);   // Q_hi K_lo
+          mma_smem_smem(dcol, sQ, sk, 128, D, true);          // Q_hi K_hi
+        } else {
+          mma_smem_smem(dcol, sQ, sk, 128, D, false);
+        }
+        mma_commit(&bar_s[b]);
+        mma_commit(&bar_empty[s]);
+        if (kb + 1 == nkb) mma_commit(bar_qfree);
       }
-      mma_commit(&bar_s[b]);
-      mma_commit(&bar_empty[s]);
+      g += nkb;
     }
   } else {
     const int row = tid & 127, cg = tid >> 7;
-    const int i = qb * 128 + row;
-    float M = -FLT_MAX, m = FLT_MAX;
-    int amax = 0, amin = 0, nmax = 0, nmin = 0;
+    int g = 0;
     bool failed = false;
-    for (int kb = 0; kb < nkb; ++kb) {
-      const int b = kb & 1;
-      if (!mbar_wait(&bar_s[b], (kb >> 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
-        failed = true;
-        break;
-      }
-      tc_fence_after();
-      const bool diag = kb == qb;
+    for (int item = blockIdx.x; item < p.nitems && !failed; item += gridDim.x) {
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
+      const int i = qb * 128 + row;
+      float M = -FLT_MAX, m = FLT_MAX;
+      int amax = 0, amin = 0, nmax = 0, nmin = 0;
+      for (int kb = 0; kb < nkb; ++kb) {
+        const int gk = g + kb, b = gk & 1;
+        if (!mbar_wait(&bar_s[b], (gk >> 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
+          failed = true;
+          break;
+        }
+        tc_fence_after();
+        const bool diag = kb == qb;
 #pragma unroll 1
-      for (int cc = 0; cc < 2; ++cc) {
-        const int c = cg * 2 + cc;
-        float v[32];
-        tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
-        tmem_ld_wait();
-        const int j0 = kb * 128 + c * 32;
-        if (diag)
-          stats_chunk<true>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
-        else
-          stats_chunk<false>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+        for (int cc = 0; cc < 2; ++cc) {
+          const int c = cg * 2 + cc;
+          float v[32];
+          tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
+          tmem_ld_wait();
+          const int j0 = kb * 128 + c * 32;
+          if (diag)
+            stats_chunk<true>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+          else
+            stats_chunk<false>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if ((tid & 31) == 0) mbar_arrive(&bar_sfree[b]);
       }
-      tc_fence_before();
-      __syncwarp();
-      if ((tid & 31) == 0) mbar_arrive(&bar_sfree[b]);
-    }
-    failed = group_any(BAR_COMPUTE, NCOMP, failed);
-    if (!failed) {
+      g += nkb;
+      failed = group_any(BAR_COMPUTE, NCOMP, failed);
+      if (failed) break;
       // combine the two column halves of each row
       if (cg == 1) {
         xch[0 * 128 + row] = M;
@@ -327,6 +354,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
         p.n_max[rw] = nmax;
         p.n_min[rw] = nmin;
       }
+      group_sync(BAR_COMPUTE, NCOMP);  // the exchange words are read before the next item writes them
     }
   }
   tc_fence_before();
@@ -334,12 +362,10 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
-static dim3 launch_grid(const Params& p) { return dim3((unsigned)p.ngrid); }
-
 cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(k_fwd_stats, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  k_fwd_stats<<<dim3(p.nqb, p.BH), NTHR, smem_bytes, s>>>(maps, p);
+  k_fwd_stats<<<launch_grid(p), NTHR, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
 }
 
