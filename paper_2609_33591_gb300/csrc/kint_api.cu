@@ -272,15 +272,21 @@ int plan_dq(Params& p) {
   // next to the K/V stages and the rows are read from global memory.
   p.ops_smem = (!p.x3 && p.d == 64) ? 1 : 0;
   p.nbuf = (2 * dp + 256 + p.d <= 512) ? 2 : 1;
+  p.nitems = p.nqb * p.BH;
   p.sm_a = 0;
   p.sm_stage0 = p.ops_smem ? 2 * 128 * p.d * 4 : 0;
   p.sm_stage_bytes = 3 * parts * ktile;
+  // One item per CTA (the kernel can loop over items, but with its own dQ staging tile
+  // the stage ring drops to two stages, which measured slower), dQ staged in the idle
+  // stage ring at the end.
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
+    p.sm_ostage = p.sm_stage0;
     const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 7), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
+      p.ngrid = p.nitems;
       return total;
     }
   }

@@ -133,13 +133,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   uint64_t* bar_sfull = bars + 2 * NS;     // [2]
   uint64_t* bar_pready = bars + 2 * NS + 2;  // [2]
   uint64_t* bar_done = bars + 2 * NS + 4;
-  uint64_t* bar_ops = bars + 2 * NS + 5;  // Q / dO rows stored in TMEM by every compute warp
-  uint64_t* bar_stg = bars + 2 * NS + 6;  // Q / dO tiles staged in smem by TMA
+  uint64_t* bar_ops = bars + 2 * NS + 5;  // Q / dO rows stored in TMEM by every compute warp (per item)
+  uint64_t* bar_stg = bars + 2 * NS + 6;  // Q / dO tiles staged in smem by TMA (per item)
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 7);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
+  uint8_t* ostg = sm + p.sm_ostage;                        // dQ staging tile
   const int tid = threadIdx.x, warp = warp_id_uniform();
-  const int bh = blockIdx.y, qb = p.nqb - 1 - blockIdx.x;
-  const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
   constexpr int W = BT / NCG;  // key columns per thread per tile
   const int dp = D * parts;
   const int cQ = 0, cdO = dp, cSG0 = 2 * dp, cdQ = cSG0 + 128 * nbuf;
@@ -167,243 +166,273 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   tc_fence_after();
   const uint32_t tmem = *tslot;
 
-  // ---- compute-thread set-up: operands Q / dO into TMEM, row constants, grid table ----
-  const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
-  const int i = qb * 128 + row;
-  const bool row_ok = i < p.T;
-  const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
-  float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
-  int nmax = 1, nmin = 1, amax = 0, amin = 0;
-  RowGrid g{};
-  if (warp < NCOMP / 32) {
-    // operand rows into TMEM (column group 0 takes Q, group 1 takes dO), handed to the
-    // MMA warp through bar_ops; the rest of the set-up runs under the first products.
-    // TF32 at d = 64: from tiles the producer staged in smem; otherwise from global rows.
-    if (p.ops_smem) {
-      if (mbar_wait(bar_stg, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-        staged_row_to_tmem(tmem, cg == 0 ? cQ : cdO, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
-    } else {
-      row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
-                  p.x3 != 0);
-    }
-    tmem_st_wait();
-    tc_fence_before();
-    __syncwarp();
-    if ((tid & 31) == 0) mbar_arrive(bar_ops);
-    if (row_ok) {
-      M = p.row_max[rw];
-      m = p.row_min[rw];
-      Wf = p.W[rw];
-      nmax = p.n_max[rw];
-      nmin = p.n_min[rw];
-      amax = p.arg_max[rw];
-      amin = p.arg_min[rw];
-      Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
-    }
-    const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
-    Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
-    g = row_grid(p, M, m);
-    if constexpr (CAL == CAL_FWM) {
-      if (tid < Kq)
-        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
-    } else if constexpr (CAL == CAL_MINMAX) {
-      for (int r = cg; r < Kq; r += NCG) {
-        const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
-        *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
-        if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
-      }
-    }
-  }
-
   if (warp == PRODUCER_WARP) {
-    if (p.ops_smem) {
-      mbar_arrive_expect_tx(bar_stg, 2 * 128 * D * 4);
-      load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb * 128, bh);
-      load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb * 128, bh);
-    }
-    for (int kt = 0; kt < nkt; ++kt) {
-      const int s = kt % NS;
-      if (kt >= NS &&
-          !mbar_wait_warp(&bar_empty[s], ((kt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-        break;
-      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      uint64_t* b = &bar_full[s];
-      mbar_arrive_expect_tx(b, 3 * parts * ktile);
-      load_rows_tile(dst, &maps.k, b, D, BT, 0, kt * BT, bh);
-      load_rows_tile(dst + parts * ktile, &maps.v, b, D, BT, 0, kt * BT, bh);
-      load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
-      if (p.x3) {
-        load_rows_tile(dst + ktile, &maps.k_lo, b, D, BT, 0, kt * BT, bh);
-        load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BT, 0, kt * BT, bh);
-        load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
+    int gt = 0, n = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
+      const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
+      if (p.ops_smem) {
+        // the staging tiles of the previous item have been copied into TMEM
+        if (n > 0 && !mbar_wait_warp(bar_ops, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        mbar_arrive_expect_tx(bar_stg, 2 * 128 * D * 4);
+        load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb * 128, bh);
+        load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb * 128, bh);
+      }
+      for (int kt = 0; kt < nkt; ++kt, ++gt) {
+        const int s = gt % NS;
+        if (gt >= NS &&
+            !mbar_wait_warp(&bar_empty[s], ((gt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        uint64_t* b = &bar_full[s];
+        mbar_arrive_expect_tx(b, 3 * parts * ktile);
+        load_rows_tile(dst, &maps.k, b, D, BT, 0, kt * BT, bh);
+        load_rows_tile(dst + parts * ktile, &maps.v, b, D, BT, 0, kt * BT, bh);
+        load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
+        if (p.x3) {
+          load_rows_tile(dst + ktile, &maps.k_lo, b, D, BT, 0, kt * BT, bh);
+          load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BT, 0, kt * BT, bh);
+          load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
+        }
       }
     }
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + cSG0;
-    bool ok = mbar_wait_warp(bar_ops, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
-    if (ok) tc_fence_after();
-    ok = ok && dq_issue_sg(p, 0, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-    for (int kt = 0; kt < nkt && ok; ++kt) {
-      const int b = kt % nbuf, s = kt % NS;
-      if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-      if (!ok) break;
-      if (!mbar_wait_warp(&bar_pready[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-      tc_fence_after();
-      const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
-      const uint32_t cS = tmem + cSG0 + 128 * b, cG = cS + 64;
-      const bool acc = kt > 0;
-      if (p.x3) {
-        mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);           // dS_hi K_hi
-        mma_tmem_smem(tmem + cdQ, cS, skt + ktile, D, BT, true);  // dS_hi K_lo
-        mma_tmem_smem(tmem + cdQ, cG, skt, D, BT, true);          // dS_lo K_hi
-      } else {
-        mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
+    int gt = 0, n = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+      const int qb = p.nqb - 1 - item / p.BH;
+      const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
+      // Q / dO of the item in TMEM (the compute warps copy them only after reading the
+      // previous item's dQ, so the first dQ product below may overwrite it)
+      ok = mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
+      if (ok) tc_fence_after();
+      ok = ok && dq_issue_sg(p, gt, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+      for (int kt = 0; kt < nkt && ok; ++kt) {
+        const int gk = gt + kt, b = gk % nbuf, s = gk % NS;
+        if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, gk + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+        if (!ok) break;
+        if (!mbar_wait_warp(&bar_pready[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint8_t* skt = sm + p.sm_stage0 + s * p.sm_stage_bytes + 2 * parts * ktile;
+        const uint32_t cS = tmem + cSG0 + 128 * b, cG = cS + 64;
+        const bool acc = kt > 0;
+        if (p.x3) {
+          mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);           // dS_hi K_hi
+          mma_tmem_smem(tmem + cdQ, cS, skt + ktile, D, BT, true);  // dS_hi K_lo
+          mma_tmem_smem(tmem + cdQ, cG, skt, D, BT, true);          // dS_lo K_hi
+        } else {
+          mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
+        }
+        mma_commit(&bar_empty[s]);
+        if (nbuf == 1 && kt + 1 < nkt)  // in order after the product reading S_0
+          ok = dq_issue_sg(p, gk + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
       }
-      mma_commit(&bar_empty[s]);
-      if (nbuf == 1 && kt + 1 < nkt)  // in order after the product reading S_0
-        ok = dq_issue_sg(p, kt + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+      gt += nkt;
+      mma_commit(bar_done);
     }
-    mma_commit(bar_done);
   } else {
-    // ---- compute warps ----
-    group_sync(BAR_COMPUTE, NCOMP);  // the grid table
-    const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
-    const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
-    const float invWf = 1.0f / Wf;
-    const float sk1 = p.scale * kLog2e, sc0 = -M * kLog2e;
-    const float Kf = (float)Kq, fk = 1.0f / Kf;
-    const uint32_t tab = (CAL == CAL_FWM) ? smem_u32(sm + p.sm_table) - 0x58000000u
-                                          : smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
-    const bool minmax = CAL == CAL_MINMAX;
-    const bool track = FULLG && CAL != CAL_SOFTMAX && row_ok && !g.nogrid && (nmax > 1 || (minmax && nmin > 1));
-    float* tie_max = p.tie_acc + rw * D;
-    float* tie_min = p.tie_acc + ((size_t)p.BH * p.T + rw) * D;
-    if (track && cg == 0) {
-      for (int k = 0; k < D; ++k) tie_max[k] = tie_min[k] = 0.f;
-      atomicOr(p.tileflags + (size_t)bh * p.nqt + i / BT, 1);
-    }
-    group_sync(BAR_COMPUTE, NCOMP);  // every column group of a row may add to its tie sums
-    float own = 0.f, cm = 0.f;
+    // ---- compute warps: items one after the other ----
+    const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
+    int gt = 0, n = 0;
     bool failed = false;
-    for (int kt = 0; kt < nkt; ++kt) {
-      const int b = kt % nbuf;
-      const bool ok = mbar_wait(&bar_sfull[b], (kt / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-      if (!ok) {
-        failed = true;
-        break;
-      }
-      tc_fence_after();
-      const int cS = cSG0 + 128 * b + cg * W, cG = cS + 64;
-      float sv[W], gv[W], out[W];
-      tmem_ldw<W>(lane_addr(tmem, cS), sv);
-      tmem_ldw<W>(lane_addr(tmem, cG), gv);
-      tmem_ld_wait();
-      const int j0 = kt * BT + cg * W;
-      if (j0 + W - 1 > qb * 128)
-        dq_chunk<CAL, FULLG, true, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
-                                      sc0, invWf, own, cm);
-      else
-        dq_chunk<CAL, FULLG, false, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab,
-                                       sk1, sc0, invWf, own, cm);
-      if (__any_sync(0xffffffffu, track)) {
-        // rare: tied extrema, the tie set is found by equality on the recomputed scores
-        uint32_t mk_max = 0, mk_min = 0;
-#pragma unroll
-        for (int jj = 0; jj < W; ++jj) {
-          const float s = __fmul_rn(sv[jj], p.scale);
-          const bool okj = track && j0 + jj <= i;
-          mk_max |= (okj && nmax > 1 && s == M) ? (1u << jj) : 0u;
-          mk_min |= (okj && minmax && nmin > 1 && s == m) ? (1u << jj) : 0u;
+    for (int item = blockIdx.x; item < p.nitems && !failed; item += gridDim.x, ++n) {
+      // ---- set-up: operands Q / dO into TMEM, row constants, grid table ----
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
+      const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
+      const int i = qb * 128 + row;
+      const bool row_ok = i < p.T;
+      const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
+      float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
+      int nmax = 1, nmin = 1, amax = 0, amin = 0;
+      RowGrid g{};
+      {
+        // operand rows into TMEM (column group 0 takes Q, group 1 takes dO), handed to the
+        // MMA warp through bar_ops; the rest of the set-up runs under the first products.
+        // TF32 at d = 64: from tiles the producer staged in smem; otherwise from global rows.
+        if (p.ops_smem) {
+          if (mbar_wait(bar_stg, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+            staged_row_to_tmem(tmem, cg == 0 ? cQ : cdO, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
+        } else {
+          row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
+                      p.x3 != 0);
         }
-        add_tied_keys(mk_max, tie_max, p.K + ((size_t)bh * p.T + j0) * D, D);
-        add_tied_keys(mk_min, tie_min, p.K + ((size_t)bh * p.T + j0) * D, D);
-      }
-      if (p.x3) {
-        float lo[W];
-#pragma unroll
-        for (int q = 0; q < W; ++q) {
-          const float h = tf32_rna(out[q]);
-          lo[q] = __fsub_rn(out[q], h);
-          out[q] = h;
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if ((tid & 31) == 0) mbar_arrive(bar_ops);
+        if (row_ok) {
+          M = p.row_max[rw];
+          m = p.row_min[rw];
+          Wf = p.W[rw];
+          nmax = p.n_max[rw];
+          nmin = p.n_min[rw];
+          amax = p.arg_max[rw];
+          amin = p.arg_min[rw];
+          Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
         }
-        tmem_stw<W>(lane_addr(tmem, cG), lo);
-      }
-      tmem_stw<W>(lane_addr(tmem, cS), out);
-      tmem_st_wait();
-      tc_fence_before();
-      __syncwarp();
-      if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
-    }
-    const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
-    if (!failed) {
-      tc_fence_after();
-      xch[cg * 128 + row] = own;
-      xch[(NCG + cg) * 128 + row] = cm;
-      group_sync(BAR_COMPUTE, NCOMP);
-      float own_t = 0.f, cm_t = 0.f;
-#pragma unroll
-      for (int q = 0; q < NCG; ++q) {
-        own_t += xch[q * 128 + row];
-        cm_t += xch[(NCG + q) * 128 + row];
-      }
-      // Eq. (full): c_m = sum gamma dw/dm; c_M = -sum gamma Delta - c_m (Delta + dw/dM + dw/dm = 0);
-      // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys.
-      const bool full = FULLG && CAL != CAL_SOFTMAX && !g.nogrid;
-      const float cmv = (full && minmax) ? cm_t : 0.f;
-      const float cMv = full ? (-own_t - cmv) : 0.f;
-      const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
-      const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
-      const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
-      // dQ rows into a swizzled tile in the idle stage ring, then one TMA store
-      uint8_t* stg = sm + p.sm_stage0;
-      for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
-        // the arg-extremum key rows first (all loads in flight before the TMEM read)
-        float4 km[8], kn[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          km[q] = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
-                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-          kn[q] = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
-                                             : make_float4(0.f, 0.f, 0.f, 0.f);
+        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
+        Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
+        g = row_grid(p, M, m);
+        if constexpr (CAL == CAL_FWM) {
+          if (tid < Kq)
+            *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+        } else if constexpr (CAL == CAL_MINMAX) {
+          for (int r = cg; r < Kq; r += NCG) {
+            const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
+            *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
+            if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
+          }
         }
-        float v[32];
-        tmem_ld32(lane_addr(tmem, cdQ + c), v);
+      }
+      group_sync(BAR_COMPUTE, NCOMP);  // the grid table
+      const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
+      const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
+      const float invWf = 1.0f / Wf;
+      const float sk1 = p.scale * kLog2e, sc0 = -M * kLog2e;
+      const float Kf = (float)Kq, fk = 1.0f / Kf;
+      const uint32_t tab = (CAL == CAL_FWM) ? smem_u32(sm + p.sm_table) - 0x58000000u
+                                            : smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
+      const bool minmax = CAL == CAL_MINMAX;
+      const bool track = FULLG && CAL != CAL_SOFTMAX && row_ok && !g.nogrid && (nmax > 1 || (minmax && nmin > 1));
+      float* tie_max = p.tie_acc + rw * D;
+      float* tie_min = p.tie_acc + ((size_t)p.BH * p.T + rw) * D;
+      if (track && cg == 0) {
+        for (int k = 0; k < D; ++k) tie_max[k] = tie_min[k] = 0.f;
+        atomicOr(p.tileflags + (size_t)bh * p.nqt + i / BT, 1);
+      }
+      group_sync(BAR_COMPUTE, NCOMP);  // every column group of a row may add to its tie sums
+      float own = 0.f, cm = 0.f;
+      for (int kt = 0; kt < nkt; ++kt) {
+        const int gk = gt + kt, b = gk % nbuf;
+        const bool ok = mbar_wait(&bar_sfull[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+        if (!ok) {
+          failed = true;
+          break;
+        }
+        tc_fence_after();
+        const int cS = cSG0 + 128 * b + cg * W, cG = cS + 64;
+        float sv[W], gv[W], out[W];
+        tmem_ldw<W>(lane_addr(tmem, cS), sv);
+        tmem_ldw<W>(lane_addr(tmem, cG), gv);
         tmem_ld_wait();
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          v[4 * q] = __fmaf_rn(cmn, kn[q].x, __fmaf_rn(cMn, km[q].x, v[4 * q])) * p.scale;
-          v[4 * q + 1] = __fmaf_rn(cmn, kn[q].y, __fmaf_rn(cMn, km[q].y, v[4 * q + 1])) * p.scale;
-          v[4 * q + 2] = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
-          v[4 * q + 3] = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
+        const int j0 = kt * BT + cg * W;
+        if (j0 + W - 1 > qb * 128)
+          dq_chunk<CAL, FULLG, true, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
+                                        sc0, invWf, own, cm);
+        else
+          dq_chunk<CAL, FULLG, false, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab,
+                                         sk1, sc0, invWf, own, cm);
+        if (__any_sync(0xffffffffu, track)) {
+          // rare: tied extrema, the tie set is found by equality on the recomputed scores
+          uint32_t mk_max = 0, mk_min = 0;
+  #pragma unroll
+          for (int jj = 0; jj < W; ++jj) {
+            const float s = __fmul_rn(sv[jj], p.scale);
+            const bool okj = track && j0 + jj <= i;
+            mk_max |= (okj && nmax > 1 && s == M) ? (1u << jj) : 0u;
+            mk_min |= (okj && minmax && nmin > 1 && s == m) ? (1u << jj) : 0u;
+          }
+          add_tied_keys(mk_max, tie_max, p.K + ((size_t)bh * p.T + j0) * D, D);
+          add_tied_keys(mk_min, tie_min, p.K + ((size_t)bh * p.T + j0) * D, D);
         }
-        row_to_staged(stg, row, c / 32, v);
+        if (p.x3) {
+          float lo[W];
+  #pragma unroll
+          for (int q = 0; q < W; ++q) {
+            const float h = tf32_rna(out[q]);
+            lo[q] = __fsub_rn(out[q], h);
+            out[q] = h;
+          }
+          tmem_stw<W>(lane_addr(tmem, cG), lo);
+        }
+        tmem_stw<W>(lane_addr(tmem, cS), out);
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
-      fence_async_smem();
-      group_sync(BAR_COMPUTE, NCOMP);
-      if (warp == 0) store_rows_tile_boxed(stg, &maps.dq, D, 64, qb * 128, bh);
-      if (row_ok && cg == 0) {
-        RowRec r;
-        r.c0 = g.c0;
-        r.k1 = g.k1;
-        r.inv_h = g.inv_h;
-        r.invWf = invWf;
-        r.ga = ga;
-        r.gb = gb;
-        r.cMn = full ? cMn : 0.f;
-        r.cmn = (full && minmax) ? cmn : 0.f;
-        r.amax = (nmax == 1) ? amax : -1;
-        r.amin = (nmin == 1) ? amin : -1;
-        r.flags = (g.nogrid ? REC_NOGRID : 0) | (nmax > 1 ? REC_TIEMAX : 0) | (nmin > 1 ? REC_TIEMIN : 0);
-        r.pad = 0;
-        r.M = M;
-        r.m = m;
-        r.sk1 = sk1;
-        r.sc0 = sc0;
-        reinterpret_cast<RowRec*>(p.rec)[rw] = r;
+      gt += nkt;
+      const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+      if (!failed) {
+        tc_fence_after();
+        if (warp == 0) tma_store_wait_read();  // the previous item's dQ tile has left the staging area
+        xch[cg * 128 + row] = own;
+        xch[(NCG + cg) * 128 + row] = cm;
+        group_sync(BAR_COMPUTE, NCOMP);
+        float own_t = 0.f, cm_t = 0.f;
+  #pragma unroll
+        for (int q = 0; q < NCG; ++q) {
+          own_t += xch[q * 128 + row];
+          cm_t += xch[(NCG + q) * 128 + row];
+        }
+        // Eq. (full): c_m = sum gamma dw/dm; c_M = -sum gamma Delta - c_m (Delta + dw/dM + dw/dm = 0);
+        // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys.
+        const bool full = FULLG && CAL != CAL_SOFTMAX && !g.nogrid;
+        const float cmv = (full && minmax) ? cm_t : 0.f;
+        const float cMv = full ? (-own_t - cmv) : 0.f;
+        const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
+        const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
+        const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
+        // dQ rows into the swizzled staging tile (its previous store has been read out),
+        // then one TMA store
+        uint8_t* stg = ostg;
+        for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
+          // the arg-extremum key rows first (all loads in flight before the TMEM read)
+          float4 km[8], kn[8];
+  #pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            km[q] = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+            kn[q] = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
+                                               : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+          float v[32];
+          tmem_ld32(lane_addr(tmem, cdQ + c), v);
+          tmem_ld_wait();
+  #pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            v[4 * q] = __fmaf_rn(cmn, kn[q].x, __fmaf_rn(cMn, km[q].x, v[4 * q])) * p.scale;
+            v[4 * q + 1] = __fmaf_rn(cmn, kn[q].y, __fmaf_rn(cMn, km[q].y, v[4 * q + 1])) * p.scale;
+            v[4 * q + 2] = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
+            v[4 * q + 3] = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
+          }
+          row_to_staged(stg, row, c / 32, v);
+        }
+        fence_async_smem();
+        group_sync(BAR_COMPUTE, NCOMP);
+        if (warp == 0) store_rows_tile_boxed(stg, &maps.dq, D, 64, qb * 128, bh, false);
+        if (row_ok && cg == 0) {
+          RowRec r;
+          r.c0 = g.c0;
+          r.k1 = g.k1;
+          r.inv_h = g.inv_h;
+          r.invWf = invWf;
+          r.ga = ga;
+          r.gb = gb;
+          r.cMn = full ? cMn : 0.f;
+          r.cmn = (full && minmax) ? cmn : 0.f;
+          r.amax = (nmax == 1) ? amax : -1;
+          r.amin = (nmin == 1) ? amin : -1;
+          r.flags = (g.nogrid ? REC_NOGRID : 0) | (nmax > 1 ? REC_TIEMAX : 0) | (nmin > 1 ? REC_TIEMIN : 0);
+          r.pad = 0;
+          r.M = M;
+          r.m = m;
+          r.sk1 = sk1;
+          r.sc0 = sc0;
+          reinterpret_cast<RowRec*>(p.rec)[rw] = r;
+        }
       }
     }
+    if (warp == 0) tma_store_wait_all();
     tc_fence_before();
   }
   __syncthreads();
@@ -769,7 +798,7 @@ static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p,
 }
 
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
-  const dim3 grid(p.nqb, p.BH);
+  const dim3 grid((unsigned)p.ngrid);
   const bool full = p.grad == 0;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX)

@@ -307,30 +307,35 @@ __device__ __forceinline__ void row_to_tmem_part(uint32_t tmem_base, int col, co
                                                  int c0, bool split) {
   const bool in = row < T;
   const float4* src = reinterpret_cast<const float4*>(X + (size_t)row * d + c0);
-  float v[N];
+  float hi[N], lo[N];
 #pragma unroll
   for (int q = 0; q < N / 4; ++q) {
     const float4 x = in ? __ldg(src + q) : make_float4(0.f, 0.f, 0.f, 0.f);
-    v[4 * q] = x.x;
-    v[4 * q + 1] = x.y;
-    v[4 * q + 2] = x.z;
-    v[4 * q + 3] = x.w;
+    hi[4 * q] = x.x;
+    hi[4 * q + 1] = x.y;
+    hi[4 * q + 2] = x.z;
+    hi[4 * q + 3] = x.w;
   }
+  if (split) {
 #pragma unroll
-  for (int c = 0; c < N; c += 32) {
-    float hi[32], lo[32];
-#pragma unroll
-    for (int q = 0; q < 32; ++q) {
-      hi[q] = v[c + q];
-      if (split) {
-        const float h = tf32_rna(hi[q]);
-        lo[q] = __fsub_rn(hi[q], h);
-        hi[q] = h;
-      }
+    for (int q = 0; q < N; ++q) {
+      const float h = tf32_rna(hi[q]);
+      lo[q] = __fsub_rn(hi[q], h);
+      hi[q] = h;
     }
-    if (split) tmem_st32(lane_addr(tmem_base, col + d + c0 + c), lo);
-    tmem_st32(lane_addr(tmem_base, col + c0 + c), hi);
+    tmem_stw<N>(lane_addr(tmem_base, col + d + c0), lo);
   }
+  tmem_stw<N>(lane_addr(tmem_base, col + c0), hi);
+}
+
+// Thread-owned row `row` of X (d fp32) into the thread's TMEM lane at columns
+// [col, col+d) (hi/lo with `split`, lo at [col+d, col+2d)), 16 columns at a time:
+// the path of the configurations without staged operands, kept small so that it
+// does not crowd the registers of the kernels' main loops.
+__device__ __forceinline__ void row_to_tmem(uint32_t tmem_base, int col, const float* X, int row, int T, int d,
+                                            bool split) {
+#pragma unroll 1
+  for (int c0 = 0; c0 < d; c0 += 16) row_to_tmem_part<16>(tmem_base, col, X, row, T, d, c0, split);
 }
 
 // Row `row` of a 128-row K-major tile staged in smem by TMA (128-byte swizzle,
@@ -352,16 +357,5 @@ __device__ __forceinline__ void staged_row_to_tmem(uint32_t tmem_base, int col, 
   }
 }
 
-// Thread-owned row `row` of X (d fp32) into the thread's TMEM lane at columns
-// [col, col+d) (hi/lo with `split`, lo at [col+d, col+2d)).
-__device__ __forceinline__ void row_to_tmem(uint32_t tmem_base, int col, const float* X, int row, int T, int d,
-                                            bool split) {
-  if (d == 64) {
-    row_to_tmem_part<64>(tmem_base, col, X, row, T, d, 0, split);
-  } else {
-    row_to_tmem_part<64>(tmem_base, col, X, row, T, d, 0, split);
-    row_to_tmem_part<64>(tmem_base, col, X, row, T, d, 64, split);
-  }
-}
 
 }  // namespace kint
