@@ -38,6 +38,23 @@ N_INPUT_SETS = 3  # rotated so that no step reads inputs the previous step left 
 TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.1 : 2.25 PFLOP/s)
 
 
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
+# one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
+# kernel sources they were taken from.
+TRAFFIC = {"src": None}
+
+
+def kernel_source_digest() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_33591_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()[:16]
+
+
 def unit_flops(B, H, T, d):
     """One causal T x T x d contraction over all heads: 2 * B*H*d*T(T+1)/2 flops."""
     return B * H * d * T * (T + 1)
@@ -282,8 +299,9 @@ def run_cuda(args, world, rank, local):
     avg_s = per_kernel[dom]["avg_us"] * 1e-6
     if bound == "tensor":
         achieved = units * unit_flops(B, H, T, d) / avg_s / 1e12
+        traffic = TRAFFIC.get(dom) if TRAFFIC.get("src") == kernel_source_digest() else None
         roof = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": tf32_peak, "unit": "TFLOP/s",
-                "frac": achieved / tf32_peak, "traffic": None,
+                "frac": achieved / tf32_peak, "traffic": traffic,
                 "peak_note": f"TF32 = (1.1 / 2.25 nominal) x {pk['source']} bf16 burst {pk['bf16']} TFLOP/s"}
     else:
         nbytes = 2 * B * H * T * d * 4
