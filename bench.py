@@ -41,7 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": None}
+TRAFFIC = {"src": "f921414081153833", "k_prep": 31479680, "k_fwd_stats": 50386432, "k_fwd_main": 95098112,
+           "k_bwd_dq": 196307968, "k_bwd_dkdv": 185556224}
 
 
 def kernel_source_digest() -> str:
