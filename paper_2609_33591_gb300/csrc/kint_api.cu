@@ -308,7 +308,9 @@ int plan_dkdv(Params& p, int sel) {
   p.sm_stage_bytes = 4 * parts * qtile + 64 * 64 + (p.calib == KINT_CALIB_MINMAX ? 64 * p.Kp * 8 : 0);
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
-    const int total = std::max(finish_plan(p, p.sm_table + 1024, 2 * p.nstage + 7), kOneCtaPerSm);
+    // FWM Nearest: the half-bin table, 2K + 3 entries of 8 bytes
+    const int table = p.calib == KINT_CALIB_FWM ? 2048 : 1024;
+    const int total = std::max(finish_plan(p, p.sm_table + table, 2 * p.nstage + 7), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       return total;

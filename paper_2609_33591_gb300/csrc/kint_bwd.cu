@@ -39,27 +39,28 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
     if constexpr (CAL == CAL_SOFTMAX) {
       const float pr = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * invWf;
       ds = pr * __fmaf_rn(gv[jj], ga, gb);  // P (g - <g>_P)
+    } else if constexpr (CAL == CAL_FWM) {
+      // k1, c0 doubled (v = 2u), Kf = 2K, tab: the half-bin table of Delta_r / h (4-byte entries)
+      const uint32_t qb = fwm_half_bits(__fmaf_rn(sv[jj], k1, c0), Kf);
+      ds = __fmaf_rn(gv[jj], ga, gb) * lds_f32(tab + qb * 4u);
     } else {
       const float u = __fmaf_rn(sv[jj], k1, c0);
       float t, rf;
       uint32_t rb;
       decode_u(u, Kf, t, rb, rf);
-      const float2 e = lds_f2(CAL == CAL_FWM ? tab + rb * 8u : tab + rb * 1024u);
+      const float2 e = lds_f2(tab + rb * 1024u);
       const float de = __fsub_rn(e.y, e.x);
       const float dlt = de * inv_h;
       const float gam = __fmaf_rn(gv[jj], ga, gb);
       ds = gam * dlt;
-      if constexpr (CAL == CAL_FWM) ds = (u < 0.0f) ? 0.f : ds;
-      if constexpr (CAL == CAL_MINMAX) {
-        if constexpr (FULLG) {
-          const float ar = __fmaf_rn(rf, -fk, 1.0f);
-          const float A = ar * __fsub_rn(e.x, dlt);
-          const float Bc = __fmaf_rn(ar, de, -fk * __fsub_rn(e.y, dlt));
-          dm = gam * __fmaf_rn(t, Bc, A);
-          dm = nogrid ? 0.f : dm;
-        }
-        ds = nogrid ? 0.f : ds;
+      if constexpr (FULLG) {
+        const float ar = __fmaf_rn(rf, -fk, 1.0f);
+        const float A = ar * __fsub_rn(e.x, dlt);
+        const float Bc = __fmaf_rn(ar, de, -fk * __fsub_rn(e.y, dlt));
+        dm = gam * __fmaf_rn(t, Bc, A);
+        dm = nogrid ? 0.f : dm;
       }
+      ds = nogrid ? 0.f : ds;
     }
     if constexpr (DIAG) {
       const bool ok = (j0 + jj) <= i;
@@ -282,8 +283,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
         g = row_grid(p, M, m);
         if constexpr (CAL == CAL_FWM) {
-          if (tid < Kq)
-            *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+          if (tid < 2 * Kq + 1 + kHalfTail)
+            *reinterpret_cast<float*>(sm + p.sm_table + tid * 4) = fwm_half_entry(p, tid - kHalfTail).y;
         } else if constexpr (CAL == CAL_MINMAX) {
           for (int r = cg; r < Kq; r += NCG) {
             const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
@@ -297,8 +298,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
       const float invWf = 1.0f / Wf;
       const float sk1 = p.scale * kLog2e, sc0 = -M * kLog2e;
-      const float Kf = (float)Kq, fk = 1.0f / Kf;
-      const uint32_t tab = (CAL == CAL_FWM) ? smem_u32(sm + p.sm_table) - 0x58000000u
+      // FWM: the half-bin table, entry q at sm_table + 4 (q + 2), addressed by the bits
+      // 0x4B000000 + q of floor(2u) (0x4B000000 * 4 = 0x2C000000 mod 2^32), and the doubled
+      // position v = 2u; MinMax: this row's pair table, r * 1024 apart
+      const float Kf = (float)(CAL == CAL_FWM ? 2 * Kq : Kq), fk = 1.0f / (float)Kq;
+      const float k1q = CAL == CAL_FWM ? 2.0f * g.k1 : g.k1, c0q = CAL == CAL_FWM ? 2.0f * g.c0 : g.c0;
+      const uint32_t tab = (CAL == CAL_FWM) ? smem_u32(sm + p.sm_table) + 4u * kHalfTail - 0x2C000000u
                                             : smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
       const bool minmax = CAL == CAL_MINMAX;
       const bool track = FULLG && CAL != CAL_SOFTMAX && row_ok && !g.nogrid && (nmax > 1 || (minmax && nmin > 1));
@@ -325,10 +330,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         tmem_ld_wait();
         const int j0 = kt * BT + cg * W;
         if (j0 + W - 1 > qb * 128)
-          dq_chunk<CAL, FULLG, true, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
+          dq_chunk<CAL, FULLG, true, W>(sv, gv, out, j0, i, k1q, c0q, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
                                         sc0, invWf, own, cm);
         else
-          dq_chunk<CAL, FULLG, false, W>(sv, gv, out, j0, i, g.k1, g.c0, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab,
+          dq_chunk<CAL, FULLG, false, W>(sv, gv, out, j0, i, k1q, c0q, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab,
                                          sk1, sc0, invWf, own, cm);
         if (__any_sync(0xffffffffu, track)) {
           // rare: tied extrema, the tie set is found by equality on the recomputed scores
@@ -411,23 +416,24 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         group_sync(BAR_COMPUTE, NCOMP);
         if (warp == 0) store_rows_tile_boxed(stg, &maps.dq, D, 64, qb * 128, bh, false);
         if (row_ok && cg == 0) {
+          // the position as the dK/dV pass forms it: softmax log2 e^{s-M}, FWM Nearest 2u, else u
+          const bool half = CAL == CAL_FWM && p.recon == REC_NEAREST;
           RowRec r;
-          r.c0 = g.c0;
-          r.k1 = g.k1;
-          r.inv_h = g.inv_h;
+          r.c0 = CAL == CAL_SOFTMAX ? sc0 : (half ? 2.0f * g.c0 : g.c0);
+          r.k1 = CAL == CAL_SOFTMAX ? sk1 : (half ? 2.0f * g.k1 : g.k1);
           r.invWf = invWf;
           r.ga = ga;
           r.gb = gb;
           r.cMn = full ? cMn : 0.f;
-          r.cmn = (full && minmax) ? cmn : 0.f;
           r.amax = (nmax == 1) ? amax : -1;
-          r.amin = (nmin == 1) ? amin : -1;
           r.flags = (g.nogrid ? REC_NOGRID : 0) | (nmax > 1 ? REC_TIEMAX : 0) | (nmin > 1 ? REC_TIEMIN : 0);
-          r.pad = 0;
+          r.inv_h = g.inv_h;
+          r.cmn = (full && minmax) ? cmn : 0.f;
+          r.amin = (nmin == 1) ? amin : -1;
+          r.pad0 = 0;
           r.M = M;
           r.m = m;
-          r.sk1 = sk1;
-          r.sc0 = sc0;
+          r.pad1 = r.pad2 = 0.f;
           reinterpret_cast<RowRec*>(p.rec)[rw] = r;
         }
       }
@@ -454,19 +460,26 @@ __device__ __forceinline__ int4 lds_i4(uint32_t addr) {
 template <int CAL, int REC, bool FULLG, bool MASKED, int W>
 __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)[W], float (&pa)[W],
                                          float (&da)[W], int j, int i0, int T, uint32_t recs, uint32_t tabs,
-                                         uint32_t fwtab, uint32_t tstride, float Kf) {
+                                         uint32_t fwtab, uint32_t tstride, float Kf, float fwm_inv_h) {
 #pragma unroll
   for (int ii = 0; ii < W; ++ii) {
     const uint32_t ra = recs + ii * 64u;  // RowRec of query row i0 + ii
-    const float4 r0 = lds_f4(ra);          // c0, k1, inv_h, invWf
-    const float4 r1 = lds_f4(ra + 16);     // ga, gb, cMn, cmn
+    const float4 r0 = lds_f4(ra);          // c0, k1, invWf, ga
+    const float4 r1 = lds_f4(ra + 16);     // gb, cMn, amax, flags
+    float4 r2 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if constexpr (CAL == CAL_MINMAX) r2 = lds_f4(ra + 32);  // inv_h, cmn, amin, -
+    const float gam = __fmaf_rn(gv[ii], r0.w, r1.x);
     float pv, ds;
     if constexpr (CAL == CAL_SOFTMAX) {
-      const float4 r3 = lds_f4(ra + 48);  // M, m, sk1, sc0
-      pv = ex2_approx(__fmaf_rn(sv[ii], r3.z, r3.w)) * r0.w;
-      ds = pv * __fmaf_rn(gv[ii], r1.x, r1.y);
+      pv = ex2_approx(__fmaf_rn(sv[ii], r0.y, r0.x)) * r0.z;
+      ds = pv * gam;
+    } else if constexpr (CAL == CAL_FWM && REC == REC_NEAREST) {
+      // record holds 2k1, 2c0; Kf = 2K; fwtab: the half-bin table of (w^N, Delta_r / h)
+      const uint32_t qb = fwm_half_bits(__fmaf_rn(sv[ii], r0.y, r0.x), Kf);
+      const float2 e = lds_f2(fwtab + qb * 8u);
+      pv = e.x * r0.z;
+      ds = gam * e.y;
     } else {
-      const int4 r2 = lds_i4(ra + 32);  // amax, amin, flags, -
       const float u = __fmaf_rn(sv[ii], r0.y, r0.x);
       float t, rf;
       uint32_t rb;
@@ -476,23 +489,22 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
       const float wl = __fmaf_rn(t, de, e.x);
       const float wn = (t >= 0.5f) ? e.y : e.x;
       float w = (REC == REC_NEAREST) ? wn : wl;
-      const float gam = __fmaf_rn(gv[ii], r1.x, r1.y);
-      ds = gam * (de * r0.z);
+      ds = gam * (de * (CAL == CAL_MINMAX ? r2.x : fwm_inv_h));
       if constexpr (CAL == CAL_FWM) {
         const bool tail = u < 0.0f;
         w = tail ? 0.f : w;
         ds = tail ? 0.f : ds;
       }
       if constexpr (CAL == CAL_MINMAX) {
-        const bool ng = (r2.z & REC_NOGRID) != 0;
+        const bool ng = (__float_as_int(r1.w) & REC_NOGRID) != 0;
         w = ng ? 1.f : w;
         ds = ng ? 0.f : ds;
       }
-      pv = w * r0.w;
-      if constexpr (FULLG) {
-        ds += (j == r2.x) ? r1.z : 0.f;
-        if constexpr (CAL == CAL_MINMAX) ds += (j == r2.y) ? r1.w : 0.f;
-      }
+      pv = w * r0.z;
+    }
+    if constexpr (FULLG && CAL != CAL_SOFTMAX) {
+      ds += (j == __float_as_int(r1.z)) ? r1.y : 0.f;
+      if constexpr (CAL == CAL_MINMAX) ds += (j == __float_as_int(r2.z)) ? r2.y : 0.f;
     }
     if constexpr (MASKED) {
       const int iq = i0 + ii;
@@ -607,8 +619,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     tc_fence_before();
     __syncwarp();
     if ((tid & 31) == 0) mbar_arrive(bar_ops);
-    if (CAL == CAL_FWM && tid < Kq)
-      *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+    if constexpr (CAL == CAL_FWM) {
+      if (REC == REC_NEAREST && tid < 2 * Kq + 1 + kHalfTail)
+        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = fwm_half_entry(p, tid - kHalfTail);
+      if (REC != REC_NEAREST && tid < Kq)
+        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+    }
   }
 
   if (warp == PRODUCER_WARP) {
@@ -679,8 +695,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     }
     mma_commit(bar_done);
   } else {
-    const float Kf = (float)Kq;
-    const uint32_t fwtab = smem_u32(sm + p.sm_table) - 0x58000000u;
+    // FWM Nearest: the half-bin table (entry q at sm_table + 8 (q + 2)) and the doubled
+    // position; FWM LERP: the pair table, entry r at sm_table + 8 r (0x4B000000 * 8 =
+    // 0x58000000 mod 2^32)
+    constexpr bool half = CAL == CAL_FWM && REC == REC_NEAREST;
+    const float Kf = (float)(half ? 2 * Kq : Kq);
+    const uint32_t fwtab = smem_u32(sm + p.sm_table) + (half ? 8u * kHalfTail : 0u) - 0x58000000u;
     group_sync(BAR_COMPUTE, NCOMP);  // the FWM table
     bool failed = false;
     const int* tflags = p.tileflags + (size_t)bh * p.nqt + qt0;
@@ -718,9 +738,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         tmem_ld_wait();
         const bool masked = (i0h < kb * 128 + 128) || (i0h + WS > p.T);
         if (masked)
-          kv_chunk<CAL, REC, FULLG, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf);
+          kv_chunk<CAL, REC, FULLG, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
+                                              p.fwm_inv_h);
         else
-          kv_chunk<CAL, REC, FULLG, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf);
+          kv_chunk<CAL, REC, FULLG, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
+                                               p.fwm_inv_h);
         if constexpr (FULLG && CAL != CAL_SOFTMAX) {
           // rows with tied extrema (flagged per 64-row tile by the dQ kernel): the tie set is
           // found by equality on the recomputed scores

@@ -71,10 +71,13 @@ __device__ __forceinline__ void tmem_stw(uint32_t taddr, const float (&v)[W]) {
 
 // Per-query-row record written by the dQ kernel for the dK/dV kernel (64 bytes).
 struct RowRec {
-  float c0, k1, inv_h, invWf;  // grid position u = acc * k1 + c0; forward 1/W
-  float ga, gb, cMn, cmn;      // gamma = g * ga + gb; extremum terms c_M / n_max, c_m / n_min
-  int amax, amin, flags, pad;  // arg-extrema; flags: 1 no grid, 2 tied maxima, 4 tied minima
-  float M, m, sk1, sc0;        // extrema; softmax e^{s-M} = 2^(acc * sk1 + sc0)
+  float c0, k1, invWf, ga;  // position acc * k1 + c0 (u; 2u for FWM Nearest; log2 e^{s-M} for softmax);
+                            // forward 1/W; gamma = g * ga + gb
+  float gb, cMn;            // c_M / n_max
+  int amax, flags;          // arg-max; flags: 1 no grid, 2 tied maxima, 4 tied minima
+  float inv_h, cmn;         // 1/h (MinMax); c_m / n_min
+  int amin, pad0;           // arg-min
+  float M, m, pad1, pad2;   // extrema
 };
 constexpr int REC_NOGRID = 1, REC_TIEMAX = 2, REC_TIEMIN = 4;
 
@@ -142,6 +145,34 @@ __device__ __forceinline__ void decode_u(float u, float Kf, float& t, uint32_t& 
   rb = __float_as_uint(fr);
 }
 
+// ---------------------------------------------------------------------------
+// FWM half-bin index.  With v = 2u (formed exactly as acc * 2k1 + 2c0) and
+// u = r + t, floor(v) = 2r + [t >= 1/2]: one floor gives both the bin r = q >> 1
+// and the Nearest endpoint (q + 1) >> 1, with the same decisions as decode_u.
+// Clamping v to [-1, 2K] sends u >= K to q = 2K and the tail u < 0 to the two
+// patterns just below 2^23 (2^23 - 1 and 2^23 - 1/2 after rounding down), so a
+// table of 2K + 3 entries, two tail entries first, is indexed by the float bits:
+// entry q sits at base + (bits - 0x4B000000) * size.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t fwm_half_bits(float v, float twoK) {
+  return __float_as_uint(__fadd_rd(fminf(fmaxf(v, -1.0f), twoK), kMagic));
+}
+constexpr int kHalfTail = 2;  // tail entries ahead of q = 0
+
+// Entry q in [-2, 2K] of the half-bin table: (w^N, Delta_r / h) with r = min(q >> 1, K - 1)
+// (zeros in the tail); Delta_r / h is rounded as the full decode path rounds it.
+__device__ __forceinline__ float2 fwm_half_entry(const Params& p, int q) {
+  if (q < 0) return make_float2(0.f, 0.f);
+  const int r = min(q >> 1, p.Kint - 1);
+  const float dlt = __fmul_rn(__fsub_rn(p.fwm_e[r + 1], p.fwm_e[r]), p.fwm_inv_h);
+  return make_float2(p.fwm_e[(q + 1) >> 1], dlt);
+}
+
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+  return v;
+}
 __device__ __forceinline__ float2 lds_f2(uint32_t addr) {
   float2 v;
   asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(addr));

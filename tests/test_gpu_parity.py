@@ -121,3 +121,21 @@ def test_many_items_per_cta(c, r, s):
     and barrier phases running on across items) are exercised; ragged T."""
     Q, K, V, dO = make_qkvdo(4, 40, 200, 64, seed=11)
     parity.check(Q, K, V, dO, _cfg(c, r, s, FU, 4), TF)
+
+
+@pytest.mark.parametrize("prec", [TF, X3])
+def test_exact_grid_points(prec):
+    """Operands in {-1, 0, 1} make every score a multiple of 1/8, so for FWM (tau = 8, K = 4,
+    h = 2) the position u = (s - M + tau) / h is exact and lands on bin edges (t = 0) and
+    midpoints (t = 1/2, where Nearest takes e_{r+1}) for many keys: the passes must take
+    the oracle's decisions there exactly."""
+    rng = np.random.default_rng(12)
+    Q = rng.integers(-1, 2, size=(1, 2, 200, 64)).astype(np.float32)
+    K = rng.integers(-1, 2, size=(1, 2, 200, 64)).astype(np.float32)
+    _, _, V, dO = make_qkvdo(1, 2, 200, 64, seed=12)
+    cfgs = (_cfg(FW, NE, PR, FU), _cfg(FW, NE, WE, FU), _cfg(FW, LE, PR, FU), _cfg(FW, NE, PR, DE),
+            _cfg(FW, NE, PR, FU, tau=2.0))  # tau = 2: h = 1/2, many keys in the tail and at u = 0
+    for cfg in cfgs:
+        rep = parity.check(Q, K, V, dO, cfg, prec)
+        assert rep["bins_flips"] == 0 and rep["ivals_flips"] == 0
+    parity.check(Q, K, V, dO, _cfg(MM, NE, WE, FU), prec)
