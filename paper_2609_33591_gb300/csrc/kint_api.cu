@@ -276,17 +276,16 @@ int plan_dq(Params& p) {
   p.sm_a = 0;
   p.sm_stage0 = p.ops_smem ? 2 * 128 * p.d * 4 : 0;
   p.sm_stage_bytes = 3 * parts * ktile;
-  // One item per CTA (the kernel can loop over items, but with its own dQ staging tile
-  // the stage ring drops to two stages, which measured slower), dQ staged in the idle
-  // stage ring at the end.
+  // One CTA per SM looping over the items (dQ goes straight from TMEM to global memory,
+  // so the stage ring keeps loading the next item's tiles under the epilogue).
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
-    p.sm_ostage = p.sm_stage0;
+    p.sm_ostage = 0;
     const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 7), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
-      p.ngrid = p.nitems;
+      p.ngrid = std::min(p.nitems, num_sms());
       return total;
     }
   }
@@ -518,8 +517,7 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     ok = ok && map_tr(&maps.kt, w.kth, BH, T, Tp, d) && map_tr(&maps.qt, w.qth, BH, T, Tp, d);
     ok = ok && map_tr(&maps.dot, w.doth, BH, T, Tp, d);
   }
-  ok = ok && map_nat(&maps.dq, dQ, BH, T, d, 64) && map_nat(&maps.dk, dK, BH, T, d, 64) &&
-       map_nat(&maps.dv, dV, BH, T, d, 64);
+  ok = ok && map_nat(&maps.dk, dK, BH, T, d, 64) && map_nat(&maps.dv, dV, BH, T, d, 64);
   if (!ok) return KINT_ERR_LAUNCH;
 
   Params pq = p;

@@ -138,7 +138,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   uint64_t* bar_stg = bars + 2 * NS + 6;  // Q / dO tiles staged in smem by TMA (per item)
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 7);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
-  uint8_t* ostg = sm + p.sm_ostage;                        // dQ staging tile
   const int tid = threadIdx.x, warp = warp_id_uniform();
   constexpr int W = BT / NCG;  // key columns per thread per tile
   const int dp = D * parts;
@@ -170,7 +169,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   if (warp == PRODUCER_WARP) {
     int gt = 0, n = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
       const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
       if (p.ops_smem) {
@@ -205,7 +204,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + cSG0;
     int gt = 0, n = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH;
       const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
       // Q / dO of the item in TMEM (the compute warps copy them only after reading the
@@ -242,10 +241,31 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   } else {
     // ---- compute warps: items one after the other ----
     const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
+    // Operand rows of the n-th item into TMEM (column group 0 takes Q, group 1 takes dO),
+    // handed to the MMA warp through bar_ops.  TF32 at d = 64: from the tiles the producer
+    // staged in smem; otherwise from global rows.  The next item's rows go in as soon as
+    // the current item's last S, g have been read (before its dQ epilogue), so the next
+    // item's first products run under that epilogue.
+    auto ops_to_tmem = [&](int n) {
+      const int item = snake_item(n);
+      const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, i = qb * 128 + row;
+      if (p.ops_smem) {
+        if (mbar_wait(bar_stg, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
+          staged_row_to_tmem(tmem, cg == 0 ? cQ : cdO, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
+      } else {
+        row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, i < p.T ? (bh + 1) * p.T : 0, D,
+                    p.x3 != 0);
+      }
+      tmem_st_wait();
+      tc_fence_before();
+      __syncwarp();
+      if ((tid & 31) == 0) mbar_arrive(bar_ops);
+    };
     int gt = 0, n = 0;
     bool failed = false;
-    for (int item = blockIdx.x; item < p.nitems && !failed; item += gridDim.x, ++n) {
-      // ---- set-up: operands Q / dO into TMEM, row constants, grid table ----
+    if (snake_item(0) < p.nitems) ops_to_tmem(0);
+    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
+      // ---- set-up: row constants, grid table (the operands are in TMEM already) ----
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
       const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
       const int i = qb * 128 + row;
@@ -255,20 +275,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       int nmax = 1, nmin = 1, amax = 0, amin = 0;
       RowGrid g{};
       {
-        // operand rows into TMEM (column group 0 takes Q, group 1 takes dO), handed to the
-        // MMA warp through bar_ops; the rest of the set-up runs under the first products.
-        // TF32 at d = 64: from tiles the producer staged in smem; otherwise from global rows.
-        if (p.ops_smem) {
-          if (mbar_wait(bar_stg, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-            staged_row_to_tmem(tmem, cg == 0 ? cQ : cdO, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
-        } else {
-          row_to_tmem(tmem, cg == 0 ? cQ : cdO, cg == 0 ? p.Q : p.dO, bh * p.T + i, row_ok ? (bh + 1) * p.T : 0, D,
-                      p.x3 != 0);
-        }
-        tmem_st_wait();
-        tc_fence_before();
-        __syncwarp();
-        if ((tid & 31) == 0) mbar_arrive(bar_ops);
         if (row_ok) {
           M = p.row_max[rw];
           m = p.row_min[rw];
@@ -365,11 +371,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
       gt += nkt;
+      // the next item's Q / dO (this item's S, g have all been read: the last tile's were)
+      if (!failed && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       failed = group_any(BAR_COMPUTE, NCOMP, !dok);
       if (!failed) {
         tc_fence_after();
-        if (warp == 0) tma_store_wait_read();  // the previous item's dQ tile has left the staging area
         xch[cg * 128 + row] = own;
         xch[(NCG + cg) * 128 + row] = cm;
         group_sync(BAR_COMPUTE, NCOMP);
@@ -387,9 +394,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
         const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
         const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
-        // dQ rows into the swizzled staging tile (its previous store has been read out),
-        // then one TMA store
-        uint8_t* stg = ostg;
+        // dQ rows straight to global memory (the stage ring is loading the next item)
         for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
           // the arg-extremum key rows first (all loads in flight before the TMEM read)
           float4 km[8], kn[8];
@@ -410,11 +415,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
             v[4 * q + 2] = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
             v[4 * q + 3] = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
           }
-          row_to_staged(stg, row, c / 32, v);
+          if (row_ok) {
+            float4* dst = reinterpret_cast<float4*>(p.dQ + rw * D + c);
+  #pragma unroll
+            for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
         }
-        fence_async_smem();
-        group_sync(BAR_COMPUTE, NCOMP);
-        if (warp == 0) store_rows_tile_boxed(stg, &maps.dq, D, 64, qb * 128, bh, false);
         if (row_ok && cg == 0) {
           // the position as the dK/dV pass forms it: softmax log2 e^{s-M}, FWM Nearest 2u, else u
           const bool half = CAL == CAL_FWM && p.recon == REC_NEAREST;
@@ -438,7 +444,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         }
       }
     }
-    if (warp == 0) tma_store_wait_all();
     tc_fence_before();
   }
   __syncthreads();

@@ -81,6 +81,15 @@ struct RowRec {
 };
 constexpr int REC_NOGRID = 1, REC_TIEMAX = 2, REC_TIEMIN = 4;
 
+// n-th work item of this CTA when the grid loops over items sorted longest first:
+// rounds of gridDim.x items taken in alternating directions (CTA 0 takes the longest
+// item of even rounds and the shortest of odd ones), which evens out the per-CTA
+// totals better than a plain stride.  With one CTA per item it is blockIdx.x.
+__device__ __forceinline__ int snake_item(int n) {
+  const int G = gridDim.x, c = blockIdx.x;
+  return n * G + ((n & 1) ? G - 1 - c : c);
+}
+
 // ---------------------------------------------------------------------------
 // Row grid.  Scores s are fp32 values of acc * scale.  The position of a key in
 // grid units is u = s * inv_h + c0:
@@ -374,17 +383,20 @@ __device__ __forceinline__ void row_to_tmem(uint32_t tmem_base, int col, const f
 // columns [col, col + d).  Chunk c (16 bytes) of a row sits at chunk c ^ (row % 8).
 __device__ __forceinline__ void staged_row_to_tmem(uint32_t tmem_base, int col, const uint8_t* tile, int row, int d) {
   const uint32_t base = smem_u32(tile) + (uint32_t)row * SW;
-  for (int pnl = 0; pnl < d / 32; ++pnl) {
-    float v[32];
+#pragma unroll 1
+  for (int h = 0; h < d / 16; ++h) {  // 16 columns (half a panel) at a time
+    const uint32_t pb = base + (uint32_t)(h >> 1) * 128u * SW;
+    float v[16];
 #pragma unroll
-    for (int c = 0; c < 8; ++c) {
-      const float4 x = lds_f4(base + (uint32_t)pnl * 128u * SW + (uint32_t)((c ^ (row & 7)) << 4));
+    for (int c = 0; c < 4; ++c) {
+      const int chunk = (h & 1) * 4 + c;
+      const float4 x = lds_f4(pb + (uint32_t)((chunk ^ (row & 7)) << 4));
       v[4 * c] = x.x;
       v[4 * c + 1] = x.y;
       v[4 * c + 2] = x.z;
       v[4 * c + 3] = x.w;
     }
-    tmem_st32(lane_addr(tmem_base, col + 32 * pnl), v);
+    tmem_st16(lane_addr(tmem_base, col + 16 * h), v);
   }
 }
 

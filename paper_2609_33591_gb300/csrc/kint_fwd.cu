@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   if (warp == PRODUCER_WARP) {
     int g = 0, n = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       if (n > 0 && !mbar_wait_warp(bar_qfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
       mbar_arrive_expect_tx(bar_q, parts * tile);
@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   } else if (warp == MMA_WARP) {
     int g = 0, n = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
       ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
       for (int kb = 0; kb < nkb && ok; ++kb) {
@@ -284,9 +284,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
     }
   } else {
     const int row = tid & 127, cg = tid >> 7;
-    int g = 0;
+    int g = 0, n = 0;
     bool failed = false;
-    for (int item = blockIdx.x; item < p.nitems && !failed; item += gridDim.x) {
+    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       const int i = qb * 128 + row;
       float M = -FLT_MAX, m = FLT_MAX;
@@ -453,7 +453,7 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
 // ---------------------------------------------------------------------------
 // Pass 2: reconstruction, normalization and P V (App. A).
 // Work items are (128-row query block, head) pairs, longest blocks first; a CTA
-// takes items blockIdx.x, blockIdx.x + gridDim.x, ... (one item per CTA when the
+// takes the items snake_item(0), snake_item(1), ... (one item per CTA when the
 // grid covers them all).  Tile counters run on across items, so the next item's Q
 // and first K/V tiles load while the current one finishes.
 // TMEM: score buffers S_b at [128 b, 128 b + 128), b < nbuf (the weights
@@ -536,7 +536,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   if (warp == PRODUCER_WARP) {
     int g = 0, n = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       // Q of the previous item is an operand until its last S product completes
       if (n > 0 && !mbar_wait_warp(bar_qfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
@@ -563,7 +563,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     const uint8_t* st0 = sm + p.sm_stage0;
     int g = 0, n = 0;
     bool ok = true;
-    for (int item = blockIdx.x; item < p.nitems && ok; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
       ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) &&
            main_issue_s(p, g, bar_full, bar_s, st0, sQ, tmem, qtile);
@@ -607,7 +607,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     const float Kf = (float)Kq;
     int g = 0, n = 0;
     bool failed = false;
-    for (int item = blockIdx.x; item < p.nitems && !failed; item += gridDim.x, ++n) {
+    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       const int i = qb * 128 + row;
       const bool row_ok = i < p.T;
