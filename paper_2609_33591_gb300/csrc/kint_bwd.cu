@@ -462,10 +462,11 @@ __device__ __forceinline__ int4 lds_i4(uint32_t addr) {
   return v;
 }
 
-template <int CAL, int REC, bool FULLG, bool MASKED, int W>
+template <int CAL, int REC, bool FULLG, bool MASKED, bool TIES, int W>
 __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)[W], float (&pa)[W],
                                          float (&da)[W], int j, int i0, int T, uint32_t recs, uint32_t tabs,
-                                         uint32_t fwtab, uint32_t tstride, float Kf, float fwm_inv_h) {
+                                         uint32_t fwtab, uint32_t tstride, float Kf, float fwm_inv_h,
+                                         float scale) {
 #pragma unroll
   for (int ii = 0; ii < W; ++ii) {
     const uint32_t ra = recs + ii * 64u;  // RowRec of query row i0 + ii
@@ -517,6 +518,19 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
       pv = ok ? pv : 0.f;
       ds = ok ? ds : 0.f;
     }
+    if constexpr (FULLG && TIES && CAL != CAL_SOFTMAX) {
+      // rows with tied extrema (flagged per 64-row query tile by the dQ kernel): the tie set
+      // is found by equality on the recomputed scores (rare, kept off the common path)
+      const int fl = __float_as_int(r1.w);
+      const int iq = i0 + ii;
+      const bool okr = (!MASKED || (iq >= j && iq < T)) && (fl & (REC_TIEMAX | REC_TIEMIN)) && !(fl & REC_NOGRID);
+      if (okr) {
+        const float2 ext = lds_f2(ra + 48);  // M, m
+        const float sc = __fmul_rn(sv[ii], scale);
+        if ((fl & REC_TIEMAX) && sc == ext.x) ds += r1.y;
+        if (CAL == CAL_MINMAX && (fl & REC_TIEMIN) && sc == ext.y) ds += r2.y;
+      }
+    }
     pa[ii] = pv;
     da[ii] = ds;
   }
@@ -549,6 +563,18 @@ __device__ __forceinline__ bool kv_issue_sg(const Params& p, int it, uint64_t* b
   return true;
 }
 
+// Producer warp of k_bwd_dkdv: TMA-stores the dV / dK tiles of its k-th item, which the
+// compute warps staged at `tile` (dV, then dK), and returns once they have been read out.
+__device__ __forceinline__ bool store_staged_dkdv(const Maps& maps, const Params& p, uint64_t* bar_ostg, int k,
+                                                  const uint8_t* tile, bool doDV, bool doDK) {
+  if (!mbar_wait_warp(bar_ostg, k & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) return false;
+  const int item = snake_item(k), kb = item / p.BH, bh = item % p.BH;
+  if (doDV) store_rows_tile_boxed(tile, &maps.dv, p.d, 64, kb * 128, bh, false);
+  if (doDK) store_rows_tile_boxed(tile + 128 * p.d * 4, &maps.dk, p.d, 64, kb * 128, bh, false);
+  tma_store_wait_read();
+  return true;
+}
+
 // ---------------------------------------------------------------------------
 // k_bwd_dkdv.  Thread t (< 256) owns key j = kb*128 + t%128 and the query half
 // t/128 of each 64-query tile.  TMEM: K [0, dp), V [dp, 2dp) (dK launches),
@@ -571,14 +597,14 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   uint64_t* bar_pready = bars + 2 * NS + 2;
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint64_t* bar_ops = bars + 2 * NS + 5;  // K / V rows stored in TMEM by every compute warp
-  uint64_t* bar_stg = bars + 2 * NS + 6;  // K / V tiles staged in smem by TMA
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 7);
+  uint64_t* bar_stg = bars + 2 * NS + 6;   // K / V tiles staged in smem by TMA
+  uint64_t* bar_ostg = bars + 2 * NS + 7;  // an item's dV / dK tiles staged in the K / V area
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 8);
   const int tid = threadIdx.x, warp = warp_id_uniform();
-  const int bh = blockIdx.y, kb = blockIdx.x;
   const int dp = D * parts;
   const int cK = 0, cV = dp, base = needV ? 2 * dp : dp;
   const int cdV = base + 128 * nbuf, cdK = cdV + (doDV ? D : 0);
-  const int qt0 = (kb * 128) / BT, nqt = (p.T + BT - 1) / BT, nit = nqt - qt0;
+  const int nqt = (p.T + BT - 1) / BT;
   const int oQ = 0, odO = parts * qtile, oQT = 2 * parts * qtile, odOT = 3 * parts * qtile;
   const int oRec = 4 * parts * qtile, oTab = oRec + BT * 64;
   const uint32_t tstride = (uint32_t)p.Kp * 8u;
@@ -597,6 +623,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     mbar_init(bar_done, 1);
     mbar_init(bar_ops, NCOMP / 32);
     mbar_init(bar_stg, 1);
+    mbar_init(bar_ostg, NCOMP / 32);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -607,208 +634,256 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-  const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
-  const int j = kb * 128 + row;
-  const bool key_ok = j < p.T;
-  if (warp < NCOMP / 32) {
-    // operand rows into TMEM: column group 0 takes K, group 1 takes V (staged tiles at
-    // TF32 d = 64, global rows otherwise)
-    if (p.ops_smem) {
-      if (mbar_wait(bar_stg, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) && (cg == 0 || needV))
-        staged_row_to_tmem(tmem, cg == 0 ? cK : cV, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
-    } else {
-      if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-      else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, key_ok ? (bh + 1) * p.T : 0, D, p.x3 != 0);
-    }
-    tmem_st_wait();
-    tc_fence_before();
-    __syncwarp();
-    if ((tid & 31) == 0) mbar_arrive(bar_ops);
-    if constexpr (CAL == CAL_FWM) {
-      if (REC == REC_NEAREST && tid < 2 * Kq + 1 + kHalfTail)
-        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = fwm_half_entry(p, tid - kHalfTail);
-      if (REC != REC_NEAREST && tid < Kq)
-        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
-    }
-  }
 
+  // Work items are (128-key block kb, head) pairs, longest first (kb = 0 meets every
+  // query tile); a CTA takes the items snake_item(0), snake_item(1), ...  Tile counters
+  // (stage ring, score buffers) run on across items.
   if (warp == PRODUCER_WARP) {
-    if (p.ops_smem) {
-      mbar_arrive_expect_tx(bar_stg, (needV ? 2 : 1) * 128 * D * 4);
-      load_rows_tile_boxed(sm + p.sm_a, &maps.k, bar_stg, D, 128, BT, 0, kb * 128, bh);
-      if (needV) load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.v, bar_stg, D, 128, BT, 0, kb * 128, bh);
+    int gt = 0, n = 0;
+    bool ok = true;
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+      const int kb = item / p.BH, bh = item % p.BH;
+      const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
+      if (p.ops_smem) {
+        // the staged K / V of the previous item have been copied into TMEM
+        if (n > 0 && !mbar_wait_warp(bar_ops, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        // the dV / dK tiles of item n - 2, staged in this area since, leave first
+        if (n >= 2 && !store_staged_dkdv(maps, p, bar_ostg, n - 2, sm + p.sm_a, doDV, doDK)) break;
+        mbar_arrive_expect_tx(bar_stg, (needV ? 2 : 1) * 128 * D * 4);
+        load_rows_tile_boxed(sm + p.sm_a, &maps.k, bar_stg, D, 128, BT, 0, kb * 128, bh);
+        if (needV) load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.v, bar_stg, D, 128, BT, 0, kb * 128, bh);
+      }
+      for (int it = 0; it < nit; ++it, ++gt) {
+        const int s = gt % NS, q0 = (qt0 + it) * BT;
+        if (gt >= NS &&
+            !mbar_wait_warp(&bar_empty[s], ((gt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        uint64_t* b = &bar_full[s];
+        const int nrows = min(BT, p.T - q0);
+        const int ntiles = 1 + (needV ? 1 : 0) + (doDK ? 1 : 0) + (doDV ? 1 : 0);
+        uint32_t bytes = ntiles * parts * qtile + nrows * 64;
+        if (CAL == CAL_MINMAX) bytes += nrows * tstride;
+        mbar_arrive_expect_tx(b, bytes);
+        load_rows_tile(dst + oQ, &maps.q, b, D, BT, 0, q0, bh);
+        if (p.x3) load_rows_tile(dst + oQ + qtile, &maps.q_lo, b, D, BT, 0, q0, bh);
+        if (needV) {
+          load_rows_tile(dst + odO, &maps.dout, b, D, BT, 0, q0, bh);
+          if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BT, 0, q0, bh);
+        }
+        if (doDK) {
+          load_rows_tile(dst + oQT, &maps.qt, b, BT, D, q0, 0, bh);
+          if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BT, D, q0, 0, bh);
+        }
+        if (doDV) {
+          load_rows_tile(dst + odOT, &maps.dot, b, BT, D, q0, 0, bh);
+          if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BT, D, q0, 0, bh);
+        }
+        const size_t r0 = (size_t)bh * p.T + q0;
+        bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
+        if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
+      }
     }
-    for (int it = 0; it < nit; ++it) {
-      const int s = it % NS, q0 = (qt0 + it) * BT;
-      if (it >= NS &&
-          !mbar_wait_warp(&bar_empty[s], ((it / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA))
-        break;
-      uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      uint64_t* b = &bar_full[s];
-      const int nrows = min(BT, p.T - q0);
-      const int ntiles = 1 + (needV ? 1 : 0) + (doDK ? 1 : 0) + (doDV ? 1 : 0);
-      uint32_t bytes = ntiles * parts * qtile + nrows * 64;
-      if (CAL == CAL_MINMAX) bytes += nrows * tstride;
-      mbar_arrive_expect_tx(b, bytes);
-      load_rows_tile(dst + oQ, &maps.q, b, D, BT, 0, q0, bh);
-      if (p.x3) load_rows_tile(dst + oQ + qtile, &maps.q_lo, b, D, BT, 0, q0, bh);
-      if (needV) {
-        load_rows_tile(dst + odO, &maps.dout, b, D, BT, 0, q0, bh);
-        if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BT, 0, q0, bh);
-      }
-      if (doDK) {
-        load_rows_tile(dst + oQT, &maps.qt, b, BT, D, q0, 0, bh);
-        if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BT, D, q0, 0, bh);
-      }
-      if (doDV) {
-        load_rows_tile(dst + odOT, &maps.dot, b, BT, D, q0, 0, bh);
-        if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BT, D, q0, 0, bh);
-      }
-      const size_t r0 = (size_t)bh * p.T + q0;
-      bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
-      if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
-    }
+    // the last-but-one item's tiles (the last item's are stored by the compute warps)
+    if (p.ops_smem && ok && n >= 2) store_staged_dkdv(maps, p, bar_ostg, n - 2, sm + p.sm_a, doDV, doDK);
+    tma_store_wait_all();
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;
-    bool ok = mbar_wait_warp(bar_ops, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
-    if (ok) tc_fence_after();
-    ok = ok && kv_issue_sg(p, 0, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
-    for (int it = 0; it < nit && ok; ++it) {
-      const int b = it % nbuf, s = it % NS;
-      if (nbuf == 2 && it + 1 < nit)
-        ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
-      if (!ok) break;
-      if (!mbar_wait_warp(&bar_pready[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-      tc_fence_after();
-      const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
-      const bool acc = it > 0;
-      if (p.x3) {
-        const uint32_t cacc = tmem + (doDV ? cdV : cdK);
-        const uint8_t* bt = st + (doDV ? odOT : oQT);
-        mma_tmem_smem(cacc, cS, bt, D, BT, acc);
-        mma_tmem_smem(cacc, cS, bt + qtile, D, BT, true);
-        mma_tmem_smem(cacc, cG, bt, D, BT, true);
-      } else {
-        if (doDV) mma_tmem_smem(tmem + cdV, cS, st + odOT, D, BT, acc);
-        if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
-      }
-      mma_commit(&bar_empty[s]);
-      if (nbuf == 1 && it + 1 < nit)
-        ok = kv_issue_sg(p, it + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
-    }
-    mma_commit(bar_done);
-  } else {
-    // FWM Nearest: the half-bin table (entry q at sm_table + 8 (q + 2)) and the doubled
-    // position; FWM LERP: the pair table, entry r at sm_table + 8 r (0x4B000000 * 8 =
-    // 0x58000000 mod 2^32)
-    constexpr bool half = CAL == CAL_FWM && REC == REC_NEAREST;
-    const float Kf = (float)(half ? 2 * Kq : Kq);
-    const uint32_t fwtab = smem_u32(sm + p.sm_table) + (half ? 8u * kHalfTail : 0u) - 0x58000000u;
-    group_sync(BAR_COMPUTE, NCOMP);  // the FWM table
-    bool failed = false;
-    const int* tflags = p.tileflags + (size_t)bh * p.nqt + qt0;
-    int tie_next = (FULLG && CAL != CAL_SOFTMAX) ? __ldg(tflags) : 0;
-    for (int it = 0; it < nit; ++it) {
-      // the tie flag of this 64-row query tile, loaded one tile ahead
-      const int tie_here = tie_next;
-      if (FULLG && CAL != CAL_SOFTMAX && it + 1 < nit) tie_next = __ldg(tflags + it + 1);
-      const int b = it % nbuf, s = it % NS;
-      const int q0 = (qt0 + it) * BT, i0 = q0 + cg * W;
-      const bool ok1 = mbar_wait(&bar_sfull[b], (it / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-      // the stage's row records arrived with its tiles (bar_full), before the products were issued
-      const bool ok2 = ok1 && mbar_wait(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-      if (!ok2) {
-        failed = true;
-        break;
-      }
-      tc_fence_after();
-      const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
-      // two 16-column halves of the thread's W columns (bounds the live registers)
-#pragma unroll 1
-      for (int h = 0; h < W / WS; ++h) {
-        const int c0 = cg * W + h * WS, i0h = q0 + c0;
-        const uint32_t recs = smem_u32(st + oRec) + c0 * 64;
-        const uint32_t tabs = smem_u32(st + oTab) + c0 * tstride - 0x58000000u;
-        const int cS = base + 128 * b + c0, cG = cS + 64;
-        float sv[WS], gv[WS], pa[WS], da[WS];
-        tmem_ldw<WS>(lane_addr(tmem, cS), sv);
-        if (needV) {
-          tmem_ldw<WS>(lane_addr(tmem, cG), gv);
-        } else {
-#pragma unroll
-          for (int q = 0; q < WS; ++q) gv[q] = 0.f;
+    int gt = 0, n = 0;
+    bool ok = true;
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+      const int kb = item / p.BH, nit = nqt - (kb * 128) / BT;
+      // K / V of the item in TMEM (the compute warps copy them only after the previous
+      // item's last S, g were read)
+      ok = mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
+      if (ok) tc_fence_after();
+      ok = ok && kv_issue_sg(p, gt, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+      for (int it = 0; it < nit && ok; ++it) {
+        const int g = gt + it, b = g % nbuf, s = g % NS;
+        if (nbuf == 2 && it + 1 < nit)
+          ok = kv_issue_sg(p, g + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+        if (!ok) break;
+        if (!mbar_wait_warp(&bar_pready[b], (g / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
+          ok = false;
+          break;
         }
-        tmem_ld_wait();
-        const bool masked = (i0h < kb * 128 + 128) || (i0h + WS > p.T);
-        if (masked)
-          kv_chunk<CAL, REC, FULLG, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
-                                              p.fwm_inv_h);
-        else
-          kv_chunk<CAL, REC, FULLG, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
-                                               p.fwm_inv_h);
-        if constexpr (FULLG && CAL != CAL_SOFTMAX) {
-          // rows with tied extrema (flagged per 64-row tile by the dQ kernel): the tie set is
-          // found by equality on the recomputed scores
-          if (tie_here) {
-            const int nr = min(WS, p.T - i0h);
-#pragma unroll
-            for (int ii = 0; ii < WS; ++ii) {
-              const RowRec& r = reinterpret_cast<const RowRec*>(st + oRec)[c0 + ii];
-              const bool okr = ii < nr && i0h + ii >= j && (r.flags & (REC_TIEMAX | REC_TIEMIN)) &&
-                               !(r.flags & REC_NOGRID);
-              const float sc = __fmul_rn(sv[ii], p.scale);
-              if (okr && (r.flags & REC_TIEMAX) && sc == r.M) da[ii] += r.cMn;
-              if (CAL == CAL_MINMAX && okr && (r.flags & REC_TIEMIN) && sc == r.m) da[ii] += r.cmn;
-            }
-          }
-        }
+        tc_fence_after();
+        const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        const uint32_t cS = tmem + base + 128 * b, cG = cS + 64;
+        const bool acc = it > 0;
         if (p.x3) {
-#pragma unroll
-          for (int q = 0; q < WS; ++q) {
-            const float x = doDV ? pa[q] : da[q];
-            const float hh = tf32_rna(x);
-            pa[q] = hh;
-            da[q] = __fsub_rn(x, hh);
-          }
-          tmem_stw<WS>(lane_addr(tmem, cS), pa);
-          tmem_stw<WS>(lane_addr(tmem, cG), da);
+          const uint32_t cacc = tmem + (doDV ? cdV : cdK);
+          const uint8_t* bt = st + (doDV ? odOT : oQT);
+          mma_tmem_smem(cacc, cS, bt, D, BT, acc);
+          mma_tmem_smem(cacc, cS, bt + qtile, D, BT, true);
+          mma_tmem_smem(cacc, cG, bt, D, BT, true);
         } else {
-          if (doDV) tmem_stw<WS>(lane_addr(tmem, cS), pa);
-          if (doDK) tmem_stw<WS>(lane_addr(tmem, cG), da);
+          if (doDV) mma_tmem_smem(tmem + cdV, cS, st + odOT, D, BT, acc);
+          if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
         }
+        mma_commit(&bar_empty[s]);
+        if (nbuf == 1 && it + 1 < nit)
+          ok = kv_issue_sg(p, g + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+      }
+      gt += nit;
+      mma_commit(bar_done);
+    }
+  } else {
+    const int row = tid & 127, cg = (tid >> 7) & (NCG - 1);
+    // K / V rows of the n-th item into TMEM (column group 0 takes K, group 1 takes V),
+    // handed to the MMA warp through bar_ops: TF32 at d = 64 from the tiles the producer
+    // staged in smem, otherwise from global rows.  The next item's rows go in as soon as
+    // the current item's last S^T, g^T have been read, so its first products run under
+    // the current item's epilogue.
+    auto ops_to_tmem = [&](int n) {
+      const int item = snake_item(n), kb = item / p.BH, bh = item % p.BH, j = kb * 128 + row;
+      if (p.ops_smem) {
+        if (mbar_wait(bar_stg, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) && (cg == 0 || needV))
+          staged_row_to_tmem(tmem, cg == 0 ? cK : cV, sm + p.sm_a + (cg == 0 ? 0 : 128 * D * 4), row, D);
+      } else {
+        const size_t lim = j < p.T ? (size_t)(bh + 1) * p.T : 0;
+        if (cg == 0) row_to_tmem(tmem, cK, p.K, bh * p.T + j, lim, D, p.x3 != 0);
+        else if (needV) row_to_tmem(tmem, cV, p.V, bh * p.T + j, lim, D, p.x3 != 0);
       }
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
-      if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
+      if ((tid & 31) == 0) mbar_arrive(bar_ops);
+    };
+    if (snake_item(0) < p.nitems) ops_to_tmem(0);
+    // FWM Nearest: the half-bin table (entry q at sm_table + 8 (q + 2)) and the doubled
+    // position; FWM LERP: the pair table, entry r at sm_table + 8 r (0x4B000000 * 8 =
+    // 0x58000000 mod 2^32)
+    constexpr bool half = CAL == CAL_FWM && REC == REC_NEAREST;
+    if constexpr (CAL == CAL_FWM) {
+      if (half && tid < 2 * Kq + 1 + kHalfTail)
+        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = fwm_half_entry(p, tid - kHalfTail);
+      if (!half && tid < Kq)
+        *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
     }
-    const bool dok = !failed && mbar_wait(bar_done, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-    failed = group_any(BAR_COMPUTE, NCOMP, !dok);
-    if (!failed) {
-      tc_fence_after();
-      // dV, dK rows into swizzled tiles in the idle stage ring, then one TMA store each
-      uint8_t* stg = sm + p.sm_stage0;
-      for (int pass = 0; pass < 2; ++pass) {
-        if (pass == 0 ? !doDV : !doDK) continue;
-        const int col = pass == 0 ? cdV : cdK;
-        const float mul = pass == 0 ? 1.0f : p.scale;
-        uint8_t* tile = stg + pass * 128 * D * 4;
-        for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
-          float v[32];
-          tmem_ld32(lane_addr(tmem, col + c), v);
-          tmem_ld_wait();
+    const float Kf = (float)(half ? 2 * Kq : Kq);
+    const uint32_t fwtab = smem_u32(sm + p.sm_table) + (half ? 8u * kHalfTail : 0u) - 0x58000000u;
+    group_sync(BAR_COMPUTE, NCOMP);  // the FWM table
+    bool failed = false;
+    int gt = 0, n = 0;
+    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
+      const int kb = item / p.BH, bh = item % p.BH;
+      const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
+      const int j = kb * 128 + row;
+      const int* tflags = p.tileflags + (size_t)bh * p.nqt + qt0;
+      int tie_next = (FULLG && CAL != CAL_SOFTMAX) ? __ldg(tflags) : 0;
+      for (int it = 0; it < nit; ++it) {
+        // the tie flag of this 64-row query tile, loaded one tile ahead
+        const int tie_here = tie_next;
+        if (FULLG && CAL != CAL_SOFTMAX && it + 1 < nit) tie_next = __ldg(tflags + it + 1);
+        const int g = gt + it, b = g % nbuf, s = g % NS;
+        const int q0 = (qt0 + it) * BT;
+        const bool ok1 = mbar_wait(&bar_sfull[b], (g / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+        // the stage's row records arrived with its tiles (bar_full), before the products were issued
+        const bool ok2 = ok1 && mbar_wait(&bar_full[s], (g / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+        if (!ok2) {
+          failed = true;
+          break;
+        }
+        tc_fence_after();
+        const uint8_t* st = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        // two 16-column halves of the thread's W columns (bounds the live registers)
+#pragma unroll 1
+        for (int h = 0; h < W / WS; ++h) {
+          const int c0 = cg * W + h * WS, i0h = q0 + c0;
+          const uint32_t recs = smem_u32(st + oRec) + c0 * 64;
+          const uint32_t tabs = smem_u32(st + oTab) + c0 * tstride - 0x58000000u;
+          const int cS = base + 128 * b + c0, cG = cS + 64;
+          float sv[WS], gv[WS], pa[WS], da[WS];
+          tmem_ldw<WS>(lane_addr(tmem, cS), sv);
+          if (needV) {
+            tmem_ldw<WS>(lane_addr(tmem, cG), gv);
+          } else {
 #pragma unroll
-          for (int q = 0; q < 32; ++q) v[q] *= mul;
-          row_to_staged(tile, row, c / 32, v);
+            for (int q = 0; q < WS; ++q) gv[q] = 0.f;
+          }
+          tmem_ld_wait();
+          const bool masked = (i0h < kb * 128 + 128) || (i0h + WS > p.T);
+          if (FULLG && CAL != CAL_SOFTMAX && tie_here)
+            kv_chunk<CAL, REC, FULLG, true, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
+                                                      p.fwm_inv_h, p.scale);
+          else if (masked)
+            kv_chunk<CAL, REC, FULLG, true, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
+                                                       Kf, p.fwm_inv_h, p.scale);
+          else
+            kv_chunk<CAL, REC, FULLG, false, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
+                                                        Kf, p.fwm_inv_h, p.scale);
+          if (p.x3) {
+#pragma unroll
+            for (int q = 0; q < WS; ++q) {
+              const float x = doDV ? pa[q] : da[q];
+              const float hh = tf32_rna(x);
+              pa[q] = hh;
+              da[q] = __fsub_rn(x, hh);
+            }
+            tmem_stw<WS>(lane_addr(tmem, cS), pa);
+            tmem_stw<WS>(lane_addr(tmem, cG), da);
+          } else {
+            if (doDV) tmem_stw<WS>(lane_addr(tmem, cS), pa);
+            if (doDK) tmem_stw<WS>(lane_addr(tmem, cG), da);
+          }
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
+      }
+      gt += nit;
+      // the next item's K / V (this item's S^T, g^T have all been read: the last tile's were)
+      if (!failed && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
+      const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+      if (!failed) {
+        tc_fence_after();
+        // dV, dK rows into swizzled tiles for TMA stores: in the K / V staging area (free now
+        // that the next item's K / V are in TMEM; the producer stores them before it stages
+        // the item after next), or, for the last item, in the idle stage ring (stored here).
+        // Without the staging area (3xTF32, d = 128, one-product launches) straight to
+        // global memory.
+        const bool last = snake_item(n + 1) >= p.nitems;
+        uint8_t* stg = last ? sm + p.sm_stage0 : sm + p.sm_a;
+        for (int pass = 0; pass < 2; ++pass) {
+          if (pass == 0 ? !doDV : !doDK) continue;
+          const int col = pass == 0 ? cdV : cdK;
+          const float mul = pass == 0 ? 1.0f : p.scale;
+          float* out = (pass == 0 ? p.dV : p.dK) + ((size_t)bh * p.T + j) * D;
+          for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
+            float v[32];
+            tmem_ld32(lane_addr(tmem, col + c), v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int q = 0; q < 32; ++q) v[q] *= mul;
+            if (p.ops_smem) {
+              row_to_staged(stg + pass * 128 * D * 4, row, c / 32, v);
+            } else if (j < p.T) {
+              float4* dst = reinterpret_cast<float4*>(out + c);
+#pragma unroll
+              for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+          }
+        }
+        if (p.ops_smem) {
+          fence_async_smem();
+          if (last) {
+            group_sync(BAR_COMPUTE, NCOMP);
+            if (warp == 0 && doDV) store_rows_tile_boxed(stg, &maps.dv, D, 64, kb * 128, bh, false);
+            if (warp == 1 && doDK) store_rows_tile_boxed(stg + 128 * D * 4, &maps.dk, D, 64, kb * 128, bh, false);
+          } else {
+            __syncwarp();
+            if ((tid & 31) == 0) mbar_arrive(bar_ostg);
+          }
         }
       }
-      fence_async_smem();
-      group_sync(BAR_COMPUTE, NCOMP);
-      if (warp == 0 && doDV) store_rows_tile_boxed(stg, &maps.dv, D, 64, kb * 128, bh);
-      if (warp == 1 && doDK) store_rows_tile_boxed(stg + 128 * D * 4, &maps.dk, D, 64, kb * 128, bh);
     }
+    if (warp < 2) tma_store_wait_all();
     tc_fence_before();
   }
   __syncthreads();
@@ -836,7 +911,7 @@ cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cud
 }
 
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
-  const dim3 grid((p.T + 127) / 128, p.BH);
+  const dim3 grid((unsigned)p.ngrid);
   const bool full = p.grad == 0, near = p.recon == REC_NEAREST;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dkdv<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
