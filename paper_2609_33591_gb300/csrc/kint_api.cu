@@ -282,7 +282,7 @@ int plan_dq(Params& p) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
     p.sm_ostage = 0;
-    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 7), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 2 * p.nstage + 8), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       p.ngrid = std::min(p.nitems, num_sms());
@@ -520,7 +520,8 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     ok = ok && map_tr(&maps.kt, w.kth, BH, T, Tp, d) && map_tr(&maps.qt, w.qth, BH, T, Tp, d);
     ok = ok && map_tr(&maps.dot, w.doth, BH, T, Tp, d);
   }
-  ok = ok && map_nat(&maps.dk, dK, BH, T, d, 64) && map_nat(&maps.dv, dV, BH, T, d, 64);
+  ok = ok && map_nat(&maps.dq, dQ, BH, T, d, 64) && map_nat(&maps.dk, dK, BH, T, d, 64) &&
+       map_nat(&maps.dv, dV, BH, T, d, 64);
   if (!ok) return KINT_ERR_LAUNCH;
 
   Params pq = p;

@@ -123,6 +123,17 @@ __device__ __forceinline__ bool dq_issue_sg(const Params& p, int kt, uint64_t* b
 // smem: stages {K [64 x d], V [64 x d], K^T [d x 64]} (hi[, lo] each) at
 // sm_stage0; the grid pair table at sm_table; exchange words at sm_rows.
 // ---------------------------------------------------------------------------
+// Producer warp of k_bwd_dq: TMA-stores the dQ tile of its k-th item, which the compute
+// warps staged at `tile`, and returns once it has been read out.
+__device__ __forceinline__ bool store_staged_dq(const Maps& maps, const Params& p, uint64_t* bar_ostg, int k,
+                                                const uint8_t* tile) {
+  if (!mbar_wait_warp(bar_ostg, k & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) return false;
+  const int item = snake_item(k), qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
+  store_rows_tile_boxed(tile, &maps.dq, p.d, 64, qb * 128, bh, false);
+  tma_store_wait_read();
+  return true;
+}
+
 template <int CAL, bool FULLG>
 __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
@@ -135,8 +146,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   uint64_t* bar_pready = bars + 2 * NS + 2;  // [2]
   uint64_t* bar_done = bars + 2 * NS + 4;
   uint64_t* bar_ops = bars + 2 * NS + 5;  // Q / dO rows stored in TMEM by every compute warp (per item)
-  uint64_t* bar_stg = bars + 2 * NS + 6;  // Q / dO tiles staged in smem by TMA (per item)
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 7);
+  uint64_t* bar_stg = bars + 2 * NS + 6;   // Q / dO tiles staged in smem by TMA (per item)
+  uint64_t* bar_ostg = bars + 2 * NS + 7;  // an item's dQ tile staged in the Q / dO area
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 8);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
   constexpr int W = BT / NCG;  // key columns per thread per tile
@@ -155,6 +167,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     mbar_init(bar_done, 1);
     mbar_init(bar_ops, NCOMP / 32);
     mbar_init(bar_stg, 1);
+    mbar_init(bar_ostg, NCOMP / 32);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -175,6 +188,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       if (p.ops_smem) {
         // the staging tiles of the previous item have been copied into TMEM
         if (n > 0 && !mbar_wait_warp(bar_ops, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        // the dQ tile of item n - 2, staged in this area since, leaves first
+        if (n >= 2 && !store_staged_dq(maps, p, bar_ostg, n - 2, sm + p.sm_a)) break;
         mbar_arrive_expect_tx(bar_stg, 2 * 128 * D * 4);
         load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb * 128, bh);
         load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb * 128, bh);
@@ -199,6 +214,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         }
       }
     }
+    // the last-but-one item's tile (the last item's is stored by the compute warps)
+    if (p.ops_smem && ok && n >= 2) store_staged_dq(maps, p, bar_ostg, n - 2, sm + p.sm_a);
+    tma_store_wait_all();
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + cSG0;
@@ -394,7 +412,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
         const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
         const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
-        // dQ rows straight to global memory (the stage ring is loading the next item)
+        // dQ rows into a swizzled tile for a TMA store: in the Q / dO staging area (free now
+        // that the next item's Q / dO are in TMEM; the producer stores it before it stages
+        // the item after next), or, for the last item, in the idle stage ring (stored here).
+        // Without the staging area (3xTF32, d = 128) straight to global memory.
+        const bool last = snake_item(n + 1) >= p.nitems;
+        uint8_t* stg = last ? sm + p.sm_stage0 : sm + p.sm_a;
         for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
           // the arg-extremum key rows first (all loads in flight before the TMEM read)
           float4 km[8], kn[8];
@@ -415,10 +438,22 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
             v[4 * q + 2] = __fmaf_rn(cmn, kn[q].z, __fmaf_rn(cMn, km[q].z, v[4 * q + 2])) * p.scale;
             v[4 * q + 3] = __fmaf_rn(cmn, kn[q].w, __fmaf_rn(cMn, km[q].w, v[4 * q + 3])) * p.scale;
           }
-          if (row_ok) {
+          if (p.ops_smem) {
+            row_to_staged(stg, row, c / 32, v);
+          } else if (row_ok) {
             float4* dst = reinterpret_cast<float4*>(p.dQ + rw * D + c);
   #pragma unroll
             for (int q = 0; q < 8; ++q) dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
+        }
+        if (p.ops_smem) {
+          fence_async_smem();
+          if (last) {
+            group_sync(BAR_COMPUTE, NCOMP);
+            if (warp == 0) store_rows_tile_boxed(stg, &maps.dq, D, 64, qb * 128, bh, false);
+          } else {
+            __syncwarp();
+            if ((tid & 31) == 0) mbar_arrive(bar_ostg);
           }
         }
         if (row_ok && cg == 0) {
@@ -444,6 +479,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         }
       }
     }
+    if (warp == 0) tma_store_wait_all();
     tc_fence_before();
   }
   __syncthreads();

@@ -25,7 +25,7 @@ enum DkvSel : int { DKV_BOTH = 0, DKV_DV = 1, DKV_DK = 2 };
 struct Maps {
   CUtensorMap q, q_lo, k, k_lo, v, v_lo, dout, dout_lo;  // natural
   CUtensorMap kt, kt_lo, vt, vt_lo, qt, qt_lo, dot, dot_lo;  // transposed
-  CUtensorMap out, out_lerp, dk, dv;  // outputs (natural, box 32 x 64 rows) for TMA stores
+  CUtensorMap out, out_lerp, dq, dk, dv;  // outputs (natural, box 32 x 64 rows) for TMA stores
 };
 
 struct Params {
