@@ -635,7 +635,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   uint64_t* bar_ops = bars + 2 * NS + 5;  // K / V rows stored in TMEM by every compute warp
   uint64_t* bar_stg = bars + 2 * NS + 6;   // K / V tiles staged in smem by TMA
   uint64_t* bar_ostg = bars + 2 * NS + 7;  // an item's dV / dK tiles staged in the K / V area
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 8);
+  // a stage's transposed tiles (Q^T, dO^T) complete on their own barrier, so the products
+  // S^T, g^T wait only for the first half of the stage's bytes
+  uint64_t* bar_fullT = bars + 2 * NS + 8;  // [NS]
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 * NS + 8);
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int dp = D * parts;
   const int cK = 0, cV = dp, base = needV ? 2 * dp : dp;
@@ -650,6 +653,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
       mbar_init(&bar_full[s], 1);
+      mbar_init(&bar_fullT[s], 1);
       mbar_init(&bar_empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -697,10 +701,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
           break;
         }
         uint8_t* dst = sm + p.sm_stage0 + s * p.sm_stage_bytes;
+        // first the operands of S^T, g^T and the row records, then the transposed tiles
         uint64_t* b = &bar_full[s];
         const int nrows = min(BT, p.T - q0);
-        const int ntiles = 1 + (needV ? 1 : 0) + (doDK ? 1 : 0) + (doDV ? 1 : 0);
-        uint32_t bytes = ntiles * parts * qtile + nrows * 64;
+        uint32_t bytes = (1 + (needV ? 1 : 0)) * parts * qtile + nrows * 64;
         if (CAL == CAL_MINMAX) bytes += nrows * tstride;
         mbar_arrive_expect_tx(b, bytes);
         load_rows_tile(dst + oQ, &maps.q, b, D, BT, 0, q0, bh);
@@ -709,17 +713,19 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
           load_rows_tile(dst + odO, &maps.dout, b, D, BT, 0, q0, bh);
           if (p.x3) load_rows_tile(dst + odO + qtile, &maps.dout_lo, b, D, BT, 0, q0, bh);
         }
-        if (doDK) {
-          load_rows_tile(dst + oQT, &maps.qt, b, BT, D, q0, 0, bh);
-          if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, b, BT, D, q0, 0, bh);
-        }
-        if (doDV) {
-          load_rows_tile(dst + odOT, &maps.dot, b, BT, D, q0, 0, bh);
-          if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, b, BT, D, q0, 0, bh);
-        }
         const size_t r0 = (size_t)bh * p.T + q0;
         bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
         if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
+        uint64_t* bt = &bar_fullT[s];
+        mbar_arrive_expect_tx(bt, ((doDK ? 1 : 0) + (doDV ? 1 : 0)) * parts * qtile);
+        if (doDK) {
+          load_rows_tile(dst + oQT, &maps.qt, bt, BT, D, q0, 0, bh);
+          if (p.x3) load_rows_tile(dst + oQT + qtile, &maps.qt_lo, bt, BT, D, q0, 0, bh);
+        }
+        if (doDV) {
+          load_rows_tile(dst + odOT, &maps.dot, bt, BT, D, q0, 0, bh);
+          if (p.x3) load_rows_tile(dst + odOT + qtile, &maps.dot_lo, bt, BT, D, q0, 0, bh);
+        }
       }
     }
     // the last-but-one item's tiles (the last item's are stored by the compute warps)
@@ -742,7 +748,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         if (nbuf == 2 && it + 1 < nit)
           ok = kv_issue_sg(p, g + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
         if (!ok) break;
-        if (!mbar_wait_warp(&bar_pready[b], (g / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
+        if (!mbar_wait_warp(&bar_pready[b], (g / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) ||
+            !mbar_wait_warp(&bar_fullT[s], (g / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
