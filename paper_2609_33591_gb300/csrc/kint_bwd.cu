@@ -90,11 +90,11 @@ __device__ __forceinline__ void add_tied_keys(uint32_t mask, float* acc, const f
 
 // MMA thread of k_bwd_dq: wait for key tile kt, then S_b = Q K^T and g_b = dO V^T
 // into score buffer b = kt % nbuf.
-__device__ __forceinline__ bool dq_issue_sg(const Params& p, int kt, uint64_t* bar_full, uint64_t* bar_sfull,
-                                            const uint8_t* st0, uint32_t cQa, uint32_t cdOa, uint32_t cSG,
-                                            int ktile) {
-  const int D = p.d, NS = p.nstage, s = kt % NS, b = kt % p.nbuf, parts = p.x3 ? 2 : 1;
-  if (!mbar_wait_warp(&bar_full[s], (kt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+__device__ __forceinline__ bool dq_issue_sg(const Params& p, RingPos stg, int b, uint64_t* bar_full,
+                                            uint64_t* bar_sfull, const uint8_t* st0, uint32_t cQa, uint32_t cdOa,
+                                            uint32_t cSG, int ktile) {
+  const int D = p.d, s = stg.i, parts = p.x3 ? 2 : 1;
+  if (!mbar_wait_warp(&bar_full[s], stg.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
   tc_fence_after();
   const uint8_t* sk = st0 + s * p.sm_stage_bytes;
   const uint8_t* sv = sk + parts * ktile;
@@ -181,6 +181,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
 
   if (warp == PRODUCER_WARP) {
     int gt = 0, n = 0;
+    RingPos ld;  // stage of the next tile loaded
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
@@ -194,10 +195,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb * 128, bh);
         load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb * 128, bh);
       }
-      for (int kt = 0; kt < nkt; ++kt, ++gt) {
-        const int s = gt % NS;
-        if (gt >= NS &&
-            !mbar_wait_warp(&bar_empty[s], ((gt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+      for (int kt = 0; kt < nkt; ++kt, ++gt, ld.next(NS)) {
+        const int s = ld.i;
+        if (gt >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
@@ -220,7 +220,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + cSG0;
-    int gt = 0, n = 0;
+    int n = 0;
+    RingPos is, ib, cs, cb;  // stage / buffer of the next S, g product and of the tile being finished
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH;
@@ -229,12 +230,18 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       // previous item's dQ, so the first dQ product below may overwrite it)
       ok = mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
       if (ok) tc_fence_after();
-      ok = ok && dq_issue_sg(p, gt, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-      for (int kt = 0; kt < nkt && ok; ++kt) {
-        const int gk = gt + kt, b = gk % nbuf, s = gk % NS;
-        if (nbuf == 2 && kt + 1 < nkt) ok = dq_issue_sg(p, gk + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+      ok = ok && dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+      is.next(NS);
+      ib.next(nbuf);
+      for (int kt = 0; kt < nkt && ok; ++kt, cs.next(NS), cb.next(nbuf)) {
+        const int b = cb.i, s = cs.i;
+        if (nbuf == 2 && kt + 1 < nkt) {
+          ok = dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+          is.next(NS);
+          ib.next(nbuf);
+        }
         if (!ok) break;
-        if (!mbar_wait_warp(&bar_pready[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
+        if (!mbar_wait_warp(&bar_pready[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
           ok = false;
           break;
         }
@@ -250,10 +257,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
           mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
         }
         mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && kt + 1 < nkt)  // in order after the product reading S_0
-          ok = dq_issue_sg(p, gk + 1, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+        if (nbuf == 1 && kt + 1 < nkt) {  // in order after the product reading S_0
+          ok = dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+          is.next(NS);
+          ib.next(nbuf);
+        }
       }
-      gt += nkt;
       mma_commit(bar_done);
     }
   } else {
@@ -279,7 +288,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       __syncwarp();
       if ((tid & 31) == 0) mbar_arrive(bar_ops);
     };
-    int gt = 0, n = 0;
+    int n = 0;
+    RingPos cb;  // score buffer of the current tile
     bool failed = false;
     if (snake_item(0) < p.nitems) ops_to_tmem(0);
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
@@ -339,9 +349,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       }
       group_sync(BAR_COMPUTE, NCOMP);  // every column group of a row may add to its tie sums
       float own = 0.f, cm = 0.f;
-      for (int kt = 0; kt < nkt; ++kt) {
-        const int gk = gt + kt, b = gk % nbuf;
-        const bool ok = mbar_wait(&bar_sfull[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+      for (int kt = 0; kt < nkt; ++kt, cb.next(nbuf)) {
+        const int b = cb.i;
+        const bool ok = mbar_wait(&bar_sfull[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
         if (!ok) {
           failed = true;
           break;
@@ -388,7 +398,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         __syncwarp();
         if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
-      gt += nkt;
       // the next item's Q / dO (this item's S, g have all been read: the last tile's were)
       if (!failed && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
@@ -572,13 +581,13 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
   }
 }
 
-// MMA thread of k_bwd_dkdv: wait for query tile it, then S^T_b = K Q^T and (dK launches)
-// g^T_b = V dO^T into score buffer b = it % nbuf.
-__device__ __forceinline__ bool kv_issue_sg(const Params& p, int it, uint64_t* bar_full, uint64_t* bar_sfull,
-                                            const uint8_t* st0, uint32_t cKa, uint32_t cVa, uint32_t cSG,
-                                            int qtile, bool needV, int oQ, int odO) {
-  const int D = p.d, NS = p.nstage, s = it % NS, b = it % p.nbuf;
-  if (!mbar_wait_warp(&bar_full[s], (it / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+// MMA thread of k_bwd_dkdv: wait for the query tile in stage st (ring position), then
+// S^T_b = K Q^T and (dK launches) g^T_b = V dO^T into score buffer b.
+__device__ __forceinline__ bool kv_issue_sg(const Params& p, RingPos stg, int b, uint64_t* bar_full,
+                                            uint64_t* bar_sfull, const uint8_t* st0, uint32_t cKa, uint32_t cVa,
+                                            uint32_t cSG, int qtile, bool needV, int oQ, int odO) {
+  const int D = p.d, s = stg.i;
+  if (!mbar_wait_warp(&bar_full[s], stg.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
   tc_fence_after();
   const uint8_t* st = st0 + s * p.sm_stage_bytes;
   const uint32_t cS = cSG + 128 * b, cG = cS + 64;
@@ -680,6 +689,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   // (stage ring, score buffers) run on across items.
   if (warp == PRODUCER_WARP) {
     int gt = 0, n = 0;
+    RingPos ld;  // stage of the next tile loaded
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
@@ -693,10 +703,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         load_rows_tile_boxed(sm + p.sm_a, &maps.k, bar_stg, D, 128, BT, 0, kb * 128, bh);
         if (needV) load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.v, bar_stg, D, 128, BT, 0, kb * 128, bh);
       }
-      for (int it = 0; it < nit; ++it, ++gt) {
-        const int s = gt % NS, q0 = (qt0 + it) * BT;
-        if (gt >= NS &&
-            !mbar_wait_warp(&bar_empty[s], ((gt / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+      for (int it = 0; it < nit; ++it, ++gt, ld.next(NS)) {
+        const int s = ld.i, q0 = (qt0 + it) * BT;
+        if (gt >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
@@ -734,7 +743,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;
-    int gt = 0, n = 0;
+    int n = 0;
+    RingPos is, ib, cs, cb;  // stage / buffer of the next S^T, g^T product and of the tile being finished
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int kb = item / p.BH, nit = nqt - (kb * 128) / BT;
@@ -742,14 +752,19 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
       // item's last S, g were read)
       ok = mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
       if (ok) tc_fence_after();
-      ok = ok && kv_issue_sg(p, gt, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
-      for (int it = 0; it < nit && ok; ++it) {
-        const int g = gt + it, b = g % nbuf, s = g % NS;
-        if (nbuf == 2 && it + 1 < nit)
-          ok = kv_issue_sg(p, g + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+      ok = ok && kv_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+      is.next(NS);
+      ib.next(nbuf);
+      for (int it = 0; it < nit && ok; ++it, cs.next(NS), cb.next(nbuf)) {
+        const int b = cb.i, s = cs.i;
+        if (nbuf == 2 && it + 1 < nit) {
+          ok = kv_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+          is.next(NS);
+          ib.next(nbuf);
+        }
         if (!ok) break;
-        if (!mbar_wait_warp(&bar_pready[b], (g / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) ||
-            !mbar_wait_warp(&bar_fullT[s], (g / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+        if (!mbar_wait_warp(&bar_pready[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) ||
+            !mbar_wait_warp(&bar_fullT[s], cs.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
@@ -768,10 +783,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
           if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
         }
         mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && it + 1 < nit)
-          ok = kv_issue_sg(p, g + 1, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+        if (nbuf == 1 && it + 1 < nit) {
+          ok = kv_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cKa, cVa, cSG, qtile, needV, oQ, odO);
+          is.next(NS);
+          ib.next(nbuf);
+        }
       }
-      gt += nit;
       mma_commit(bar_done);
     }
   } else {
@@ -811,22 +828,23 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     const uint32_t fwtab = smem_u32(sm + p.sm_table) + (half ? 8u * kHalfTail : 0u) - 0x58000000u;
     group_sync(BAR_COMPUTE, NCOMP);  // the FWM table
     bool failed = false;
-    int gt = 0, n = 0;
+    int n = 0;
+    RingPos cs, cb;  // stage and score buffer of the current tile
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
       const int j = kb * 128 + row;
       const int* tflags = p.tileflags + (size_t)bh * p.nqt + qt0;
       int tie_next = (FULLG && CAL != CAL_SOFTMAX) ? __ldg(tflags) : 0;
-      for (int it = 0; it < nit; ++it) {
+      for (int it = 0; it < nit; ++it, cs.next(NS), cb.next(nbuf)) {
         // the tie flag of this 64-row query tile, loaded one tile ahead
         const int tie_here = tie_next;
         if (FULLG && CAL != CAL_SOFTMAX && it + 1 < nit) tie_next = __ldg(tflags + it + 1);
-        const int g = gt + it, b = g % nbuf, s = g % NS;
+        const int b = cb.i, s = cs.i;
         const int q0 = (qt0 + it) * BT;
-        const bool ok1 = mbar_wait(&bar_sfull[b], (g / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
+        const bool ok1 = mbar_wait(&bar_sfull[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
         // the stage's row records arrived with its tiles (bar_full), before the products were issued
-        const bool ok2 = ok1 && mbar_wait(&bar_full[s], (g / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+        const bool ok2 = ok1 && mbar_wait(&bar_full[s], cs.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
         if (!ok2) {
           failed = true;
           break;
@@ -879,7 +897,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         __syncwarp();
         if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
-      gt += nit;
       // the next item's K / V (this item's S^T, g^T have all been read: the last tile's were)
       if (!failed && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);

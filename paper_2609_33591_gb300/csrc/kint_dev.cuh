@@ -81,6 +81,20 @@ struct RowRec {
 };
 constexpr int REC_NOGRID = 1, REC_TIEMAX = 2, REC_TIEMIN = 4;
 
+// Position in a ring of n slots used round robin (pipeline stages, score buffers): the
+// slot and the parity of its current use, since the uses of one slot alternate the
+// phases of its mbarriers.  Kept as counters, so the per-tile paths divide nothing.
+struct RingPos {
+  int i = 0;
+  uint32_t ph = 0;
+  __device__ __forceinline__ void next(int n) {
+    if (++i == n) {
+      i = 0;
+      ph ^= 1u;
+    }
+  }
+};
+
 // n-th work item of this CTA when the grid loops over items sorted longest first:
 // rounds of gridDim.x items taken in alternating directions (CTA 0 takes the longest
 // item of even rounds and the shortest of odd ones), which evens out the per-CTA
