@@ -230,6 +230,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   // Work items as in pass 2: (query block, head), longest first, strided over the grid.
   if (warp == PRODUCER_WARP) {
     int g = 0, n = 0;
+    RingPos ld;  // stage of the next K tile loaded
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
@@ -237,9 +238,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
       mbar_arrive_expect_tx(bar_q, parts * tile);
       load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
       if (p.x3) load_rows_tile(sQ + tile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-      for (int kb = 0; kb < nkb; ++kb, ++g) {
-        const int s = g % NS;
-        if (g >= NS && !mbar_wait_warp(&bar_empty[s], ((g / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+      for (int kb = 0; kb < nkb; ++kb, ++g, ld.next(NS)) {
+        const int s = ld.i;
+        if (g >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
@@ -251,18 +252,19 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
     }
   } else if (warp == MMA_WARP) {
     int g = 0, n = 0;
+    RingPos cs;  // stage of the current K tile
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
       ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-      for (int kb = 0; kb < nkb && ok; ++kb) {
-        const int gk = g + kb, s = gk % NS, b = gk & 1;
+      for (int kb = 0; kb < nkb && ok; ++kb, cs.next(NS)) {
+        const int gk = g + kb, s = cs.i, b = gk & 1;
         // S_b was last read two tiles ago
         if (gk >= 2 && !mbar_wait_warp(&bar_sfree[b], ((gk >> 1) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
           ok = false;
           break;
         }
-        if (!mbar_wait_warp(&bar_full[s], (gk / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+        if (!mbar_wait_warp(&bar_full[s], cs.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
@@ -465,12 +467,13 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ const uint8_t* stgl_of(const uint8_t* ostg, int d) { return ostg + 128 * d * 4; }
 
-// MMA warp of k_fwd_main: wait for the K/V stage of global tile gt, S_b = Q K^T into
-// score buffer b = gt % nbuf, commit to bar_s[b].
-__device__ __forceinline__ bool main_issue_s(const Params& p, int gt, uint64_t* bar_full, uint64_t* bar_s,
-                                             const uint8_t* st0, const uint8_t* sQ, uint32_t tmem, int qtile) {
-  const int NS = p.nstage, s = gt % NS, b = gt % p.nbuf, D = p.d;
-  if (!mbar_wait_warp(&bar_full[s], (gt / NS) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
+// MMA warp of k_fwd_main: wait for the K/V stage st (ring position), S_b = Q K^T into
+// score buffer b, commit to bar_s[b].
+__device__ __forceinline__ bool main_issue_s(const Params& p, RingPos stg, int b, uint64_t* bar_full,
+                                             uint64_t* bar_s, const uint8_t* st0, const uint8_t* sQ, uint32_t tmem,
+                                             int qtile) {
+  const int s = stg.i, D = p.d;
+  if (!mbar_wait_warp(&bar_full[s], stg.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) return false;
   tc_fence_after();
   const uint8_t* sk = st0 + s * p.sm_stage_bytes;
   const uint32_t dcol = tmem + b * 128;
@@ -535,6 +538,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
 
   if (warp == PRODUCER_WARP) {
     int g = 0, n = 0;
+    RingPos ld;  // stage of the next K/V tile loaded
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
@@ -543,9 +547,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       mbar_arrive_expect_tx(bar_q, parts * qtile);
       load_rows_tile(sQ, &maps.q, bar_q, D, 128, 0, qb * 128, bh);
       if (p.x3) load_rows_tile(sQ + qtile, &maps.q_lo, bar_q, D, 128, 0, qb * 128, bh);
-      for (int kb = 0; kb < nkb; ++kb, ++g) {
-        const int s = g % NS;
-        if (g >= NS && !mbar_wait_warp(&bar_empty[s], ((g / NS) - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+      for (int kb = 0; kb < nkb; ++kb, ++g, ld.next(NS)) {
+        const int s = ld.i;
+        if (g >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
           ok = false;
           break;
         }
@@ -562,20 +566,25 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     int g = 0, n = 0;
+    RingPos is, ib, cs, cb;  // stage / buffer of the next S product and of the tile being finished
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
       ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) &&
-           main_issue_s(p, g, bar_full, bar_s, st0, sQ, tmem, qtile);
+           main_issue_s(p, is, ib.i, bar_full, bar_s, st0, sQ, tmem, qtile);
+      is.next(NS);
+      ib.next(nbuf);
       if (ok && nkb == 1) mma_commit(bar_qfree);
-      for (int kb = 0; kb < nkb && ok; ++kb) {
-        const int gk = g + kb, b = gk % nbuf, s = gk % NS;
+      for (int kb = 0; kb < nkb && ok; ++kb, cs.next(NS), cb.next(nbuf)) {
+        const int b = cb.i, s = cs.i;
         // S(kb+1) goes to the other buffer, whose last reader P V(kb-1) precedes it in issue order
         if (nbuf == 2 && kb + 1 < nkb) {
-          if (!main_issue_s(p, gk + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+          if (!main_issue_s(p, is, ib.i, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+          is.next(NS);
+          ib.next(nbuf);
           if (kb + 2 == nkb) mma_commit(bar_qfree);
         }
-        if (!mbar_wait_warp(&bar_pready[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
+        if (!mbar_wait_warp(&bar_pready[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
         // the item's first P V overwrites O: the previous item's epilogue must have read it
         if (kb == 0 && n > 0 && !mbar_wait_warp(bar_ofree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC))
           break;
@@ -595,7 +604,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
         mma_commit(&bar_empty[s]);
         // one buffer: S(kb+1) overwrites the weights P V(kb) reads, in issue order after it
         if (nbuf == 1 && kb + 1 < nkb) {
-          if (!main_issue_s(p, gk + 1, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+          if (!main_issue_s(p, is, ib.i, bar_full, bar_s, st0, sQ, tmem, qtile)) break;
+          is.next(NS);
+          ib.next(nbuf);
           if (kb + 2 == nkb) mma_commit(bar_qfree);
         }
       }
@@ -606,6 +617,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     const int row = tid & 127, cg = tid >> 7;
     const float Kf = (float)Kq;
     int g = 0, n = 0;
+    RingPos cb;  // score buffer of the current tile
     bool failed = false;
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
@@ -637,9 +649,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       group_sync(BAR_COMPUTE, NCOMP);
 
       float Wm = 0.f, Wl = 0.f;
-      for (int kb = 0; kb < nkb && !failed; ++kb) {
-        const int gk = g + kb, b = gk % nbuf;
-        if (!mbar_wait(&bar_s[b], (gk / nbuf) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
+      for (int kb = 0; kb < nkb && !failed; ++kb, cb.next(nbuf)) {
+        const int gk = g + kb, b = cb.i;
+        if (!mbar_wait(&bar_s[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
           failed = true;
           break;
         }
