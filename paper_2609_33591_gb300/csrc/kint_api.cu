@@ -336,25 +336,31 @@ cudaError_t traced(const char* name, cudaStream_t s, F&& launch) {
   return e;
 }
 
-cudaError_t prep(const float* X, float* nat_hi, float* nat_lo, float* tr_hi, float* tr_lo, int BH, int T, int Tp,
-                 int d, bool split, cudaStream_t s, const float* Y = nullptr, float* dot = nullptr) {
-  return traced("k_prep", s,
-                [&] { return launch_prep(X, nat_hi, nat_lo, tr_hi, tr_lo, BH, T, Tp, d, split, s, Y, dot); });
+// The operand copies of one pass, all in one launch.
+struct PrepList {
+  PrepJobs jobs{};
+  void add(const float* X, float* nat_hi, float* nat_lo, float* tr_hi, float* tr_lo, const float* Y = nullptr,
+           float* dot = nullptr) {
+    jobs.j[jobs.n++] = PrepJob{X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot};
+  }
+};
+cudaError_t prep(const PrepList& l, int BH, int T, int Tp, int d, bool split, cudaStream_t s) {
+  return traced("k_prep", s, [&] { return launch_prep(l.jobs, BH, T, Tp, d, split, s); });
 }
 
 // Forward prep + pass 1 (shared by kint_attn_fwd and kint_attn_debug_bins).
 int forward_prologue(const float* Q, const float* K, const float* V, const Params& p, const Workspace& w,
                      Maps& maps, cudaStream_t s) {
   const int BH = p.BH, T = p.T, d = p.d, Tp = round_up(T, 32);
+  PrepList pl;
   if (p.x3) {
-    if (prep(Q, w.qh, w.ql, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (prep(K, w.kh, w.kl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (prep(V, nullptr, nullptr, w.vth, w.vtl, BH, T, Tp, d, true, s) != cudaSuccess)
-      return KINT_ERR_LAUNCH;
+    pl.add(Q, w.qh, w.ql, nullptr, nullptr);
+    pl.add(K, w.kh, w.kl, nullptr, nullptr);
+    pl.add(V, nullptr, nullptr, w.vth, w.vtl);
   } else {
-    if (prep(V, nullptr, nullptr, w.vth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
-      return KINT_ERR_LAUNCH;
+    pl.add(V, nullptr, nullptr, w.vth, nullptr);
   }
+  if (prep(pl, BH, T, Tp, d, p.x3 != 0, s) != cudaSuccess) return KINT_ERR_LAUNCH;
   std::memset(&maps, 0, sizeof(maps));
   bool ok = true;
   if (p.x3) {
@@ -489,20 +495,18 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   if (cudaMemsetAsync(p.tileflags, 0, (size_t)BH * p.nqt * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
 
   // Operand copies: K-major transposes (and 3xTF32 splits).
+  PrepList pl;
   if (p.x3) {
-    if (prep(Q, w.qh, w.ql, w.qth, w.qtl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (prep(K, w.kh, w.kl, w.kth, w.ktl, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (prep(V, w.vh, w.vl, nullptr, nullptr, BH, T, Tp, d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
-    if (prep(dO, w.doh, w.dol, w.doth, w.dotl, BH, T, Tp, d, true, s, p.Ostar, w.gbar) != cudaSuccess)
-      return KINT_ERR_LAUNCH;
+    pl.add(Q, w.qh, w.ql, w.qth, w.qtl);
+    pl.add(K, w.kh, w.kl, w.kth, w.ktl);
+    pl.add(V, w.vh, w.vl, nullptr, nullptr);
+    pl.add(dO, w.doh, w.dol, w.doth, w.dotl, p.Ostar, w.gbar);
   } else {
-    if (prep(Q, nullptr, nullptr, w.qth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
-      return KINT_ERR_LAUNCH;
-    if (prep(K, nullptr, nullptr, w.kth, nullptr, BH, T, Tp, d, false, s) != cudaSuccess)
-      return KINT_ERR_LAUNCH;
-    if (prep(dO, nullptr, nullptr, w.doth, nullptr, BH, T, Tp, d, false, s, p.Ostar, w.gbar) != cudaSuccess)
-      return KINT_ERR_LAUNCH;
+    pl.add(Q, nullptr, nullptr, w.qth, nullptr);
+    pl.add(K, nullptr, nullptr, w.kth, nullptr);
+    pl.add(dO, nullptr, nullptr, w.doth, nullptr, p.Ostar, w.gbar);
   }
+  if (prep(pl, BH, T, Tp, d, p.x3 != 0, s) != cudaSuccess) return KINT_ERR_LAUNCH;
   Maps maps;
   std::memset(&maps, 0, sizeof(maps));
   bool ok = true;

@@ -13,67 +13,80 @@ namespace kint {
 // ---------------------------------------------------------------------------
 // Operand preparation (HBM-bound).  tcgen05.mma kind::tf32 reads both operands
 // K-major, so every second-stage product (P V, dS K, P^T dO, dS^T Q) reads a
-// transposed copy X^T [BH][d][Tp].  3xTF32 also needs tf32 hi/lo splits.  With
-// DOT the block also forms the row dot products dot[t] = X_t . Y_t (the
-// backward's <g>_{P*} = dO_i . O*_i, App. B) from the rows it already holds.
-// CTA = 64 rows of one head, all d columns in 64-column steps; float4 loads and
-// stores, a padded 64 x 65 shared tile per step.
+// transposed copy X^T [BH][d][Tp].  3xTF32 also needs tf32 hi/lo splits.  A job
+// with Y also forms the row dot products dot[t] = X_t . Y_t (the backward's
+// <g>_{P*} = dO_i . O*_i, App. B) from the rows it already holds.
+// One launch serves up to four tensors (blockIdx.z picks the job).  CTA = 64 rows
+// of one head, all d columns in 64-column steps; 128 threads, eight float4 loads
+// and stores each per step (all in flight together), a padded 64 x 65 shared tile.
+// Small CTAs keep a launch of 1536 CTAs per tensor inside one wave of the GPU.
 // ---------------------------------------------------------------------------
-template <bool SPLIT, bool DOT>
-__global__ void __launch_bounds__(256) k_prep(const float* __restrict__ X, const float* __restrict__ Y,
-                                              float* __restrict__ nat_hi, float* __restrict__ nat_lo,
-                                              float* __restrict__ tr_hi, float* __restrict__ tr_lo,
-                                              float* __restrict__ dot, int T, int Tp, int d) {
+template <bool SPLIT>
+__global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs jobs, int T, int Tp, int d) {
   __shared__ float hs[64][65];
   __shared__ float ls[SPLIT ? 64 : 1][65];
+  const PrepJob& J = jobs.j[blockIdx.z];
   const int t0 = blockIdx.x * 64, bh = blockIdx.y, tid = threadIdx.x;
-  const int r = tid >> 4, c4 = tid & 15;  // load phase: rows r + 16 q, columns 4 c4 .. 4 c4 + 3
-  const int k = tid >> 4, tq = tid & 15;  // store phase: output rows k + 16 q, keys 4 tq .. 4 tq + 3
+  const int r = tid >> 4, c4 = tid & 15;  // load phase: rows r + 8 q, columns 4 c4 .. 4 c4 + 3
+  const int k = tid >> 4, tq = tid & 15;  // store phase: output rows k + 8 q, keys 4 tq .. 4 tq + 3
   const size_t nat = (size_t)bh * T * d, tr = (size_t)bh * d * Tp;
-  float dacc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int k0 = 0; k0 < d; k0 += 64) {
+  const bool dotj = J.Y != nullptr;
+  float dacc[8];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int rr = r + 16 * q, t = t0 + rr;
-      const size_t off = nat + (size_t)t * d + k0 + 4 * c4;
-      float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (t < T) x = __ldg(reinterpret_cast<const float4*>(X + off));
-      if constexpr (DOT) {
+  for (int q = 0; q < 8; ++q) dacc[q] = 0.f;
+  for (int k0 = 0; k0 < d; k0 += 64) {
+    float4 x[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int t = t0 + r + 8 * q;
+      x[q] = t < T ? __ldg(reinterpret_cast<const float4*>(J.X + nat + (size_t)t * d + k0 + 4 * c4))
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    if (dotj) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int t = t0 + r + 8 * q;
         if (t < T) {
-          const float4 y = __ldg(reinterpret_cast<const float4*>(Y + off));
-          dacc[q] = __fmaf_rn(x.x, y.x, dacc[q]);
-          dacc[q] = __fmaf_rn(x.y, y.y, dacc[q]);
-          dacc[q] = __fmaf_rn(x.z, y.z, dacc[q]);
-          dacc[q] = __fmaf_rn(x.w, y.w, dacc[q]);
+          const float4 y = __ldg(reinterpret_cast<const float4*>(J.Y + nat + (size_t)t * d + k0 + 4 * c4));
+          dacc[q] = __fmaf_rn(x[q].x, y.x, dacc[q]);
+          dacc[q] = __fmaf_rn(x[q].y, y.y, dacc[q]);
+          dacc[q] = __fmaf_rn(x[q].z, y.z, dacc[q]);
+          dacc[q] = __fmaf_rn(x[q].w, y.w, dacc[q]);
         }
       }
+    }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int rr = r + 8 * q, t = t0 + rr;
+      float4 v = x[q];
       if constexpr (SPLIT) {
         float4 h, l;
-        h.x = tf32_rna(x.x); l.x = __fsub_rn(x.x, h.x);
-        h.y = tf32_rna(x.y); l.y = __fsub_rn(x.y, h.y);
-        h.z = tf32_rna(x.z); l.z = __fsub_rn(x.z, h.z);
-        h.w = tf32_rna(x.w); l.w = __fsub_rn(x.w, h.w);
-        if (t < T && nat_hi) {
-          *reinterpret_cast<float4*>(nat_hi + off) = h;
-          *reinterpret_cast<float4*>(nat_lo + off) = l;
+        h.x = tf32_rna(v.x); l.x = __fsub_rn(v.x, h.x);
+        h.y = tf32_rna(v.y); l.y = __fsub_rn(v.y, h.y);
+        h.z = tf32_rna(v.z); l.z = __fsub_rn(v.z, h.z);
+        h.w = tf32_rna(v.w); l.w = __fsub_rn(v.w, h.w);
+        if (t < T && J.nat_hi) {
+          const size_t off = nat + (size_t)t * d + k0 + 4 * c4;
+          *reinterpret_cast<float4*>(J.nat_hi + off) = h;
+          *reinterpret_cast<float4*>(J.nat_lo + off) = l;
         }
-        x = h;
+        v = h;
         ls[rr][4 * c4] = l.x; ls[rr][4 * c4 + 1] = l.y; ls[rr][4 * c4 + 2] = l.z; ls[rr][4 * c4 + 3] = l.w;
       }
-      hs[rr][4 * c4] = x.x; hs[rr][4 * c4 + 1] = x.y; hs[rr][4 * c4 + 2] = x.z; hs[rr][4 * c4 + 3] = x.w;
+      hs[rr][4 * c4] = v.x; hs[rr][4 * c4 + 1] = v.y; hs[rr][4 * c4 + 2] = v.z; hs[rr][4 * c4 + 3] = v.w;
     }
     __syncthreads();
-    if (tr_hi) {
+    if (J.tr_hi) {
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int kk = k + 16 * q, t = t0 + 4 * tq;
+      for (int q = 0; q < 8; ++q) {
+        const int kk = k + 8 * q, t = t0 + 4 * tq;
         if (t < Tp) {
           const size_t off = tr + (size_t)(k0 + kk) * Tp + t;
-          *reinterpret_cast<float4*>(tr_hi + off) =
+          *reinterpret_cast<float4*>(J.tr_hi + off) =
               make_float4(hs[4 * tq][kk], hs[4 * tq + 1][kk], hs[4 * tq + 2][kk], hs[4 * tq + 3][kk]);
           if constexpr (SPLIT) {
-            if (tr_lo)
-              *reinterpret_cast<float4*>(tr_lo + off) =
+            if (J.tr_lo)
+              *reinterpret_cast<float4*>(J.tr_lo + off) =
                   make_float4(ls[4 * tq][kk], ls[4 * tq + 1][kk], ls[4 * tq + 2][kk], ls[4 * tq + 3][kk]);
           }
         }
@@ -81,32 +94,25 @@ __global__ void __launch_bounds__(256) k_prep(const float* __restrict__ X, const
     }
     __syncthreads();
   }
-  if constexpr (DOT) {
+  if (dotj) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < 8; ++q) {
       float v = dacc[q];
 #pragma unroll
       for (int o = 8; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-      const int t = t0 + r + 16 * q;
-      if (c4 == 0 && t < T) dot[(size_t)bh * T + t] = v;
+      const int t = t0 + r + 8 * q;
+      if (c4 == 0 && t < T) J.dot[(size_t)bh * T + t] = v;
     }
   }
 }
 
-cudaError_t launch_prep(const float* X, float* nat_hi, float* nat_lo, float* tr_hi, float* tr_lo, int BH, int T,
-                        int Tp, int d, bool split, cudaStream_t s, const float* Y, float* dot) {
-  dim3 grid((Tp + 63) / 64, BH), block(256);
-  if (dot) {
-    if (split)
-      k_prep<true, true><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
-    else
-      k_prep<false, true><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
-  } else {
-    if (split)
-      k_prep<true, false><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
-    else
-      k_prep<false, false><<<grid, block, 0, s>>>(X, Y, nat_hi, nat_lo, tr_hi, tr_lo, dot, T, Tp, d);
-  }
+cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, cudaStream_t s) {
+  if (jobs.n <= 0) return cudaSuccess;
+  dim3 grid((Tp + 63) / 64, BH, jobs.n), block(128);
+  if (split)
+    k_prep<true><<<grid, block, 0, s>>>(jobs, T, Tp, d);
+  else
+    k_prep<false><<<grid, block, 0, s>>>(jobs, T, Tp, d);
   return cudaGetLastError();
 }
 
