@@ -309,7 +309,7 @@ int plan_dkdv(Params& p, int sel) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     // FWM Nearest: the half-bin table, 2K + 3 entries of 8 bytes
     const int table = p.calib == KINT_CALIB_FWM ? 2048 : 1024;
-    const int total = std::max(finish_plan(p, p.sm_table + table, 3 * p.nstage + 8), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_table + table, 4 * p.nstage + 8), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       // one CTA per SM looping over the (key block, head) items

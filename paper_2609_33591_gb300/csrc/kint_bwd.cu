@@ -647,7 +647,11 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   // a stage's transposed tiles (Q^T, dO^T) complete on their own barrier, so the products
   // S^T, g^T wait only for the first half of the stage's bytes
   uint64_t* bar_fullT = bars + 2 * NS + 8;  // [NS]
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 * NS + 8);
+  // the first half of a stage (Q, dO, row records) is free once the compute warps are done
+  // with the tile (S^T, g^T completed before they started); the transposed half once the
+  // products dV, dK that read it complete (bar_empty)
+  uint64_t* bar_emptyA = bars + 3 * NS + 8;  // [NS]
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 4 * NS + 8);
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const int dp = D * parts;
   const int cK = 0, cV = dp, base = needV ? 2 * dp : dp;
@@ -664,6 +668,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_fullT[s], 1);
       mbar_init(&bar_empty[s], 1);
+      mbar_init(&bar_emptyA[s], NCOMP / 32);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
@@ -705,7 +710,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
       }
       for (int it = 0; it < nit; ++it, ++gt, ld.next(NS)) {
         const int s = ld.i, q0 = (qt0 + it) * BT;
-        if (gt >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+        if (gt >= NS && !mbar_wait_warp(&bar_emptyA[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
           ok = false;
           break;
         }
@@ -725,6 +730,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         const size_t r0 = (size_t)bh * p.T + q0;
         bulk_load(dst + oRec, reinterpret_cast<const RowRec*>(p.rec) + r0, nrows * 64, b);
         if (CAL == CAL_MINMAX) bulk_load(dst + oTab, p.rtab + r0 * p.Kp * 2, nrows * tstride, b);
+        if (gt >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
         uint64_t* bt = &bar_fullT[s];
         mbar_arrive_expect_tx(bt, ((doDK ? 1 : 0) + (doDV ? 1 : 0)) * parts * qtile);
         if (doDK) {
@@ -892,6 +901,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
             if (doDK) tmem_stw<WS>(lane_addr(tmem, cG), da);
           }
         }
+        __syncwarp();
+        if ((tid & 31) == 0) mbar_arrive(&bar_emptyA[s]);  // the stage's records are read
         tmem_st_wait();
         tc_fence_before();
         __syncwarp();
