@@ -148,7 +148,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   uint64_t* bar_ops = bars + 2 * NS + 5;  // Q / dO rows stored in TMEM by every compute warp (per item)
   uint64_t* bar_stg = bars + 2 * NS + 6;   // Q / dO tiles staged in smem by TMA (per item)
   uint64_t* bar_ostg = bars + 2 * NS + 7;  // an item's dQ tile staged in the Q / dO area
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2 * NS + 8);
+  // K and V of a stage are free once S, g of the tile completed (the compute warps, which
+  // waited for them, arrive); K^T once the dQ product reading it completes (bar_empty)
+  uint64_t* bar_emptyA = bars + 2 * NS + 8;  // [NS]
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 * NS + 8);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
   constexpr int W = BT / NCG;  // key columns per thread per tile
@@ -159,6 +162,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     for (int s = 0; s < NS; ++s) {
       mbar_init(&bar_full[s], 1);
       mbar_init(&bar_empty[s], 1);
+      mbar_init(&bar_emptyA[s], NCOMP / 32);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
@@ -197,7 +201,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       }
       for (int kt = 0; kt < nkt; ++kt, ++gt, ld.next(NS)) {
         const int s = ld.i;
-        if (gt >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+        if (gt >= NS && !mbar_wait_warp(&bar_emptyA[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
           ok = false;
           break;
         }
@@ -206,12 +210,16 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         mbar_arrive_expect_tx(b, 3 * parts * ktile);
         load_rows_tile(dst, &maps.k, b, D, BT, 0, kt * BT, bh);
         load_rows_tile(dst + parts * ktile, &maps.v, b, D, BT, 0, kt * BT, bh);
-        load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
         if (p.x3) {
           load_rows_tile(dst + ktile, &maps.k_lo, b, D, BT, 0, kt * BT, bh);
           load_rows_tile(dst + parts * ktile + ktile, &maps.v_lo, b, D, BT, 0, kt * BT, bh);
-          load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
         }
+        if (gt >= NS && !mbar_wait_warp(&bar_empty[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA)) {
+          ok = false;
+          break;
+        }
+        load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
+        if (p.x3) load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
       }
     }
     // the last-but-one item's tile (the last item's is stored by the compute warps)
@@ -289,7 +297,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
       if ((tid & 31) == 0) mbar_arrive(bar_ops);
     };
     int n = 0;
-    RingPos cb;  // score buffer of the current tile
+    RingPos cb, cs;  // score buffer and stage of the current tile
     bool failed = false;
     if (snake_item(0) < p.nitems) ops_to_tmem(0);
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
@@ -356,6 +364,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
           failed = true;
           break;
         }
+        // S, g of the tile completed: its K and V may be reloaded
+        if ((tid & 31) == 0) mbar_arrive(&bar_emptyA[cs.i]);
+        cs.next(NS);
         tc_fence_after();
         const int cS = cSG0 + 128 * b + cg * W, cG = cS + 64;
         float sv[W], gv[W], out[W];
