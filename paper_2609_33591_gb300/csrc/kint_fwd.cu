@@ -540,7 +540,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *tslot;
+  // All 512 columns are allocated, so the allocation starts at lane 0, column 0; a
+  // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
+  if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
+  constexpr uint32_t tmem = 0;
 
   if (warp == PRODUCER_WARP) {
     int g = 0, n = 0;
