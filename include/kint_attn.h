@@ -71,11 +71,12 @@ typedef enum { KINT_PREC_TF32 = 0, KINT_PREC_3XTF32 = 1 } kint_prec;
  * arrays are caller-owned device memory of B*H*T elements unless noted. */
 typedef struct {
   float* row_max;    /* M_i = max_j s_ij over valid keys (App. A) */
-  float* row_min;    /* m_i = min_j s_ij (written for FWM too, as a diagnostic) */
+  float* row_min;    /* m_i = min_j s_ij; MinMax only (the FWM and softmax grids are
+                        anchored at M_i alone): otherwise set to +inf */
   int32_t* arg_max;  /* lowest j with s_ij == M_i */
-  int32_t* arg_min;  /* lowest j with s_ij == m_i */
+  int32_t* arg_min;  /* lowest j with s_ij == m_i; -1 when row_min is not computed */
   int32_t* n_max;    /* number of keys tied at M_i (the extremum gradient is split evenly) */
-  int32_t* n_min;    /* number of keys tied at m_i */
+  int32_t* n_min;    /* number of keys tied at m_i; 0 when row_min is not computed */
   float* W;          /* W^N = sum w^N (Nearest) or W^L (LERP); softmax: sum e^{s - M} */
   float* W_lerp;     /* W^L; required for Prob-STE, may be NULL otherwise */
   float* O_lerp;     /* [B,H,T,d] P^L V; required for Prob-STE, may be NULL otherwise */

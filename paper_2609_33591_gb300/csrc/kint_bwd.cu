@@ -432,7 +432,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
         const bool full = FULLG && CAL != CAL_SOFTMAX && !g.nogrid;
         const float cmv = (full && minmax) ? cm_t : 0.f;
         const float cMv = full ? (-own_t - cmv) : 0.f;
-        const float cMn = cMv / (float)nmax, cmn = cmv / (float)nmin;
+        // (n_min is 0 where the minimum side was not computed, and c_m is 0 there)
+        const float cMn = cMv / (float)nmax, cmn = (minmax && nmin > 0) ? cmv / (float)nmin : 0.f;
         const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
         const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
         // dQ rows into a swizzled tile for a TMA store: in the Q / dO staging area (free now

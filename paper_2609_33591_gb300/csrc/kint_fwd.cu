@@ -130,7 +130,9 @@ cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool
 // taken while a lane's running extremum can still move) the lanes whose chunk
 // reaches their running extremum count the chunk's equal keys with a bit mask;
 // its lowest set bit is the lowest index.  Masked keys (j > i) take -inf / +inf.
-template <bool DIAG>
+// MIN: also the minimum side, which only the MinMax grid spans (FWM and the softmax
+// comparator are anchored at M alone).
+template <bool DIAG, bool MIN>
 __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float scale, float& M, float& m,
                                             int& amax, int& amin, int& nmax, int& nmin) {
   float hi[16], lo[16];
@@ -147,17 +149,17 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
       b2 = ob ? b2 : INFINITY;
     }
     hi[jj] = fmaxf(a, b);
-    lo[jj] = fminf(a2, b2);
+    if constexpr (MIN) lo[jj] = fminf(a2, b2);
   }
 #pragma unroll
   for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll
     for (int jj = 0; jj < w; ++jj) {
       hi[jj] = fmaxf(hi[jj], hi[jj + w]);
-      lo[jj] = fminf(lo[jj], lo[jj + w]);
+      if constexpr (MIN) lo[jj] = fminf(lo[jj], lo[jj + w]);
     }
-  const float cmax = hi[0], cmin = lo[0];
-  const bool um = cmax >= M, un = cmin <= m;
+  const float cmax = hi[0], cmin = MIN ? lo[0] : 0.f;
+  const bool um = cmax >= M, un = MIN && cmin <= m;
   if (__any_sync(0xffffffffu, um)) {
     uint32_t mk = 0;
 #pragma unroll
@@ -175,7 +177,7 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
       }
     }
   }
-  if (__any_sync(0xffffffffu, un)) {
+  if (MIN && __any_sync(0xffffffffu, un)) {
     uint32_t mk = 0;
 #pragma unroll
     for (int jj = 0; jj < 32; ++jj) {
@@ -196,6 +198,7 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
 
 static dim3 launch_grid(const Params& p) { return dim3((unsigned)p.ngrid); }
 
+template <bool MIN>
 __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, tile = D * 512, parts = p.x3 ? 2 : 1, NS = p.nstage;
@@ -315,9 +318,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
           tmem_ld_wait();
           const int j0 = kb * 128 + c * 32;
           if (diag)
-            stats_chunk<true>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+            stats_chunk<true, MIN>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
           else
-            stats_chunk<false>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+            stats_chunk<false, MIN>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
         }
         tc_fence_before();
         __syncwarp();
@@ -347,12 +350,18 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
         } else if (M1 == M) {
           nmax += nmax1;
         }
-        if (m1 < m || (m1 == m && nmin1 > 0 && amin1 < amin)) amin = (m1 < m || nmin == 0) ? amin1 : min(amin, amin1);
-        if (m1 < m) {
-          nmin = nmin1;
-          m = m1;
-        } else if (m1 == m) {
-          nmin += nmin1;
+        if (MIN) {
+          if (m1 < m || (m1 == m && nmin1 > 0 && amin1 < amin)) amin = (m1 < m || nmin == 0) ? amin1 : min(amin, amin1);
+          if (m1 < m) {
+            nmin = nmin1;
+            m = m1;
+          } else if (m1 == m) {
+            nmin += nmin1;
+          }
+        } else {  // not computed: +inf, index -1, count 0
+          m = INFINITY;
+          amin = -1;
+          nmin = 0;
         }
         const size_t rw = (size_t)bh * p.T + i;
         p.row_max[rw] = M;
@@ -371,9 +380,10 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
 }
 
 cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(k_fwd_stats, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+  auto kern = p.calib == CAL_MINMAX ? k_fwd_stats<true> : k_fwd_stats<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  k_fwd_stats<<<launch_grid(p), NTHR, smem_bytes, s>>>(maps, p);
+  kern<<<launch_grid(p), NTHR, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
 }
 
