@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "f921414081153833", "k_prep": 31479680, "k_fwd_stats": 50386432, "k_fwd_main": 95098112,
-           "k_bwd_dq": 196307968, "k_bwd_dkdv": 185556224}
+TRAFFIC = {"src": "9c7391497459bd11", "k_prep": 81723520, "k_fwd_stats": 50369792, "k_fwd_main": 94741504,
+           "k_bwd_dq": 189582848, "k_bwd_dkdv": 273446144}
 
 
 def kernel_source_digest() -> str:
@@ -209,7 +209,9 @@ KERNEL_WORK = {
     "k_fwd_main": ("tensor", 1),   # PV (its QK^T is a recomputation)
     "k_bwd_dq": ("tensor", 2),     # dP = dO V^T, dQ = dS K
     "k_bwd_dkdv": ("tensor", 2),   # dV = P^T dO, dK = dS^T Q (S^T, dP^T are recomputations)
-    "k_prep": ("hbm", None),       # one read + one write of a [B,H,T,d] fp32 tensor
+    # per launch, [B,H,T,d] fp32 tensor passes: the forward launch reads V and writes V^T (2),
+    # the backward one reads Q, K, dO and O* and writes three transposes (7); 4.5 on average
+    "k_prep": ("hbm", 4.5),
 }
 
 
@@ -305,7 +307,7 @@ def run_cuda(args, world, rank, local):
                 "frac": achieved / tf32_peak, "traffic": traffic,
                 "peak_note": f"TF32 = (1.1 / 2.25 nominal) x {pk['source']} bf16 burst {pk['bf16']} TFLOP/s"}
     else:
-        nbytes = 2 * B * H * T * d * 4
+        nbytes = units * B * H * T * d * 4
         achieved = nbytes / avg_s / 1e9
         roof = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / pk["hbm_gbs"], "traffic": None}
