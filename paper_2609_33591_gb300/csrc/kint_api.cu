@@ -282,7 +282,7 @@ int plan_dq(Params& p) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
     p.sm_ostage = 0;
-    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 3 * p.nstage + 8), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 3 * p.nstage + 10), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       p.ngrid = std::min(p.nitems, num_sms());

@@ -135,7 +135,7 @@ __device__ __forceinline__ bool store_staged_dq(const Maps& maps, const Params& 
 }
 
 template <int CAL, bool FULLG>
-__global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int ktile = BT * D * 4;
@@ -151,7 +151,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
   // K and V of a stage are free once S, g of the tile completed (the compute warps, which
   // waited for them, arrive); K^T once the dQ product reading it completes (bar_empty)
   uint64_t* bar_emptyA = bars + 2 * NS + 8;  // [NS]
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 * NS + 8);
+  // score buffer b free again: the dQ product that read its dS completed (MMA2 -> MMA warp)
+  uint64_t* bar_dqdone = bars + 3 * NS + 8;  // [2]
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 3 * NS + 10);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
   constexpr int W = BT / NCG;  // key columns per thread per tile
@@ -167,6 +169,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
       mbar_init(&bar_pready[b], NCOMP / 32);
+      mbar_init(&bar_dqdone[b], 1);
     }
     mbar_init(bar_done, 1);
     mbar_init(bar_ops, NCOMP / 32);
@@ -229,29 +232,39 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
     if (p.ops_smem && ok && n >= 2) store_staged_dq(maps, p, bar_ostg, n - 2, sm + p.sm_a);
     tma_store_wait_all();
   } else if (warp == MMA_WARP) {
+    // S, g of every tile, into score buffer b once the dQ product that read the buffer's
+    // previous dS has completed (bar_dqdone)
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cQa = tmem + cQ, cdOa = tmem + cdO, cSG = tmem + cSG0;
-    int n = 0;
-    RingPos is, ib, cs, cb;  // stage / buffer of the next S, g product and of the tile being finished
+    int n = 0, g = 0;
+    RingPos is, ib;  // stage and buffer of the next S, g product
     bool ok = true;
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH;
       const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
-      // Q / dO of the item in TMEM (the compute warps copy them only after reading the
-      // previous item's dQ, so the first dQ product below may overwrite it)
+      // Q / dO of the item in TMEM (copied by the compute warps once the previous item's
+      // last S, g were read)
       ok = mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
       if (ok) tc_fence_after();
-      ok = ok && dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-      is.next(NS);
-      ib.next(nbuf);
+      for (int kt = 0; kt < nkt && ok; ++kt, ++g, is.next(NS), ib.next(nbuf)) {
+        if (g >= nbuf &&
+            !mbar_wait_warp(&bar_dqdone[ib.i], ib.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
+          ok = false;
+          break;
+        }
+        ok = dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
+      }
+    }
+  } else if (warp == MMA2_WARP) {
+    // dQ += dS K of every tile once the compute warps wrote its dS
+    RingPos cs, cb;  // stage and buffer of the tile being finished
+    int n = 0;
+    bool ok = true;
+    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+      const int qb = p.nqb - 1 - item / p.BH;
+      const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
       for (int kt = 0; kt < nkt && ok; ++kt, cs.next(NS), cb.next(nbuf)) {
         const int b = cb.i, s = cs.i;
-        if (nbuf == 2 && kt + 1 < nkt) {
-          ok = dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-          is.next(NS);
-          ib.next(nbuf);
-        }
-        if (!ok) break;
         if (!mbar_wait_warp(&bar_pready[b], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
           ok = false;
           break;
@@ -268,11 +281,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dq(const __grid_constant__ Maps
           mma_tmem_smem(tmem + cdQ, cS, skt, D, BT, acc);
         }
         mma_commit(&bar_empty[s]);
-        if (nbuf == 1 && kt + 1 < nkt) {  // in order after the product reading S_0
-          ok = dq_issue_sg(p, is, ib.i, bar_full, bar_sfull, st0, cQa, cdOa, cSG, ktile);
-          is.next(NS);
-          ib.next(nbuf);
-        }
+        mma_commit(&bar_dqdone[b]);
       }
       mma_commit(bar_done);
     }
@@ -981,22 +990,23 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
 
 // ---------------------------------------------------------------------------
 template <class K>
-static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s,
+                           int nthr = NTHR) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<grid, NTHR, smem_bytes, s>>>(maps, p);
+  kern<<<grid, nthr, smem_bytes, s>>>(maps, p);
   return cudaGetLastError();
 }
 
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   const dim3 grid((unsigned)p.ngrid);
   const bool full = p.grad == 0;
-  if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s);
+  if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
   if (p.calib == CAL_MINMAX)
-    return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s)
-                : launch3(k_bwd_dq<CAL_MINMAX, false>, grid, maps, p, smem_bytes, s);
-  return full ? launch3(k_bwd_dq<CAL_FWM, true>, grid, maps, p, smem_bytes, s)
-              : launch3(k_bwd_dq<CAL_FWM, false>, grid, maps, p, smem_bytes, s);
+    return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
+                : launch3(k_bwd_dq<CAL_MINMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
+  return full ? launch3(k_bwd_dq<CAL_FWM, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
+              : launch3(k_bwd_dq<CAL_FWM, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
 }
 
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {

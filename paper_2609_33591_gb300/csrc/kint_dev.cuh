@@ -49,6 +49,10 @@ constexpr int NCOMP = 128 * NCG;
 constexpr int NTHR = NCOMP + 64;
 constexpr int MMA_WARP = NCOMP / 32;
 constexpr int PRODUCER_WARP = NCOMP / 32 + 1;
+// The dQ kernel issues its two kinds of products from two warps on different SM
+// sub-partitions: S, g from MMA_WARP, dQ from MMA2_WARP.
+constexpr int MMA2_WARP = NCOMP / 32 + 2;
+constexpr int NTHR_DQ = NTHR + 32;
 constexpr int BAR_COMPUTE = 1;  // named barrier id of the compute group
 
 // W-column TMEM row access (W = 16 or 32).
