@@ -308,10 +308,38 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
       __syncwarp();
       if ((tid & 31) == 0) mbar_arrive(bar_ops);
     };
+    // The row statistics of an item, loaded one item ahead (under the previous item's epilogue).
+    struct RowIn {
+      float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
+      int nmax = 1, nmin = 1, amax = 0, amin = 0;
+    };
+    auto load_row_stats = [&](int n) {
+      RowIn r;
+      const int item = snake_item(n);
+      const int i = (p.nqb - 1 - item / p.BH) * 128 + row;
+      if (i < p.T) {
+        const size_t rw = (size_t)(item % p.BH) * p.T + i;
+        r.M = p.row_max[rw];
+        r.m = p.row_min[rw];
+        r.Wf = p.W[rw];
+        r.nmax = p.n_max[rw];
+        r.nmin = p.n_min[rw];
+        r.amax = p.arg_max[rw];
+        r.amin = p.arg_min[rw];
+        r.Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
+        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
+        r.Ws = prob ? p.W_lerp[rw] : r.Wf;
+      }
+      return r;
+    };
     int n = 0;
     RingPos cb, cs;  // score buffer and stage of the current tile
     bool failed = false;
-    if (snake_item(0) < p.nitems) ops_to_tmem(0);
+    RowIn nx;
+    if (snake_item(0) < p.nitems) {
+      ops_to_tmem(0);
+      nx = load_row_stats(0);
+    }
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       // ---- set-up: row constants, grid table (the operands are in TMEM already) ----
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
@@ -319,35 +347,24 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
       const int i = qb * 128 + row;
       const bool row_ok = i < p.T;
       const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
-      float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
-      int nmax = 1, nmin = 1, amax = 0, amin = 0;
-      RowGrid g{};
-      {
-        if (row_ok) {
-          M = p.row_max[rw];
-          m = p.row_min[rw];
-          Wf = p.W[rw];
-          nmax = p.n_max[rw];
-          nmin = p.n_min[rw];
-          amax = p.arg_max[rw];
-          amin = p.arg_min[rw];
-          Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
-        }
-        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
-        Ws = prob ? (row_ok ? p.W_lerp[rw] : 1.f) : Wf;
-        g = row_grid(p, M, m);
-        if constexpr (CAL == CAL_FWM) {
-          if (tid < 2 * Kq + 1 + kHalfTail)
-            *reinterpret_cast<float*>(sm + p.sm_table + tid * 4) = fwm_half_entry(p, tid - kHalfTail).y;
-        } else if constexpr (CAL == CAL_MINMAX) {
-          for (int r = cg; r < Kq; r += NCG) {
-            const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
-            *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
-            if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
-          }
+      const float M = nx.M, m = nx.m, Wf = nx.Wf, Ws = nx.Ws, Dg = nx.Dg;
+      const int nmax = nx.nmax, nmin = nx.nmin, amax = nx.amax, amin = nx.amin;
+      const RowGrid g = row_grid(p, M, m);
+      if constexpr (CAL == CAL_FWM) {  // the same for every item
+        if (n == 0 && tid < 2 * Kq + 1 + kHalfTail)
+          *reinterpret_cast<float*>(sm + p.sm_table + tid * 4) = fwm_half_entry(p, tid - kHalfTail).y;
+      } else if constexpr (CAL == CAL_MINMAX) {
+        for (int r = cg; r < Kq; r += NCG) {
+          const float2 e = make_float2(grid_value(p, g, r), grid_value(p, g, r + 1));
+          *reinterpret_cast<float2*>(sm + p.sm_table + (size_t)r * 1024 + row * 8) = e;
+          if (row_ok) *reinterpret_cast<float2*>(p.rtab + (rw * p.Kp + r) * 2) = e;
         }
       }
-      group_sync(BAR_COMPUTE, NCOMP);  // the grid table
+      // the arg-extremum key rows the epilogue reads, into L2 ahead of it
+      if (FULLG && CAL != CAL_SOFTMAX && row_ok) {
+        prefetch_l2(p.K + ((size_t)bh * p.T + amax) * D + cg * (D / NCG));
+        if (CAL == CAL_MINMAX) prefetch_l2(p.K + ((size_t)bh * p.T + amin) * D + cg * (D / NCG));
+      }
       const float ga = CAL == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
       const float gb = CAL == CAL_SOFTMAX ? -Dg : -Dg * ga;
       const float invWf = 1.0f / Wf;
@@ -367,7 +384,8 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         for (int k = 0; k < D; ++k) tie_max[k] = tie_min[k] = 0.f;
         atomicOr(p.tileflags + (size_t)bh * p.nqt + i / BT, 1);
       }
-      group_sync(BAR_COMPUTE, NCOMP);  // every column group of a row may add to its tie sums
+      // the grid table, and the zeroed tie sums (every column group of a row may add to them)
+      group_sync(BAR_COMPUTE, NCOMP);
       float own = 0.f, cm = 0.f;
       for (int kt = 0; kt < nkt; ++kt, cb.next(nbuf)) {
         const int b = cb.i;
@@ -422,7 +440,11 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
       // the next item's Q / dO (this item's S, g have all been read: the last tile's were)
-      if (!failed && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
+      // and its row statistics
+      if (!failed && snake_item(n + 1) < p.nitems) {
+        ops_to_tmem(n + 1);
+        nx = load_row_stats(n + 1);
+      }
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       failed = group_any(BAR_COMPUTE, NCOMP, !dok);
       if (!failed) {
