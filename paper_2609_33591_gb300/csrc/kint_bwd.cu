@@ -75,6 +75,35 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
   }
 }
 
+// Warp-cooperative gather of one 128-byte row segment per lane into the warp's 4 KB smem
+// slot: lane l passes the address of its segment (null: zeros).  Each asynchronous copy
+// instruction moves four whole segments (eight lanes each, 16 bytes per lane); 16-byte
+// chunks are swizzled by row, so both the copies and the reads are conflict-free.
+// gather_rows128_issue starts the copies; gather_rows128_read waits for them and hands
+// lane l its segment.
+__device__ __forceinline__ void gather_rows128_issue(const float* mine, float4* slot) {
+  const int l = threadIdx.x & 31;
+  const unsigned long long mp = reinterpret_cast<unsigned long long>(mine);
+  __syncwarp();  // the slot's previous contents have been read
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const int r = 4 * k + (l >> 3), ch = l & 7;
+    const unsigned long long src = __shfl_sync(0xffffffffu, mp, r);
+    const uint32_t dst = smem_u32(slot + r * 8 + (ch ^ (r & 7)));
+    const unsigned long long gsrc = src ? src + 16ull * ch : mp;  // any valid address when zero-filled
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(gsrc), "r"(src ? 16 : 0)
+                 : "memory");
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void gather_rows128_read(const float4* slot, float4 (&out)[8]) {
+  const int l = threadIdx.x & 31;
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncwarp();
+#pragma unroll
+  for (int q = 0; q < 8; ++q) out[q] = slot[l * 8 + (q ^ (l & 7))];
+}
+
 // Adds key rows j0 + b (b a set bit of `mask`) of K (rows of d floats from `k0`) to
 // the tie sum `acc` (rare path, kept rolled).
 __device__ __forceinline__ void add_tied_keys(uint32_t mask, float* acc, const float* k0, int d) {
@@ -445,6 +474,15 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         ops_to_tmem(n + 1);
         nx = load_row_stats(n + 1);
       }
+      if (p.ops_smem && FULLG && CAL != CAL_SOFTMAX) {
+        // the epilogue's arg-max key rows (this thread's column half), gathered into the dO half
+        // of the staging area (read by every warp's copy above: hence the barrier) while the
+        // item's last product completes
+        group_sync(BAR_COMPUTE, NCOMP);
+        const bool own_row = !failed && row_ok && !g.nogrid && nmax == 1;
+        gather_rows128_issue(own_row ? p.K + ((size_t)bh * p.T + amax) * D + cg * (D / NCG) : nullptr,
+                             reinterpret_cast<float4*>(sm + p.sm_a + 128 * D * 4) + warp * 256);
+      }
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       failed = group_any(BAR_COMPUTE, NCOMP, !dok);
       if (!failed) {
@@ -474,14 +512,36 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         const bool last = snake_item(n + 1) >= p.nitems;
         uint8_t* stg = last ? sm + p.sm_stage0 : sm + p.sm_a;
         for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
-          // the arg-extremum key rows first (all loads in flight before the TMEM read)
+          // the arg-extremum key rows (128 bytes of each: this column half).  With the staging
+          // area, the warp gathers its 32 rows cooperatively (four whole lines per load) into
+          // its 4 KB slot of the free dO half of that area, then each thread reads its row back;
+          // otherwise every thread loads its own row (32 lines per load).
           float4 km[8], kn[8];
+          if (p.ops_smem && FULLG && CAL != CAL_SOFTMAX) {
+            // the arg-max rows were requested before the wait for the item's last product
+            // (tie sums, complete only now, are read directly)
+            float4* slot = reinterpret_cast<float4*>(sm + p.sm_a + 128 * D * 4) + warp * 256;
+            gather_rows128_read(slot, km);
+            if (row_ok && full && nmax > 1) {
   #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            km[q] = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
-                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-            kn[q] = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
-                                               : make_float4(0.f, 0.f, 0.f, 0.f);
+              for (int q = 0; q < 8; ++q) km[q] = reinterpret_cast<const float4*>(tie_max + c)[q];
+            }
+            if (minmax) {
+              gather_rows128_issue(full && row_ok ? kmin + c : nullptr, slot);
+              gather_rows128_read(slot, kn);
+            }
+          } else {
+  #pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              km[q] = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+              kn[q] = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
+                                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+          }
+          if (!minmax) {
+  #pragma unroll
+            for (int q = 0; q < 8; ++q) kn[q] = make_float4(0.f, 0.f, 0.f, 0.f);
           }
           float v[32];
           tmem_ld32(lane_addr(tmem, cdQ + c), v);
