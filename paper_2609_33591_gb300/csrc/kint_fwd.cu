@@ -638,13 +638,22 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     int g = 0, n = 0;
     RingPos cb;  // score buffer of the current tile
     bool failed = false;
+    // the row extrema of an item, loaded one item ahead (under the previous item's epilogue)
+    auto load_extrema = [&](int n, float& M, float& m) {
+      const int item = snake_item(n);
+      const int i = (p.nqb - 1 - item / p.BH) * 128 + row;
+      const size_t rw = (size_t)(item % p.BH) * p.T + i;
+      M = i < p.T ? p.row_max[rw] : 0.0f;
+      m = i < p.T ? p.row_min[rw] : 0.0f;
+    };
+    float nM = 0.f, nm = 0.f;
+    if (snake_item(0) < p.nitems) load_extrema(0, nM, nm);
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       const int i = qb * 128 + row;
       const bool row_ok = i < p.T;
       const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
-      const float M = row_ok ? p.row_max[rw] : 0.0f;
-      const float m = row_ok ? p.row_min[rw] : 0.0f;
+      const float M = nM, m = nm;
       const RowGrid gr = row_grid(p, M, m);
       const float sk1 = p.scale * 1.4426950408889634f, sc0 = -M * 1.4426950408889634f;  // softmax, base 2
       // Pair tables, entry r = (e_r, e_{r+1}), r = 0..K-1, addressed by the float bits
@@ -712,6 +721,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
         if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
       g += nkb;
+      if (snake_item(n + 1) < p.nitems) load_extrema(n + 1, nM, nm);
       if (!failed) failed = !mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       failed = group_any(BAR_COMPUTE, NCOMP, failed);
       if (failed) break;
