@@ -213,6 +213,8 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_trigger();
+  pdl_wait();  // everything below may read what the previous kernel wrote
   // All 512 columns are allocated, so the allocation starts at lane 0, column 0; a
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
@@ -793,6 +795,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_trigger();
+  pdl_wait();  // everything below may read what the previous kernel wrote
   // All 512 columns are allocated, so the allocation starts at lane 0, column 0; a
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
@@ -1076,8 +1080,7 @@ static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p,
                            int nthr = NTHR) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<grid, nthr, smem_bytes, s>>>(maps, p);
-  return cudaGetLastError();
+  return launch_pdl(kern, grid, dim3(nthr), smem_bytes, s, maps, p);
 }
 
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {

@@ -27,6 +27,7 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
   __shared__ float ls[SPLIT ? 64 : 1][65];
   const PrepJob& J = jobs.j[blockIdx.z];
   const int t0 = blockIdx.x * 64, bh = blockIdx.y, tid = threadIdx.x;
+  pdl_wait();
   const int r = tid >> 4, c4 = tid & 15;  // load phase: rows r + 8 q, columns 4 c4 .. 4 c4 + 3
   const int k = tid >> 4, tq = tid & 15;  // store phase: output rows k + 8 q, keys 4 tq .. 4 tq + 3
   const size_t nat = (size_t)bh * T * d, tr = (size_t)bh * d * Tp;
@@ -109,11 +110,7 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
 cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, cudaStream_t s) {
   if (jobs.n <= 0) return cudaSuccess;
   dim3 grid((Tp + 63) / 64, BH, jobs.n), block(128);
-  if (split)
-    k_prep<true><<<grid, block, 0, s>>>(jobs, T, Tp, d);
-  else
-    k_prep<false><<<grid, block, 0, s>>>(jobs, T, Tp, d);
-  return cudaGetLastError();
+  return launch_pdl(split ? k_prep<true> : k_prep<false>, grid, block, 0, s, jobs, T, Tp, d);
 }
 
 // ---------------------------------------------------------------------------
@@ -234,6 +231,8 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_trigger();
+  pdl_wait();  // everything below may read what the previous kernel wrote
   const uint32_t tmem = *tslot;
 
   // Work items as in pass 2: (query block, head), longest first, strided over the grid.
@@ -383,8 +382,7 @@ cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, 
   auto kern = p.calib == CAL_MINMAX ? k_fwd_stats<true> : k_fwd_stats<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<launch_grid(p), NTHR, smem_bytes, s>>>(maps, p);
-  return cudaGetLastError();
+  return launch_pdl(kern, launch_grid(p), dim3(NTHR), smem_bytes, s, maps, p);
 }
 
 // ---------------------------------------------------------------------------
@@ -550,6 +548,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_trigger();
+  pdl_wait();  // everything below may read what the previous kernel wrote
   // All 512 columns are allocated, so the allocation starts at lane 0, column 0; a
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
@@ -786,8 +786,7 @@ static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_byt
   auto kern = k_fwd_main<CAL, REC, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  kern<<<launch_grid(p), NTHR, smem_bytes, s>>>(maps, p);
-  return cudaGetLastError();
+  return launch_pdl(kern, launch_grid(p), dim3(NTHR), smem_bytes, s, maps, p);
 }
 
 cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {

@@ -24,6 +24,14 @@ enum : unsigned {
 // receive its device address as a plain pointer argument.
 __device__ __forceinline__ void dev_flag(unsigned* status, unsigned bits) { atomicOr(status, bits); }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start while its predecessor in the stream finishes; pdl_wait()
+// returns once the predecessor grid has completed and its memory is visible (a no-op
+// without such a predecessor), so every kernel calls it before its first global access.
+// pdl_trigger() lets the successor be scheduled (onto SMs this grid has left).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // Bring the 128-byte line holding p into L2 (no register result, no wait).
 __device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
 
