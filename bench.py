@@ -262,29 +262,62 @@ def run_cuda(args, world, rank, local):
     torch.cuda.synchronize()
     kint.check_status()
 
-    # per-kernel events through the library's launch-trace hook, during the timed steps
-    events = {}
-    launches = [0]
-    cur_stream = torch.cuda.current_stream()
+    # launches per step, counted through the library's launch hook
+    per_step = [0]
+    kint.kint_set_launch_callback(lambda name, phase, stream: per_step.__setitem__(0, per_step[0] + (phase == 0)))
+    step(0)
+    kint.kint_set_launch_callback(None)
+    torch.cuda.synchronize()
 
-    def on_launch(name, phase, stream):
-        if phase == 0:
-            launches[0] += 1
-            ev = torch.cuda.Event(enable_timing=True)
-            ev.record(cur_stream)
-            events.setdefault(name, []).append([ev, None])
-        else:
-            ev = torch.cuda.Event(enable_timing=True)
-            ev.record(cur_stream)
-            events[name][-1][1] = ev
+    # The timed steps replay one CUDA graph per input set (the same kernels and launch
+    # attributes as the stream calls; the launch overhead of the Python binding stays out)
+    graphs = []
+    try:
+        cs = torch.cuda.Stream()
+        cs.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(cs):
+            for i in range(N_INPUT_SETS):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=cs):
+                    step(i)
+                graphs.append(g)
+        torch.cuda.current_stream().wait_stream(cs)
+        for g in graphs:
+            g.replay()
+        torch.cuda.synchronize()
+        kint.check_status()
+        launch_mode, run_step = "cuda_graph", (lambda i: graphs[i % N_INPUT_SETS].replay())
+    except Exception:  # capture unsupported here: plain stream launches
+        graphs = []
+        launch_mode, run_step = "stream", step
+        torch.cuda.synchronize()
 
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
-    kint.kint_set_launch_callback(on_launch)
-    ms = timed(args.steps, step)
-    kint.kint_set_launch_callback(None)
+    ms = timed(args.steps, run_step)
     clocks = sampler.stop()
+    kint.check_status()
+    launches = [per_step[0] * args.steps]
+
+    # Per-kernel durations: CUDA events on the launching stream around every launch, over a
+    # second pass of stream-launched steps (events between launches would otherwise stretch
+    # the timed steps by about 25 us each)
+    events = {}
+    cur_stream = torch.cuda.current_stream()
+
+    def on_launch(name, phase, stream):
+        ev = torch.cuda.Event(enable_timing=True)
+        ev.record(cur_stream)
+        if phase == 0:
+            events.setdefault(name, []).append([ev, None])
+        else:
+            events[name][-1][1] = ev
+
+    n_kt = max(3, min(args.steps, 200))
+    kint.kint_set_launch_callback(on_launch)
+    timed(n_kt, step)
+    kint.kint_set_launch_callback(None)
     kint.check_status()
 
     per_kernel = {}
@@ -316,11 +349,14 @@ def run_cuda(args, world, rank, local):
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "tf32", "data": "synthetic",
             "config": {"workload": WORKLOAD, **SHAPE, **{k: v for k, v in VARIANT.items()}, "prec": "tf32",
+                       "launch": launch_mode,
                        "parallelism": f"replicas x{world} (b,h)-sharded, no collective",
                        "l2": f"{N_INPUT_SETS} rotating input sets of {4 * B * H * T * d * 4 >> 20} MiB each; "
                              "per-step traffic (>300 MB) exceeds the 129 MB L2"},
             "tf32_peak_frac": value / world / tf32_peak,
-            "roofline": roof, "kernels": per_kernel, "gpu_launches": launches[0], "clocks": clocks}
+            "roofline": roof, "kernels": per_kernel,
+            "kernel_timing": f"CUDA events around each launch on its stream, over a second pass of {n_kt} steps",
+            "gpu_launches": launches[0], "clocks": clocks}
 
     # plain softmax built the same way, and the 3xTF32 mode, on the same inputs
     soft = kint.Config(Kint=4, calib=kint.CALIB_SOFTMAX, tau=8.0, recon=kint.RECON_LERP, ste=0, grad=0)
@@ -341,23 +377,51 @@ def run_cuda(args, world, rank, local):
     line["x3tf32_mode"] = {"value": job_value(flops_step, world, ms3), "unit": UNIT, "ms_per_step": ms3}
     del ws_f3, ws_b3
 
-    # end to end through the public API: pinned host inputs in, results (O, dQ, dK, dV) out, every step
+    # End to end through the public API: every step copies its inputs in from pinned host
+    # memory and its results (O, dQ, dK, dV) out.  The copies run on their own streams into
+    # and out of two alternating device buffer sets, so step i's compute overlaps step i+1's
+    # input copy and step i-1's output copy (host -> device and device -> host at once).
     pin_in = [torch.from_numpy(x).pin_memory() for x in (Qh, Kh, Vh, dOh)]
     pin_out = [torch.empty(B, H, T, d).pin_memory() for _ in range(4)]
-    dq, dk, dv = grads
-    q, k, v, do = sets[0]
+    ins = [tuple(torch.empty_like(sets[0][0]) for _ in range(4)) for _ in range(2)]
+    outs = [tuple(torch.empty_like(sets[0][0]) for _ in range(4)) for _ in range(2)]
+    s_c = torch.cuda.current_stream()
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    ev = {k: [torch.cuda.Event() for _ in range(2)] for k in ("in", "done", "out")}
+    used = set()
 
     def e2e_step(i):
-        for dst, src in zip((q, k, v, do), pin_in):
-            dst.copy_(src, non_blocking=True)
-        kint.forward(q, k, v, cfg, prec, O=O, stats=st, ws=ws_f)
-        kint.backward(q, k, v, O, do, st, cfg, prec, grads=grads, ws=ws_b)
-        for dst, src in zip(pin_out, (O, dq, dk, dv)):
-            dst.copy_(src, non_blocking=True)
+        b = i % 2
+        q, k, v, do = ins[b]
+        Ob, dq, dk, dv = outs[b]
+        with torch.cuda.stream(s_in):
+            if ("done", b) in used:
+                s_in.wait_event(ev["done"][b])  # the compute that read this input set finished
+            for dst, src in zip(ins[b], pin_in):
+                dst.copy_(src, non_blocking=True)
+            ev["in"][b].record(s_in)
+        s_c.wait_event(ev["in"][b])
+        if ("out", b) in used:
+            s_c.wait_event(ev["out"][b])  # this output set has been copied out
+        kint.forward(q, k, v, cfg, prec, O=Ob, stats=st, ws=ws_f)
+        kint.backward(q, k, v, Ob, do, st, cfg, prec, grads=(dq, dk, dv), ws=ws_b)
+        ev["done"][b].record(s_c)
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(ev["done"][b])
+            for dst, src in zip(pin_out, outs[b]):
+                dst.copy_(src, non_blocking=True)
+            ev["out"][b].record(s_out)
+        used.update((("done", b), ("out", b)))
 
-    e2e_step(0)
+    def e2e_run(n):
+        s_in.wait_stream(s_c)  # the first copy starts inside the timed region
+        for i in range(n):
+            e2e_step(i)
+        s_c.wait_stream(s_out)  # the timed region ends with the last results on the host side
+
+    e2e_run(2)
     n_e2e = max(3, min(args.steps, 100))
-    ms_e2e = timed(n_e2e, e2e_step)
+    ms_e2e = timed(1, lambda i: e2e_run(n_e2e)) / n_e2e
     line["e2e"] = {"value": job_value(flops_step, world, ms_e2e), "unit": UNIT,
                    "h2d_bytes_per_step": sum(t.numel() * 4 for t in pin_in),
                    "d2h_bytes_per_step": sum(t.numel() * 4 for t in pin_out), "ms_per_step": ms_e2e}
