@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "9c7391497459bd11", "k_prep": 81723520, "k_fwd_stats": 50369792, "k_fwd_main": 94741504,
-           "k_bwd_dq": 189582848, "k_bwd_dkdv": 273446144}
+TRAFFIC = {"src": "39fdcaaf2b05d70a", "k_prep": 81601408, "k_fwd_stats": 50368000, "k_fwd_main": 93910784,
+           "k_bwd_dq": 194736896, "k_bwd_dkdv": 273436928}
 
 
 def kernel_source_digest() -> str:
