@@ -345,7 +345,7 @@ struct PrepList {
   }
 };
 cudaError_t prep(const PrepList& l, int BH, int T, int Tp, int d, bool split, cudaStream_t s) {
-  return traced("k_prep", s, [&] { return launch_prep(l.jobs, BH, T, Tp, d, split, s); });
+  return traced("k_prep", s, [&] { return launch_prep(l.jobs, BH, T, Tp, d, split, num_sms(), s); });
 }
 
 // Forward prep + pass 1 (shared by kint_attn_fwd and kint_attn_debug_bins).

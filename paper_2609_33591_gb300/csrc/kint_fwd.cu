@@ -16,72 +16,73 @@ namespace kint {
 // transposed copy X^T [BH][d][Tp].  3xTF32 also needs tf32 hi/lo splits.  A job
 // with Y also forms the row dot products dot[t] = X_t . Y_t (the backward's
 // <g>_{P*} = dO_i . O*_i, App. B) from the rows it already holds.
-// One launch serves up to four tensors (blockIdx.z picks the job).  CTA = 64 rows
-// of one head, all d columns in 64-column steps; 128 threads, eight float4 loads
-// and stores each per step (all in flight together), a padded 64 x 65 shared tile.
-// Small CTAs keep a launch of 1536 CTAs per tensor inside one wave of the GPU.
+// One launch serves up to four tensors.  The work units (job, head, 32-row block)
+// are spread over a grid of a few CTAs per SM that loop over them, so the launch
+// has no partial last wave; a unit moves all d columns in 64-column steps through a
+// padded 32 x 65 shared tile (128 threads, four float4 loads and stores each).
 // ---------------------------------------------------------------------------
 template <bool SPLIT>
-__global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs jobs, int T, int Tp, int d) {
-  __shared__ float hs[64][65];
-  __shared__ float ls[SPLIT ? 64 : 1][65];
-  const PrepJob& J = jobs.j[blockIdx.z];
-  const int t0 = blockIdx.x * 64, bh = blockIdx.y, tid = threadIdx.x;
-  pdl_wait();
+__global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs jobs, int T, int Tp, int d,
+                                              int BH) {
+  __shared__ float hs[32][65];
+  __shared__ float ls[SPLIT ? 32 : 1][65];
+  const int tid = threadIdx.x;
   const int r = tid >> 4, c4 = tid & 15;  // load phase: rows r + 8 q, columns 4 c4 .. 4 c4 + 3
-  const int k = tid >> 4, tq = tid & 15;  // store phase: output rows k + 8 q, keys 4 tq .. 4 tq + 3
-  const size_t nat = (size_t)bh * T * d, tr = (size_t)bh * d * Tp;
-  const bool dotj = J.Y != nullptr;
-  float dacc[8];
+  const int k = tid >> 3, tq = tid & 7;   // store phase: output rows k + 16 q, keys 4 tq .. 4 tq + 3
+  const int ntb = Tp / 32, per_job = BH * ntb, units = jobs.n * per_job;
+  pdl_wait();
+  for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    const PrepJob& J = jobs.j[u / per_job];
+    const int bh = (u % per_job) / ntb, t0 = (u % ntb) * 32;
+    const size_t nat = (size_t)bh * T * d, tr = (size_t)bh * d * Tp;
+    const bool dotj = J.Y != nullptr;
+    float dacc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int k0 = 0; k0 < d; k0 += 64) {
+      float4 x[4];
 #pragma unroll
-  for (int q = 0; q < 8; ++q) dacc[q] = 0.f;
-  for (int k0 = 0; k0 < d; k0 += 64) {
-    float4 x[8];
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int t = t0 + r + 8 * q;
-      x[q] = t < T ? __ldg(reinterpret_cast<const float4*>(J.X + nat + (size_t)t * d + k0 + 4 * c4))
-                   : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    if (dotj) {
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
+      for (int q = 0; q < 4; ++q) {
         const int t = t0 + r + 8 * q;
-        if (t < T) {
-          const float4 y = __ldg(reinterpret_cast<const float4*>(J.Y + nat + (size_t)t * d + k0 + 4 * c4));
-          dacc[q] = __fmaf_rn(x[q].x, y.x, dacc[q]);
-          dacc[q] = __fmaf_rn(x[q].y, y.y, dacc[q]);
-          dacc[q] = __fmaf_rn(x[q].z, y.z, dacc[q]);
-          dacc[q] = __fmaf_rn(x[q].w, y.w, dacc[q]);
+        x[q] = t < T ? __ldg(reinterpret_cast<const float4*>(J.X + nat + (size_t)t * d + k0 + 4 * c4))
+                     : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+      if (dotj) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int t = t0 + r + 8 * q;
+          if (t < T) {
+            const float4 y = __ldg(reinterpret_cast<const float4*>(J.Y + nat + (size_t)t * d + k0 + 4 * c4));
+            dacc[q] = __fmaf_rn(x[q].x, y.x, dacc[q]);
+            dacc[q] = __fmaf_rn(x[q].y, y.y, dacc[q]);
+            dacc[q] = __fmaf_rn(x[q].z, y.z, dacc[q]);
+            dacc[q] = __fmaf_rn(x[q].w, y.w, dacc[q]);
+          }
         }
       }
-    }
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int rr = r + 8 * q, t = t0 + rr;
-      float4 v = x[q];
-      if constexpr (SPLIT) {
-        float4 h, l;
-        h.x = tf32_rna(v.x); l.x = __fsub_rn(v.x, h.x);
-        h.y = tf32_rna(v.y); l.y = __fsub_rn(v.y, h.y);
-        h.z = tf32_rna(v.z); l.z = __fsub_rn(v.z, h.z);
-        h.w = tf32_rna(v.w); l.w = __fsub_rn(v.w, h.w);
-        if (t < T && J.nat_hi) {
-          const size_t off = nat + (size_t)t * d + k0 + 4 * c4;
-          *reinterpret_cast<float4*>(J.nat_hi + off) = h;
-          *reinterpret_cast<float4*>(J.nat_lo + off) = l;
+      for (int q = 0; q < 4; ++q) {
+        const int rr = r + 8 * q, t = t0 + rr;
+        float4 v = x[q];
+        if constexpr (SPLIT) {
+          float4 h, l;
+          h.x = tf32_rna(v.x); l.x = __fsub_rn(v.x, h.x);
+          h.y = tf32_rna(v.y); l.y = __fsub_rn(v.y, h.y);
+          h.z = tf32_rna(v.z); l.z = __fsub_rn(v.z, h.z);
+          h.w = tf32_rna(v.w); l.w = __fsub_rn(v.w, h.w);
+          if (t < T && J.nat_hi) {
+            const size_t off = nat + (size_t)t * d + k0 + 4 * c4;
+            *reinterpret_cast<float4*>(J.nat_hi + off) = h;
+            *reinterpret_cast<float4*>(J.nat_lo + off) = l;
+          }
+          v = h;
+          ls[rr][4 * c4] = l.x; ls[rr][4 * c4 + 1] = l.y; ls[rr][4 * c4 + 2] = l.z; ls[rr][4 * c4 + 3] = l.w;
         }
-        v = h;
-        ls[rr][4 * c4] = l.x; ls[rr][4 * c4 + 1] = l.y; ls[rr][4 * c4 + 2] = l.z; ls[rr][4 * c4 + 3] = l.w;
+        hs[rr][4 * c4] = v.x; hs[rr][4 * c4 + 1] = v.y; hs[rr][4 * c4 + 2] = v.z; hs[rr][4 * c4 + 3] = v.w;
       }
-      hs[rr][4 * c4] = v.x; hs[rr][4 * c4 + 1] = v.y; hs[rr][4 * c4 + 2] = v.z; hs[rr][4 * c4 + 3] = v.w;
-    }
-    __syncthreads();
-    if (J.tr_hi) {
+      __syncthreads();
+      if (J.tr_hi) {
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int kk = k + 8 * q, t = t0 + 4 * tq;
-        if (t < Tp) {
+        for (int q = 0; q < 4; ++q) {
+          const int kk = k + 16 * q, t = t0 + 4 * tq;
           const size_t off = tr + (size_t)(k0 + kk) * Tp + t;
           *reinterpret_cast<float4*>(J.tr_hi + off) =
               make_float4(hs[4 * tq][kk], hs[4 * tq + 1][kk], hs[4 * tq + 2][kk], hs[4 * tq + 3][kk]);
@@ -92,25 +93,26 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
           }
         }
       }
+      __syncthreads();
     }
-    __syncthreads();
-  }
-  if (dotj) {
+    if (dotj) {
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      float v = dacc[q];
+      for (int q = 0; q < 4; ++q) {
+        float v = dacc[q];
 #pragma unroll
-      for (int o = 8; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-      const int t = t0 + r + 8 * q;
-      if (c4 == 0 && t < T) J.dot[(size_t)bh * T + t] = v;
+        for (int o = 8; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        const int t = t0 + r + 8 * q;
+        if (c4 == 0 && t < T) J.dot[(size_t)bh * T + t] = v;
+      }
     }
   }
 }
 
-cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, cudaStream_t s) {
+cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, int nsm, cudaStream_t s) {
   if (jobs.n <= 0) return cudaSuccess;
-  dim3 grid((Tp + 63) / 64, BH, jobs.n), block(128);
-  return launch_pdl(split ? k_prep<true> : k_prep<false>, grid, block, 0, s, jobs, T, Tp, d);
+  const int units = jobs.n * BH * (Tp / 32);
+  dim3 grid((unsigned)(units < 6 * nsm ? units : 6 * nsm)), block(128);
+  return launch_pdl(split ? k_prep<true> : k_prep<false>, grid, block, 0, s, jobs, T, Tp, d, BH);
 }
 
 // ---------------------------------------------------------------------------

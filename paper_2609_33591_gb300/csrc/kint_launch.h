@@ -18,7 +18,8 @@ struct PrepJobs {
   PrepJob j[4];
   int n;
 };
-cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, cudaStream_t s);
+// nsm: SMs of the device (the grid is a few CTAs per SM looping over the work units)
+cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, int nsm, cudaStream_t s);
 
 // Launch with programmatic stream serialization: the kernel may be scheduled while the
 // previous kernel in the stream finishes; every kernel of the library waits for its
