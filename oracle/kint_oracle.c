@@ -16,6 +16,9 @@
  *   App. B "FWM" paragraph                        -> FWM calibration gradient
  *   Eq. (wste) / Eq. (pste), App. B Weight-STE / Prob-STE paragraphs
  *   App. B "Detach (legacy)"                      -> detached extrema
+ *   supplement "Single-channel ablation" and "Local gradient decomposition"
+ *                                                 -> max_only / min_only modes
+ *                                                  (g_self + g_M, g_self + g_m)
  *   App. B "Softmax", App. A "Softmax"            -> the comparator
  *   Table "Edge cases" (App. A)                   -> degenerate rows, ties,
  *                                                  midpoint rounding, window edge
@@ -329,7 +332,7 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
       const double gamma = (R->g[j] - D) / Wst;           /* normalization Jacobian */
       const double Delta = (R->e[r + 1] - R->e[r]) / h;   /* secant slope */
       R->dS[j] = gamma * Delta;                           /* own-score term */
-      if (p->grad == KOR_FULL) {
+      if (p->grad != KOR_DETACH) {
         if (p->calib == KOR_MINMAX) {
           /* Eq. (calgrad) */
           const double rho = (r + t) / K;
@@ -344,12 +347,14 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
         }
       }
     }
-    if (p->grad == KOR_FULL) {
+    if (p->grad != KOR_DETACH) {
       /* Eq. (full): the extremum terms go to the arg-max / arg-min keys, split
-       * evenly among ties. */
+       * evenly among ties; the single-channel modes keep one of the two. */
+      const int use_M = p->grad == KOR_FULL || p->grad == KOR_MAX_ONLY;
+      const int use_m = p->grad == KOR_FULL || p->grad == KOR_MIN_ONLY;
       for (int j = 0; j < n; ++j) {
-        if (R->s[j] == R->M) R->dS[j] += cM / R->nmax;
-        if (p->calib == KOR_MINMAX && R->s[j] == R->m) R->dS[j] += cm / R->nmin;
+        if (use_M && R->s[j] == R->M) R->dS[j] += cM / R->nmax;
+        if (use_m && p->calib == KOR_MINMAX && R->s[j] == R->m) R->dS[j] += cm / R->nmin;
       }
     }
   }
@@ -444,7 +449,7 @@ static int check_params(const kor_params* p) {
   if (p->calib < 0 || p->calib > 2) return -1;
   if (p->calib != KOR_SOFTMAX && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
   if (p->calib == KOR_FWM && !(p->tau > 0.0)) return -1;
-  if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 1) return -1;
+  if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 3) return -1;
   return 0;
 }
 

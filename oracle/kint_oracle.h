@@ -27,7 +27,11 @@ typedef float kor_in;
 enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2 };
 enum { KOR_LERP = 0, KOR_NEAREST = 1 };
 enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
-enum { KOR_FULL = 0, KOR_DETACH = 1 };
+/* Backward modes: the full calibration gradient (Eq. full), detached extrema (App. B
+ * "Detach (legacy)"), and the single-channel ablations that keep only the maximum's or
+ * only the minimum's calibration term (App. "Single-channel ablation":
+ * g_max_only = g_self + g_M, g_min_only = g_self + g_m). */
+enum { KOR_FULL = 0, KOR_DETACH = 1, KOR_MAX_ONLY = 2, KOR_MIN_ONLY = 3 };
 
 /* Codes of the per-key decision arrays (bins: Nearest index l in 0..K,
  * ivals: interval index r in 0..K-1). */
@@ -40,7 +44,7 @@ typedef struct {
   double tau; /* FWM window in nats */
   int recon;  /* KOR_LERP / KOR_NEAREST */
   int ste;    /* KOR_WEIGHT / KOR_PROB (ignored for LERP) */
-  int grad;   /* KOR_FULL / KOR_DETACH */
+  int grad;   /* KOR_FULL / KOR_DETACH / KOR_MAX_ONLY / KOR_MIN_ONLY */
   int nthreads; /* <= 0: all online cores */
 } kor_params;
 
@@ -65,8 +69,8 @@ typedef struct {
   double* dQ;   /* [B,H,T,d] */
   double* dK;   /* [B,H,T,d] */
   double* dV;   /* [B,H,T,d] */
-  double* cM;   /* [B,H,T] sum_j gamma_j dw_j/dM (0 under detach) */
-  double* cm;   /* [B,H,T] sum_j gamma_j dw_j/dm (MinMax, full) */
+  double* cM;   /* [B,H,T] sum_j gamma_j dw_j/dM (0 under detach; computed in every other mode) */
+  double* cm;   /* [B,H,T] sum_j gamma_j dw_j/dm (MinMax; 0 under detach) */
   double* dsum; /* [B,H,T] sum_j dL/ds_ij */
   double* dabs; /* [B,H,T] sum_j |dL/ds_ij| */
   double* dS;   /* [B,H,T,T] dL/ds (optional, small cases) */

@@ -12,7 +12,7 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle import Config, MINMAX, FWM, SOFTMAX, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH
+from oracle import Config, MINMAX, FWM, SOFTMAX, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH, MAX_ONLY, MIN_ONLY
 from tests import witness
 
 ALL_COMBOS = [(c, r, s, g) for c in (MINMAX, FWM) for r in (LERP, NEAREST) for s in (WEIGHT, PROB)
@@ -308,6 +308,49 @@ def test_matches_autograd_witness(calib, recon, ste, grad, Kint):
     O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
     for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
         assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+# --- Single-channel ablations (supplement "Single-channel ablation", "Local gradient decomposition") ---
+
+@pytest.mark.parametrize("calib,recon,ste", [(MINMAX, LERP, WEIGHT), (MINMAX, NEAREST, PROB), (MINMAX, NEAREST, WEIGHT),
+                                             (FWM, NEAREST, PROB), (FWM, LERP, WEIGHT)])
+@pytest.mark.parametrize("grad", [MAX_ONLY, MIN_ONLY])
+def test_single_channel_matches_autograd_witness(calib, recon, ste, grad):
+    """max_only keeps the maximum's channel (the witness detaches m only), min_only the minimum's
+    (M detached); the forward is unchanged."""
+    Q, K, V, dO = rand_inputs(1, 2, 12, 8, 17, scale=2.0)
+    cfg = Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad)
+    f = oracle.forward(Q, K, V, cfg)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+    for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+        assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+@pytest.mark.parametrize("calib,recon,ste", [(MINMAX, LERP, WEIGHT), (MINMAX, NEAREST, PROB), (FWM, NEAREST, PROB)])
+def test_gradient_decomposition_identity(calib, recon, ste):
+    """g_full = g_self + g_M + g_m with g_max_only = g_self + g_M, g_min_only = g_self + g_m and
+    g_detach = g_self, so full + detach = max_only + min_only in every linear image of dS (dQ, dK);
+    dV and the calibration sums do not depend on the mode (except detach, which has none).
+    For FWM (no minimum channel) max_only is full and min_only is detach."""
+    Q, K, V, dO = rand_inputs(1, 2, 16, 8, 19, scale=2.0)
+    out = {}
+    for g in (FULL, DETACH, MAX_ONLY, MIN_ONLY):
+        cfg = Config(Kint=4, calib=calib, tau=3.0, recon=recon, ste=ste, grad=g)
+        out[g] = oracle.backward(Q, K, V, dO, cfg)
+    for n in ("dQ", "dK"):
+        lhs = out[FULL][n] + out[DETACH][n]
+        rhs = out[MAX_ONLY][n] + out[MIN_ONLY][n]
+        assert np.max(np.abs(lhs - rhs)) <= 1e-12 * max(1.0, np.max(np.abs(lhs)))
+        assert np.max(np.abs(out[MAX_ONLY][n] - out[FULL][n])) > 0 or calib == FWM
+        if calib == FWM:
+            assert np.array_equal(out[MAX_ONLY][n], out[FULL][n])
+            assert np.array_equal(out[MIN_ONLY][n], out[DETACH][n])
+    for g in (DETACH, MAX_ONLY, MIN_ONLY):
+        assert np.array_equal(out[g]["dV"], out[FULL]["dV"])
+    for g in (MAX_ONLY, MIN_ONLY):
+        assert np.array_equal(out[g]["cM"], out[FULL]["cM"]) and np.array_equal(out[g]["cm"], out[FULL]["cm"])
+    assert not out[DETACH]["cM"].any()
 
 
 def test_ties_split_evenly_like_autograd():

@@ -18,7 +18,7 @@ import torch
 MINMAX, FWM, SOFTMAX = 0, 1, 2
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
-FULL, DETACH = 0, 1
+FULL, DETACH, MAX_ONLY, MIN_ONLY = 0, 1, 2, 3
 
 
 def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
@@ -28,8 +28,11 @@ def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
         return torch.softmax(S.masked_fill(~valid, -math.inf), dim=-1)
     M = S.masked_fill(~valid, -math.inf).amax(dim=-1, keepdim=True)
     m = S.masked_fill(~valid, math.inf).amin(dim=-1, keepdim=True)
-    if cfg.grad == DETACH:
-        M, m = M.detach(), m.detach()
+    # detach stops both extremum channels; the single-channel ablations stop one
+    if cfg.grad in (DETACH, MIN_ONLY):
+        M = M.detach()
+    if cfg.grad in (DETACH, MAX_ONLY):
+        m = m.detach()
     z = S - M
     if cfg.calib == MINMAX:
         span = M - m
