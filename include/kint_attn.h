@@ -59,9 +59,17 @@ typedef enum { KINT_RECON_LERP = 0, KINT_RECON_NEAREST = 1 } kint_recon;
 /* Surrogate placement (Sec. 3 Eqs. wste / pste).  Ignored under LERP, where the
  * two placements coincide (w^N = w^L). */
 typedef enum { KINT_STE_WEIGHT = 0, KINT_STE_PROB = 1 } kint_ste;
-/* Backward mode: full calibration gradient (Eq. full) or detached extrema
- * (App. B "Detach (legacy)").  The forward does not depend on it. */
-typedef enum { KINT_GRAD_FULL = 0, KINT_GRAD_DETACH = 1 } kint_grad;
+/* Backward mode: full calibration gradient (Eq. full), detached extrema
+ * (App. B "Detach (legacy)"), or one extremum channel only (supplement
+ * "Single-channel ablation": max_only keeps the c_M term, min_only the c_m term;
+ * for FWM, which has no minimum channel, max_only equals full and min_only
+ * equals detach).  The forward does not depend on it. */
+typedef enum {
+  KINT_GRAD_FULL = 0,
+  KINT_GRAD_DETACH = 1,
+  KINT_GRAD_MAX_ONLY = 2,
+  KINT_GRAD_MIN_ONLY = 3
+} kint_grad;
 /* Tensor-core arithmetic: plain TF32 products (the precision the paper trains
  * with, App. C "Numerics and hardware"), or 3xTF32 (hi/lo operand splitting,
  * fp32-level accuracy). */
@@ -80,6 +88,11 @@ typedef struct {
   float* W;          /* W^N = sum w^N (Nearest) or W^L (LERP); softmax: sum e^{s - M} */
   float* W_lerp;     /* W^L; required for Prob-STE, may be NULL otherwise */
   float* O_lerp;     /* [B,H,T,d] P^L V; required for Prob-STE, may be NULL otherwise */
+  float* c_M;        /* optional side output of kint_attn_bwd (NULL: not written): the row's
+                        calibration sum c_M = sum_j gamma_j dw_j/dM (supplement "Local gradient
+                        decomposition", the M channel); 0 under detach and for softmax */
+  float* c_m;        /* optional side output of kint_attn_bwd: c_m = sum_j gamma_j dw_j/dm
+                        (MinMax; 0 otherwise) */
 } kint_rowstats;
 
 /*
@@ -111,8 +124,9 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
  *   gamma_j = (g_j - <g>_{P*}) / W*, g_j = dO_i . V_j, where (P*, W*) is
  *     (P^N, W^N) for Nearest + Weight-STE and (P^L, W^L) otherwise;
  *   dS_ij = gamma_j Delta_j + [j tied at M_i] c_M / n_max + [j tied at m_i] c_m / n_min
- *     (c_m only for MinMax; both zero under detach; FWM tail keys get 0;
- *      degenerate MinMax rows get 0);
+ *     (c_m only for MinMax; both dropped under detach, c_m under max_only, c_M under
+ *      min_only; FWM tail keys get 0; degenerate MinMax rows get 0);
+ *   st->c_M, st->c_m, when non-NULL, receive the per-row sums c_M, c_m (16-byte aligned);
  *   dQ = dS K / sqrt(d), dK = dS^T Q / sqrt(d), dV = P^T dO with the forward P.
  * dQ, dK, dV are overwritten.
  *   O        in:  forward output

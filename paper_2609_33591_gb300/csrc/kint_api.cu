@@ -163,7 +163,7 @@ int validate(const Common& c, int causal) {
   if (c.B < 1 || c.H < 1 || c.T < 1 || c.d < 1) return KINT_ERR_ARG;
   if (causal != 1) return KINT_ERR_ARG;
   if (c.calib < 0 || c.calib > 2 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
-      c.grad > 1 || c.prec < 0 || c.prec > 1)
+      c.grad > 3 || c.prec < 0 || c.prec > 1)
     return KINT_ERR_ARG;
   if (c.calib != KINT_CALIB_SOFTMAX && (c.Kint < 1 || c.Kint > KMAX)) return KINT_ERR_ARG;
   if (c.calib == KINT_CALIB_FWM && !(c.tau > 0.0f && std::isfinite(c.tau))) return KINT_ERR_ARG;
@@ -385,6 +385,7 @@ int check_stats(const kint_rowstats* st, bool prob) {
   for (const void* q : ptrs)
     if (!aligned16(q)) return KINT_ERR_ALIGN;
   if (prob && (!aligned16(st->W_lerp) || !aligned16(st->O_lerp))) return KINT_ERR_ALIGN;
+  if ((st->c_M && !aligned16(st->c_M)) || (st->c_m && !aligned16(st->c_m))) return KINT_ERR_ALIGN;
   return KINT_OK;
 }
 
@@ -400,6 +401,7 @@ void set_stats(Params& p, const kint_rowstats* st) {
   p.arg_max = st->arg_max; p.arg_min = st->arg_min;
   p.n_max = st->n_max; p.n_min = st->n_min;
   p.W = st->W; p.W_lerp = st->W_lerp; p.O_lerp = st->O_lerp;
+  p.cM_out = st->c_M; p.cm_out = st->c_m;
 }
 
 bool is_prob(const Common& c) {

@@ -499,12 +499,15 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
           cm_t += xch[(NCG + q) * 128 + row];
         }
         // Eq. (full): c_m = sum gamma dw/dm; c_M = -sum gamma Delta - c_m (Delta + dw/dM + dw/dm = 0);
-        // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys.
+        // FWM: c_M = -sum_window gamma Delta.  Split evenly over tied keys; the single-channel
+        // modes (max_only, min_only) apply one of the two sums.
         const bool full = FULLG && CAL != CAL_SOFTMAX && !g.nogrid;
         const float cmv = (full && minmax) ? cm_t : 0.f;
         const float cMv = full ? (-own_t - cmv) : 0.f;
+        const bool use_M = p.grad != GRAD_MIN_ONLY, use_m = p.grad != GRAD_MAX_ONLY;
         // (n_min is 0 where the minimum side was not computed, and c_m is 0 there)
-        const float cMn = cMv / (float)nmax, cmn = (minmax && nmin > 0) ? cmv / (float)nmin : 0.f;
+        const float cMn = use_M ? cMv / (float)nmax : 0.f;
+        const float cmn = (use_m && minmax && nmin > 0) ? cmv / (float)nmin : 0.f;
         const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
         const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
         // dQ rows into a swizzled tile for a TMA store: in the Q / dO staging area (free now
@@ -574,6 +577,8 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
           }
         }
         if (row_ok && cg == 0) {
+          if (p.cM_out) p.cM_out[rw] = cMv;
+          if (p.cm_out) p.cm_out[rw] = cmv;
           // the position as the dK/dV pass forms it: softmax log2 e^{s-M}, FWM Nearest 2u, else u
           const bool half = CAL == CAL_FWM && p.recon == REC_NEAREST;
           RowRec r;
@@ -1085,7 +1090,7 @@ static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p,
 
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   const dim3 grid((unsigned)p.ngrid);
-  const bool full = p.grad == 0;
+  const bool full = p.grad != GRAD_DETACH;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
   if (p.calib == CAL_MINMAX)
     return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
@@ -1096,7 +1101,7 @@ cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cud
 
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   const dim3 grid((unsigned)p.ngrid);
-  const bool full = p.grad == 0, near = p.recon == REC_NEAREST;
+  const bool full = p.grad != GRAD_DETACH, near = p.recon == REC_NEAREST;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dkdv<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
     if (near)

@@ -8,6 +8,7 @@ namespace kint {
 
 enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2 };
 enum Recon : int { REC_LERP = 0, REC_NEAREST = 1 };
+enum Grad : int { GRAD_FULL = 0, GRAD_DETACH = 1, GRAD_MAX_ONLY = 2, GRAD_MIN_ONLY = 3 };
 
 constexpr int KMAX = 64;  // largest number of intervals K
 
@@ -59,6 +60,7 @@ struct Params {
   int nqt;                  // ceil(T / 64)
   float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
   const float* gbar;        // [BH*T] <g>_{P*} = dO_i . O*_i (workspace, written by the dO prep)
+  float *cM_out, *cm_out;   // optional [BH*T] side outputs of the backward: c_M, c_m per row
   uint8_t *bins, *ivals;
 };
 

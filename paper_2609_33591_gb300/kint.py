@@ -20,7 +20,7 @@ from . import build as _build
 CALIB_MINMAX, CALIB_FWM, CALIB_SOFTMAX = 0, 1, 2
 RECON_LERP, RECON_NEAREST = 0, 1
 STE_WEIGHT, STE_PROB = 0, 1
-GRAD_FULL, GRAD_DETACH = 0, 1
+GRAD_FULL, GRAD_DETACH, GRAD_MAX_ONLY, GRAD_MIN_ONLY = 0, 1, 2, 3
 PREC_TF32, PREC_3XTF32 = 0, 1
 CODE_NOGRID, CODE_TAIL, CODE_MASKED = 253, 254, 255
 
@@ -45,7 +45,7 @@ class KintError(RuntimeError):
 
 class kint_rowstats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("row_max", "row_min", "arg_max", "arg_min", "n_max", "n_min", "W",
-                                               "W_lerp", "O_lerp")]
+                                               "W_lerp", "O_lerp", "c_M", "c_m")]
 
 
 _lock = threading.Lock()
@@ -204,16 +204,21 @@ def kint_set_launch_callback(fn) -> None:
 
 # ---- conveniences that allocate with torch ---------------------------------------------------
 
-def alloc_rowstats(B, H, T, d, device, prob: bool) -> dict:
+def alloc_rowstats(B, H, T, d, device, prob: bool, calib_sums: bool = False) -> dict:
+    """Row statistics for one forward/backward pair.  ``calib_sums`` adds the backward's
+    optional per-row outputs c_M and c_m."""
     f = dict(device=device, dtype=torch.float32)
     i = dict(device=device, dtype=torch.int32)
     st = {"row_max": torch.empty(B, H, T, **f), "row_min": torch.empty(B, H, T, **f),
           "arg_max": torch.empty(B, H, T, **i), "arg_min": torch.empty(B, H, T, **i),
           "n_max": torch.empty(B, H, T, **i), "n_min": torch.empty(B, H, T, **i), "W": torch.empty(B, H, T, **f),
-          "W_lerp": None, "O_lerp": None}
+          "W_lerp": None, "O_lerp": None, "c_M": None, "c_m": None}
     if prob:
         st["W_lerp"] = torch.empty(B, H, T, **f)
         st["O_lerp"] = torch.empty(B, H, T, d, **f)
+    if calib_sums:
+        st["c_M"] = torch.empty(B, H, T, **f)
+        st["c_m"] = torch.empty(B, H, T, **f)
     return st
 
 

@@ -14,6 +14,7 @@ MM, FW, SM = kint.CALIB_MINMAX, kint.CALIB_FWM, kint.CALIB_SOFTMAX
 LE, NE = kint.RECON_LERP, kint.RECON_NEAREST
 WE, PR = kint.STE_WEIGHT, kint.STE_PROB
 FU, DE = kint.GRAD_FULL, kint.GRAD_DETACH
+MX, MN = kint.GRAD_MAX_ONLY, kint.GRAD_MIN_ONLY
 X3, TF = kint.PREC_3XTF32, kint.PREC_TF32
 
 COMBOS = [(c, r, s, g) for c in (MM, FW) for r in (LE, NE) for s in (WE, PR) for g in (FU, DE)]
@@ -50,6 +51,15 @@ def test_all_variants_3xtf32_ragged(c, r, s, g, Kint):
 def test_all_variants_tf32(c, r, s, g):
     Q, K, V, dO = make_qkvdo(2, 2, 200, 64, seed=2)
     parity.check(Q, K, V, dO, _cfg(c, r, s, g, 4), TF)
+
+
+@pytest.mark.parametrize("g", [MX, MN])
+@pytest.mark.parametrize("c,r,s", [(MM, LE, WE), (MM, NE, PR), (MM, NE, WE), (FW, NE, WE), (FW, LE, PR)])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_single_channel_modes(c, r, s, g, prec):
+    """max_only / min_only backward (one extremum term of Eq. full kept); T = 300 is ragged."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=11)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, g, 8), prec)
 
 
 @pytest.mark.parametrize("prec", [X3, TF])
