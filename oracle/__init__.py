@@ -27,7 +27,7 @@ _SO64 = os.path.join(_BUILD, "liboracle64.so")    # fp64 inputs, same arithmetic
 MINMAX, FWM, SOFTMAX = 0, 1, 2
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
-FULL, DETACH, MAX_ONLY, MIN_ONLY = 0, 1, 2, 3
+FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4
 CODE_NOGRID, CODE_TAIL, CODE_MASKED = 253, 254, 255
 
 _lock = threading.Lock()

@@ -15,7 +15,8 @@
  *   Eq. (calgrad), Eq. (full), App. B "Full calibration gradient (MinMax)"
  *   App. B "FWM" paragraph                        -> FWM calibration gradient
  *   Eq. (wste) / Eq. (pste), App. B Weight-STE / Prob-STE paragraphs
- *   App. B "Detach (legacy)"                      -> detached extrema
+ *   App. B "Detach (legacy)"                      -> detached extrema, and its P1
+ *                                                  control (zero-sum projection)
  *   supplement "Single-channel ablation" and "Local gradient decomposition"
  *                                                 -> max_only / min_only modes
  *                                                  (g_self + g_M, g_self + g_m)
@@ -332,7 +333,7 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
       const double gamma = (R->g[j] - D) / Wst;           /* normalization Jacobian */
       const double Delta = (R->e[r + 1] - R->e[r]) / h;   /* secant slope */
       R->dS[j] = gamma * Delta;                           /* own-score term */
-      if (p->grad != KOR_DETACH) {
+      if (p->grad != KOR_DETACH && p->grad != KOR_DETACH_PROJ) {
         if (p->calib == KOR_MINMAX) {
           /* Eq. (calgrad) */
           const double rho = (r + t) / K;
@@ -347,7 +348,16 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
         }
       }
     }
-    if (p->grad != KOR_DETACH) {
+    if (p->grad == KOR_DETACH_PROJ) {
+      /* P1 control (App. B, "Detach (legacy)"): keep the detached terms and subtract their
+       * mean over the causal row, g'_ij = g_ij - (1/(i+1)) sum_{k<=i} g_ik, so that every
+       * row sums to zero.  The mean is taken over all n = i + 1 causal keys, FWM tail keys
+       * (detached term 0) included. */
+      double mean = 0.0;
+      for (int j = 0; j < n; ++j) mean += R->dS[j];
+      mean /= n;
+      for (int j = 0; j < n; ++j) R->dS[j] -= mean;
+    } else if (p->grad != KOR_DETACH) {
       /* Eq. (full): the extremum terms go to the arg-max / arg-min keys, split
        * evenly among ties; the single-channel modes keep one of the two. */
       const int use_M = p->grad == KOR_FULL || p->grad == KOR_MAX_ONLY;
@@ -449,7 +459,7 @@ static int check_params(const kor_params* p) {
   if (p->calib < 0 || p->calib > 2) return -1;
   if (p->calib != KOR_SOFTMAX && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
   if (p->calib == KOR_FWM && !(p->tau > 0.0)) return -1;
-  if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 3) return -1;
+  if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 4) return -1;
   return 0;
 }
 

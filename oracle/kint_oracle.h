@@ -30,8 +30,10 @@ enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
 /* Backward modes: the full calibration gradient (Eq. full), detached extrema (App. B
  * "Detach (legacy)"), and the single-channel ablations that keep only the maximum's or
  * only the minimum's calibration term (App. "Single-channel ablation":
- * g_max_only = g_self + g_M, g_min_only = g_self + g_m). */
-enum { KOR_FULL = 0, KOR_DETACH = 1, KOR_MAX_ONLY = 2, KOR_MIN_ONLY = 3 };
+ * g_max_only = g_self + g_M, g_min_only = g_self + g_m), and the P1 control of App. B
+ * "Detach (legacy)": the detached score gradient projected, per causal row, onto the
+ * zero-sum subspace (g'_ij = g_ij - (1/(i+1)) sum_{k<=i} g_ik). */
+enum { KOR_FULL = 0, KOR_DETACH = 1, KOR_MAX_ONLY = 2, KOR_MIN_ONLY = 3, KOR_DETACH_PROJ = 4 };
 
 /* Codes of the per-key decision arrays (bins: Nearest index l in 0..K,
  * ivals: interval index r in 0..K-1). */
@@ -44,7 +46,7 @@ typedef struct {
   double tau; /* FWM window in nats */
   int recon;  /* KOR_LERP / KOR_NEAREST */
   int ste;    /* KOR_WEIGHT / KOR_PROB (ignored for LERP) */
-  int grad;   /* KOR_FULL / KOR_DETACH / KOR_MAX_ONLY / KOR_MIN_ONLY */
+  int grad;   /* KOR_FULL / KOR_DETACH / KOR_MAX_ONLY / KOR_MIN_ONLY / KOR_DETACH_PROJ */
   int nthreads; /* <= 0: all online cores */
 } kor_params;
 

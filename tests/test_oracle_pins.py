@@ -12,7 +12,8 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle import Config, MINMAX, FWM, SOFTMAX, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH, MAX_ONLY, MIN_ONLY
+from oracle import Config, MINMAX, FWM, SOFTMAX, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH, MAX_ONLY, MIN_ONLY, \
+    DETACH_PROJ
 from tests import witness
 
 ALL_COMBOS = [(c, r, s, g) for c in (MINMAX, FWM) for r in (LERP, NEAREST) for s in (WEIGHT, PROB)
@@ -475,3 +476,48 @@ def test_decision_override_roundtrip():
     h = oracle.forward(Q, K, V, cfg, override={**ov, "bins": bins})
     changed = np.where(np.any(h["O"] != f["O"], axis=-1))
     assert list(changed[2]) == [i]
+
+
+# --- P1 control: detached gradient projected onto the zero-sum subspace (App. B "Detach (legacy)") ---
+
+@pytest.mark.parametrize("calib,recon,ste,tau", [(MINMAX, LERP, WEIGHT, 3.0), (MINMAX, NEAREST, PROB, 3.0),
+                                                 (MINMAX, NEAREST, WEIGHT, 3.0), (FWM, NEAREST, PROB, 1.0),
+                                                 (FWM, LERP, WEIGHT, 1.0)])
+def test_projection_matches_autograd_witness(calib, recon, ste, tau):
+    """The witness detaches M and m and centres the score gradient over each causal row with a
+    hook; tau = 1 puts FWM keys in the zero tail, whose centred gradient is -mean."""
+    Q, K, V, dO = rand_inputs(1, 2, 14, 8, 23, scale=2.0)
+    cfg = Config(Kint=4, calib=calib, tau=tau, recon=recon, ste=ste, grad=DETACH_PROJ)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    _, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+    for a, w in ((b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+        assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+@pytest.mark.parametrize("calib,recon,ste", [(MINMAX, LERP, WEIGHT), (MINMAX, NEAREST, PROB), (FWM, NEAREST, WEIGHT)])
+def test_projection_removes_only_the_common_mode(calib, recon, ste):
+    """Every causal row of the projected dS sums to zero; it differs from the detached dS by one
+    constant per row (the differences between keys are kept); dV, the forward and the absence of
+    calibration sums are those of detach; rows whose detached terms are all zero stay zero."""
+    T = 20
+    Q, K, V, dO = rand_inputs(1, 2, T, 8, 29, scale=2.0)
+    out = {}
+    for g in (DETACH, DETACH_PROJ):
+        cfg = Config(Kint=4, calib=calib, tau=1.5, recon=recon, ste=ste, grad=g)
+        out[g] = oracle.backward(Q, K, V, dO, cfg, want_dS=True)
+    dp, dd = out[DETACH_PROJ]["dS"], out[DETACH]["dS"]
+    for b in range(1):
+        for h in range(2):
+            for i in range(T):
+                row_p, row_d = dp[b, h, i, :i + 1], dd[b, h, i, :i + 1]
+                scale = max(1e-300, np.sum(np.abs(row_d)))
+                assert abs(np.sum(row_p)) <= 1e-13 * scale
+                shift = row_p - row_d
+                assert np.max(np.abs(shift - shift[0])) <= 1e-13 * scale
+                assert np.all(dp[b, h, i, i + 1:] == 0)
+                if not np.any(row_d):
+                    assert not np.any(row_p)
+    assert np.array_equal(out[DETACH_PROJ]["dV"], out[DETACH]["dV"])
+    assert not out[DETACH_PROJ]["cM"].any() and not out[DETACH_PROJ]["cm"].any()
+    # the detached gradient is not zero-sum in general (App. B), so the projection changes dQ, dK
+    assert np.max(np.abs(out[DETACH_PROJ]["dK"] - out[DETACH]["dK"])) > 1e-6

@@ -18,7 +18,7 @@ import torch
 MINMAX, FWM, SOFTMAX = 0, 1, 2
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
-FULL, DETACH, MAX_ONLY, MIN_ONLY = 0, 1, 2, 3
+FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4
 
 
 def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
@@ -29,9 +29,9 @@ def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
     M = S.masked_fill(~valid, -math.inf).amax(dim=-1, keepdim=True)
     m = S.masked_fill(~valid, math.inf).amin(dim=-1, keepdim=True)
     # detach stops both extremum channels; the single-channel ablations stop one
-    if cfg.grad in (DETACH, MIN_ONLY):
+    if cfg.grad in (DETACH, DETACH_PROJ, MIN_ONLY):
         M = M.detach()
-    if cfg.grad in (DETACH, MAX_ONLY):
+    if cfg.grad in (DETACH, DETACH_PROJ, MAX_ONLY):
         m = m.detach()
     z = S - M
     if cfg.calib == MINMAX:
@@ -84,6 +84,10 @@ def attention(Q, K, V, dO, cfg):
     T, d = Qt.shape[-2], Qt.shape[-1]
     S = Qt @ Kt.transpose(-1, -2) / math.sqrt(d)
     valid = torch.ones(T, T, dtype=torch.bool).tril().expand(S.shape)
+    if cfg.grad == DETACH_PROJ and cfg.calib != SOFTMAX:
+        # P1: the gradient reaching the scores is centred over each causal row
+        vf = valid.to(S.dtype)
+        S.register_hook(lambda gS: (gS - (gS * vf).sum(-1, keepdim=True) / vf.sum(-1, keepdim=True)) * vf)
     P = probs(S, valid, cfg)
     O = P @ Vt
     (O * torch.tensor(np.asarray(dO, dtype=np.float64))).sum().backward()
