@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "ad277cc1cfb4c562", "k_prep": 82498304, "k_fwd_stats": 50371584, "k_fwd_main": 93692672,
-           "k_bwd_dq": 193934848, "k_bwd_dkdv": 274213632}
+TRAFFIC = {"src": "380726be8a630b41", "k_prep": 82461568, "k_fwd_stats": 50369024, "k_fwd_main": 93682688,
+           "k_bwd_dq": 193184768, "k_bwd_dkdv": 274102528}
 
 
 def kernel_source_digest() -> str:

@@ -63,12 +63,16 @@ typedef enum { KINT_STE_WEIGHT = 0, KINT_STE_PROB = 1 } kint_ste;
  * (App. B "Detach (legacy)"), or one extremum channel only (supplement
  * "Single-channel ablation": max_only keeps the c_M term, min_only the c_m term;
  * for FWM, which has no minimum channel, max_only equals full and min_only
- * equals detach).  The forward does not depend on it. */
+ * equals detach), or the P1 control of App. B "Detach (legacy)": the detached score
+ * gradient projected onto the zero-sum subspace of each causal row,
+ * dS'_ij = dS_ij - (1/(i+1)) sum_{k<=i} dS_ik (tail keys included).  The forward does not
+ * depend on it; softmax ignores it. */
 typedef enum {
   KINT_GRAD_FULL = 0,
   KINT_GRAD_DETACH = 1,
   KINT_GRAD_MAX_ONLY = 2,
-  KINT_GRAD_MIN_ONLY = 3
+  KINT_GRAD_MIN_ONLY = 3,
+  KINT_GRAD_DETACH_PROJ = 4
 } kint_grad;
 /* Tensor-core arithmetic: plain TF32 products (the precision the paper trains
  * with, App. C "Numerics and hardware"), or 3xTF32 (hi/lo operand splitting,
@@ -126,7 +130,10 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
  *   dS_ij = gamma_j Delta_j + [j tied at M_i] c_M / n_max + [j tied at m_i] c_m / n_min
  *     (c_m only for MinMax; both dropped under detach, c_m under max_only, c_M under
  *      min_only; FWM tail keys get 0; degenerate MinMax rows get 0);
- *   st->c_M, st->c_m, when non-NULL, receive the per-row sums c_M, c_m (16-byte aligned);
+ *     under detach_proj each causal row of the detached dS then loses its mean;
+ *   st->c_M, st->c_m, when non-NULL, receive the per-row sums c_M, c_m (16-byte aligned;
+ *     the sums are written whether or not the mode applies them, 0 under detach and
+ *     detach_proj);
  *   dQ = dS K / sqrt(d), dK = dS^T Q / sqrt(d), dV = P^T dO with the forward P.
  * dQ, dK, dV are overwritten.
  *   O        in:  forward output

@@ -163,7 +163,7 @@ int validate(const Common& c, int causal) {
   if (c.B < 1 || c.H < 1 || c.T < 1 || c.d < 1) return KINT_ERR_ARG;
   if (causal != 1) return KINT_ERR_ARG;
   if (c.calib < 0 || c.calib > 2 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
-      c.grad > 3 || c.prec < 0 || c.prec > 1)
+      c.grad > 4 || c.prec < 0 || c.prec > 1)
     return KINT_ERR_ARG;
   if (c.calib != KINT_CALIB_SOFTMAX && (c.Kint < 1 || c.Kint > KMAX)) return KINT_ERR_ARG;
   if (c.calib == KINT_CALIB_FWM && !(c.tau > 0.0f && std::isfinite(c.tau))) return KINT_ERR_ARG;
@@ -298,7 +298,9 @@ int plan_dkdv(Params& p, int sel) {
   // TF32 at d = 64, both products: K and V staged in smem by TMA (see plan_dq)
   p.ops_smem = (!p.x3 && p.d == 64 && doDV && doDK) ? 1 : 0;
   const int base = doDK ? 2 * dp : dp;
-  const int acc = (doDV ? p.d : 0) + (doDK ? p.d : 0);
+  // accumulators, and under 3xTF32 (one product per launch) the cross-term accumulator
+  const int acc = (doDV ? p.d : 0) + (doDK ? p.d : 0) + (p.x3 ? p.d : 0);
+  if (p.x3 && doDV && doDK) return -1;
   if (base + 128 + acc > 512) return -1;
   p.dkv_sel = sel;
   p.nbuf = (base + 256 + acc <= 512) ? 2 : 1;
@@ -530,6 +532,9 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
        map_nat(&maps.dv, dV, BH, T, d, 64);
   if (!ok) return KINT_ERR_LAUNCH;
 
+  // P1 projection: key prefix sums into the tie-sum buffer (unused by the detached modes)
+  if (c.grad == KINT_GRAD_DETACH_PROJ && c.calib != KINT_CALIB_SOFTMAX)
+    if ((rc = launch_rc(traced("k_kcum", s, [&] { return launch_kcum(K, w.tie, BH, T, d, s); })))) return rc;
   Params pq = p;
   const int smem_dq = plan_dq(pq);
   if (smem_dq < 0 || smem_dq > kSmemLimit) return KINT_ERR_UNSUPPORTED;

@@ -67,10 +67,8 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
       ds = ok ? ds : 0.f;
       dm = ok ? dm : 0.f;
     }
-    if constexpr (FULLG && CAL != CAL_SOFTMAX) {
-      own += ds;
-      if constexpr (CAL == CAL_MINMAX) cm += dm;
-    }
+    if constexpr (CAL != CAL_SOFTMAX) own += ds;  // (detached too: the P1 row mean)
+    if constexpr (FULLG && CAL == CAL_MINMAX) cm += dm;
     out[jj] = ds;
   }
 }
@@ -505,10 +503,15 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         const float cmv = (full && minmax) ? cm_t : 0.f;
         const float cMv = full ? (-own_t - cmv) : 0.f;
         const bool use_M = p.grad != GRAD_MIN_ONLY, use_m = p.grad != GRAD_MAX_ONLY;
+        // P1 control (detached, App. B): dS_ij - mu_i over the causal row, mu_i = sum_j dS_ij / (i + 1),
+        // adds -mu_i C_i to dQ_i, C_i = sum_{j<=i} K_j (prefix sums, in the tie-sum buffer, which
+        // the detached modes do not use); the dK/dV pass subtracts mu_i from every causal dS_ij
+        const bool p1 = !FULLG && CAL != CAL_SOFTMAX && p.grad == GRAD_DETACH_PROJ;
+        const float mu = p1 ? own_t / (float)(i + 1) : 0.f;
         // (n_min is 0 where the minimum side was not computed, and c_m is 0 there)
-        const float cMn = use_M ? cMv / (float)nmax : 0.f;
+        const float cMn = p1 ? -mu : (use_M ? cMv / (float)nmax : 0.f);
         const float cmn = (use_m && minmax && nmin > 0) ? cmv / (float)nmin : 0.f;
-        const float* kmax = (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
+        const float* kmax = p1 ? tie_max : (nmax == 1) ? p.K + ((size_t)bh * p.T + amax) * D : tie_max;
         const float* kmin = (nmin == 1) ? p.K + ((size_t)bh * p.T + amin) * D : tie_min;
         // dQ rows into a swizzled tile for a TMA store: in the Q / dO staging area (free now
         // that the next item's Q / dO are in TMEM; the producer stores it before it stages
@@ -538,8 +541,8 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
           } else {
   #pragma unroll
             for (int q = 0; q < 8; ++q) {
-              km[q] = (row_ok && full) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
-                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+              km[q] = (row_ok && (full || p1)) ? __ldg(reinterpret_cast<const float4*>(kmax + c) + q)
+                                               : make_float4(0.f, 0.f, 0.f, 0.f);
               kn[q] = (row_ok && full && minmax) ? __ldg(reinterpret_cast<const float4*>(kmin + c) + q)
                                                  : make_float4(0.f, 0.f, 0.f, 0.f);
             }
@@ -587,7 +590,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
           r.invWf = invWf;
           r.ga = ga;
           r.gb = gb;
-          r.cMn = full ? cMn : 0.f;
+          r.cMn = full ? cMn : mu;  // detached: the P1 row mean (0 without the projection)
           r.amax = (nmax == 1) ? amax : -1;
           r.flags = (g.nogrid ? REC_NOGRID : 0) | (nmax > 1 ? REC_TIEMAX : 0) | (nmin > 1 ? REC_TIEMIN : 0);
           r.inv_h = g.inv_h;
@@ -620,7 +623,7 @@ __device__ __forceinline__ int4 lds_i4(uint32_t addr) {
   return v;
 }
 
-template <int CAL, int REC, bool FULLG, bool MASKED, bool TIES, int W>
+template <int CAL, int REC, bool FULLG, bool PROJ, bool MASKED, bool TIES, int W>
 __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)[W], float (&pa)[W],
                                          float (&da)[W], int j, int i0, int T, uint32_t recs, uint32_t tabs,
                                          uint32_t fwtab, uint32_t tstride, float Kf, float fwm_inv_h,
@@ -669,6 +672,8 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
     if constexpr (FULLG && CAL != CAL_SOFTMAX) {
       ds += (j == __float_as_int(r1.z)) ? r1.y : 0.f;
       if constexpr (CAL == CAL_MINMAX) ds += (j == __float_as_int(r2.z)) ? r2.y : 0.f;
+    } else if constexpr (PROJ && CAL != CAL_SOFTMAX) {
+      ds = __fsub_rn(ds, r1.y);  // detached, P1 projection: minus the row mean
     }
     if constexpr (MASKED) {
       const int iq = i0 + ii;
@@ -742,7 +747,7 @@ __device__ __forceinline__ bool store_staged_dkdv(const Maps& maps, const Params
 // smem stage: Q | dO | Q^T | dO^T tiles (hi[, lo]), the 64 RowRecs of the tile,
 // and (MinMax) their grid pair tables; FWM's shared table at sm_table.
 // ---------------------------------------------------------------------------
-template <int CAL, int REC, bool FULLG>
+template <int CAL, int REC, bool FULLG, bool PROJ = false>
 __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
@@ -769,6 +774,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   const int dp = D * parts;
   const int cK = 0, cV = dp, base = needV ? 2 * dp : dp;
   const int cdV = base + 128 * nbuf, cdK = cdV + (doDV ? D : 0);
+  // 3xTF32 (one product per launch): the two cross terms accumulate apart from hi x hi.
+  // The tensor core rounds each accumulation step toward zero, so a dK / dV row summed
+  // over a whole causal column (up to T / 8 x 3 steps) drifts by about one unit in the
+  // last place per step; keeping the cross terms out of the main accumulator cuts its
+  // steps by three, and the two sums meet in fp32 in the epilogue.
+  const int cdC = cdK + (doDK ? D : 0);
   const int nqt = (p.T + BT - 1) / BT;
   const int oQ = 0, odO = parts * qtile, oQT = 2 * parts * qtile, odOT = 3 * parts * qtile;
   const int oRec = 4 * parts * qtile, oTab = oRec + BT * 64;
@@ -902,9 +913,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         if (p.x3) {
           const uint32_t cacc = tmem + (doDV ? cdV : cdK);
           const uint8_t* bt = st + (doDV ? odOT : oQT);
-          mma_tmem_smem(cacc, cS, bt, D, BT, acc);
-          mma_tmem_smem(cacc, cS, bt + qtile, D, BT, true);
-          mma_tmem_smem(cacc, cG, bt, D, BT, true);
+          mma_tmem_smem(cacc, cS, bt, D, BT, acc);                   // hi x hi
+          mma_tmem_smem(tmem + cdC, cS, bt + qtile, D, BT, acc);     // hi x lo
+          mma_tmem_smem(tmem + cdC, cG, bt, D, BT, true);            // lo x hi
         } else {
           if (doDV) mma_tmem_smem(tmem + cdV, cS, st + odOT, D, BT, acc);
           if (doDK) mma_tmem_smem(tmem + cdK, cG, st + oQT, D, BT, acc);
@@ -996,13 +1007,13 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
           tmem_ld_wait();
           const bool masked = (i0h < kb * 128 + 128) || (i0h + WS > p.T);
           if (FULLG && CAL != CAL_SOFTMAX && tie_here)
-            kv_chunk<CAL, REC, FULLG, true, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
+            kv_chunk<CAL, REC, FULLG, PROJ, true, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
                                                       p.fwm_inv_h, p.scale);
           else if (masked)
-            kv_chunk<CAL, REC, FULLG, true, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
+            kv_chunk<CAL, REC, FULLG, PROJ, true, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
                                                        Kf, p.fwm_inv_h, p.scale);
           else
-            kv_chunk<CAL, REC, FULLG, false, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
+            kv_chunk<CAL, REC, FULLG, PROJ, false, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
                                                         Kf, p.fwm_inv_h, p.scale);
           if (p.x3) {
 #pragma unroll
@@ -1047,6 +1058,13 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
           for (int c = cg * (D / NCG); c < (cg + 1) * (D / NCG); c += 32) {
             float v[32];
             tmem_ld32(lane_addr(tmem, col + c), v);
+            if (p.x3) {
+              float w[32];
+              tmem_ld32(lane_addr(tmem, cdC + c), w);
+              tmem_ld_wait();
+#pragma unroll
+              for (int q = 0; q < 32; ++q) v[q] += w[q];
+            }
             tmem_ld_wait();
 #pragma unroll
             for (int q = 0; q < 32; ++q) v[q] *= mul;
@@ -1080,6 +1098,44 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
 }
 
 // ---------------------------------------------------------------------------
+// Key prefix sums C_i = sum_{j<=i} K_j of every head ([BH][T][d], fp32), for the P1
+// control of App. B ("Detach (legacy)"): projecting the detached dS onto the zero-sum
+// subspace of each causal row adds -mu_i C_i to dQ_i.  One CTA per (head, 32-column
+// slice): its warps take consecutive row segments (lane = column, 128-byte rows), sum
+// them, exchange the segment totals through shared memory and write running sums (the
+// second pass re-reads the segment, from L2).
+// ---------------------------------------------------------------------------
+constexpr int KCUM_WARPS = 16;
+__global__ void __launch_bounds__(KCUM_WARPS * 32) k_kcum(const float* __restrict__ K, float* __restrict__ C,
+                                                          int T, int d) {
+  __shared__ float part[KCUM_WARPS][32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nsl = d / 32;
+  const int bh = blockIdx.x / nsl, col = (blockIdx.x % nsl) * 32 + lane;
+  const int seg = (T + KCUM_WARPS - 1) / KCUM_WARPS;
+  const int t0 = min(T, w * seg), t1 = min(T, t0 + seg);
+  const float* src = K + (size_t)bh * T * d + col;
+  float* dst = C + (size_t)bh * T * d + col;
+  pdl_wait();  // (the dQ kernel's wait on this launch then also covers the operand prep)
+  float sum = 0.f;
+#pragma unroll 4
+  for (int t = t0; t < t1; ++t) sum += __ldg(src + (size_t)t * d);
+  part[w][lane] = sum;
+  __syncthreads();
+  pdl_trigger();
+  float run = 0.f;
+  for (int q = 0; q < w; ++q) run += part[q][lane];
+#pragma unroll 4
+  for (int t = t0; t < t1; ++t) {
+    run += __ldg(src + (size_t)t * d);
+    dst[(size_t)t * d] = run;
+  }
+}
+
+cudaError_t launch_kcum(const float* K, float* C, int BH, int T, int d, cudaStream_t s) {
+  return launch_pdl(k_kcum, dim3((unsigned)(BH * (d / 32))), dim3(KCUM_WARPS * 32), 0, s, K, C, T, d);
+}
+
+// ---------------------------------------------------------------------------
 template <class K>
 static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s,
                            int nthr = NTHR) {
@@ -1090,7 +1146,7 @@ static cudaError_t launch3(K kern, dim3 grid, const Maps& maps, const Params& p,
 
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   const dim3 grid((unsigned)p.ngrid);
-  const bool full = p.grad != GRAD_DETACH;
+  const bool full = p.grad != GRAD_DETACH && p.grad != GRAD_DETACH_PROJ;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
   if (p.calib == CAL_MINMAX)
     return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
@@ -1101,20 +1157,25 @@ cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cud
 
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   const dim3 grid((unsigned)p.ngrid);
-  const bool full = p.grad != GRAD_DETACH, near = p.recon == REC_NEAREST;
+  const bool proj = p.grad == GRAD_DETACH_PROJ, full = p.grad != GRAD_DETACH && !proj;
+  const bool near = p.recon == REC_NEAREST;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dkdv<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
     if (near)
       return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)
-                  : launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
+             : proj ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, false, true>, grid, maps, p, smem_bytes, s)
+                    : launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
     return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, true>, grid, maps, p, smem_bytes, s)
-                : launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+           : proj ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
+                  : launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   }
   if (near)
     return full ? launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)
-                : launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
+           : proj ? launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, false, true>, grid, maps, p, smem_bytes, s)
+                  : launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
   return full ? launch3(k_bwd_dkdv<CAL_FWM, REC_LERP, true>, grid, maps, p, smem_bytes, s)
-              : launch3(k_bwd_dkdv<CAL_FWM, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+         : proj ? launch3(k_bwd_dkdv<CAL_FWM, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
+                : launch3(k_bwd_dkdv<CAL_FWM, REC_LERP, false>, grid, maps, p, smem_bytes, s);
 }
 
 }  // namespace kint

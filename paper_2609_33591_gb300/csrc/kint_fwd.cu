@@ -157,7 +157,9 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
       hi[jj] = fmaxf(hi[jj], hi[jj + w]);
       if constexpr (MIN) lo[jj] = fminf(lo[jj], lo[jj + w]);
     }
-  const float cmax = hi[0], cmin = MIN ? lo[0] : 0.f;
+  const float cmax = hi[0];
+  float cmin = 0.f;
+  if constexpr (MIN) cmin = lo[0];
   const bool um = cmax >= M, un = MIN && cmin <= m;
   if (__any_sync(0xffffffffu, um)) {
     uint32_t mk = 0;

@@ -43,5 +43,7 @@ cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, 
 cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
+// C = running sums of the key rows of every head, [BH][T][d] (the P1 projection)
+cudaError_t launch_kcum(const float* K, float* C, int BH, int T, int d, cudaStream_t s);
 
 }  // namespace kint

@@ -8,7 +8,7 @@ namespace kint {
 
 enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2 };
 enum Recon : int { REC_LERP = 0, REC_NEAREST = 1 };
-enum Grad : int { GRAD_FULL = 0, GRAD_DETACH = 1, GRAD_MAX_ONLY = 2, GRAD_MIN_ONLY = 3 };
+enum Grad : int { GRAD_FULL = 0, GRAD_DETACH = 1, GRAD_MAX_ONLY = 2, GRAD_MIN_ONLY = 3, GRAD_DETACH_PROJ = 4 };
 
 constexpr int KMAX = 64;  // largest number of intervals K
 

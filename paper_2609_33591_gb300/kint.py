@@ -20,7 +20,7 @@ from . import build as _build
 CALIB_MINMAX, CALIB_FWM, CALIB_SOFTMAX = 0, 1, 2
 RECON_LERP, RECON_NEAREST = 0, 1
 STE_WEIGHT, STE_PROB = 0, 1
-GRAD_FULL, GRAD_DETACH, GRAD_MAX_ONLY, GRAD_MIN_ONLY = 0, 1, 2, 3
+GRAD_FULL, GRAD_DETACH, GRAD_MAX_ONLY, GRAD_MIN_ONLY, GRAD_DETACH_PROJ = 0, 1, 2, 3, 4
 PREC_TF32, PREC_3XTF32 = 0, 1
 CODE_NOGRID, CODE_TAIL, CODE_MASKED = 253, 254, 255
 

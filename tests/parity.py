@@ -125,7 +125,7 @@ def check(Q, K, V, dO, cfg: kint.Config, prec, *, want_bwd=True, tol=None, repor
         # the per-row calibration sums of Eq. (full), exactly zero where they are not formed
         scale = float(np.max(b["dabs"] + np.abs(b["cM"]) + np.abs(b["cm"]))) if b["dabs"].size else 0.0
         for n, on in (("c_M", "cM"), ("c_m", "cm")):
-            if cfg.grad == kint.GRAD_DETACH or cfg.calib == kint.CALIB_SOFTMAX or \
+            if cfg.grad in (kint.GRAD_DETACH, kint.GRAD_DETACH_PROJ) or cfg.calib == kint.CALIB_SOFTMAX or \
                     (n == "c_m" and cfg.calib != kint.CALIB_MINMAX):
                 assert not g[n].any(), f"{n} not zero where the mode forms no calibration sum"
             elif g[n].size:

@@ -44,6 +44,7 @@ def test_workspace_sizes():
     (dict(B=0), -1), (dict(T=0), -1), (dict(Kint=0), -1), (dict(Kint=65), -1),
     (dict(calib=1, tau=0.0), -1), (dict(calib=7), -1), (dict(causal=0), -1), (dict(d=96), -2),
     (dict(d=128, prec=1), -2), (dict(Kint=33, prec=1), -2), (dict(Kint=33, d=128), -2),
+    (dict(grad=-1), -1), (dict(grad=5), -1),
 ])
 def test_argument_errors_are_returned_before_any_launch(kw, code):
     args = dict(B=1, H=1, T=8, d=64, Kint=4, calib=0, tau=8.0, recon=0, ste=0, grad=0, causal=1, prec=0)
@@ -69,6 +70,16 @@ def test_null_stats_and_alignment_and_workspace():
     assert lib.kint_attn_fwd(odd, p, p, p, ctypes.byref(full), *args, p, 1 << 30, None) == -3
     assert lib.kint_attn_fwd(p, p, p, p, ctypes.byref(full), *args, p, 16, None) == -4
     assert lib.kint_attn_fwd(p, p, p, p, ctypes.byref(full), *args, None, 1 << 30, None) == -4
+
+
+def test_bwd_side_output_alignment():
+    """The optional c_M / c_m outputs of kint_attn_bwd must be 16-byte aligned like every buffer."""
+    lib = kint.load()
+    p = ctypes.c_void_p(256)
+    st = kint.kint_rowstats(*([256] * 7 + [None, None, 260, None]))
+    rc = lib.kint_attn_bwd(p, p, p, p, p, ctypes.byref(st), p, p, p, 1, 1, 8, 64, 4, 0, 8.0, 0, 0, 0, 1, 0,
+                           p, 1 << 30, None)
+    assert rc == -3
 
 
 def test_strerror_covers_every_code():

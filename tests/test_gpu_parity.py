@@ -15,6 +15,7 @@ LE, NE = kint.RECON_LERP, kint.RECON_NEAREST
 WE, PR = kint.STE_WEIGHT, kint.STE_PROB
 FU, DE = kint.GRAD_FULL, kint.GRAD_DETACH
 MX, MN = kint.GRAD_MAX_ONLY, kint.GRAD_MIN_ONLY
+PJ = kint.GRAD_DETACH_PROJ
 X3, TF = kint.PREC_3XTF32, kint.PREC_TF32
 
 COMBOS = [(c, r, s, g) for c in (MM, FW) for r in (LE, NE) for s in (WE, PR) for g in (FU, DE)]
@@ -60,6 +61,31 @@ def test_single_channel_modes(c, r, s, g, prec):
     """max_only / min_only backward (one extremum term of Eq. full kept); T = 300 is ragged."""
     Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=11)
     parity.check(Q, K, V, dO, _cfg(c, r, s, g, 8), prec)
+
+
+@pytest.mark.parametrize("c,r,s", [(MM, LE, WE), (MM, NE, PR), (FW, NE, WE), (FW, LE, PR)])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_zero_sum_projection(c, r, s, prec):
+    """P1 control: detached dS minus its causal-row mean (tau = 3 puts FWM keys in the tail);
+    T = 300 spans three query blocks and a ragged tail."""
+    Q, K, V, dO = make_qkvdo(2, 2, 300, 64, seed=13)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, PJ, 8, tau=3.0), prec)
+
+
+@pytest.mark.parametrize("c,r,s", [(MM, LE, WE), (MM, NE, PR), (FW, NE, PR), (FW, LE, WE)])
+def test_full_length_rows_3xtf32(c, r, s):
+    """T = 1024 (the GPT-2 context): dK and dV of the first keys sum over every query row, the
+    longest accumulation chains of the backward, and must still meet the 3xTF32 tolerance."""
+    Q, K, V, dO = make_qkvdo(1, 1, 1024, 64, seed=15)
+    parity.check(Q, K, V, dO, _cfg(c, r, s, FU), X3)
+
+
+@pytest.mark.parametrize("T", [1, 2, 65, 1024])
+def test_zero_sum_projection_lengths(T):
+    """Short rows (T = 1: the one causal key of row 0 keeps 0) and a full-length head."""
+    Q, K, V, dO = make_qkvdo(1, 1, T, 64, seed=14)
+    for cfg in (_cfg(MM, NE, WE, PJ), _cfg(FW, NE, PR, PJ)):
+        parity.check(Q, K, V, dO, cfg, X3)
 
 
 @pytest.mark.parametrize("prec", [X3, TF])
