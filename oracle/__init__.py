@@ -24,11 +24,11 @@ _BUILD = os.path.join(_HERE, "_build")
 _SO = os.path.join(_BUILD, "liboracle.so")        # fp32 inputs
 _SO64 = os.path.join(_BUILD, "liboracle64.so")    # fp64 inputs, same arithmetic
 
-MINMAX, FWM, SOFTMAX = 0, 1, 2
+MINMAX, FWM, SOFTMAX, FWM_RESOLVED = 0, 1, 2, 3
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
 FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4
-CODE_NOGRID, CODE_TAIL, CODE_MASKED = 253, 254, 255
+CODE_NOGRID, CODE_TAIL, CODE_MASKED, CODE_OFFSET = 253, 254, 255, 128
 
 _lock = threading.Lock()
 _libs = {}

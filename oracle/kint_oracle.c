@@ -14,6 +14,9 @@
  *   App. B "LERP own-score slope"                 -> Delta (secant)
  *   Eq. (calgrad), Eq. (full), App. B "Full calibration gradient (MinMax)"
  *   App. B "FWM" paragraph                        -> FWM calibration gradient
+ *   App. "Tail policy in the MinMax -> FWM change" -> the resolved grid (FWM's
+ *                                                  step and origin, continued
+ *                                                  below -tau, no zero tail)
  *   Eq. (wste) / Eq. (pste), App. B Weight-STE / Prob-STE paragraphs
  *   App. B "Detach (legacy)"                      -> detached extrema, and its P1
  *                                                  control (zero-sum projection)
@@ -63,6 +66,7 @@ typedef struct {
 /* Per-thread row workspace, sized T. */
 typedef struct {
   double *s, *z, *t, *wL, *wN, *P, *Pst, *g, *dS;
+  double *er0, *er1; /* per key: the grid values e^{b_r}, e^{b_{r+1}} of its interval */
   int *r, *l, *tail, *code_l, *code_r;
   double* e; /* K+1 grid values e^{b_r} */
   double* margin;
@@ -92,6 +96,19 @@ static double decision_distance_u(double u, int K) {
     }
   }
   return best;
+}
+
+/* The same for the resolved grid, whose switches continue below u = 0: every
+ * n / 2 with n <= 2K - 1 (bin edges n + 1/2, interval switches n <= K - 1). */
+static double decision_distance_resolved(double u, int K) {
+  if (u >= K - 0.5) return u - (K - 0.5);
+  return fabs(u - floor(2.0 * u + 0.5) / 2.0);
+}
+
+/* Stored decision code of an index under the resolved policy. */
+static int resolved_code(int idx) {
+  const int c = idx + KOR_CODE_OFFSET;
+  return c < 0 ? 0 : (c > 252 ? 252 : c);
 }
 
 /*
@@ -140,6 +157,8 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
     R->margin[j] = INFINITY;
     R->code_l[j] = KOR_CODE_NOGRID;
     R->code_r[j] = KOR_CODE_NOGRID;
+    R->er0[j] = 0.0;
+    R->er1[j] = 0.0;
   }
 
   if (p->calib == KOR_SOFTMAX) {
@@ -157,7 +176,9 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
     }
   } else {
     /* Grid.  MinMax: z_min = m - M, h = (M - m)/K, b_r = z_min + r h.
-     *        FWM:    h = tau/K, b_r = -tau + r h.                     */
+     *        FWM:    h = tau/K, b_r = -tau + r h  (resolved: the same
+     *                grid for every integer r <= K, no tail).           */
+    const int resolved = (p->calib == KOR_FWM_RESOLVED);
     if (p->calib == KOR_MINMAX) {
       R->b0 = R->m - R->M;
       R->h = (R->M - R->m) / K;
@@ -176,10 +197,11 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
         tail = (z < -p->tau);        /* zero tail below the window, strict */
         zc = clampd(z, -p->tau, 0.0); /* z~ = clip(z, -tau, 0) */
       }
-      /* r = clip(floor((z - b_0)/h), 0, K-1), t = clip((z - b_r)/h, 0, 1) */
+      /* r = clip(floor((z - b_0)/h), 0, K-1), t = clip((z - b_r)/h, 0, 1);
+       * resolved: r = min(floor(u), K-1), unbounded below */
       const double u = (zc - b0) / h;
       int r = (int)floor(u);
-      if (r < 0) r = 0;
+      if (r < 0 && !resolved) r = 0;
       if (r > K - 1) r = K - 1;
       double t = clampd((zc - (b0 + r * h)) / h, 0.0, 1.0);
       /* Nearest grid centre: l = r + [t >= 1/2] (midpoint rounds up) */
@@ -189,17 +211,24 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
       double mg = INFINITY;
       if (p->calib == KOR_FWM) mg = fabs(z + p->tau);
       if (!tail) {
-        double du = decision_distance_u(u, K) * h;
+        double du = (resolved ? decision_distance_resolved(u, K) : decision_distance_u(u, K)) * h;
         if (du < mg) mg = du;
       }
       R->margin[j] = mg;
 
       if (J->ov && J->ov->bins) {
-        /* Decision-aligned re-run: take the given bin / interval / tail choice. */
+        /* Decision-aligned re-run: take the given bin / interval / tail choice
+         * (resolved: a saturated code 0 keeps this row's own choice). */
         const size_t idx = ((size_t)bh * T + i) * T + j;
         const int cb = J->ov->bins[idx];
-        tail = (cb == KOR_CODE_TAIL);
-        if (!tail) {
+        tail = !resolved && (cb == KOR_CODE_TAIL);
+        if (resolved) {
+          if (cb != 0) {
+            l = cb - KOR_CODE_OFFSET;
+            if (J->ov->ivals) r = J->ov->ivals[idx] - KOR_CODE_OFFSET;
+            t = clampd((zc - (b0 + r * h)) / h, 0.0, 1.0);
+          }
+        } else if (!tail) {
           l = cb;
           if (J->ov->ivals) r = J->ov->ivals[idx];
           t = clampd((zc - (b0 + r * h)) / h, 0.0, 1.0);
@@ -215,10 +244,15 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
         R->code_l[j] = KOR_CODE_TAIL;
         R->code_r[j] = KOR_CODE_TAIL;
       } else {
-        R->wL[j] = (1.0 - t) * R->e[r] + t * R->e[r + 1]; /* LERP */
-        R->wN[j] = R->e[l];                               /* Nearest */
-        R->code_l[j] = l;
-        R->code_r[j] = r;
+        /* grid values e^{b_r}: the table, or for the resolved grid below the
+         * window the same expression at the negative index */
+        R->er0[j] = r >= 0 ? R->e[r] : exp(b0 + r * h);
+        R->er1[j] = r + 1 >= 0 ? R->e[r + 1] : exp(b0 + (r + 1) * h);
+        const double eN = l >= 0 ? R->e[l] : exp(b0 + l * h);
+        R->wL[j] = (1.0 - t) * R->er0[j] + t * R->er1[j]; /* LERP */
+        R->wN[j] = eN;                                   /* Nearest */
+        R->code_l[j] = resolved ? resolved_code(l) : l;
+        R->code_r[j] = resolved ? resolved_code(r) : r;
       }
     }
   }
@@ -331,19 +365,19 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
       const int r = R->r[j];
       const double t = R->t[j];
       const double gamma = (R->g[j] - D) / Wst;           /* normalization Jacobian */
-      const double Delta = (R->e[r + 1] - R->e[r]) / h;   /* secant slope */
+      const double Delta = (R->er1[j] - R->er0[j]) / h;   /* secant slope */
       R->dS[j] = gamma * Delta;                           /* own-score term */
       if (p->grad != KOR_DETACH && p->grad != KOR_DETACH_PROJ) {
         if (p->calib == KOR_MINMAX) {
           /* Eq. (calgrad) */
           const double rho = (r + t) / K;
-          const double X = ((1.0 - t) * r * R->e[r] + t * (r + 1) * R->e[r + 1]) / K;
+          const double X = ((1.0 - t) * r * R->er0[j] + t * (r + 1) * R->er1[j]) / K;
           const double dwdM = -R->wL[j] - Delta * rho + X;
           const double dwdm = -Delta * (1.0 - rho) + R->wL[j] - X;
           cM += gamma * dwdM;
           cm += gamma * dwdm;
         } else {
-          /* FWM: dw/dM = -Delta for in-window keys, no m term. */
+          /* FWM: dw/dM = -Delta for in-window keys (resolved: every key), no m term. */
           cM += gamma * (-Delta);
         }
       }
@@ -402,7 +436,8 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
 
 static int row_alloc(row_t* R, int T, int K) {
   memset(R, 0, sizeof(*R));
-  double** dptrs[] = {&R->s, &R->z, &R->t, &R->wL, &R->wN, &R->P, &R->Pst, &R->g, &R->dS, &R->margin};
+  double** dptrs[] = {&R->s, &R->z, &R->t, &R->wL, &R->wN, &R->P, &R->Pst, &R->g, &R->dS, &R->margin,
+                      &R->er0, &R->er1};
   for (size_t k = 0; k < sizeof(dptrs) / sizeof(dptrs[0]); ++k) {
     *dptrs[k] = (double*)calloc((size_t)T, sizeof(double));
     if (!*dptrs[k]) return -1;
@@ -417,7 +452,7 @@ static int row_alloc(row_t* R, int T, int K) {
 }
 
 static void row_free(row_t* R) {
-  double* dp[] = {R->s, R->z, R->t, R->wL, R->wN, R->P, R->Pst, R->g, R->dS, R->margin, R->e};
+  double* dp[] = {R->s, R->z, R->t, R->wL, R->wN, R->P, R->Pst, R->g, R->dS, R->margin, R->e, R->er0, R->er1};
   for (size_t k = 0; k < sizeof(dp) / sizeof(dp[0]); ++k) free(dp[k]);
   int* ip[] = {R->r, R->l, R->tail, R->code_l, R->code_r};
   for (size_t k = 0; k < sizeof(ip) / sizeof(ip[0]); ++k) free(ip[k]);
@@ -456,9 +491,9 @@ static void* worker(void* arg) {
 
 static int check_params(const kor_params* p) {
   if (!p || p->B < 1 || p->H < 1 || p->T < 1 || p->d < 1) return -1;
-  if (p->calib < 0 || p->calib > 2) return -1;
+  if (p->calib < 0 || p->calib > 3) return -1;
   if (p->calib != KOR_SOFTMAX && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
-  if (p->calib == KOR_FWM && !(p->tau > 0.0)) return -1;
+  if ((p->calib == KOR_FWM || p->calib == KOR_FWM_RESOLVED) && !(p->tau > 0.0)) return -1;
   if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 4) return -1;
   return 0;
 }
@@ -468,6 +503,10 @@ static int run(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_
   if (check_params(p) != 0) return -1;
   /* the uint8 decision codes hold l in 0..K and need K + 1 < KOR_CODE_NOGRID */
   if (fo && (fo->bins || fo->ivals) && p->Kint >= KOR_CODE_NOGRID - 1) return -1;
+  /* resolved: codes l + KOR_CODE_OFFSET <= 252 */
+  if (p->calib == KOR_FWM_RESOLVED && ((fo && (fo->bins || fo->ivals)) || (ov && ov->bins)) &&
+      p->Kint > 252 - KOR_CODE_OFFSET)
+    return -1;
   job_t J;
   memset(&J, 0, sizeof(J));
   J.p = p;

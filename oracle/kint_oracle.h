@@ -24,7 +24,10 @@ typedef double kor_in;
 typedef float kor_in;
 #endif
 
-enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2 };
+/* Calibrations: MinMax, FWM, the softmax comparator, and FWM's "resolved" tail policy
+ * (App. "Tail policy in the MinMax -> FWM change"): FWM's step tau/K and origin -tau,
+ * with the grid continued below -tau (negative indices) instead of a zero tail. */
+enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2, KOR_FWM_RESOLVED = 3 };
 enum { KOR_LERP = 0, KOR_NEAREST = 1 };
 enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
 /* Backward modes: the full calibration gradient (Eq. full), detached extrema (App. B
@@ -36,14 +39,17 @@ enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
 enum { KOR_FULL = 0, KOR_DETACH = 1, KOR_MAX_ONLY = 2, KOR_MIN_ONLY = 3, KOR_DETACH_PROJ = 4 };
 
 /* Codes of the per-key decision arrays (bins: Nearest index l in 0..K,
- * ivals: interval index r in 0..K-1). */
-enum { KOR_CODE_NOGRID = 253, KOR_CODE_TAIL = 254, KOR_CODE_MASKED = 255 };
+ * ivals: interval index r in 0..K-1).  Under the resolved policy the indices run
+ * below zero and are stored as index + KOR_CODE_OFFSET, saturated to [0, 252]
+ * (code 0 stands for every index <= -128; such keys carry weights below
+ * e^{-tau - 128 tau/K}). */
+enum { KOR_CODE_NOGRID = 253, KOR_CODE_TAIL = 254, KOR_CODE_MASKED = 255, KOR_CODE_OFFSET = 128 };
 
 typedef struct {
   int B, H, T, d;
   int Kint;   /* K, number of intervals */
-  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX */
-  double tau; /* FWM window in nats */
+  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX / KOR_FWM_RESOLVED */
+  double tau; /* FWM window in nats (also the resolved grid's origin) */
   int recon;  /* KOR_LERP / KOR_NEAREST */
   int ste;    /* KOR_WEIGHT / KOR_PROB (ignored for LERP) */
   int grad;   /* KOR_FULL / KOR_DETACH / KOR_MAX_ONLY / KOR_MIN_ONLY / KOR_DETACH_PROJ */

@@ -12,12 +12,14 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle import Config, MINMAX, FWM, SOFTMAX, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH, MAX_ONLY, MIN_ONLY, \
-    DETACH_PROJ
+from oracle import Config, MINMAX, FWM, SOFTMAX, FWM_RESOLVED, LERP, NEAREST, WEIGHT, PROB, FULL, DETACH, \
+    MAX_ONLY, MIN_ONLY, DETACH_PROJ
 from tests import witness
 
 ALL_COMBOS = [(c, r, s, g) for c in (MINMAX, FWM) for r in (LERP, NEAREST) for s in (WEIGHT, PROB)
               for g in (FULL, DETACH)]
+RES = FWM_RESOLVED
+RES_COMBOS = [(RES, r, s, g) for r in (LERP, NEAREST) for s in (WEIGHT, PROB) for g in (FULL, DETACH)]
 
 
 def rand_inputs(B, H, T, d, seed, scale=1.0, f64=False):
@@ -51,7 +53,7 @@ def scores_np(Q, K):
 
 # --- P1: rows sum to one (App. A "Normalization") ------------------------------------------------
 
-@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + [(SOFTMAX, LERP, WEIGHT, FULL)])
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + RES_COMBOS + [(SOFTMAX, LERP, WEIGHT, FULL)])
 def test_rows_sum_to_one(calib, recon, ste, grad):
     Q, K, _, _ = rand_inputs(2, 2, 40, 16, 1, scale=2.0)
     V = np.ones_like(Q)
@@ -164,14 +166,16 @@ def test_lerp_k1_closed_form():
 
 # --- P4: K -> infinity, against textbook interpolation bounds ------------------------------------
 
-@pytest.mark.parametrize("calib", [MINMAX, FWM])
+@pytest.mark.parametrize("calib", [MINMAX, FWM, FWM_RESOLVED])
 def test_convergence_to_softmax(calib):
     T, d = 16, 16
     Q, K, _, _ = rand_inputs(8, 1, T, d, 5, scale=2.5)
     V = np.broadcast_to(eye_values(T, d), (8, 1, T, d)).copy()
     S = scores_np(Q, K)
     span = max(S[b, 0, i, : i + 1].max() - S[b, 0, i, : i + 1].min() for b in range(8) for i in range(T))
-    tau = span + 1.0  # FWM window covering every row: no tail
+    # FWM window covering every row: no tail.  The resolved grid needs no such window: with a
+    # 1-nat window most keys sit below it, on the continued grid of the same step.
+    tau = 1.0 if calib == FWM_RESOLVED else span + 1.0
     Ks = [2 ** k for k in range(2, 13)]
     errs = {LERP: [], NEAREST: []}
     for Kint in Ks:
@@ -372,7 +376,7 @@ def test_ties_split_evenly_like_autograd():
 
 # --- P6 / P8: zero-sum identity, shift invariance, the per-key calibration identity --------------
 
-@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS)
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + RES_COMBOS)
 def test_zero_sum_identity(calib, recon, ste, grad):
     Q, K, V, dO = rand_inputs(1, 2, 48, 16, 9, scale=2.0)
     cfg = Config(Kint=8, calib=calib, tau=3.0, recon=recon, ste=ste, grad=grad)
@@ -385,7 +389,7 @@ def test_zero_sum_identity(calib, recon, ste, grad):
         assert np.median(rho) > 1e-3  # detach violates it (App. B "Detach")
 
 
-@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS)
+@pytest.mark.parametrize("calib,recon,ste,grad", ALL_COMBOS + RES_COMBOS)
 def test_key_shift_invariance(calib, recon, ste, grad):
     """K' = K + 1 k0^T adds Q_i.k0/sqrt(d) to every score of row i: F(s + c1) = F(s), so O and dV are
     unchanged; dQ' = dQ + (sum_j dS_ij) k0 / sqrt(d), which is dQ exactly under the full gradient."""
@@ -521,3 +525,117 @@ def test_projection_removes_only_the_common_mode(calib, recon, ste):
     assert not out[DETACH_PROJ]["cM"].any() and not out[DETACH_PROJ]["cm"].any()
     # the detached gradient is not zero-sum in general (App. B), so the projection changes dQ, dK
     assert np.max(np.abs(out[DETACH_PROJ]["dK"] - out[DETACH]["dK"])) > 1e-6
+
+
+# --- Resolved tail policy (App. "Tail policy in the MinMax -> FWM change") --------------------------
+
+@pytest.mark.parametrize("calib,recon,ste,grad", RES_COMBOS + [(RES, NEAREST, PROB, DETACH_PROJ),
+                                                               (RES, LERP, WEIGHT, DETACH_PROJ)])
+@pytest.mark.parametrize("Kint", [1, 4])
+def test_resolved_matches_autograd_witness(calib, recon, ste, grad, Kint):
+    """The witness continues FWM's grid below -tau (floor unclipped below, no tail); tau = 1 puts
+    most keys of these rows below the window."""
+    Q, K, V, dO = rand_inputs(1, 2, 12, 8, 31, scale=2.0)
+    cfg = Config(Kint=Kint, calib=calib, tau=1.0, recon=recon, ste=ste, grad=grad)
+    f = oracle.forward(Q, K, V, cfg, decisions=True)
+    assert np.any(f["ivals"][f["ivals"] != oracle.CODE_MASKED] < oracle.CODE_OFFSET)  # negative indices occur
+    b = oracle.backward(Q, K, V, dO, cfg)
+    O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+    for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+        assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+@pytest.mark.parametrize("recon,ste,grad", [(LERP, WEIGHT, FULL), (NEAREST, WEIGHT, FULL), (NEAREST, PROB, FULL),
+                                            (NEAREST, PROB, DETACH), (LERP, PROB, DETACH_PROJ)])
+def test_resolved_is_fwm_when_no_key_leaves_the_window(recon, ste, grad):
+    """Inside the window both policies use the same grid values (the paper: in-window weights
+    bit-identical), so with a window wider than every row's span they agree bit for bit."""
+    Q, K, V, dO = rand_inputs(1, 2, 20, 8, 33, scale=1.5)
+    S = scores_np(Q, K)
+    tau = 1.0 + max(S[0, h, i, : i + 1].max() - S[0, h, i, : i + 1].min() for h in range(2) for i in range(20))
+    out = {}
+    for c in (FWM, RES):
+        cfg = Config(Kint=4, calib=c, tau=tau, recon=recon, ste=ste, grad=grad)
+        out[c] = (oracle.forward(Q, K, V, cfg, decisions=True), oracle.backward(Q, K, V, dO, cfg))
+    for n in ("O", "W"):
+        assert np.array_equal(out[FWM][0][n], out[RES][0][n])
+    for n in ("dQ", "dK", "dV", "cM"):
+        assert np.array_equal(out[FWM][1][n], out[RES][1][n])
+    live = out[FWM][0]["bins"] != oracle.CODE_MASKED
+    assert np.array_equal(out[FWM][0]["bins"][live].astype(int) + oracle.CODE_OFFSET,
+                          out[RES][0]["bins"][live].astype(int))
+
+
+def test_resolved_brute_force_on_lattice():
+    """Nearest index by scanning every grid point b_l = -tau + l h, l = -60..K (ties go up), LERP
+    weight from the interval that contains z, on score lattices reaching 11 steps below the
+    window; the stored codes are index + 128."""
+    rng = np.random.default_rng(35)
+    Kint, T, tau = 4, 16, 2.0
+    h = tau / Kint
+    for trial in range(40):
+        ks = rng.integers(0, 61, size=T)
+        ks[rng.integers(0, T)] = 0
+        targets = 1.0 - 0.125 * ks  # 1/8 lattice: grid points and Nearest midpoints of h = 1/2
+        Q, K = lattice_qk(targets)
+        cfg = Config(Kint=Kint, calib=RES, tau=tau, recon=NEAREST)
+        out = oracle.forward(Q, K, eye_values(T, 16), cfg, decisions=True)
+        out_l = oracle.forward(Q, K, eye_values(T, 16), Config(Kint=Kint, calib=RES, tau=tau, recon=LERP))
+        z = targets - targets.max()
+        grid = {l: -tau + l * h for l in range(-60, Kint + 1)}
+        ell, rr, wl, wn = [], [], [], []
+        for zj in z:
+            best, best_l = math.inf, None
+            for l, b in sorted(grid.items()):
+                if abs(zj - b) <= best:  # equal distance: the larger index wins
+                    best, best_l = abs(zj - b), l
+            r = min(max(l for l, b in grid.items() if b <= zj), Kint - 1)
+            t = min(max((zj - grid[r]) / h, 0.0), 1.0)
+            ell.append(best_l + 128)
+            rr.append(r + 128)
+            wn.append(math.exp(grid[best_l]))
+            wl.append((1 - t) * math.exp(grid[r]) + t * math.exp(grid[r + 1]))
+        wl, wn = np.array(wl), np.array(wn)
+        last = T - 1
+        assert np.array_equal(out["bins"][0, 0, last], ell), (trial, targets)
+        assert np.array_equal(out["ivals"][0, 0, last], rr), (trial, targets)
+        assert np.allclose(out["O"][0, 0, last, :T], wn / wn.sum(), rtol=0, atol=1e-15)
+        assert np.allclose(out_l["O"][0, 0, last, :T], wl / wl.sum(), rtol=0, atol=1e-15)
+
+
+@pytest.mark.parametrize("recon", [LERP, NEAREST])
+def test_resolved_on_grid_scores_is_softmax(recon):
+    """Scores on the grid's own points (multiples of h = tau/K from the row max, far below the
+    window too) are reconstructed exactly, w = e^z, so the resolved operator is softmax there;
+    FWM, which zeroes keys below -tau, is not."""
+    T, tau, Kint = 16, 1.0, 4
+    rng = np.random.default_rng(37)
+    ks = rng.integers(0, 40, size=T)
+    ks[3] = 0
+    targets = -0.25 * ks  # h = 1/4: every score on a grid point, down to 39 steps below the max
+    Q, K = lattice_qk(targets)
+    V = eye_values(T, 16)
+    z = targets - targets.max()
+    pe = np.exp(z) / np.exp(z).sum()
+    res = oracle.forward(Q, K, V, Config(Kint=Kint, calib=RES, tau=tau, recon=recon))
+    fwm = oracle.forward(Q, K, V, Config(Kint=Kint, calib=FWM, tau=tau, recon=recon))
+    assert np.allclose(res["O"][0, 0, T - 1, :T], pe, rtol=1e-13, atol=0)
+    assert np.max(np.abs(fwm["O"][0, 0, T - 1, :T] - pe)) > 1e-3
+
+
+def test_resolved_decision_override_roundtrip():
+    Q, K, V, dO = rand_inputs(1, 1, 20, 8, 39, scale=2.0)
+    cfg = Config(Kint=4, calib=RES, tau=1.0, recon=NEAREST, ste=PROB)
+    f = oracle.forward(Q, K, V, cfg, decisions=True)
+    ov = {"bins": f["bins"], "ivals": f["ivals"], "amax": f["amax"], "amin": f["amin"]}
+    g = oracle.forward(Q, K, V, cfg, override=ov)
+    assert np.array_equal(f["O"], g["O"])
+    bins = f["bins"].copy()
+    i = 17
+    below = [j for j in range(i + 1) if 0 < bins[0, 0, i, j] < oracle.CODE_OFFSET]  # keys below the window
+    assert below
+    j = below[0]
+    bins[0, 0, i, j] += 1
+    hh = oracle.forward(Q, K, V, cfg, override={**ov, "bins": bins})
+    changed = np.where(np.any(hh["O"] != f["O"], axis=-1))
+    assert list(changed[2]) == [i]

@@ -15,7 +15,7 @@ import math
 import numpy as np
 import torch
 
-MINMAX, FWM, SOFTMAX = 0, 1, 2
+MINMAX, FWM, SOFTMAX, FWM_RESOLVED = 0, 1, 2, 3
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
 FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4
@@ -41,13 +41,21 @@ def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
         b0 = m - M
         zc = z
         tail = torch.zeros_like(valid)
-    else:
+    elif cfg.calib == FWM:
         h = torch.full_like(M, cfg.tau / K)
         b0 = torch.full_like(M, -cfg.tau)
         tail = z < -cfg.tau
         zc = z.clamp(-cfg.tau, 0.0)
+    else:
+        # resolved tail policy: FWM's grid, continued below -tau (no tail, no clip)
+        h = torch.full_like(M, cfg.tau / K)
+        b0 = torch.full_like(M, -cfg.tau)
+        tail = torch.zeros_like(valid)
+        zc = z
     u = (zc - b0) / h
-    r = torch.floor(u.detach()).clamp(0, K - 1)
+    r = torch.floor(u.detach()).clamp(max=K - 1)
+    if cfg.calib != FWM_RESOLVED:
+        r = r.clamp(min=0)
     b_lo = b0 + r * h
     b_hi = b0 + (r + 1) * h
     # With r = clip(floor(u), 0, K-1) the position t lies in [0, 1] up to rounding; its clip only
