@@ -422,9 +422,25 @@ def run_cuda(args, world, rank, local):
     e2e_run(2)
     n_e2e = max(3, min(args.steps, 100))
     ms_e2e = timed(1, lambda i: e2e_run(n_e2e)) / n_e2e
+    # the same copies with no compute: the host link's floor for one end-to-end step
+    def copies_only(i):
+        b = i % 2
+        s_in.wait_stream(s_c)
+        s_out.wait_stream(s_c)
+        with torch.cuda.stream(s_in):
+            for dst, src in zip(ins[b], pin_in):
+                dst.copy_(src, non_blocking=True)
+        with torch.cuda.stream(s_out):
+            for dst, src in zip(pin_out, outs[b]):
+                dst.copy_(src, non_blocking=True)
+        s_c.wait_stream(s_in)
+        s_c.wait_stream(s_out)
+
+    ms_link = timed(n_e2e, copies_only)
     line["e2e"] = {"value": job_value(flops_step, world, ms_e2e), "unit": UNIT,
                    "h2d_bytes_per_step": sum(t.numel() * 4 for t in pin_in),
-                   "d2h_bytes_per_step": sum(t.numel() * 4 for t in pin_out), "ms_per_step": ms_e2e}
+                   "d2h_bytes_per_step": sum(t.numel() * 4 for t in pin_out), "ms_per_step": ms_e2e,
+                   "copies_only_ms_per_step": ms_link, "link_bound_frac": ms_link / ms_e2e}
     kint.check_status()
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

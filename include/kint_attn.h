@@ -52,8 +52,17 @@ extern "C" {
 #define KINT_ERR_SCRATCH_LIMIT (-8) /* kint_attn_fwd_noalloc: problem needs more than KINT_NOALLOC_SCRATCH_BYTES */
 
 /* Calibration (Sec. 3 "Objects and calibration"; App. A "MinMax grid", "FWM";
- * App. A "Softmax" is the exact-exponential comparator). */
-typedef enum { KINT_CALIB_MINMAX = 0, KINT_CALIB_FWM = 1, KINT_CALIB_SOFTMAX = 2 } kint_calib;
+ * App. A "Softmax" is the exact-exponential comparator).  FWM_RESOLVED is the
+ * "resolved" tail policy of App. "Tail policy in the MinMax -> FWM change": FWM's
+ * step tau/K and origin -tau, with the grid continued below -tau (negative indices)
+ * instead of a zero tail; its grid values below the window come from the exponential
+ * unit (ex2.approx), in-window values from the same table as FWM. */
+typedef enum {
+  KINT_CALIB_MINMAX = 0,
+  KINT_CALIB_FWM = 1,
+  KINT_CALIB_SOFTMAX = 2,
+  KINT_CALIB_FWM_RESOLVED = 3
+} kint_calib;
 /* Reconstruction (Sec. 3 "Reconstruction"; App. A "LERP", "Nearest"). */
 typedef enum { KINT_RECON_LERP = 0, KINT_RECON_NEAREST = 1 } kint_recon;
 /* Surrogate placement (Sec. 3 Eqs. wste / pste).  Ignored under LERP, where the
@@ -149,7 +158,9 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
  * Decision dump for parity checks: for every (b, h, i, j) the Nearest index
  * l_ij = r + [t >= 1/2] in 0..K (bins) and the interval index r_ij in 0..K-1
  * (ivals), with 254 for FWM tail keys (z < -tau), 255 for masked keys (j > i)
- * and 253 where no grid exists (degenerate MinMax rows, softmax).  Either
+ * and 253 where no grid exists (degenerate MinMax rows, softmax); under
+ * FWM_RESOLVED both indices run below zero and are stored as index + 128,
+ * saturated to [0, 252] (0: index <= -128).  Either
  * output may be NULL.  Needs the row statistics of kint_attn_fwd on the same
  * inputs and the forward's workspace size.  bins, ivals: [B,H,T,T] uint8.
  */

@@ -162,11 +162,12 @@ struct Common {
 int validate(const Common& c, int causal) {
   if (c.B < 1 || c.H < 1 || c.T < 1 || c.d < 1) return KINT_ERR_ARG;
   if (causal != 1) return KINT_ERR_ARG;
-  if (c.calib < 0 || c.calib > 2 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
+  if (c.calib < 0 || c.calib > 3 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
       c.grad > 4 || c.prec < 0 || c.prec > 1)
     return KINT_ERR_ARG;
   if (c.calib != KINT_CALIB_SOFTMAX && (c.Kint < 1 || c.Kint > KMAX)) return KINT_ERR_ARG;
-  if (c.calib == KINT_CALIB_FWM && !(c.tau > 0.0f && std::isfinite(c.tau))) return KINT_ERR_ARG;
+  if ((c.calib == KINT_CALIB_FWM || c.calib == KINT_CALIB_FWM_RESOLVED) && !(c.tau > 0.0f && std::isfinite(c.tau)))
+    return KINT_ERR_ARG;
   if (c.d != 64 && c.d != 128) return KINT_ERR_UNSUPPORTED;
   if (c.prec == KINT_PREC_3XTF32 && c.d != 64) return KINT_ERR_UNSUPPORTED;
   // MinMax keeps a (K x 128)-pair grid table per query block in shared memory;
@@ -189,10 +190,13 @@ Params base_params(const Common& c, unsigned* status) {
   p.nqb = (c.T + 127) / 128;
   p.tau = c.tau;
   p.scale = (float)(1.0 / std::sqrt((double)c.d));
-  if (c.calib == KINT_CALIB_FWM) {
+  if (c.calib == KINT_CALIB_FWM || c.calib == KINT_CALIB_FWM_RESOLVED) {
     p.fwm_inv_h = (float)((double)c.Kint / (double)c.tau);
     for (int r = 0; r <= c.Kint; ++r)
       p.fwm_e[r] = (float)std::exp(-(double)c.tau + (double)r * (double)c.tau / (double)c.Kint);
+    const double log2e = 1.4426950408889634;
+    p.fwm_hl = (float)((double)c.tau / (double)c.Kint * log2e);
+    p.fwm_b0l = (float)(-(double)c.tau * log2e);
   }
   p.wait_ns = g_wait_ns;
   p.status = status;
@@ -230,7 +234,7 @@ int plan_stats(Params& p) {
 int plan_main(Params& p, int mode) {
   const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
   // (e_r, e_{r+1}) pairs: per row for MinMax ([K][128]), one shared [K] for FWM
-  const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : (p.calib == KINT_CALIB_FWM ? 1024 : 0);
+  const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : (p.calib == KINT_CALIB_FWM || p.calib == KINT_CALIB_FWM_RESOLVED ? 1024 : 0);
   const bool useA2 = mode == PV_MAIN_LERP || p.x3;
   const int cols1 = 128 + (useA2 ? 128 : 0) + p.d + (mode == PV_MAIN_LERP ? p.d : 0);
   const int ostage = (mode == PV_MAIN_LERP ? 2 : 1) * 128 * p.d * 4;  // O (and O_lerp) staging tiles
@@ -310,7 +314,7 @@ int plan_dkdv(Params& p, int sel) {
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     // FWM Nearest: the half-bin table, 2K + 3 entries of 8 bytes
-    const int table = p.calib == KINT_CALIB_FWM ? 2048 : 1024;
+    const int table = (p.calib == KINT_CALIB_FWM || p.calib == KINT_CALIB_FWM_RESOLVED) ? 2048 : 1024;
     const int total = std::max(finish_plan(p, p.sm_table + table, 4 * p.nstage + 8), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;

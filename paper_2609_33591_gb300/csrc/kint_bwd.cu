@@ -32,17 +32,24 @@ template <int CAL, bool FULLG, bool DIAG, int W>
 __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)[W], float (&out)[W], int j0,
                                          int i, float k1, float c0, float inv_h, float ga, float gb, bool nogrid,
                                          float Kf, float fk, uint32_t tab, float sk1, float sc0, float invWf,
-                                         float& own, float& cm) {
+                                         float hl, float b0l, float& own, float& cm) {
 #pragma unroll
   for (int jj = 0; jj < W; ++jj) {
     float ds, dm = 0.f;
     if constexpr (CAL == CAL_SOFTMAX) {
       const float pr = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * invWf;
       ds = pr * __fmaf_rn(gv[jj], ga, gb);  // P (g - <g>_P)
-    } else if constexpr (CAL == CAL_FWM) {
+    } else if constexpr (fwm_like(CAL)) {
       // k1, c0 doubled (v = 2u), Kf = 2K, tab: the half-bin table of Delta_r / h (4-byte entries)
-      const uint32_t qb = fwm_half_bits(__fmaf_rn(sv[jj], k1, c0), Kf);
-      ds = __fmaf_rn(gv[jj], ga, gb) * lds_f32(tab + qb * 4u);
+      const float v = __fmaf_rn(sv[jj], k1, c0);
+      const uint32_t qb = fwm_half_bits(v, Kf);
+      float dl = lds_f32(tab + qb * 4u);
+      if constexpr (CAL == CAL_FWMR) {
+        // resolved: below the window the secant of the continued grid (u = v / 2 exactly)
+        const BelowPair bp = resolved_below(__fmul_rn(v, 0.5f), hl, b0l);
+        dl = v < 0.0f ? __fmul_rn(__fsub_rn(bp.e1, bp.e0), inv_h) : dl;
+      }
+      ds = __fmaf_rn(gv[jj], ga, gb) * dl;
     } else {
       const float u = __fmaf_rn(sv[jj], k1, c0);
       float t, rf;
@@ -379,7 +386,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
       const float M = nx.M, m = nx.m, Wf = nx.Wf, Ws = nx.Ws, Dg = nx.Dg;
       const int nmax = nx.nmax, nmin = nx.nmin, amax = nx.amax, amin = nx.amin;
       const RowGrid g = row_grid(p, M, m);
-      if constexpr (CAL == CAL_FWM) {  // the same for every item
+      if constexpr (fwm_like(CAL)) {  // the same for every item
         if (n == 0 && tid < 2 * Kq + 1 + kHalfTail)
           *reinterpret_cast<float*>(sm + p.sm_table + tid * 4) = fwm_half_entry(p, tid - kHalfTail).y;
       } else if constexpr (CAL == CAL_MINMAX) {
@@ -401,9 +408,9 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
       // FWM: the half-bin table, entry q at sm_table + 4 (q + 2), addressed by the bits
       // 0x4B000000 + q of floor(2u) (0x4B000000 * 4 = 0x2C000000 mod 2^32), and the doubled
       // position v = 2u; MinMax: this row's pair table, r * 1024 apart
-      const float Kf = (float)(CAL == CAL_FWM ? 2 * Kq : Kq), fk = 1.0f / (float)Kq;
-      const float k1q = CAL == CAL_FWM ? 2.0f * g.k1 : g.k1, c0q = CAL == CAL_FWM ? 2.0f * g.c0 : g.c0;
-      const uint32_t tab = (CAL == CAL_FWM) ? smem_u32(sm + p.sm_table) + 4u * kHalfTail - 0x2C000000u
+      const float Kf = (float)(fwm_like(CAL) ? 2 * Kq : Kq), fk = 1.0f / (float)Kq;
+      const float k1q = fwm_like(CAL) ? 2.0f * g.k1 : g.k1, c0q = fwm_like(CAL) ? 2.0f * g.c0 : g.c0;
+      const uint32_t tab = fwm_like(CAL) ? smem_u32(sm + p.sm_table) + 4u * kHalfTail - 0x2C000000u
                                             : smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
       const bool minmax = CAL == CAL_MINMAX;
       const bool track = FULLG && CAL != CAL_SOFTMAX && row_ok && !g.nogrid && (nmax > 1 || (minmax && nmin > 1));
@@ -435,10 +442,10 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         const int j0 = kt * BT + cg * W;
         if (j0 + W - 1 > qb * 128)
           dq_chunk<CAL, FULLG, true, W>(sv, gv, out, j0, i, k1q, c0q, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab, sk1,
-                                        sc0, invWf, own, cm);
+                                        sc0, invWf, g.hl, g.b0l, own, cm);
         else
           dq_chunk<CAL, FULLG, false, W>(sv, gv, out, j0, i, k1q, c0q, g.inv_h, ga, gb, g.nogrid, Kf, fk, tab,
-                                         sk1, sc0, invWf, own, cm);
+                                         sk1, sc0, invWf, g.hl, g.b0l, own, cm);
         if (__any_sync(0xffffffffu, track)) {
           // rare: tied extrema, the tie set is found by equality on the recomputed scores
           uint32_t mk_max = 0, mk_min = 0;
@@ -583,7 +590,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
           if (p.cM_out) p.cM_out[rw] = cMv;
           if (p.cm_out) p.cm_out[rw] = cmv;
           // the position as the dK/dV pass forms it: softmax log2 e^{s-M}, FWM Nearest 2u, else u
-          const bool half = CAL == CAL_FWM && p.recon == REC_NEAREST;
+          const bool half = fwm_like(CAL) && p.recon == REC_NEAREST;
           RowRec r;
           r.c0 = CAL == CAL_SOFTMAX ? sc0 : (half ? 2.0f * g.c0 : g.c0);
           r.k1 = CAL == CAL_SOFTMAX ? sk1 : (half ? 2.0f * g.k1 : g.k1);
@@ -627,7 +634,7 @@ template <int CAL, int REC, bool FULLG, bool PROJ, bool MASKED, bool TIES, int W
 __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)[W], float (&pa)[W],
                                          float (&da)[W], int j, int i0, int T, uint32_t recs, uint32_t tabs,
                                          uint32_t fwtab, uint32_t tstride, float Kf, float fwm_inv_h,
-                                         float scale) {
+                                         float scale, float hl, float b0l) {
 #pragma unroll
   for (int ii = 0; ii < W; ++ii) {
     const uint32_t ra = recs + ii * 64u;  // RowRec of query row i0 + ii
@@ -640,10 +647,17 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
     if constexpr (CAL == CAL_SOFTMAX) {
       pv = ex2_approx(__fmaf_rn(sv[ii], r0.y, r0.x)) * r0.z;
       ds = pv * gam;
-    } else if constexpr (CAL == CAL_FWM && REC == REC_NEAREST) {
+    } else if constexpr (fwm_like(CAL) && REC == REC_NEAREST) {
       // record holds 2k1, 2c0; Kf = 2K; fwtab: the half-bin table of (w^N, Delta_r / h)
-      const uint32_t qb = fwm_half_bits(__fmaf_rn(sv[ii], r0.y, r0.x), Kf);
-      const float2 e = lds_f2(fwtab + qb * 8u);
+      const float v = __fmaf_rn(sv[ii], r0.y, r0.x);
+      const uint32_t qb = fwm_half_bits(v, Kf);
+      float2 e = lds_f2(fwtab + qb * 8u);
+      if constexpr (CAL == CAL_FWMR) {
+        // resolved: below the window, (w^N, Delta_r / h) of the continued grid (u = v / 2 exactly)
+        const BelowPair bp = resolved_below(__fmul_rn(v, 0.5f), hl, b0l);
+        const float2 eb = make_float2(bp.t >= 0.5f ? bp.e1 : bp.e0, __fmul_rn(__fsub_rn(bp.e1, bp.e0), fwm_inv_h));
+        e = v < 0.0f ? eb : e;
+      }
       pv = e.x * r0.z;
       ds = gam * e.y;
     } else {
@@ -651,7 +665,13 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
       float t, rf;
       uint32_t rb;
       decode_u(u, Kf, t, rb, rf);
-      const float2 e = lds_f2(CAL == CAL_FWM ? fwtab + rb * 8u : tabs + ii * tstride + rb * 8u);
+      float2 e = lds_f2(fwm_like(CAL) ? fwtab + rb * 8u : tabs + ii * tstride + rb * 8u);
+      if constexpr (CAL == CAL_FWMR) {
+        const BelowPair bp = resolved_below(u, hl, b0l);
+        const bool below = u < 0.0f;
+        t = below ? bp.t : t;
+        e = below ? make_float2(bp.e0, bp.e1) : e;
+      }
       const float de = __fsub_rn(e.y, e.x);
       const float wl = __fmaf_rn(t, de, e.x);
       const float wn = (t >= 0.5f) ? e.y : e.x;
@@ -955,8 +975,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     // FWM Nearest: the half-bin table (entry q at sm_table + 8 (q + 2)) and the doubled
     // position; FWM LERP: the pair table, entry r at sm_table + 8 r (0x4B000000 * 8 =
     // 0x58000000 mod 2^32)
-    constexpr bool half = CAL == CAL_FWM && REC == REC_NEAREST;
-    if constexpr (CAL == CAL_FWM) {
+    constexpr bool half = fwm_like(CAL) && REC == REC_NEAREST;
+    if constexpr (fwm_like(CAL)) {
       if (half && tid < 2 * Kq + 1 + kHalfTail)
         *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = fwm_half_entry(p, tid - kHalfTail);
       if (!half && tid < Kq)
@@ -1008,13 +1028,13 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
           const bool masked = (i0h < kb * 128 + 128) || (i0h + WS > p.T);
           if (FULLG && CAL != CAL_SOFTMAX && tie_here)
             kv_chunk<CAL, REC, FULLG, PROJ, true, true, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride, Kf,
-                                                      p.fwm_inv_h, p.scale);
+                                                      p.fwm_inv_h, p.scale, p.fwm_hl, p.fwm_b0l);
           else if (masked)
             kv_chunk<CAL, REC, FULLG, PROJ, true, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
-                                                       Kf, p.fwm_inv_h, p.scale);
+                                                       Kf, p.fwm_inv_h, p.scale, p.fwm_hl, p.fwm_b0l);
           else
             kv_chunk<CAL, REC, FULLG, PROJ, false, false, WS>(sv, gv, pa, da, j, i0h, p.T, recs, tabs, fwtab, tstride,
-                                                        Kf, p.fwm_inv_h, p.scale);
+                                                        Kf, p.fwm_inv_h, p.scale, p.fwm_hl, p.fwm_b0l);
           if (p.x3) {
 #pragma unroll
             for (int q = 0; q < WS; ++q) {
@@ -1151,6 +1171,9 @@ cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cud
   if (p.calib == CAL_MINMAX)
     return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
                 : launch3(k_bwd_dq<CAL_MINMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
+  if (p.calib == CAL_FWMR)
+    return full ? launch3(k_bwd_dq<CAL_FWMR, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
+                : launch3(k_bwd_dq<CAL_FWMR, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
   return full ? launch3(k_bwd_dq<CAL_FWM, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
               : launch3(k_bwd_dq<CAL_FWM, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
 }
@@ -1168,6 +1191,15 @@ cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, c
     return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, true>, grid, maps, p, smem_bytes, s)
            : proj ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
                   : launch3(k_bwd_dkdv<CAL_MINMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+  }
+  if (p.calib == CAL_FWMR) {
+    if (near)
+      return full ? launch3(k_bwd_dkdv<CAL_FWMR, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)
+             : proj ? launch3(k_bwd_dkdv<CAL_FWMR, REC_NEAREST, false, true>, grid, maps, p, smem_bytes, s)
+                    : launch3(k_bwd_dkdv<CAL_FWMR, REC_NEAREST, false>, grid, maps, p, smem_bytes, s);
+    return full ? launch3(k_bwd_dkdv<CAL_FWMR, REC_LERP, true>, grid, maps, p, smem_bytes, s)
+           : proj ? launch3(k_bwd_dkdv<CAL_FWMR, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
+                  : launch3(k_bwd_dkdv<CAL_FWMR, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   }
   if (near)
     return full ? launch3(k_bwd_dkdv<CAL_FWM, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)

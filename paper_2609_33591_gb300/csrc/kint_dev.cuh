@@ -119,12 +119,15 @@ __device__ __forceinline__ int snake_item(int n) {
 // ---------------------------------------------------------------------------
 struct RowGrid {
   float inv_h, c0, h, b0;
+  float hl, b0l;  // resolved grid: e_r = 2^(r hl + b0l)
   float k1;     // scale * inv_h: u = acc * k1 + c0 straight from the raw accumulator
   bool nogrid;  // degenerate MinMax row (M - m <= 1e-12) or softmax
 };
 
 __device__ __forceinline__ RowGrid row_grid(const Params& p, float M, float m) {
   RowGrid g;
+  g.hl = p.fwm_hl;
+  g.b0l = p.fwm_b0l;
   if (p.calib == CAL_MINMAX) {
     const float span = __fsub_rn(M, m);
     g.nogrid = !(span > 1e-12f);
@@ -134,7 +137,7 @@ __device__ __forceinline__ RowGrid row_grid(const Params& p, float M, float m) {
     g.c0 = -__fmul_rn(m, g.inv_h);
     g.b0 = __fsub_rn(m, M);
     g.k1 = __fmul_rn(p.scale, g.inv_h);
-  } else if (p.calib == CAL_FWM) {
+  } else if (fwm_like(p.calib)) {
     g.nogrid = false;
     g.h = __fdiv_rn(p.tau, (float)p.Kint);
     g.inv_h = p.fwm_inv_h;
@@ -219,28 +222,24 @@ __device__ __forceinline__ float ex2_approx(float x) {
 // Grid value e^{b_r}, r = 0..K.  MinMax: b_r = b0 + r h from the row's own
 // extrema (device expf, K + 1 calls per row).  FWM: host table.
 __device__ __forceinline__ float grid_value(const Params& p, const RowGrid& g, int r) {
-  if (p.calib == CAL_FWM) return p.fwm_e[r];
+  if (fwm_like(p.calib)) return p.fwm_e[r];
   return expf(__fmaf_rn((float)r, g.h, g.b0));
 }
 
-// Per-key decisions of App. A from the grid position u.
-struct KeyPos {
-  int r;     // interval index, clip(floor(u), 0, K-1)
-  int l;     // Nearest index, r + [t >= 1/2]
-  float t;   // position in the interval, clip(u - r, 0, 1)
-  bool tail; // FWM zero tail (z < -tau)
+// Resolved tail policy (App. "Tail policy in the MinMax -> FWM change"): below the
+// window (u < 0) FWM's grid continues with negative indices, r = floor(u), t = u - r
+// (exact), and the grid values e^{-tau + r tau/K} = 2^(r hl + b0l) come from the
+// exponential unit (far below the window they flush to zero).  Only read where u < 0.
+struct BelowPair {
+  float t, e0, e1;  // position in the interval, e_r, e_{r+1}
 };
-
-__device__ __forceinline__ KeyPos key_pos(const Params& p, float u) {
-  KeyPos k;
-  k.tail = (p.calib == CAL_FWM) && (u < 0.0f);
-  const float uc = fminf(fmaxf(u, 0.0f), (float)p.Kint);
-  int r = __float2int_rd(uc);
-  r = min(r, p.Kint - 1);
-  k.r = r;
-  k.t = fminf(fmaxf(__fsub_rn(uc, (float)r), 0.0f), 1.0f);
-  k.l = r + (k.t >= 0.5f ? 1 : 0);
-  return k;
+__device__ __forceinline__ BelowPair resolved_below(float u, float hl, float b0l) {
+  BelowPair b;
+  const float rf = floorf(u);
+  b.t = __fsub_rn(u, rf);
+  b.e0 = ex2_approx(__fmaf_rn(rf, hl, b0l));
+  b.e1 = ex2_approx(__fmaf_rn(__fadd_rn(rf, 1.0f), hl, b0l));
+  return b;
 }
 
 // ---------------------------------------------------------------------------

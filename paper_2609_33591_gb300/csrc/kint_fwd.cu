@@ -412,7 +412,14 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
       uint32_t rb;
       decode_u(u, Kf, t, rb, rf);
       // MinMax: this row's table, rows 1024 bytes apart; FWM: one shared table, entries 8 bytes apart
-      const float2 e = lds_f2(CAL == CAL_FWM ? tab + rb * 8u : tab + rb * 1024u);
+      float2 e = lds_f2(fwm_like(CAL) ? tab + rb * 8u : tab + rb * 1024u);
+      if constexpr (CAL == CAL_FWMR) {
+        // below the window: the continued grid (negative r)
+        const BelowPair bp = resolved_below(u, g.hl, g.b0l);
+        const bool below = u < 0.0f;
+        t = below ? bp.t : t;
+        e = below ? make_float2(bp.e0, bp.e1) : e;
+      }
       wl = __fmaf_rn(t, __fsub_rn(e.y, e.x), e.x);
       float wn = (t >= 0.5f) ? e.y : e.x;
       if constexpr (CAL == CAL_FWM) {
@@ -440,7 +447,10 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
   wl_sum += wl_acc;
 }
 
-// Decision codes of one chunk for kint_attn_debug_bins (not on the timed path).
+// Decision codes of one chunk for kint_attn_debug_bins (not on the timed path, but
+// inlined into the main loop: the calibration is a template parameter so that each
+// instantiation carries only its own branch).
+template <int CAL>
 __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, int i, int bh, const RowGrid& g) {
   if (i >= p.T) return;
   for (int jj = 0; jj < 32; ++jj) {
@@ -448,15 +458,22 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
     if (j >= p.T) break;
     uint8_t cb = 255, ci = 255;
     if (j <= i) {
-      if (p.calib == CAL_SOFTMAX || g.nogrid) {
+      if (CAL == CAL_SOFTMAX || g.nogrid) {
         cb = ci = 253;
       } else {
         const float u = __fmaf_rn(v[jj], g.k1, g.c0);
         float t, rf;
         uint32_t rb;
         decode_u(u, (float)p.Kint, t, rb, rf);
-        if (p.calib == CAL_FWM && u < 0.0f) {
+        if (CAL == CAL_FWM && u < 0.0f) {
           cb = ci = 254;
+        } else if constexpr (CAL == CAL_FWMR) {
+          // resolved: indices run below zero, stored as index + 128 saturated to [0, 252]
+          const int r = u < 0.0f ? (int)floorf(u) : (int)rf;
+          const float tt = u < 0.0f ? __fsub_rn(u, floorf(u)) : t;
+          const int l = r + (tt >= 0.5f ? 1 : 0);
+          ci = (uint8_t)min(max(r + 128, 0), 252);
+          cb = (uint8_t)min(max(l + 128, 0), 252);
         } else {
           const int r = (int)rf;
           ci = (uint8_t)r;
@@ -665,7 +682,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       // ([K][128], 1024 bytes per r: rb * 1024 wraps to r * 1024); FWM's grid is the
       // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r).
       uint32_t tab;
-      if constexpr (CAL == CAL_FWM) {
+      if constexpr (fwm_like(CAL)) {
         tab = smem_u32(sm + p.sm_table) - 0x58000000u;
         if (n == 0 && tid < Kq)
           *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
@@ -696,7 +713,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
           tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
           tmem_ld_wait();
           const int j0 = kb * 128 + c * 32;
-          if (p.debug) fwd_debug_codes(p, v, j0, i, bh, gr);
+          if (p.debug) fwd_debug_codes<CAL>(p, v, j0, i, bh, gr);
           if (diag)
             fwd_chunk<CAL, REC, MODE, true>(v, a1, a2, j0, i, gr, Kf, tab, sk1, sc0, Wm, Wl);
           else
@@ -801,6 +818,12 @@ cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, c
     if (mode == PV_MAIN) return launch_main_t<CAL_MINMAX, REC_NEAREST, 0>(maps, p, smem_bytes, s);
     if (mode == PV_MAIN_LERP) return launch_main_t<CAL_MINMAX, REC_NEAREST, 1>(maps, p, smem_bytes, s);
     return launch_main_t<CAL_MINMAX, REC_NEAREST, 2>(maps, p, smem_bytes, s);
+  }
+  if (p.calib == CAL_FWMR) {
+    if (p.recon == REC_LERP) return launch_main_t<CAL_FWMR, REC_LERP, 0>(maps, p, smem_bytes, s);
+    if (mode == PV_MAIN) return launch_main_t<CAL_FWMR, REC_NEAREST, 0>(maps, p, smem_bytes, s);
+    if (mode == PV_MAIN_LERP) return launch_main_t<CAL_FWMR, REC_NEAREST, 1>(maps, p, smem_bytes, s);
+    return launch_main_t<CAL_FWMR, REC_NEAREST, 2>(maps, p, smem_bytes, s);
   }
   if (p.recon == REC_LERP) return launch_main_t<CAL_FWM, REC_LERP, 0>(maps, p, smem_bytes, s);
   if (mode == PV_MAIN) return launch_main_t<CAL_FWM, REC_NEAREST, 0>(maps, p, smem_bytes, s);

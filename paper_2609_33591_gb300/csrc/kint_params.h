@@ -6,7 +6,10 @@
 
 namespace kint {
 
-enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2 };
+enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2, CAL_FWMR = 3 };
+// FWM's grid (step tau/K, origin -tau), with a zero tail below the window (FWM) or
+// continued below it with negative indices (CAL_FWMR, the "resolved" tail policy)
+__host__ __device__ constexpr bool fwm_like(int cal) { return cal == CAL_FWM || cal == CAL_FWMR; }
 enum Recon : int { REC_LERP = 0, REC_NEAREST = 1 };
 enum Grad : int { GRAD_FULL = 0, GRAD_DETACH = 1, GRAD_MAX_ONLY = 2, GRAD_MIN_ONLY = 3, GRAD_DETACH_PROJ = 4 };
 
@@ -34,6 +37,7 @@ struct Params {
   int BH, nqb;  // number of 128-row query blocks
   float tau, scale;       // scale = 1/sqrt(d)
   float fwm_inv_h;        // K / tau (FWM), host-rounded
+  float fwm_hl, fwm_b0l;  // (tau / K) log2 e and -tau log2 e (resolved grid below the window)
   float fwm_e[KMAX + 2];  // FWM grid values e^{-tau + r tau/K}, r = 0..K (host fp64 -> fp32)
   int pv_sel, dkv_sel, debug;
   unsigned long long wait_ns;

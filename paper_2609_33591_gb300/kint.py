@@ -17,7 +17,7 @@ import torch
 
 from . import build as _build
 
-CALIB_MINMAX, CALIB_FWM, CALIB_SOFTMAX = 0, 1, 2
+CALIB_MINMAX, CALIB_FWM, CALIB_SOFTMAX, CALIB_FWM_RESOLVED = 0, 1, 2, 3
 RECON_LERP, RECON_NEAREST = 0, 1
 STE_WEIGHT, STE_PROB = 0, 1
 GRAD_FULL, GRAD_DETACH, GRAD_MAX_ONLY, GRAD_MIN_ONLY, GRAD_DETACH_PROJ = 0, 1, 2, 3, 4

@@ -10,7 +10,7 @@ from tests import parity
 
 pytestmark = pytest.mark.gpu
 
-MM, FW, SM = kint.CALIB_MINMAX, kint.CALIB_FWM, kint.CALIB_SOFTMAX
+MM, FW, SM, FR = kint.CALIB_MINMAX, kint.CALIB_FWM, kint.CALIB_SOFTMAX, kint.CALIB_FWM_RESOLVED
 LE, NE = kint.RECON_LERP, kint.RECON_NEAREST
 WE, PR = kint.STE_WEIGHT, kint.STE_PROB
 FU, DE = kint.GRAD_FULL, kint.GRAD_DETACH
@@ -86,6 +86,22 @@ def test_zero_sum_projection_lengths(T):
     Q, K, V, dO = make_qkvdo(1, 1, T, 64, seed=14)
     for cfg in (_cfg(MM, NE, WE, PJ), _cfg(FW, NE, PR, PJ)):
         parity.check(Q, K, V, dO, cfg, X3)
+
+
+@pytest.mark.parametrize("r,s,g", [(r, s, g) for r in (LE, NE) for s in (WE, PR) for g in (FU, DE)] + [(NE, PR, PJ)])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_resolved_tail_policy(r, s, g, prec):
+    """FWM's grid continued below -tau (App. "Tail policy"): tau = 3 at these score scales puts
+    most keys below the window, on negative grid indices; T = 300 is ragged."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=16)
+    parity.check(Q, K, V, dO, _cfg(FR, r, s, g, 4, tau=3.0), prec)
+
+
+@pytest.mark.parametrize("Kint,tau", [(1, 1.0), (16, 8.0), (64, 4.0)])
+def test_resolved_tail_policy_grids(Kint, tau):
+    """Coarse and fine steps: K = 1 with a 1-nat window, K = 64 (h = 1/16) far below the window."""
+    Q, K, V, dO = make_qkvdo(1, 2, 200, 64, seed=17)
+    parity.check(Q, K, V, dO, _cfg(FR, NE, PR, FU, Kint, tau=tau), X3 if Kint <= 32 else TF)
 
 
 @pytest.mark.parametrize("prec", [X3, TF])
