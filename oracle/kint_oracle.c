@@ -24,6 +24,8 @@
  *                                                 -> max_only / min_only modes
  *                                                  (g_self + g_M, g_self + g_m)
  *   App. B "Softmax", App. A "Softmax"            -> the comparator
+ *   App. "Reduced-precision exponential baselines" -> FP8-rounded exponential
+ *                                                  (E4M3 forward, fp32-exp backward)
  *   Table "Edge cases" (App. A)                   -> degenerate rows, ties,
  *                                                  midpoint rounding, window edge
  *
@@ -111,6 +113,31 @@ static int resolved_code(int idx) {
   return c < 0 ? 0 : (c > 252 ? 252 : c);
 }
 
+/* OCP E4M3 ("fn": bias 7, 3 mantissa bits, no infinities).  Codes 0..0x3F in
+ * increasing order cover [0, 1.875]: code = (exponent field << 3) | mantissa,
+ * subnormals (exponent field 0) m * 2^-9, normals (1 + m/8) 2^(e - 7). */
+static double e4m3_value(int code) {
+  const int e = code >> 3, m = code & 7;
+  return e == 0 ? ldexp((double)m, -9) : ldexp(1.0 + m / 8.0, e - 7);
+}
+
+/* Round 0 <= w <= 1 to the nearest E4M3 value, ties to the even code (even
+ * mantissa), by scanning every code.  Returns the code; *mg receives the
+ * distance, in z = ln w units, from w to the nearer edge of its rounding cell. */
+static int e4m3_round(double w, double* mg) {
+  int best = 0;
+  for (int c = 1; c <= 0x3F; ++c) {
+    const double dc = fabs(w - e4m3_value(c)), db = fabs(w - e4m3_value(best));
+    if (dc < db || (dc == db && (c & 1) == 0)) best = c;
+  }
+  const double lo = best > 0 ? 0.5 * (e4m3_value(best - 1) + e4m3_value(best)) : 0.0;
+  const double hi = 0.5 * (e4m3_value(best) + e4m3_value(best + 1));
+  const double lz = log(w);
+  const double dlo = lo > 0.0 ? lz - log(lo) : INFINITY, dhi = log(hi) - lz;
+  *mg = dlo < dhi ? dlo : dhi;
+  return best;
+}
+
 /*
  * Forward quantities of causal row i of head bh (App. A).  Fills R.
  */
@@ -166,6 +193,20 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
     for (int j = 0; j < n; ++j) {
       R->wL[j] = exp(R->z[j]);
       R->wN[j] = R->wL[j];
+    }
+  } else if (p->calib == KOR_EXP_FP8) {
+    /* w^exp_j = e^{z_j}, rounded to E4M3 and returned to full precision: the
+     * forward weight (App. "Reduced-precision exponential baselines").  The
+     * exponential itself is kept for the backward. */
+    for (int j = 0; j < n; ++j) {
+      const double we = exp(R->z[j]);
+      double mg;
+      int code = e4m3_round(we, &mg);
+      if (J->ov && J->ov->bins) code = J->ov->bins[((size_t)bh * T + i) * T + j]; /* decision-aligned re-run */
+      R->er0[j] = we;
+      R->wL[j] = R->wN[j] = e4m3_value(code);
+      R->code_l[j] = R->code_r[j] = code;
+      R->margin[j] = mg;
     }
   } else if (p->calib == KOR_MINMAX && (R->M - R->m) <= DEGENERATE_EPS) {
     /* Degenerate MinMax row: weights 1, P uniform (Table "Edge cases"). */
@@ -341,6 +382,26 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
     double D = 0.0;
     for (int j = 0; j < n; ++j) D += R->P[j] * R->g[j];
     for (int j = 0; j < n; ++j) R->dS[j] = R->P[j] * (R->g[j] - D);
+  } else if (p->calib == KOR_EXP_FP8) {
+    /* Normalization Jacobian at the rounded weights, gamma_j = (g_j - <g>_P) / W;
+     * the rounding passes the gradient unchanged and dw_j/dz_j = e^{z_j}.  With
+     * z = s - M the row max collects -sum_j dL/dz_j (split among ties); it has no
+     * minimum channel. */
+    double D = 0.0;
+    for (int j = 0; j < n; ++j) D += R->P[j] * R->g[j];
+    double own = 0.0;
+    for (int j = 0; j < n; ++j) {
+      R->dS[j] = (R->g[j] - D) / R->W_N * R->er0[j];
+      own += R->dS[j];
+    }
+    if (p->grad == KOR_DETACH_PROJ) {
+      for (int j = 0; j < n; ++j) R->dS[j] -= own / n;
+    } else if (p->grad != KOR_DETACH) {
+      cM = -own;
+      if (p->grad == KOR_FULL || p->grad == KOR_MAX_ONLY)
+        for (int j = 0; j < n; ++j)
+          if (R->s[j] == R->M) R->dS[j] += cM / R->nmax;
+    }
   } else if (R->degenerate) {
     /* Degenerate MinMax row: zero gradient (Table "Edge cases"). */
     for (int j = 0; j < n; ++j) R->dS[j] = 0.0;
@@ -491,8 +552,8 @@ static void* worker(void* arg) {
 
 static int check_params(const kor_params* p) {
   if (!p || p->B < 1 || p->H < 1 || p->T < 1 || p->d < 1) return -1;
-  if (p->calib < 0 || p->calib > 3) return -1;
-  if (p->calib != KOR_SOFTMAX && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
+  if (p->calib < 0 || p->calib > 4) return -1;
+  if (p->calib != KOR_SOFTMAX && p->calib != KOR_EXP_FP8 && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
   if ((p->calib == KOR_FWM || p->calib == KOR_FWM_RESOLVED) && !(p->tau > 0.0)) return -1;
   if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 4) return -1;
   return 0;

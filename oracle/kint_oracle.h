@@ -27,7 +27,11 @@ typedef float kor_in;
 /* Calibrations: MinMax, FWM, the softmax comparator, and FWM's "resolved" tail policy
  * (App. "Tail policy in the MinMax -> FWM change"): FWM's step tau/K and origin -tau,
  * with the grid continued below -tau (negative indices) instead of a zero tail. */
-enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2, KOR_FWM_RESOLVED = 3 };
+/* KOR_EXP_FP8 is the FP8-rounded exponential baseline (App. "Reduced-precision
+ * exponential baselines"): w = E4M3(e^{z}) forward, the fp32 exponential's derivative
+ * backward (identity surrogate on the rounding), the row max on the gradient path;
+ * K, tau, the reconstruction and the STE placement do not apply to it. */
+enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2, KOR_FWM_RESOLVED = 3, KOR_EXP_FP8 = 4 };
 enum { KOR_LERP = 0, KOR_NEAREST = 1 };
 enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
 /* Backward modes: the full calibration gradient (Eq. full), detached extrema (App. B
@@ -42,13 +46,14 @@ enum { KOR_FULL = 0, KOR_DETACH = 1, KOR_MAX_ONLY = 2, KOR_MIN_ONLY = 3, KOR_DET
  * ivals: interval index r in 0..K-1).  Under the resolved policy the indices run
  * below zero and are stored as index + KOR_CODE_OFFSET, saturated to [0, 252]
  * (code 0 stands for every index <= -128; such keys carry weights below
- * e^{-tau - 128 tau/K}). */
+ * e^{-tau - 128 tau/K}).  Under KOR_EXP_FP8 both arrays hold the E4M3 byte of
+ * the rounded weight (0x00 = 0 .. 0x38 = 1). */
 enum { KOR_CODE_NOGRID = 253, KOR_CODE_TAIL = 254, KOR_CODE_MASKED = 255, KOR_CODE_OFFSET = 128 };
 
 typedef struct {
   int B, H, T, d;
   int Kint;   /* K, number of intervals */
-  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX / KOR_FWM_RESOLVED */
+  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX / KOR_FWM_RESOLVED / KOR_EXP_FP8 */
   double tau; /* FWM window in nats (also the resolved grid's origin) */
   int recon;  /* KOR_LERP / KOR_NEAREST */
   int ste;    /* KOR_WEIGHT / KOR_PROB (ignored for LERP) */

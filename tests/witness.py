@@ -15,7 +15,7 @@ import math
 import numpy as np
 import torch
 
-MINMAX, FWM, SOFTMAX, FWM_RESOLVED = 0, 1, 2, 3
+MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8 = 0, 1, 2, 3, 4
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
 FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4
@@ -34,6 +34,13 @@ def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
     if cfg.grad in (DETACH, DETACH_PROJ, MAX_ONLY):
         m = m.detach()
     z = S - M
+    if cfg.calib == EXP_FP8:
+        # E4M3-rounded exponential forward (torch's float8 cast), the exponential's own
+        # derivative backward: w = fp8(e^z) + (e^z - sg(e^z))
+        we = torch.exp(z.masked_fill(~valid, -math.inf))
+        w = we.detach().to(torch.float8_e4m3fn).to(S.dtype) + (we - we.detach())
+        w = torch.where(valid, w, torch.zeros_like(w))
+        return w / w.sum(-1, keepdim=True)
     if cfg.calib == MINMAX:
         span = M - m
         degenerate = span <= 1e-12
