@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "380726be8a630b41", "k_prep": 82461568, "k_fwd_stats": 50369024, "k_fwd_main": 93682688,
-           "k_bwd_dq": 193184768, "k_bwd_dkdv": 274102528}
+TRAFFIC = {"src": "caee8376817f7757", "k_prep": 82507264, "k_fwd_stats": 50368256, "k_fwd_main": 92466688,
+           "k_bwd_dq": 181998336, "k_bwd_dkdv": 258794240}
 
 
 def kernel_source_digest() -> str:
@@ -364,6 +364,10 @@ def run_cuda(args, world, rank, local):
     ms_soft = timed(n_cmp, lambda i: step(i, soft, prec))
     line["softmax_comparator"] = {"value": job_value(flops_step, world, ms_soft), "unit": UNIT,
                                   "ms_per_step": ms_soft}
+    # the FP8-rounded exponential baseline (E4M3(e^z) forward, e^z backward) on the same inputs
+    e8 = kint.Config(Kint=4, calib=kint.CALIB_EXP_FP8, tau=8.0, recon=kint.RECON_LERP, ste=0, grad=0)
+    ms_e8 = timed(n_cmp, lambda i: step(i, e8, prec))
+    line["exp_fp8_baseline"] = {"value": job_value(flops_step, world, ms_e8), "unit": UNIT, "ms_per_step": ms_e8}
     ws_f3 = kint.workspace(B, H, T, d, kint.PREC_3XTF32, 0, dev)
     ws_b3 = kint.workspace(B, H, T, d, kint.PREC_3XTF32, 1, dev)
 
@@ -422,21 +426,23 @@ def run_cuda(args, world, rank, local):
     e2e_run(2)
     n_e2e = max(3, min(args.steps, 100))
     ms_e2e = timed(1, lambda i: e2e_run(n_e2e)) / n_e2e
-    # the same copies with no compute: the host link's floor for one end-to-end step
-    def copies_only(i):
-        b = i % 2
+    # the same copies with no compute, each direction streaming back to back on its own
+    # stream: the host link's floor for the end-to-end steps
+    def copies_only(n):
         s_in.wait_stream(s_c)
         s_out.wait_stream(s_c)
-        with torch.cuda.stream(s_in):
-            for dst, src in zip(ins[b], pin_in):
-                dst.copy_(src, non_blocking=True)
-        with torch.cuda.stream(s_out):
-            for dst, src in zip(pin_out, outs[b]):
-                dst.copy_(src, non_blocking=True)
+        for i in range(n):
+            with torch.cuda.stream(s_in):
+                for dst, src in zip(ins[i % 2], pin_in):
+                    dst.copy_(src, non_blocking=True)
+            with torch.cuda.stream(s_out):
+                for dst, src in zip(pin_out, outs[i % 2]):
+                    dst.copy_(src, non_blocking=True)
         s_c.wait_stream(s_in)
         s_c.wait_stream(s_out)
 
-    ms_link = timed(n_e2e, copies_only)
+    copies_only(2)
+    ms_link = timed(1, lambda i: copies_only(n_e2e)) / n_e2e
     line["e2e"] = {"value": job_value(flops_step, world, ms_e2e), "unit": UNIT,
                    "h2d_bytes_per_step": sum(t.numel() * 4 for t in pin_in),
                    "d2h_bytes_per_step": sum(t.numel() * 4 for t in pin_out), "ms_per_step": ms_e2e,

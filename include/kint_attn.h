@@ -61,8 +61,16 @@ typedef enum {
   KINT_CALIB_MINMAX = 0,
   KINT_CALIB_FWM = 1,
   KINT_CALIB_SOFTMAX = 2,
-  KINT_CALIB_FWM_RESOLVED = 3
+  KINT_CALIB_FWM_RESOLVED = 3,
+  KINT_CALIB_EXP_FP8 = 4
 } kint_calib;
+/* KINT_CALIB_EXP_FP8 is the FP8-rounded exponential baseline of App. "Reduced-precision
+ * exponential baselines": w = E4M3(e^{s - M}) (round to nearest even) in the forward, the
+ * exponential's own derivative e^{s - M} in the backward (identity surrogate on the
+ * rounding, normalization Jacobian at the rounded weights), the row max M on the gradient
+ * path as the maximum channel (full / max_only keep it; detach, min_only drop it).  Kint,
+ * tau, recon and ste are not used (they must still be valid values); the exponential is
+ * ex2.approx, as for the softmax comparator. */
 /* Reconstruction (Sec. 3 "Reconstruction"; App. A "LERP", "Nearest"). */
 typedef enum { KINT_RECON_LERP = 0, KINT_RECON_NEAREST = 1 } kint_recon;
 /* Surrogate placement (Sec. 3 Eqs. wste / pste).  Ignored under LERP, where the
@@ -160,7 +168,8 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
  * (ivals), with 254 for FWM tail keys (z < -tau), 255 for masked keys (j > i)
  * and 253 where no grid exists (degenerate MinMax rows, softmax); under
  * FWM_RESOLVED both indices run below zero and are stored as index + 128,
- * saturated to [0, 252] (0: index <= -128).  Either
+ * saturated to [0, 252] (0: index <= -128); under EXP_FP8 both hold the E4M3
+ * byte of the rounded weight (0x00 = 0 .. 0x38 = 1).  Either
  * output may be NULL.  Needs the row statistics of kint_attn_fwd on the same
  * inputs and the forward's workspace size.  bins, ivals: [B,H,T,T] uint8.
  */

@@ -39,6 +39,9 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
     if constexpr (CAL == CAL_SOFTMAX) {
       const float pr = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * invWf;
       ds = pr * __fmaf_rn(gv[jj], ga, gb);  // P (g - <g>_P)
+    } else if constexpr (CAL == CAL_EXP8) {
+      // gamma e^{z}: the exponential's derivative through the rounding's identity surrogate
+      ds = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * __fmaf_rn(gv[jj], ga, gb);
     } else if constexpr (fwm_like(CAL)) {
       // k1, c0 doubled (v = 2u), Kf = 2K, tab: the half-bin table of Delta_r / h (4-byte entries)
       const float v = __fmaf_rn(sv[jj], k1, c0);
@@ -363,7 +366,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         r.amax = p.arg_max[rw];
         r.amin = p.arg_min[rw];
         r.Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
-        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && CAL != CAL_SOFTMAX);
+        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && !exp_like(CAL));
         r.Ws = prob ? p.W_lerp[rw] : r.Wf;
       }
       return r;
@@ -592,8 +595,8 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
           // the position as the dK/dV pass forms it: softmax log2 e^{s-M}, FWM Nearest 2u, else u
           const bool half = fwm_like(CAL) && p.recon == REC_NEAREST;
           RowRec r;
-          r.c0 = CAL == CAL_SOFTMAX ? sc0 : (half ? 2.0f * g.c0 : g.c0);
-          r.k1 = CAL == CAL_SOFTMAX ? sk1 : (half ? 2.0f * g.k1 : g.k1);
+          r.c0 = exp_like(CAL) ? sc0 : (half ? 2.0f * g.c0 : g.c0);
+          r.k1 = exp_like(CAL) ? sk1 : (half ? 2.0f * g.k1 : g.k1);
           r.invWf = invWf;
           r.ga = ga;
           r.gb = gb;
@@ -647,6 +650,11 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
     if constexpr (CAL == CAL_SOFTMAX) {
       pv = ex2_approx(__fmaf_rn(sv[ii], r0.y, r0.x)) * r0.z;
       ds = pv * gam;
+    } else if constexpr (CAL == CAL_EXP8) {
+      // forward P from the E4M3-rounded weight; dS from the exponential itself
+      const float we = ex2_approx(__fmaf_rn(sv[ii], r0.y, r0.x));
+      pv = e4m3_rn(we) * r0.z;
+      ds = gam * we;
     } else if constexpr (fwm_like(CAL) && REC == REC_NEAREST) {
       // record holds 2k1, 2c0; Kf = 2K; fwtab: the half-bin table of (w^N, Delta_r / h)
       const float v = __fmaf_rn(sv[ii], r0.y, r0.x);
@@ -1168,6 +1176,9 @@ cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cud
   const dim3 grid((unsigned)p.ngrid);
   const bool full = p.grad != GRAD_DETACH && p.grad != GRAD_DETACH_PROJ;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dq<CAL_SOFTMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
+  if (p.calib == CAL_EXP8)
+    return full ? launch3(k_bwd_dq<CAL_EXP8, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
+                : launch3(k_bwd_dq<CAL_EXP8, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
   if (p.calib == CAL_MINMAX)
     return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
                 : launch3(k_bwd_dq<CAL_MINMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
@@ -1183,6 +1194,10 @@ cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, c
   const bool proj = p.grad == GRAD_DETACH_PROJ, full = p.grad != GRAD_DETACH && !proj;
   const bool near = p.recon == REC_NEAREST;
   if (p.calib == CAL_SOFTMAX) return launch3(k_bwd_dkdv<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+  if (p.calib == CAL_EXP8)
+    return full ? launch3(k_bwd_dkdv<CAL_EXP8, REC_LERP, true>, grid, maps, p, smem_bytes, s)
+           : proj ? launch3(k_bwd_dkdv<CAL_EXP8, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
+                  : launch3(k_bwd_dkdv<CAL_EXP8, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
     if (near)
       return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)

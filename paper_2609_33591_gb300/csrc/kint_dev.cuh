@@ -145,7 +145,7 @@ __device__ __forceinline__ RowGrid row_grid(const Params& p, float M, float m) {
     g.b0 = -p.tau;
     g.k1 = __fmul_rn(p.scale, g.inv_h);
   } else {
-    g.nogrid = true;
+    g.nogrid = p.calib != CAL_EXP8;  // (the FP8 exponential keeps the row max's gradient channel)
     g.h = 1.0f;
     g.inv_h = 1.0f;
     g.c0 = 0.0f;
@@ -224,6 +224,24 @@ __device__ __forceinline__ float ex2_approx(float x) {
 __device__ __forceinline__ float grid_value(const Params& p, const RowGrid& g, int r) {
   if (fwm_like(p.calib)) return p.fwm_e[r];
   return expf(__fmaf_rn((float)r, g.h, g.b0));
+}
+
+// FP8-rounded exponential (App. "Reduced-precision exponential baselines"): 0 <= w <= 1
+// to the nearest OCP E4M3 value, ties to even.  Normals (w >= 2^-6) keep 3 mantissa bits:
+// adding 2^19 - 1 plus the kept LSB to the bit pattern and clearing the 20 dropped bits
+// rounds to nearest even (a mantissa carry moves into the exponent).  Below 2^-6 the
+// format's subnormals are the multiples of 2^-9: rint(w 2^9) 2^-9.  Both are exact.
+__device__ __forceinline__ float e4m3_rn(float w) {
+  uint32_t u = __float_as_uint(w);
+  u = (u + 0x7FFFFu + ((u >> 20) & 1u)) & 0xFFF00000u;
+  const float wsub = __fmul_rn(rintf(__fmul_rn(w, 512.0f)), 0.001953125f);
+  return w < 0.015625f ? wsub : __uint_as_float(u);
+}
+// The E4M3 byte of an E4M3 value in [0, 1] (for the decision dump).
+__device__ __forceinline__ int e4m3_code(float wr) {
+  if (wr < 0.015625f) return (int)__fmul_rn(wr, 512.0f);
+  const uint32_t u = __float_as_uint(wr);
+  return ((int)((u >> 23) & 0xFFu) - 127 + 7) << 3 | (int)((u >> 20) & 7u);
 }
 
 // Resolved tail policy (App. "Tail policy in the MinMax -> FWM change"): below the

@@ -406,6 +406,8 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
     float wm, wl = 0.f;
     if constexpr (CAL == CAL_SOFTMAX) {
       wm = ex2_approx(__fmaf_rn(v[jj], sk1, sc0));  // e^{s - M} (App. A, Softmax)
+    } else if constexpr (CAL == CAL_EXP8) {
+      wm = e4m3_rn(ex2_approx(__fmaf_rn(v[jj], sk1, sc0)));  // E4M3(e^{s - M})
     } else {
       const float u = __fmaf_rn(v[jj], g.k1, g.c0);
       float t, rf;
@@ -451,14 +453,17 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
 // inlined into the main loop: the calibration is a template parameter so that each
 // instantiation carries only its own branch).
 template <int CAL>
-__device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, int i, int bh, const RowGrid& g) {
+__device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, int i, int bh, const RowGrid& g,
+                                float sk1, float sc0) {
   if (i >= p.T) return;
   for (int jj = 0; jj < 32; ++jj) {
     const int j = j0 + jj;
     if (j >= p.T) break;
     uint8_t cb = 255, ci = 255;
     if (j <= i) {
-      if (CAL == CAL_SOFTMAX || g.nogrid) {
+      if constexpr (CAL == CAL_EXP8) {
+        cb = ci = (uint8_t)e4m3_code(e4m3_rn(ex2_approx(__fmaf_rn(v[jj], sk1, sc0))));
+      } else if (CAL == CAL_SOFTMAX || g.nogrid) {
         cb = ci = 253;
       } else {
         const float u = __fmaf_rn(v[jj], g.k1, g.c0);
@@ -713,7 +718,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
           tmem_ld32(lane_addr(tmem, b * 128 + c * 32), v);
           tmem_ld_wait();
           const int j0 = kb * 128 + c * 32;
-          if (p.debug) fwd_debug_codes<CAL>(p, v, j0, i, bh, gr);
+          if (p.debug) fwd_debug_codes<CAL>(p, v, j0, i, bh, gr, sk1, sc0);
           if (diag)
             fwd_chunk<CAL, REC, MODE, true>(v, a1, a2, j0, i, gr, Kf, tab, sk1, sc0, Wm, Wl);
           else
@@ -813,6 +818,7 @@ static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_byt
 cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
   const int mode = p.pv_sel;
   if (p.calib == CAL_SOFTMAX) return launch_main_t<CAL_SOFTMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
+  if (p.calib == CAL_EXP8) return launch_main_t<CAL_EXP8, REC_LERP, 0>(maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
     if (p.recon == REC_LERP) return launch_main_t<CAL_MINMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
     if (mode == PV_MAIN) return launch_main_t<CAL_MINMAX, REC_NEAREST, 0>(maps, p, smem_bytes, s);

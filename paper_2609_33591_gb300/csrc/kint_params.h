@@ -6,10 +6,13 @@
 
 namespace kint {
 
-enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2, CAL_FWMR = 3 };
+enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2, CAL_FWMR = 3, CAL_EXP8 = 4 };
 // FWM's grid (step tau/K, origin -tau), with a zero tail below the window (FWM) or
 // continued below it with negative indices (CAL_FWMR, the "resolved" tail policy)
 __host__ __device__ constexpr bool fwm_like(int cal) { return cal == CAL_FWM || cal == CAL_FWMR; }
+// weights from the exponential unit instead of a grid: the softmax comparator, and
+// CAL_EXP8, the FP8-rounded exponential baseline (E4M3(e^z) forward, e^z backward)
+__host__ __device__ constexpr bool exp_like(int cal) { return cal == CAL_SOFTMAX || cal == CAL_EXP8; }
 enum Recon : int { REC_LERP = 0, REC_NEAREST = 1 };
 enum Grad : int { GRAD_FULL = 0, GRAD_DETACH = 1, GRAD_MAX_ONLY = 2, GRAD_MIN_ONLY = 3, GRAD_DETACH_PROJ = 4 };
 

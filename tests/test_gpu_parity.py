@@ -11,6 +11,7 @@ from tests import parity
 pytestmark = pytest.mark.gpu
 
 MM, FW, SM, FR = kint.CALIB_MINMAX, kint.CALIB_FWM, kint.CALIB_SOFTMAX, kint.CALIB_FWM_RESOLVED
+E8 = kint.CALIB_EXP_FP8
 LE, NE = kint.RECON_LERP, kint.RECON_NEAREST
 WE, PR = kint.STE_WEIGHT, kint.STE_PROB
 FU, DE = kint.GRAD_FULL, kint.GRAD_DETACH
@@ -102,6 +103,27 @@ def test_resolved_tail_policy_grids(Kint, tau):
     """Coarse and fine steps: K = 1 with a 1-nat window, K = 64 (h = 1/16) far below the window."""
     Q, K, V, dO = make_qkvdo(1, 2, 200, 64, seed=17)
     parity.check(Q, K, V, dO, _cfg(FR, NE, PR, FU, Kint, tau=tau), X3 if Kint <= 32 else TF)
+
+
+@pytest.mark.parametrize("g", [FU, DE, PJ])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_fp8_exponential_baseline(g, prec):
+    """E4M3(e^z) forward, e^z backward, row max on the gradient path; the E4M3 byte of every weight
+    is a decision (compared exactly outside the guard band).  T = 300 is ragged."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=18)
+    rep = parity.check(Q, K, V, dO, _cfg(E8, LE, WE, g), prec)
+    if prec == X3:  # fp32-accurate scores: a rounding decision flips only within a few ulps
+        assert rep["bins_flips"] <= 0.001 * 300 * 301
+
+
+def test_fp8_exponential_value_set():
+    """Scores spread so that every E4M3 level below 1 and the underflow to zero occur: the GPU's
+    codes take exactly the format's 56 nonzero values and 0."""
+    Q, K, V, dO = make_qkvdo(1, 4, 256, 64, seed=19)
+    g = parity.run_gpu(Q * 1.5, K, V, dO, _cfg(E8, LE, WE, FU), X3, want_bwd=False)
+    codes = g["bins"][g["bins"] != 255]
+    assert codes.max() == 0x38 and codes.min() == 0
+    assert len(set(codes[codes > 0].tolist())) == 56
 
 
 @pytest.mark.parametrize("prec", [X3, TF])
