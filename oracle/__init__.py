@@ -60,7 +60,7 @@ _P = ctypes.c_void_p
 
 class _FwdOut(ctypes.Structure):
     _fields_ = [(n, _P) for n in ("O", "M", "m", "amax", "amin", "nmax", "nmin", "W", "WL", "OL",
-                                  "bins", "ivals", "margin", "row_margin")]
+                                  "bins", "ivals", "margin", "row_margin", "probe")]
 
 
 class _BwdOut(ctypes.Structure):
@@ -130,8 +130,11 @@ def _override(ov):
     return o, keep
 
 
+PROBE_NAMES = ("span", "h", "entropy", "frac_below6", "top_mass", "eff_buckets", "tv")
+
+
 def forward(Q, K, V, cfg: Config, *, decisions: bool = False, lerp_out: bool = False, override=None,
-            nthreads: int = 0, f64: bool = False) -> dict:
+            nthreads: int = 0, f64: bool = False, probes: bool = False) -> dict:
     """Forward of K-interval attention in fp64.  Q, K, V: [B, H, T, d], taken
     as fp32 (or as fp64 with ``f64=True``).
 
@@ -149,6 +152,8 @@ def forward(Q, K, V, cfg: Config, *, decisions: bool = False, lerp_out: bool = F
     }
     if lerp_out:
         out["OL"] = np.zeros((B, H, T, d))
+    if probes:
+        out["probe"] = np.zeros((len(PROBE_NAMES), B, H, T))
     if decisions:
         out["bins"] = np.zeros((B, H, T, T), np.uint8)
         out["ivals"] = np.zeros((B, H, T, T), np.uint8)

@@ -26,6 +26,10 @@
  *   App. B "Softmax", App. A "Softmax"            -> the comparator
  *   App. "Reduced-precision exponential baselines" -> FP8-rounded exponential
  *                                                  (E4M3 forward, fp32-exp backward)
+ *   App. "Geometry probe"                         -> per-row probes: span, width,
+ *                                                  softmax entropy, mass below -6,
+ *                                                  top-bucket mass, effective buckets,
+ *                                                  total variation to softmax
  *   Table "Edge cases" (App. A)                   -> degenerate rows, ties,
  *                                                  midpoint rounding, window edge
  *
@@ -313,7 +317,7 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
 static void fwd_row_outputs(const job_t* J, int bh, int i, row_t* R) {
   const kor_params* p = J->p;
   const kor_fwd_out* fo = J->fo;
-  const int T = p->T, d = p->d, n = R->n;
+  const int T = p->T, d = p->d, n = R->n, K = p->Kint;
   const size_t row = (size_t)bh * T + i;
   const kor_in* Vh = J->V + (size_t)bh * T * d;
   const int hard = (p->calib != KOR_SOFTMAX && p->recon == KOR_NEAREST);
@@ -345,6 +349,45 @@ static void fwd_row_outputs(const job_t* J, int bh, int i, row_t* R) {
       if (fo->ivals) fo->ivals[idx] = (uint8_t)(valid ? R->code_r[j] : KOR_CODE_MASKED);
       if (fo->margin) fo->margin[idx] = valid ? R->margin[j] : INFINITY;
     }
+  }
+  if (fo->probe) {
+    /* Geometry probe (App. "Geometry probe"), on the operator's own fp64 scores:
+     * P^E = softmax(s); buckets are the operator's levels (Nearest: l in 0..K;
+     * LERP: interval r in 0..K-1), with FWM's tail keys as one more bucket and a
+     * degenerate MinMax row as a single bucket; the top bucket is l = K (Nearest)
+     * or r = K-1 (LERP). */
+    const size_t plane = (size_t)p->B * p->H * T;
+    double Z = 0.0;
+    for (int j = 0; j < n; ++j) Z += exp(R->z[j]);
+    double H = 0.0, below = 0.0, top = 0.0, tv = 0.0;
+    double* mass = (double*)calloc((size_t)K + 3, sizeof(double));
+    const int nearest = (p->recon == KOR_NEAREST);
+    for (int j = 0; j < n; ++j) {
+      const double pe = exp(R->z[j]) / Z;
+      if (pe > 0.0) H -= pe * log(pe);
+      if (R->z[j] < -6.0) below += 1.0;
+      tv += fabs(R->P[j] - pe);
+      int bkt, is_top;
+      if (R->degenerate) {
+        bkt = 0;
+        is_top = 1;
+      } else if (R->tail[j]) {
+        bkt = K + 1;
+        is_top = 0;
+      } else {
+        bkt = nearest ? R->l[j] : R->r[j];
+        is_top = nearest ? (R->l[j] == K) : (R->r[j] == K - 1);
+      }
+      if (mass) mass[bkt] += pe;
+      if (is_top) top += pe;
+    }
+    double Hq = 0.0;
+    for (int b = 0; b <= K + 1 && mass; ++b)
+      if (mass[b] > 0.0) Hq -= mass[b] * log(mass[b]);
+    free(mass);
+    const double vals[KOR_PROBES] = {R->degenerate ? 0.0 : R->M - R->m, R->degenerate ? 0.0 : R->h, H, below / n,
+                                     top, exp(Hq), 0.5 * tv};
+    for (int k = 0; k < KOR_PROBES; ++k) fo->probe[k * plane + row] = vals[k];
   }
   if (fo->row_margin) {
     /* Gap between the extremum and the runner-up (a different score value),
@@ -564,6 +607,8 @@ static int run(const kor_params* p, const kor_in* Q, const kor_in* K, const kor_
   if (check_params(p) != 0) return -1;
   /* the uint8 decision codes hold l in 0..K and need K + 1 < KOR_CODE_NOGRID */
   if (fo && (fo->bins || fo->ivals) && p->Kint >= KOR_CODE_NOGRID - 1) return -1;
+  /* the probes are defined for the grid calibrations MinMax and FWM */
+  if (fo && fo->probe && p->calib != KOR_MINMAX && p->calib != KOR_FWM) return -1;
   /* resolved: codes l + KOR_CODE_OFFSET <= 252 */
   if (p->calib == KOR_FWM_RESOLVED && ((fo && (fo->bins || fo->ivals)) || (ov && ov->bins)) &&
       p->Kint > 252 - KOR_CODE_OFFSET)

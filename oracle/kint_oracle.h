@@ -76,7 +76,12 @@ typedef struct {
   uint8_t* ivals;     /* [B,H,T,T] interval index r / codes */
   double* margin;     /* [B,H,T,T] distance (score units) to the nearest decision boundary */
   double* row_margin; /* [B,H,T] gap between an extremum and its runner-up */
+  double* probe;      /* [7][B,H,T] geometry probe of each row (MinMax / FWM only), in order:
+                         span M - m; native width h; softmax entropy H(P^E); fraction of keys
+                         with z < -6; top-bucket mass; effective buckets exp H(q); TV(P, P^E) */
 } kor_fwd_out;
+
+enum { KOR_PROBES = 7 };
 
 typedef struct {
   double* dQ;   /* [B,H,T,d] */

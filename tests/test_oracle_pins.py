@@ -735,3 +735,78 @@ def test_fp8_rows_sum_to_one_and_decision_override():
     g = oracle.forward(Q, K, V, cfg, override={**ov, "bins": bins})
     changed = np.argwhere(np.any(g["O"] != f["O"], axis=-1))
     assert changed.tolist() == [[1, 0, i]]
+
+
+# --- Geometry probe (App. "Geometry probe") --------------------------------------------------------
+
+def _probe(out, name):
+    return out["probe"][oracle.PROBE_NAMES.index(name)]
+
+
+@pytest.mark.parametrize("calib,recon", [(MINMAX, LERP), (MINMAX, NEAREST), (FWM, NEAREST), (FWM, LERP)])
+def test_probe_entropy_tv_span_against_library_routines(calib, recon):
+    """Softmax entropy and softmax itself from scipy; the operator's own P from its output with V = I;
+    span, width and the share of keys below z = -6 from the scores."""
+    scipy_special = pytest.importorskip("scipy.special")
+    scipy_stats = pytest.importorskip("scipy.stats")
+    T, d, Kint, tau = 16, 16, 4, 3.0
+    Q, K, _, _ = rand_inputs(2, 2, T, d, 47, scale=3.0)
+    cfg = Config(Kint=Kint, calib=calib, tau=tau, recon=recon)
+    out = oracle.forward(Q, K, eye_values(T, d)[None, None].repeat(2, 0).repeat(2, 1), cfg, probes=True)
+    S = scores_np(Q, K)
+    for b in range(2):
+        for h in range(2):
+            for i in range(T):
+                s = S[b, h, i, : i + 1]
+                pe = scipy_special.softmax(s)
+                P = out["O"][b, h, i, : i + 1]
+                assert abs(_probe(out, "entropy")[b, h, i] - scipy_stats.entropy(pe)) < 1e-12
+                assert abs(_probe(out, "tv")[b, h, i] - 0.5 * np.abs(P - pe).sum()) < 1e-12
+                span = s.max() - s.min()
+                assert abs(_probe(out, "span")[b, h, i] - span) < 1e-12
+                assert abs(_probe(out, "h")[b, h, i] - (span / Kint if calib == MINMAX else tau / Kint)) < 1e-12
+                assert _probe(out, "frac_below6")[b, h, i] == np.mean(s - s.max() < -6.0)
+
+
+@pytest.mark.parametrize("calib,recon", [(MINMAX, NEAREST), (MINMAX, LERP), (FWM, NEAREST), (FWM, LERP)])
+def test_probe_buckets_brute_force_on_lattice(calib, recon):
+    """Top-bucket mass and effective buckets exp H(q) from a brute-force bucket assignment (the
+    lattice scan of the bins pin) and numpy softmax masses."""
+    rng = np.random.default_rng(48)
+    Kint, T, tau = 4, 16, 2.0
+    for trial in range(30):
+        ks = rng.integers(0, 25, size=T)
+        ks[rng.integers(0, T)] = 0
+        if calib == MINMAX:
+            ks[rng.integers(0, T)] = 16
+        targets = 1.0 - 0.125 * ks
+        Q, K = lattice_qk(targets)
+        out = oracle.forward(Q, K, eye_values(T, 16), Config(Kint=Kint, calib=calib, tau=tau, recon=recon),
+                             probes=True)
+        z = targets - targets.max()
+        if calib == MINMAX:
+            b = [z.min() + r * (0 - z.min()) / Kint for r in range(Kint + 1)]
+            tail = np.zeros(T, bool)
+        else:
+            b = [-tau + r * tau / Kint for r in range(Kint + 1)]
+            tail = z < -tau
+        ell, r_idx, _, _ = brute_force_row(z, b, tail)
+        pe = np.exp(z) / np.exp(z).sum()
+        bucket = np.where(tail, Kint + 1, ell if recon == NEAREST else r_idx)
+        top = (~tail) & ((ell == Kint) if recon == NEAREST else (r_idx == Kint - 1))
+        q = np.array([pe[bucket == k].sum() for k in range(Kint + 2)])
+        q = q[q > 0]
+        assert abs(_probe(out, "top_mass")[0, 0, T - 1] - pe[top].sum()) < 1e-12, trial
+        assert abs(_probe(out, "eff_buckets")[0, 0, T - 1] - np.exp(-(q * np.log(q)).sum())) < 1e-12, trial
+
+
+def test_probe_degenerate_and_single_key_rows():
+    """Row 0 (one key) and all-equal MinMax rows: one bucket holding all the mass, no span."""
+    T = 12
+    Q = np.zeros((1, 1, T, 8), np.float32)
+    K = rand_inputs(1, 1, T, 8, 49)[1]
+    out = oracle.forward(Q, K, eye_values(T, 8)[:, :8] if T <= 8 else np.zeros((1, 1, T, 8), np.float32),
+                         Config(Kint=4, calib=MINMAX, recon=NEAREST), probes=True)
+    for n, v in (("span", 0.0), ("h", 0.0), ("top_mass", 1.0), ("eff_buckets", 1.0), ("tv", 0.0), ("frac_below6", 0.0)):
+        assert np.allclose(_probe(out, n)[0, 0], v, atol=1e-12), n
+    assert np.allclose(_probe(out, "entropy")[0, 0], np.log(np.arange(1, T + 1)), atol=1e-12)
