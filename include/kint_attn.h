@@ -163,6 +163,26 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
                   kint_prec prec, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * Geometry probe (App. "Geometry probe"), MinMax and FWM only: pass 1 on Q, K (into st,
+ * as kint_attn_fwd writes it), then per causal row i of every head, from the fp32 scores
+ * the operator uses, into probe[k * B*H*T + (b*H + h)*T + i] for k =
+ *   0  span M - m (0 for a degenerate MinMax row)
+ *   1  native width h: (M - m)/K (MinMax), tau/K (FWM); 0 for a degenerate row
+ *   2  softmax entropy H(P^E), P^E = softmax of the row's scores
+ *   3  share of the row's i + 1 keys with z = s - M < -6
+ *   4  top-bucket mass: P^E mass on keys in the top level (Nearest, l = K) or the top
+ *      interval (LERP, r = K - 1); 1 for a degenerate row
+ *   5  effective buckets exp H(q), q_b the P^E mass of bucket b: the Nearest levels l or the
+ *      LERP intervals r, FWM tail keys as one more bucket, a degenerate row as one bucket
+ *   6  total variation 1/2 sum_j |P_j - P^E_j| to the operator's forward P
+ * probe: device, [7][B,H,T] fp32, 16-byte aligned, caller-owned.  The workspace is the
+ * forward's (kint_attn_workspace_bytes(..., 0)).  Diagnostic: not on the training path.
+ */
+int kint_attn_probe(const float* Q, const float* K, const kint_rowstats* st, float* probe, int B, int H, int T,
+                    int d, int Kint, kint_calib calib, float tau, kint_recon recon, int causal, kint_prec prec,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+/*
  * Decision dump for parity checks: for every (b, h, i, j) the Nearest index
  * l_ij = r + [t >= 1/2] in 0..K (bins) and the interval index r_ij in 0..K-1
  * (ivals), with 254 for FWM tail keys (z < -tau), 255 for masked keys (j > i)

@@ -1,6 +1,6 @@
 """Build libkint.so in-tree with nvcc for sm_103a (no torch extension machinery).
 
-The three translation units are compiled in parallel and linked against the
+The translation units are compiled in parallel and linked against the
 shared CUDA runtime (the one PyTorch also loads), with an rpath to the CUDA
 toolkit so the library also loads on its own.
 """
@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libkint.so")
-SOURCES = ["kint_api.cu", "kint_fwd.cu", "kint_bwd.cu"]
+SOURCES = ["kint_api.cu", "kint_fwd.cu", "kint_bwd.cu", "kint_probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

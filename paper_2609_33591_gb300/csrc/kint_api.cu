@@ -232,6 +232,22 @@ int plan_stats(Params& p) {
   return total;
 }
 
+// Geometry probe: pass 1's layout, 8 x 128 exchange words and a [2][128][K + 2] float
+// bucket-mass array per CTA; one CTA per SM.
+int plan_probe(Params& p) {
+  const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
+  p.nitems = p.nqb * p.BH;
+  p.sm_a = 0;
+  p.sm_stage0 = parts * tile;
+  p.sm_stage_bytes = parts * tile;
+  p.nstage = 2;
+  p.sm_rows = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+  p.sm_table = p.sm_rows + 8 * 128 * 4;
+  const int total = finish_plan(p, p.sm_table + 2 * 128 * (p.Kint + 2) * 4, 6 + 2 * p.nstage);
+  p.ngrid = std::min(p.nitems, num_sms());
+  return total;
+}
+
 // mode: PV_MAIN / PV_MAIN_LERP / PV_LERP.  Picks the TMEM score double-buffering
 // and the deepest K/V ring that fit.
 int plan_main(Params& p, int mode) {
@@ -597,6 +613,52 @@ int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const k
   pm.bins = bins;
   pm.ivals = ivals;
   return launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); }));
+}
+
+int kint_attn_probe(const float* Q, const float* K, const kint_rowstats* st, float* probe, int B, int H, int T,
+                    int d, int Kint, kint_calib calib, float tau, kint_recon recon, int causal, kint_prec prec,
+                    void* workspace, size_t workspace_bytes, void* stream) {
+  const Common c{B, H, T, d, Kint, (int)calib, (int)recon, 0, 0, (int)prec, tau};
+  int rc = validate(c, causal);
+  if (rc) return rc;
+  if (calib != KINT_CALIB_MINMAX && calib != KINT_CALIB_FWM) return KINT_ERR_UNSUPPORTED;
+  if (!Q || !K || !probe) return KINT_ERR_ARG;
+  if ((rc = check_stats(st, false))) return rc;
+  if (!aligned16(Q) || !aligned16(K) || !aligned16(probe)) return KINT_ERR_ALIGN;
+  const size_t need = kint_attn_workspace_bytes(B, H, T, d, prec, 0);
+  if (!workspace || workspace_bytes < need) return KINT_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return KINT_ERR_ALIGN;
+  unsigned* status = nullptr;
+  if ((rc = device_setup(&status))) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+  Params p = base_params(c, status);
+  set_stats(p, st);
+  p.Q = Q; p.K = K;
+  p.probe = probe;
+  const Workspace w = plan_workspace(static_cast<char*>(workspace), p.BH, T, d, p.x3 != 0, false);
+  Maps maps;
+  std::memset(&maps, 0, sizeof(maps));
+  bool ok = true;
+  if (p.x3) {
+    PrepList pl;
+    pl.add(Q, w.qh, w.ql, nullptr, nullptr);
+    pl.add(K, w.kh, w.kl, nullptr, nullptr);
+    if (prep(pl, p.BH, T, round_up(T, 32), d, true, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+    ok = map_nat(&maps.q, w.qh, p.BH, T, d, 128) && map_nat(&maps.q_lo, w.ql, p.BH, T, d, 128) &&
+         map_nat(&maps.k, w.kh, p.BH, T, d, 128) && map_nat(&maps.k_lo, w.kl, p.BH, T, d, 128);
+  } else {
+    ok = map_nat(&maps.q, Q, p.BH, T, d, 128) && map_nat(&maps.k, K, p.BH, T, d, 128);
+  }
+  if (!ok) return KINT_ERR_LAUNCH;
+  // pass 1 (row extrema), then the probe's two sweeps
+  Params ps = p;
+  const int smem_s = plan_stats(ps);
+  if ((rc = launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem_s, s); })))) return rc;
+  Params pp = p;
+  const int smem_p = plan_probe(pp);
+  if (smem_p < 0 || smem_p > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  return launch_rc(traced("k_fwd_probe", s, [&] { return launch_fwd_probe(maps, pp, smem_p, s); }));
 }
 
 int kint_get_status(void* stream, unsigned* detail) {

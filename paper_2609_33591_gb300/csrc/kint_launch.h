@@ -43,6 +43,9 @@ cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, 
 cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
+// Geometry probe: per-row span, width, softmax entropy, share below -6, top-bucket mass,
+// effective buckets and total variation to softmax, into p.probe
+cudaError_t launch_fwd_probe(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 // C = running sums of the key rows of every head, [BH][T][d] (the P1 projection)
 cudaError_t launch_kcum(const float* K, float* C, int BH, int T, int d, cudaStream_t s);
 

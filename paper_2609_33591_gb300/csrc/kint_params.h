@@ -68,6 +68,7 @@ struct Params {
   float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
   const float* gbar;        // [BH*T] <g>_{P*} = dO_i . O*_i (workspace, written by the dO prep)
   float *cM_out, *cm_out;   // optional [BH*T] side outputs of the backward: c_M, c_m per row
+  float* probe;             // [7][BH*T] geometry probe outputs
   uint8_t *bins, *ivals;
 };
 

@@ -30,7 +30,7 @@ ERRORS = {0: "KINT_OK", -1: "KINT_ERR_ARG", -2: "KINT_ERR_UNSUPPORTED", -3: "KIN
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 # Every symbol include/kint_attn.h declares.
-EXPORTS = ("kint_attn_workspace_bytes", "kint_attn_fwd", "kint_attn_bwd", "kint_attn_debug_bins",
+EXPORTS = ("kint_attn_workspace_bytes", "kint_attn_fwd", "kint_attn_bwd", "kint_attn_debug_bins", "kint_attn_probe",
            "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns", "kint_set_launch_callback",
            "kint_attn_fwd_noalloc")
 
@@ -75,6 +75,9 @@ def load(build_if_missing: bool = True):
             lib.kint_attn_debug_bins.argtypes = [vp, vp, vp, ctypes.POINTER(kint_rowstats), vp, vp, i, i, i, i, i,
                                                  i, f, i, i, i, i, vp, sz, vp]
             lib.kint_attn_debug_bins.restype = i
+            lib.kint_attn_probe.argtypes = [vp, vp, ctypes.POINTER(kint_rowstats), vp, i, i, i, i, i, i, f, i, i, i,
+                                            vp, sz, vp]
+            lib.kint_attn_probe.restype = i
             lib.kint_get_status.argtypes = [vp, ctypes.POINTER(ctypes.c_uint)]
             lib.kint_get_status.restype = i
             lib.kint_strerror.argtypes = [i]
@@ -165,6 +168,15 @@ def kint_attn_fwd_noalloc(Q, K, V, O, st: dict, B, H, T, d, Kint, calib, tau, re
                                         float(tau), recon, ste, grad, causal, prec, _stream(stream))
 
 
+def kint_attn_probe(Q, K, st: dict, probe, B, H, T, d, Kint, calib, tau, recon, causal, prec, workspace,
+                    stream=None) -> int:
+    s = _stats_struct(st)
+    return load().kint_attn_probe(_p(Q), _p(K), ctypes.byref(s), _p(probe), B, H, T, d, Kint, calib, float(tau), recon,
+                                  causal, prec, _p(workspace),
+                                  0 if workspace is None else workspace.numel() * workspace.element_size(),
+                                  _stream(stream))
+
+
 def kint_attn_debug_bins(Q, K, V, st: dict, bins, ivals, B, H, T, d, Kint, calib, tau, recon, ste, causal, prec,
                          workspace, stream=None) -> int:
     s = _stats_struct(st)
@@ -253,6 +265,20 @@ def backward(Q, K, V, O, dO, stats, cfg: Config, prec=PREC_TF32, *, grads=None, 
     _check(kint_attn_bwd(Q, K, V, O, dO, stats, dQ, dK, dV, B, H, T, d, cfg.Kint, cfg.calib, cfg.tau, cfg.recon,
                          cfg.ste, cfg.grad, 1, prec, ws, stream), "kint_attn_bwd")
     return dQ, dK, dV
+
+
+PROBE_NAMES = ("span", "h", "entropy", "frac_below6", "top_mass", "eff_buckets", "tv")
+
+
+def probe(Q, K, cfg: Config, prec=PREC_TF32, *, stats=None, ws=None, stream=None) -> dict:
+    """Per-row geometry probe [B, H, T] for each of PROBE_NAMES (MinMax and FWM)."""
+    B, H, T, d = _shape(Q)
+    out = torch.empty(len(PROBE_NAMES), B, H, T, dtype=torch.float32, device=Q.device)
+    stats = alloc_rowstats(B, H, T, d, Q.device, False) if stats is None else stats
+    ws = workspace(B, H, T, d, prec, 0, Q.device) if ws is None else ws
+    _check(kint_attn_probe(Q, K, stats, out, B, H, T, d, cfg.Kint, cfg.calib, cfg.tau, cfg.recon, 1, prec, ws,
+                           stream), "kint_attn_probe")
+    return dict(zip(PROBE_NAMES, out.unbind(0)))
 
 
 def debug_bins(Q, K, V, stats, cfg: Config, prec=PREC_TF32, *, ws=None, stream=None):

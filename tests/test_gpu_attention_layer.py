@@ -36,6 +36,7 @@ class _OracleAttention(torch.autograd.Function):
 
 
 def _rel(a, ref):
+    a, ref = a.detach(), ref.detach()
     return float((a.double() - ref).abs().max() / ref.abs().max())
 
 

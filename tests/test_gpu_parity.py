@@ -213,3 +213,39 @@ def test_exact_grid_points(prec):
         rep = parity.check(Q, K, V, dO, cfg, prec)
         assert rep["bins_flips"] == 0 and rep["ivals_flips"] == 0
     parity.check(Q, K, V, dO, _cfg(MM, NE, WE, FU), prec)
+
+
+@pytest.mark.parametrize("c,r", [(MM, LE), (MM, NE), (FW, NE), (FW, LE)])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_geometry_probe(c, r, prec):
+    """kint_attn_probe against the oracle's probes, decision-aligned (the oracle takes the GPU's
+    bins and extrema, as in the parity check); T = 300 is ragged, Q x 2 spreads the rows so that
+    keys below z = -6 and FWM tail keys occur."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=20)
+    Q = Q * 2.0
+    cfg = _cfg(c, r, WE, FU, 4, tau=3.0)
+    dev = torch.device("cuda:0")
+    q, k, v = (torch.from_numpy(np.ascontiguousarray(x)).to(dev) for x in (Q, K, V))
+    pr = kint.probe(q, k, cfg, prec)
+    O, st = kint.forward(q, k, v, cfg, prec)
+    bins, ivals = kint.debug_bins(q, k, v, st, cfg, prec)
+    torch.cuda.synchronize()
+    kint.check_status()
+    amin = st["arg_min"].cpu().numpy() if c == MM else None
+    ov = {"bins": bins.cpu().numpy(), "ivals": ivals.cpu().numpy(), "amax": st["arg_max"].cpu().numpy()}
+    if amin is not None:
+        ov["amin"] = amin
+    f = parity.oracle.forward(Q, K, V, parity.to_oracle_cfg(cfg), probes=True, override=ov)
+    tol = 2e-5 if prec == X3 else 5e-3
+    # "z < -6" is a decision too: a key within the score rounding of -6 may count either way
+    S = np.einsum("bhid,bhjd->bhij", Q.astype(np.float64), K.astype(np.float64)) / 8.0
+    causal = np.tril(np.ones((300, 300), bool))
+    z = np.where(causal, S - np.where(causal, S, -np.inf).max(-1, keepdims=True), 0.0)
+    band = parity.BAND_REL[prec] * (np.abs(S).max() + 1.0)
+    near = (causal & (np.abs(z + 6.0) <= band)).sum(-1) / np.arange(1, 301)
+    for n, ref in zip(parity.oracle.PROBE_NAMES, f["probe"]):
+        got = pr[n].cpu().numpy().astype(np.float64)
+        err = np.abs(got - ref) / (1.0 + np.abs(ref))
+        if n == "frac_below6":
+            err = np.maximum(np.abs(got - ref) - near, 0.0)
+        assert err.max() <= tol, f"{n}: {err.max():.3g}"
