@@ -106,12 +106,14 @@ typedef struct {
   int32_t* arg_min;  /* lowest j with s_ij == m_i; -1 when row_min is not computed */
   int32_t* n_max;    /* number of keys tied at M_i (the extremum gradient is split evenly) */
   int32_t* n_min;    /* number of keys tied at m_i; 0 when row_min is not computed */
-  float* W;          /* W^N = sum w^N (Nearest) or W^L (LERP); softmax: sum e^{s - M} */
+  float* W;          /* W^N = sum w^N (Nearest) or W^L (LERP); softmax: sum e^{s - M};
+                        EXP_FP8: sum E4M3(e^{s - M}) */
   float* W_lerp;     /* W^L; required for Prob-STE, may be NULL otherwise */
   float* O_lerp;     /* [B,H,T,d] P^L V; required for Prob-STE, may be NULL otherwise */
   float* c_M;        /* optional side output of kint_attn_bwd (NULL: not written): the row's
                         calibration sum c_M = sum_j gamma_j dw_j/dM (supplement "Local gradient
-                        decomposition", the M channel); 0 under detach and for softmax */
+                        decomposition", the M channel; EXP_FP8: -sum_j gamma_j e^{z_j}); 0 under
+                        detach, detach_proj and for softmax */
   float* c_m;        /* optional side output of kint_attn_bwd: c_m = sum_j gamma_j dw_j/dm
                         (MinMax; 0 otherwise) */
 } kint_rowstats;
@@ -129,8 +131,8 @@ size_t kint_attn_workspace_bytes(int B, int H, int T, int d, kint_prec prec, int
  *   Q, K, V  in:  [B,H,T,d]
  *   O        out: [B,H,T,d]
  *   st       out: row statistics (struct itself is host memory, read during the call)
- *   Kint     number of intervals K, 1..64 (ignored for softmax)
- *   tau      FWM window in nats, > 0 (ignored otherwise)
+ *   Kint     number of intervals K, 1..64 (ignored for softmax and EXP_FP8)
+ *   tau      FWM window in nats, > 0 (FWM and FWM_RESOLVED; ignored otherwise)
  *   workspace, workspace_bytes: device scratch of at least
  *            kint_attn_workspace_bytes(B, H, T, d, prec, 0) bytes
  */
@@ -146,7 +148,8 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
  *     (P^N, W^N) for Nearest + Weight-STE and (P^L, W^L) otherwise;
  *   dS_ij = gamma_j Delta_j + [j tied at M_i] c_M / n_max + [j tied at m_i] c_m / n_min
  *     (c_m only for MinMax; both dropped under detach, c_m under max_only, c_M under
- *      min_only; FWM tail keys get 0; degenerate MinMax rows get 0);
+ *      min_only; FWM tail keys get 0; degenerate MinMax rows get 0; FWM_RESOLVED has no
+ *      tail; EXP_FP8 uses gamma at the rounded weights and e^{z_j} in place of Delta_j);
  *     under detach_proj each causal row of the detached dS then loses its mean;
  *   st->c_M, st->c_m, when non-NULL, receive the per-row sums c_M, c_m (16-byte aligned;
  *     the sums are written whether or not the mode applies them, 0 under detach and
