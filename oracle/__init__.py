@@ -24,7 +24,7 @@ _BUILD = os.path.join(_HERE, "_build")
 _SO = os.path.join(_BUILD, "liboracle.so")        # fp32 inputs
 _SO64 = os.path.join(_BUILD, "liboracle64.so")    # fp64 inputs, same arithmetic
 
-MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8 = 0, 1, 2, 3, 4
+MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8, EXP_BF16 = 0, 1, 2, 3, 4, 5
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
 FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4

@@ -26,6 +26,8 @@
  *   App. B "Softmax", App. A "Softmax"            -> the comparator
  *   App. "Reduced-precision exponential baselines" -> FP8-rounded exponential
  *                                                  (E4M3 forward, fp32-exp backward)
+ *                                                  and BF16 exponential (bf16 casts
+ *                                                  and bf16 chain rule)
  *   App. "Geometry probe"                         -> per-row probes: span, width,
  *                                                  softmax entropy, mass below -6,
  *                                                  top-bucket mass, effective buckets,
@@ -142,6 +144,52 @@ static int e4m3_round(double w, double* mg) {
   return best;
 }
 
+/* bfloat16: 8 significant bits, fp32's exponent range.  Round to nearest, ties to
+ * even (x = f 2^e with f in [1/2, 1): the significand is f 2^8 in [128, 256)), and
+ * flush magnitudes below 2^-126 to zero. */
+static double bf16_rne(double x) {
+  if (fabs(x) < ldexp(1.0, -126)) return 0.0;
+  int e;
+  const double f = frexp(x, &e);
+  double r = f * 256.0;
+  const double fl = floor(r), fr = r - fl;
+  r = (fr > 0.5 || (fr == 0.5 && fmod(fl, 2.0) != 0.0)) ? fl + 1.0 : fl;
+  return ldexp(r, e - 8);
+}
+
+/* Low byte of the bfloat16 bit pattern of a bfloat16 value v (0 for zero):
+ * bits = sign | (E + 127) << 7 | m for v = +-(1 + m/128) 2^E. */
+static int bf16_low_byte(double v) {
+  if (v == 0.0) return 0;
+  int e;
+  const double f = frexp(fabs(v), &e); /* |v| = f 2^e, f in [1/2, 1) */
+  const int E = e - 1, m = (int)(f * 256.0) - 128;
+  return (((E + 127) & 1) << 7) | m;
+}
+
+/* The bfloat16 neighbour of x (the rounded value or the next one either way)
+ * whose low byte is c; the rounded value itself when none matches. */
+static double bf16_with_low_byte(double x, int c) {
+  const double r = bf16_rne(x);
+  if (r == 0.0 || bf16_low_byte(r) == c) return r;
+  int e;
+  frexp(fabs(r), &e);
+  const double ulp = ldexp(1.0, e - 8);
+  const double cand[2] = {r - ulp, r + ulp};
+  for (int k = 0; k < 2; ++k)
+    if (bf16_low_byte(bf16_rne(cand[k])) == c) return bf16_rne(cand[k]);
+  return r;
+}
+
+/* Distance from x to the nearest bfloat16 rounding midpoint (x != 0). */
+static double bf16_margin(double x) {
+  int e;
+  frexp(fabs(x), &e);
+  const double half = ldexp(1.0, e - 9); /* half an ulp of x's binade */
+  const double r = bf16_rne(x);
+  return fabs(half - fabs(x - r));
+}
+
 /*
  * Forward quantities of causal row i of head bh (App. A).  Fills R.
  */
@@ -210,6 +258,28 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
       R->er0[j] = we;
       R->wL[j] = R->wN[j] = e4m3_value(code);
       R->code_l[j] = R->code_r[j] = code;
+      R->margin[j] = mg;
+    }
+  } else if (p->calib == KOR_EXP_BF16) {
+    /* z rounded to bfloat16, its exponential rounded to bfloat16: the forward weight
+     * (App. "Reduced-precision exponential baselines").  Both roundings are decisions:
+     * their codes are the low bytes, their margin the distance (in z) to a midpoint. */
+    for (int j = 0; j < n; ++j) {
+      const size_t idx = ((size_t)bh * T + i) * T + j;
+      const int ov = J->ov && J->ov->bins;
+      const double zb = ov ? bf16_with_low_byte(R->z[j], J->ov->bins[idx]) : bf16_rne(R->z[j]);
+      const double ez = exp(zb);
+      const double w = (ov && J->ov->ivals) ? bf16_with_low_byte(ez, J->ov->ivals[idx]) : bf16_rne(ez);
+      R->er0[j] = w;
+      R->wL[j] = R->wN[j] = w;
+      R->code_l[j] = bf16_low_byte(zb);
+      R->code_r[j] = bf16_low_byte(w);
+      double mg = INFINITY;
+      if (R->z[j] != 0.0) mg = bf16_margin(R->z[j]);
+      if (ez > 0.0 && ez != 1.0) {
+        const double me = bf16_margin(ez) / ez; /* relative: in z units */
+        if (me < mg) mg = me;
+      }
       R->margin[j] = mg;
     }
   } else if (p->calib == KOR_MINMAX && (R->M - R->m) <= DEGENERATE_EPS) {
@@ -425,6 +495,26 @@ static void bwd_row(const job_t* J, int bh, int i, row_t* R) {
     double D = 0.0;
     for (int j = 0; j < n; ++j) D += R->P[j] * R->g[j];
     for (int j = 0; j < n; ++j) R->dS[j] = R->P[j] * (R->g[j] - D);
+  } else if (p->calib == KOR_EXP_BF16) {
+    /* The chain rule through the casts in bfloat16: the gradient reaching the bfloat16
+     * weight is bf16(gamma_j), gamma_j = (g_j - <g>_P) / W; the exponential's backward
+     * multiplies it by its bfloat16 output, rounded to bfloat16; the cast of z passes it
+     * on.  The row max collects -sum_j dL/dz_j (split among ties). */
+    double D = 0.0;
+    for (int j = 0; j < n; ++j) D += R->P[j] * R->g[j];
+    double own = 0.0;
+    for (int j = 0; j < n; ++j) {
+      R->dS[j] = bf16_rne(bf16_rne((R->g[j] - D) / R->W_N) * R->er0[j]);
+      own += R->dS[j];
+    }
+    if (p->grad == KOR_DETACH_PROJ) {
+      for (int j = 0; j < n; ++j) R->dS[j] -= own / n;
+    } else if (p->grad != KOR_DETACH) {
+      cM = -own;
+      if (p->grad == KOR_FULL || p->grad == KOR_MAX_ONLY)
+        for (int j = 0; j < n; ++j)
+          if (R->s[j] == R->M) R->dS[j] += cM / R->nmax;
+    }
   } else if (p->calib == KOR_EXP_FP8) {
     /* Normalization Jacobian at the rounded weights, gamma_j = (g_j - <g>_P) / W;
      * the rounding passes the gradient unchanged and dw_j/dz_j = e^{z_j}.  With
@@ -595,8 +685,10 @@ static void* worker(void* arg) {
 
 static int check_params(const kor_params* p) {
   if (!p || p->B < 1 || p->H < 1 || p->T < 1 || p->d < 1) return -1;
-  if (p->calib < 0 || p->calib > 4) return -1;
-  if (p->calib != KOR_SOFTMAX && p->calib != KOR_EXP_FP8 && (p->Kint < 1 || p->Kint > (1 << 20))) return -1;
+  if (p->calib < 0 || p->calib > 5) return -1;
+  if (p->calib != KOR_SOFTMAX && p->calib != KOR_EXP_FP8 && p->calib != KOR_EXP_BF16 &&
+      (p->Kint < 1 || p->Kint > (1 << 20)))
+    return -1;
   if ((p->calib == KOR_FWM || p->calib == KOR_FWM_RESOLVED) && !(p->tau > 0.0)) return -1;
   if (p->recon < 0 || p->recon > 1 || p->ste < 0 || p->ste > 1 || p->grad < 0 || p->grad > 4) return -1;
   return 0;

@@ -31,7 +31,12 @@ typedef float kor_in;
  * exponential baselines"): w = E4M3(e^{z}) forward, the fp32 exponential's derivative
  * backward (identity surrogate on the rounding), the row max on the gradient path;
  * K, tau, the reconstruction and the STE placement do not apply to it. */
-enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2, KOR_FWM_RESOLVED = 3, KOR_EXP_FP8 = 4 };
+/* KOR_EXP_BF16 is the BF16 exponential baseline of the same appendix: z = s - M rounded to
+ * bfloat16, its exponential rounded to bfloat16 (w), P = w / sum w; the backward is the
+ * chain rule through those casts in bfloat16 arithmetic: dL/dz_j = bf16(bf16(gamma_j) w_j),
+ * the row max on the gradient path.  bfloat16 rounding is to nearest even; magnitudes
+ * below 2^-126 flush to zero. */
+enum { KOR_MINMAX = 0, KOR_FWM = 1, KOR_SOFTMAX = 2, KOR_FWM_RESOLVED = 3, KOR_EXP_FP8 = 4, KOR_EXP_BF16 = 5 };
 enum { KOR_LERP = 0, KOR_NEAREST = 1 };
 enum { KOR_WEIGHT = 0, KOR_PROB = 1 };
 /* Backward modes: the full calibration gradient (Eq. full), detached extrema (App. B
@@ -47,13 +52,15 @@ enum { KOR_FULL = 0, KOR_DETACH = 1, KOR_MAX_ONLY = 2, KOR_MIN_ONLY = 3, KOR_DET
  * below zero and are stored as index + KOR_CODE_OFFSET, saturated to [0, 252]
  * (code 0 stands for every index <= -128; such keys carry weights below
  * e^{-tau - 128 tau/K}).  Under KOR_EXP_FP8 both arrays hold the E4M3 byte of
- * the rounded weight (0x00 = 0 .. 0x38 = 1). */
+ * the rounded weight (0x00 = 0 .. 0x38 = 1).  Under KOR_EXP_BF16 bins holds the low
+ * byte of the bfloat16 bits of the rounded z and ivals that of the rounded weight
+ * (the low byte tells apart the two bfloat16 neighbours of a value). */
 enum { KOR_CODE_NOGRID = 253, KOR_CODE_TAIL = 254, KOR_CODE_MASKED = 255, KOR_CODE_OFFSET = 128 };
 
 typedef struct {
   int B, H, T, d;
   int Kint;   /* K, number of intervals */
-  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX / KOR_FWM_RESOLVED / KOR_EXP_FP8 */
+  int calib;  /* KOR_MINMAX / KOR_FWM / KOR_SOFTMAX / KOR_FWM_RESOLVED / KOR_EXP_FP8 / KOR_EXP_BF16 */
   double tau; /* FWM window in nats (also the resolved grid's origin) */
   int recon;  /* KOR_LERP / KOR_NEAREST */
   int ste;    /* KOR_WEIGHT / KOR_PROB (ignored for LERP) */

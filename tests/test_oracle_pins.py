@@ -12,8 +12,8 @@ import numpy as np
 import pytest
 
 import oracle
-from oracle import Config, MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8, LERP, NEAREST, WEIGHT, PROB, FULL, \
-    DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ
+from oracle import Config, MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8, EXP_BF16, LERP, NEAREST, WEIGHT, PROB, \
+    FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ
 from tests import witness
 
 ALL_COMBOS = [(c, r, s, g) for c in (MINMAX, FWM) for r in (LERP, NEAREST) for s in (WEIGHT, PROB)
@@ -810,3 +810,54 @@ def test_probe_degenerate_and_single_key_rows():
     for n, v in (("span", 0.0), ("h", 0.0), ("top_mass", 1.0), ("eff_buckets", 1.0), ("tv", 0.0), ("frac_below6", 0.0)):
         assert np.allclose(_probe(out, n)[0, 0], v, atol=1e-12), n
     assert np.allclose(_probe(out, "entropy")[0, 0], np.log(np.arange(1, T + 1)), atol=1e-12)
+
+
+# --- BF16 exponential baseline (App. "Reduced-precision exponential baselines") --------------------
+
+@pytest.mark.parametrize("grad", [FULL, DETACH, DETACH_PROJ, MAX_ONLY, MIN_ONLY])
+def test_bf16_matches_autograd_witness(grad):
+    """The witness casts z to torch.bfloat16, takes torch.exp in bfloat16 and casts back; autograd
+    supplies the bfloat16 chain rule the oracle writes out."""
+    Q, K, V, dO = rand_inputs(1, 2, 16, 8, 51, scale=2.0)
+    cfg = Config(Kint=4, calib=EXP_BF16, grad=grad)
+    f = oracle.forward(Q, K, V, cfg)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    O, dQ, dK, dV = witness.attention(Q, K, V, dO, cfg)
+    for a, w in ((f["O"], O), (b["dQ"], dQ), (b["dK"], dK), (b["dV"], dV)):
+        assert np.max(np.abs(a - w)) <= 1e-10 * max(1.0, np.max(np.abs(w)))
+
+
+def test_bf16_codes_are_torch_bfloat16_bits():
+    """The decision codes are the low bytes of torch's bfloat16 bit patterns of z and of e^{bf16(z)}."""
+    torch = pytest.importorskip("torch")
+    z = -np.round(np.linspace(0.0, 12.0, 63) * 1024) / 1024
+    T, d = 64, 64
+    Q = np.zeros((1, 1, T, d), np.float32)
+    K = np.zeros((1, 1, T, d), np.float32)
+    Q[0, 0, :, 0] = 8.0
+    K[0, 0, :, 0] = np.concatenate([[0.0], z])
+    out = oracle.forward(Q, K, eye_values(T, d), Config(Kint=4, calib=EXP_BF16), decisions=True)
+    zb = torch.tensor(np.concatenate([[0.0], z])).to(torch.bfloat16)
+    wb = torch.exp(zb)
+    lo = lambda t: (t.view(torch.int16).to(torch.int32) & 0xFF).numpy()
+    assert np.array_equal(out["bins"][0, 0, T - 1], lo(zb))
+    assert np.array_equal(out["ivals"][0, 0, T - 1], lo(wb))
+    O = out["O"][0, 0, T - 1]
+    assert np.allclose(O / O[0], wb.to(torch.float64).numpy(), rtol=1e-14, atol=0)
+
+
+def test_bf16_zero_sum_and_override():
+    Q, K, V, dO = rand_inputs(1, 2, 24, 8, 53, scale=2.0)
+    cfg = Config(Kint=4, calib=EXP_BF16, grad=FULL)
+    b = oracle.backward(Q, K, V, dO, cfg)
+    live = b["dabs"] > 0
+    assert np.max(np.abs(b["dsum"][live]) / b["dabs"][live]) < 1e-13
+    f = oracle.forward(Q, K, V, cfg, decisions=True)
+    ov = {"bins": f["bins"], "ivals": f["ivals"], "amax": f["amax"], "amin": f["amin"]}
+    assert np.array_equal(oracle.forward(Q, K, V, cfg, override=ov)["O"], f["O"])
+    iv = f["ivals"].copy()
+    i, j = 20, 3
+    iv[0, 1, i, j] ^= 1  # the other bfloat16 neighbour of that key's weight
+    g = oracle.forward(Q, K, V, cfg, override={**ov, "ivals": iv})
+    changed = np.argwhere(np.any(g["O"] != f["O"], axis=-1))
+    assert changed.tolist() == [[0, 1, i]]

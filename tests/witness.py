@@ -15,7 +15,7 @@ import math
 import numpy as np
 import torch
 
-MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8 = 0, 1, 2, 3, 4
+MINMAX, FWM, SOFTMAX, FWM_RESOLVED, EXP_FP8, EXP_BF16 = 0, 1, 2, 3, 4, 5
 LERP, NEAREST = 0, 1
 WEIGHT, PROB = 0, 1
 FULL, DETACH, MAX_ONLY, MIN_ONLY, DETACH_PROJ = 0, 1, 2, 3, 4
@@ -39,6 +39,12 @@ def probs(S: torch.Tensor, valid: torch.Tensor, cfg) -> torch.Tensor:
         # derivative backward: w = fp8(e^z) + (e^z - sg(e^z))
         we = torch.exp(z.masked_fill(~valid, -math.inf))
         w = we.detach().to(torch.float8_e4m3fn).to(S.dtype) + (we - we.detach())
+        w = torch.where(valid, w, torch.zeros_like(w))
+        return w / w.sum(-1, keepdim=True)
+    if cfg.calib == EXP_BF16:
+        # z cast to bfloat16, the exponential evaluated in bfloat16, cast back; autograd then
+        # differentiates through the casts in bfloat16 arithmetic
+        w = torch.exp(z.masked_fill(~valid, 0.0).to(torch.bfloat16)).to(S.dtype)
         w = torch.where(valid, w, torch.zeros_like(w))
         return w / w.sum(-1, keepdim=True)
     if cfg.calib == MINMAX:
