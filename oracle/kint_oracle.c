@@ -274,7 +274,9 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
       R->wL[j] = R->wN[j] = w;
       R->code_l[j] = bf16_low_byte(zb);
       R->code_r[j] = bf16_low_byte(w);
-      double mg = INFINITY;
+      /* z = 0 (the row max) is itself a boundary: every z of either sign near 0 has its own
+       * bfloat16 code, so a row max that another key ties within rounding moves it */
+      double mg = 0.0;
       if (R->z[j] != 0.0) mg = bf16_margin(R->z[j]);
       if (ez > 0.0 && ez != 1.0) {
         const double me = bf16_margin(ez) / ez; /* relative: in z units */
