@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "f13b8f9bd983badb", "k_prep": 82543104, "k_fwd_stats": 50366976, "k_fwd_main": 92420608,
-           "k_bwd_dq": 182365952, "k_bwd_dkdv": 261233152}
+TRAFFIC = {"src": "3c0af8e07a6451c9", "k_prep": 82473856, "k_fwd_stats": 50369536, "k_fwd_main": 93726976,
+           "k_bwd_dq": 194415616, "k_bwd_dkdv": 274723840}
 
 
 def kernel_source_digest() -> str:

@@ -62,8 +62,14 @@ typedef enum {
   KINT_CALIB_FWM = 1,
   KINT_CALIB_SOFTMAX = 2,
   KINT_CALIB_FWM_RESOLVED = 3,
-  KINT_CALIB_EXP_FP8 = 4
+  KINT_CALIB_EXP_FP8 = 4,
+  KINT_CALIB_EXP_BF16 = 5
 } kint_calib;
+/* KINT_CALIB_EXP_BF16 is the BF16 exponential baseline of the same appendix: z = s - M
+ * rounded to bfloat16, w = e^z rounded to bfloat16 (round to nearest even; the exponential
+ * is ex2.approx, flushing below 2^-126), P = w / sum w; the backward is the chain rule
+ * through the casts in bfloat16 arithmetic, dL/dz_j = bf16(bf16(gamma_j) w_j), with the
+ * row max on the gradient path as for EXP_FP8.  Kint, tau, recon, ste: as for EXP_FP8. */
 /* KINT_CALIB_EXP_FP8 is the FP8-rounded exponential baseline of App. "Reduced-precision
  * exponential baselines": w = E4M3(e^{s - M}) (round to nearest even) in the forward, the
  * exponential's own derivative e^{s - M} in the backward (identity surrogate on the
@@ -192,7 +198,8 @@ int kint_attn_probe(const float* Q, const float* K, const kint_rowstats* st, flo
  * and 253 where no grid exists (degenerate MinMax rows, softmax); under
  * FWM_RESOLVED both indices run below zero and are stored as index + 128,
  * saturated to [0, 252] (0: index <= -128); under EXP_FP8 both hold the E4M3
- * byte of the rounded weight (0x00 = 0 .. 0x38 = 1).  Either
+ * byte of the rounded weight (0x00 = 0 .. 0x38 = 1); under EXP_BF16 bins holds the low
+ * byte of the bfloat16 bits of z and ivals that of the weight.  Either
  * output may be NULL.  Needs the row statistics of kint_attn_fwd on the same
  * inputs and the forward's workspace size.  bins, ivals: [B,H,T,T] uint8.
  */

@@ -162,10 +162,10 @@ struct Common {
 int validate(const Common& c, int causal) {
   if (c.B < 1 || c.H < 1 || c.T < 1 || c.d < 1) return KINT_ERR_ARG;
   if (causal != 1) return KINT_ERR_ARG;
-  if (c.calib < 0 || c.calib > 4 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
+  if (c.calib < 0 || c.calib > 5 || c.recon < 0 || c.recon > 1 || c.ste < 0 || c.ste > 1 || c.grad < 0 ||
       c.grad > 4 || c.prec < 0 || c.prec > 1)
     return KINT_ERR_ARG;
-  const bool grid = c.calib != KINT_CALIB_SOFTMAX && c.calib != KINT_CALIB_EXP_FP8;
+  const bool grid = c.calib != KINT_CALIB_SOFTMAX && c.calib != KINT_CALIB_EXP_FP8 && c.calib != KINT_CALIB_EXP_BF16;
   if (grid && (c.Kint < 1 || c.Kint > KMAX)) return KINT_ERR_ARG;
   if ((c.calib == KINT_CALIB_FWM || c.calib == KINT_CALIB_FWM_RESOLVED) && !(c.tau > 0.0f && std::isfinite(c.tau)))
     return KINT_ERR_ARG;
@@ -184,7 +184,8 @@ Params base_params(const Common& c, unsigned* status) {
   Params p;
   std::memset(&p, 0, sizeof(p));
   p.B = c.B; p.H = c.H; p.T = c.T; p.d = c.d;
-  const bool exp_w = c.calib == KINT_CALIB_SOFTMAX || c.calib == KINT_CALIB_EXP_FP8;  // no grid
+  const bool exp_w = c.calib == KINT_CALIB_SOFTMAX || c.calib == KINT_CALIB_EXP_FP8 ||
+                     c.calib == KINT_CALIB_EXP_BF16;  // no grid
   p.Kint = exp_w ? 1 : c.Kint;
   p.calib = c.calib; p.recon = c.recon; p.ste = c.ste; p.grad = c.grad;
   if (exp_w) p.recon = p.ste = 0;  // (neither a reconstruction nor a surrogate placement applies)
@@ -430,8 +431,8 @@ void set_stats(Params& p, const kint_rowstats* st) {
 }
 
 bool is_prob(const Common& c) {
-  return c.calib != KINT_CALIB_SOFTMAX && c.calib != KINT_CALIB_EXP_FP8 && c.recon == KINT_RECON_NEAREST &&
-         c.ste == KINT_STE_PROB;
+  return c.calib != KINT_CALIB_SOFTMAX && c.calib != KINT_CALIB_EXP_FP8 && c.calib != KINT_CALIB_EXP_BF16 &&
+         c.recon == KINT_RECON_NEAREST && c.ste == KINT_STE_PROB;
 }
 
 }  // namespace

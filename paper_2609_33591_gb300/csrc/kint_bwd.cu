@@ -42,6 +42,11 @@ __device__ __forceinline__ void dq_chunk(const float (&sv)[W], const float (&gv)
     } else if constexpr (CAL == CAL_EXP8) {
       // gamma e^{z}: the exponential's derivative through the rounding's identity surrogate
       ds = ex2_approx(__fmaf_rn(sv[jj], sk1, sc0)) * __fmaf_rn(gv[jj], ga, gb);
+    } else if constexpr (CAL == CAL_EXPB) {
+      // the bfloat16 chain rule: bf16(bf16(gamma) w), w = bf16(e^{bf16(z)}); k1, c0 = scale, -M
+      float zb;
+      const float w = bf16_exp_weight(__fadd_rn(__fmul_rn(sv[jj], k1), c0), zb);
+      ds = bf16_rn(__fmul_rn(bf16_rn(__fmaf_rn(gv[jj], ga, gb)), w));
     } else if constexpr (fwm_like(CAL)) {
       // k1, c0 doubled (v = 2u), Kf = 2K, tab: the half-bin table of Delta_r / h (4-byte entries)
       const float v = __fmaf_rn(sv[jj], k1, c0);
@@ -366,7 +371,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         r.amax = p.arg_max[rw];
         r.amin = p.arg_min[rw];
         r.Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
-        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && !exp_like(CAL));
+        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && !gridless(CAL));
         r.Ws = prob ? p.W_lerp[rw] : r.Wf;
       }
       return r;
@@ -655,6 +660,12 @@ __device__ __forceinline__ void kv_chunk(const float (&sv)[W], const float (&gv)
       const float we = ex2_approx(__fmaf_rn(sv[ii], r0.y, r0.x));
       pv = e4m3_rn(we) * r0.z;
       ds = gam * we;
+    } else if constexpr (CAL == CAL_EXPB) {
+      // record holds -M, scale: z = acc * scale - M; the bfloat16 chain rule
+      float zb;
+      const float w = bf16_exp_weight(__fadd_rn(__fmul_rn(sv[ii], r0.y), r0.x), zb);
+      pv = w * r0.z;
+      ds = bf16_rn(__fmul_rn(bf16_rn(gam), w));
     } else if constexpr (fwm_like(CAL) && REC == REC_NEAREST) {
       // record holds 2k1, 2c0; Kf = 2K; fwtab: the half-bin table of (w^N, Delta_r / h)
       const float v = __fmaf_rn(sv[ii], r0.y, r0.x);
@@ -1179,6 +1190,9 @@ cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cud
   if (p.calib == CAL_EXP8)
     return full ? launch3(k_bwd_dq<CAL_EXP8, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
                 : launch3(k_bwd_dq<CAL_EXP8, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
+  if (p.calib == CAL_EXPB)
+    return full ? launch3(k_bwd_dq<CAL_EXPB, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
+                : launch3(k_bwd_dq<CAL_EXPB, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
   if (p.calib == CAL_MINMAX)
     return full ? launch3(k_bwd_dq<CAL_MINMAX, true>, grid, maps, p, smem_bytes, s, NTHR_DQ)
                 : launch3(k_bwd_dq<CAL_MINMAX, false>, grid, maps, p, smem_bytes, s, NTHR_DQ);
@@ -1198,6 +1212,10 @@ cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, c
     return full ? launch3(k_bwd_dkdv<CAL_EXP8, REC_LERP, true>, grid, maps, p, smem_bytes, s)
            : proj ? launch3(k_bwd_dkdv<CAL_EXP8, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
                   : launch3(k_bwd_dkdv<CAL_EXP8, REC_LERP, false>, grid, maps, p, smem_bytes, s);
+  if (p.calib == CAL_EXPB)
+    return full ? launch3(k_bwd_dkdv<CAL_EXPB, REC_LERP, true>, grid, maps, p, smem_bytes, s)
+           : proj ? launch3(k_bwd_dkdv<CAL_EXPB, REC_LERP, false, true>, grid, maps, p, smem_bytes, s)
+                  : launch3(k_bwd_dkdv<CAL_EXPB, REC_LERP, false>, grid, maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
     if (near)
       return full ? launch3(k_bwd_dkdv<CAL_MINMAX, REC_NEAREST, true>, grid, maps, p, smem_bytes, s)

@@ -2,6 +2,7 @@
 // (Sec. 3 "Objects and calibration", App. A), the per-key decisions and weights
 // (App. A "LERP", "Nearest"), and the tile movement / tensor-core helpers.
 #pragma once
+#include <cuda_bf16.h>
 #include <cstdint>
 #include <cuda.h>
 #include "kint_params.h"
@@ -145,12 +146,13 @@ __device__ __forceinline__ RowGrid row_grid(const Params& p, float M, float m) {
     g.b0 = -p.tau;
     g.k1 = __fmul_rn(p.scale, g.inv_h);
   } else {
-    g.nogrid = p.calib != CAL_EXP8;  // (the FP8 exponential keeps the row max's gradient channel)
+    // (the FP8 and BF16 exponentials keep the row max's gradient channel)
+    g.nogrid = p.calib != CAL_EXP8 && p.calib != CAL_EXPB;
     g.h = 1.0f;
     g.inv_h = 1.0f;
-    g.c0 = 0.0f;
+    g.c0 = -M;  // z = acc * scale - M (the BF16 exponential rounds z itself)
     g.b0 = 0.0f;
-    g.k1 = 1.0f;
+    g.k1 = p.scale;
   }
   return g;
 }
@@ -224,6 +226,19 @@ __device__ __forceinline__ float ex2_approx(float x) {
 __device__ __forceinline__ float grid_value(const Params& p, const RowGrid& g, int r) {
   if (fwm_like(p.calib)) return p.fwm_e[r];
   return expf(__fmaf_rn((float)r, g.h, g.b0));
+}
+
+// BF16 exponential (App. "Reduced-precision exponential baselines"): round to the nearest
+// bfloat16, ties to even (the CUDA conversion), and the low byte of its bit pattern (the
+// decision code: it tells apart the two bfloat16 neighbours of a value).
+__device__ __forceinline__ float bf16_rn(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+__device__ __forceinline__ int bf16_low_byte(float x) {
+  return (int)(__bfloat16_as_ushort(__float2bfloat16_rn(x)) & 0xFFu);
+}
+// w = bf16(e^{bf16(z)}) from z, and the pair (bf16(z), w) for the decision dump
+__device__ __forceinline__ float bf16_exp_weight(float z, float& zb) {
+  zb = bf16_rn(z);
+  return bf16_rn(ex2_approx(__fmul_rn(zb, 1.4426950408889634f)));
 }
 
 // FP8-rounded exponential (App. "Reduced-precision exponential baselines"): 0 <= w <= 1

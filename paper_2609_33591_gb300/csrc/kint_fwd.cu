@@ -408,6 +408,9 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
       wm = ex2_approx(__fmaf_rn(v[jj], sk1, sc0));  // e^{s - M} (App. A, Softmax)
     } else if constexpr (CAL == CAL_EXP8) {
       wm = e4m3_rn(ex2_approx(__fmaf_rn(v[jj], sk1, sc0)));  // E4M3(e^{s - M})
+    } else if constexpr (CAL == CAL_EXPB) {
+      float zb;
+      wm = bf16_exp_weight(__fadd_rn(__fmul_rn(v[jj], g.k1), g.c0), zb);  // bf16(e^{bf16(s - M)})
     } else {
       const float u = __fmaf_rn(v[jj], g.k1, g.c0);
       float t, rf;
@@ -463,6 +466,11 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
     if (j <= i) {
       if constexpr (CAL == CAL_EXP8) {
         cb = ci = (uint8_t)e4m3_code(e4m3_rn(ex2_approx(__fmaf_rn(v[jj], sk1, sc0))));
+      } else if constexpr (CAL == CAL_EXPB) {
+        float zb;
+        const float w = bf16_exp_weight(__fadd_rn(__fmul_rn(v[jj], g.k1), g.c0), zb);
+        cb = (uint8_t)bf16_low_byte(zb);
+        ci = (uint8_t)bf16_low_byte(w);
       } else if (CAL == CAL_SOFTMAX || g.nogrid) {
         cb = ci = 253;
       } else {
@@ -819,6 +827,7 @@ cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, c
   const int mode = p.pv_sel;
   if (p.calib == CAL_SOFTMAX) return launch_main_t<CAL_SOFTMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
   if (p.calib == CAL_EXP8) return launch_main_t<CAL_EXP8, REC_LERP, 0>(maps, p, smem_bytes, s);
+  if (p.calib == CAL_EXPB) return launch_main_t<CAL_EXPB, REC_LERP, 0>(maps, p, smem_bytes, s);
   if (p.calib == CAL_MINMAX) {
     if (p.recon == REC_LERP) return launch_main_t<CAL_MINMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
     if (mode == PV_MAIN) return launch_main_t<CAL_MINMAX, REC_NEAREST, 0>(maps, p, smem_bytes, s);

@@ -6,13 +6,16 @@
 
 namespace kint {
 
-enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2, CAL_FWMR = 3, CAL_EXP8 = 4 };
+enum Calib : int { CAL_MINMAX = 0, CAL_FWM = 1, CAL_SOFTMAX = 2, CAL_FWMR = 3, CAL_EXP8 = 4, CAL_EXPB = 5 };
 // FWM's grid (step tau/K, origin -tau), with a zero tail below the window (FWM) or
 // continued below it with negative indices (CAL_FWMR, the "resolved" tail policy)
 __host__ __device__ constexpr bool fwm_like(int cal) { return cal == CAL_FWM || cal == CAL_FWMR; }
 // weights from the exponential unit instead of a grid: the softmax comparator, and
 // CAL_EXP8, the FP8-rounded exponential baseline (E4M3(e^z) forward, e^z backward)
 __host__ __device__ constexpr bool exp_like(int cal) { return cal == CAL_SOFTMAX || cal == CAL_EXP8; }
+// no grid at all (no reconstruction, no surrogate placement): the above and CAL_EXPB, the
+// BF16 exponential baseline (z and e^z rounded to bfloat16, bfloat16 chain rule backward)
+__host__ __device__ constexpr bool gridless(int cal) { return exp_like(cal) || cal == CAL_EXPB; }
 enum Recon : int { REC_LERP = 0, REC_NEAREST = 1 };
 enum Grad : int { GRAD_FULL = 0, GRAD_DETACH = 1, GRAD_MAX_ONLY = 2, GRAD_MIN_ONLY = 3, GRAD_DETACH_PROJ = 4 };
 

@@ -17,7 +17,7 @@ import torch
 
 from . import build as _build
 
-CALIB_MINMAX, CALIB_FWM, CALIB_SOFTMAX, CALIB_FWM_RESOLVED, CALIB_EXP_FP8 = 0, 1, 2, 3, 4
+CALIB_MINMAX, CALIB_FWM, CALIB_SOFTMAX, CALIB_FWM_RESOLVED, CALIB_EXP_FP8, CALIB_EXP_BF16 = 0, 1, 2, 3, 4, 5
 RECON_LERP, RECON_NEAREST = 0, 1
 STE_WEIGHT, STE_PROB = 0, 1
 GRAD_FULL, GRAD_DETACH, GRAD_MAX_ONLY, GRAD_MIN_ONLY, GRAD_DETACH_PROJ = 0, 1, 2, 3, 4
@@ -112,7 +112,7 @@ class Config:
 
     @property
     def prob(self) -> bool:
-        return self.calib not in (CALIB_SOFTMAX, CALIB_EXP_FP8) and self.recon == RECON_NEAREST and \
+        return self.calib not in (CALIB_SOFTMAX, CALIB_EXP_FP8, CALIB_EXP_BF16) and self.recon == RECON_NEAREST and \
             self.ste == STE_PROB
 
 

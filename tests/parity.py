@@ -30,6 +30,11 @@ BAND_REL = {kint.PREC_3XTF32: 16 * 2.0 ** -22, kint.PREC_TF32: 16 * 2.0 ** -11}
 # than against their own size, and held to four times the output tolerance (one fp32 sum
 # over up to T keys, against the tensor-core sums of the outputs).
 SUM_TOL_FACTOR = 4.0
+# The BF16 exponential baseline computes its score gradient in bfloat16 (dL/dz = bf16(bf16(gamma) w)):
+# a gamma within the GPU's rounding of a bfloat16 midpoint rounds to the other neighbour, one
+# bfloat16 unit (2^-8 relative) on that key, twice at most; dQ, dK and the calibration sums are
+# held to that, 2^-7 normwise.
+BF16_GRAD_TOL = 2.0 ** -7
 
 
 def to_oracle_cfg(cfg: kint.Config) -> oracle.Config:
@@ -137,6 +142,8 @@ def check(Q, K, V, dO, cfg: kint.Config, prec, *, want_bwd=True, tol=None, repor
     rep["errors"] = errs
     for n, e in errs.items():
         t = tol * SUM_TOL_FACTOR if n in ("c_M", "c_m") else tol
+        if cfg.calib == kint.CALIB_EXP_BF16 and n in ("dQ", "dK", "c_M", "c_m"):
+            t = max(t, BF16_GRAD_TOL)
         assert e <= t, f"{n}: normwise error {e:.3g} > {t:g} ({rep})"
     if report is not None:
         report.update(rep)

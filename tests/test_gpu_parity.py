@@ -11,7 +11,7 @@ from tests import parity
 pytestmark = pytest.mark.gpu
 
 MM, FW, SM, FR = kint.CALIB_MINMAX, kint.CALIB_FWM, kint.CALIB_SOFTMAX, kint.CALIB_FWM_RESOLVED
-E8 = kint.CALIB_EXP_FP8
+E8, EB = kint.CALIB_EXP_FP8, kint.CALIB_EXP_BF16
 LE, NE = kint.RECON_LERP, kint.RECON_NEAREST
 WE, PR = kint.STE_WEIGHT, kint.STE_PROB
 FU, DE = kint.GRAD_FULL, kint.GRAD_DETACH
@@ -114,6 +114,17 @@ def test_fp8_exponential_baseline(g, prec):
     rep = parity.check(Q, K, V, dO, _cfg(E8, LE, WE, g), prec)
     if prec == X3:  # fp32-accurate scores: a rounding decision flips only within a few ulps
         assert rep["bins_flips"] <= 0.001 * 300 * 301
+
+
+@pytest.mark.parametrize("g", [FU, DE, PJ])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_bf16_exponential_baseline(g, prec):
+    """bf16(e^{bf16(z)}) forward (both roundings compared as decisions through their bfloat16 low
+    bytes), bfloat16 chain-rule backward; T = 300 is ragged."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=22)
+    rep = parity.check(Q, K, V, dO, _cfg(EB, LE, WE, g), prec)
+    if prec == X3:
+        assert rep["errors"]["dV"] <= 1e-5 and rep["errors"]["O"] <= 1e-5
 
 
 def test_fp8_exponential_value_set():
