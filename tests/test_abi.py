@@ -86,3 +86,29 @@ def test_strerror_covers_every_code():
     for code in kint.ERRORS:
         assert kint.strerror(code) != "unknown error code"
     assert kint.strerror(12345) == "unknown error code"
+
+
+def test_torch_entry_points_refuse_host_tensors():
+    """The product path has no CPU fallback: the tensor-level API and the autograd layer refuse
+    host tensors before any call into the library."""
+    import torch
+    from paper_2609_33591_gb300.attention import KIntSelfAttention, kint_attention
+    q = torch.zeros(1, 1, 8, 64)
+    for call in (lambda: kint.forward(q, q, q, kint.Config()), lambda: kint.probe(q, q, kint.Config()),
+                 lambda: kint_attention(q, q, q, kint.Config()),
+                 lambda: KIntSelfAttention(128, 2)(torch.zeros(1, 8, 128))):
+        with pytest.raises(ValueError):
+            call()
+
+
+def test_probe_argument_errors():
+    """kint_attn_probe: MinMax and FWM only; arguments are checked before any launch."""
+    lib = kint.load()
+    p = ctypes.c_void_p(256)
+    st = kint.kint_rowstats(*([256] * 7 + [None, None]))
+    args = (1, 1, 8, 64, 4)
+    assert lib.kint_attn_probe(p, p, ctypes.byref(st), p, *args, kint.CALIB_SOFTMAX, 8.0, 0, 1, 0, p, 1 << 30,
+                               None) == -2
+    assert lib.kint_attn_probe(p, p, ctypes.byref(st), None, *args, kint.CALIB_FWM, 8.0, 0, 1, 0, p, 1 << 30,
+                               None) == -1
+    assert lib.kint_attn_probe(p, p, ctypes.byref(st), p, *args, kint.CALIB_FWM, 8.0, 0, 1, 0, p, 16, None) == -4
