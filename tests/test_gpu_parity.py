@@ -116,17 +116,6 @@ def test_fp8_exponential_baseline(g, prec):
         assert rep["bins_flips"] <= 0.001 * 300 * 301
 
 
-@pytest.mark.parametrize("g", [FU, DE, PJ])
-@pytest.mark.parametrize("prec", [X3, TF])
-def test_bf16_exponential_baseline(g, prec):
-    """bf16(e^{bf16(z)}) forward (both roundings compared as decisions through their bfloat16 low
-    bytes), bfloat16 chain-rule backward; T = 300 is ragged."""
-    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=22)
-    rep = parity.check(Q, K, V, dO, _cfg(EB, LE, WE, g), prec)
-    if prec == X3:
-        assert rep["errors"]["dV"] <= 1e-5 and rep["errors"]["O"] <= 1e-5
-
-
 def test_fp8_exponential_value_set():
     """Scores spread so that every E4M3 level below 1 and the underflow to zero occur: the GPU's
     codes take exactly the format's 56 nonzero values and 0."""
@@ -260,3 +249,14 @@ def test_geometry_probe(c, r, prec):
         if n == "frac_below6":
             err = np.maximum(np.abs(got - ref) - near, 0.0)
         assert err.max() <= tol, f"{n}: {err.max():.3g}"
+
+
+@pytest.mark.parametrize("g", [FU, DE, PJ])
+@pytest.mark.parametrize("prec", [X3, TF])
+def test_bf16_exponential_baseline(g, prec):
+    """bf16(e^{bf16(z)}) forward (both roundings compared as decisions through their bfloat16 low
+    bytes), bfloat16 chain-rule backward; T = 300 is ragged."""
+    Q, K, V, dO = make_qkvdo(1, 2, 300, 64, seed=22)
+    rep = parity.check(Q, K, V, dO, _cfg(EB, LE, WE, g), prec)
+    if prec == X3:
+        assert rep["errors"]["dV"] <= 1e-5 and rep["errors"]["O"] <= 1e-5
