@@ -219,7 +219,7 @@ def _fd_setup(seed, calib, tau):
     raise RuntimeError("no well-separated seed")
 
 
-@pytest.mark.parametrize("calib", [MINMAX, FWM, SOFTMAX])
+@pytest.mark.parametrize("calib", [MINMAX, FWM, SOFTMAX, FWM_RESOLVED])
 def test_lerp_full_gradient_matches_finite_differences(calib):
     tau = 2.0
     Q, K, V, dO = _fd_setup(10, calib, tau)
