@@ -185,7 +185,9 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
  *      LERP intervals r, FWM tail keys as one more bucket, a degenerate row as one bucket
  *   6  total variation 1/2 sum_j |P_j - P^E_j| to the operator's forward P
  * probe: device, [7][B,H,T] fp32, 16-byte aligned, caller-owned.  The workspace is the
- * forward's (kint_attn_workspace_bytes(..., 0)).  Diagnostic: not on the training path.
+ * forward's (kint_attn_workspace_bytes(..., 0)).  The per-CTA bucket masses take
+ * 1 KB x (K + 2) of shared memory: TF32 at d = 64 supports every K, 3xTF32 and d = 128
+ * K <= 27 (KINT_ERR_UNSUPPORTED above).  Diagnostic: not on the training path.
  */
 int kint_attn_probe(const float* Q, const float* K, const kint_rowstats* st, float* probe, int B, int H, int T,
                     int d, int Kint, kint_calib calib, float tau, kint_recon recon, int causal, kint_prec prec,
