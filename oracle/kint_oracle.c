@@ -264,6 +264,11 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
     /* z rounded to bfloat16, its exponential rounded to bfloat16: the forward weight
      * (App. "Reduced-precision exponential baselines").  Both roundings are decisions:
      * their codes are the low bytes, their margin the distance (in z) to a midpoint. */
+    /* The row max key has z = 0 exactly; its code moves only if another key takes over as
+     * the row max, i.e. by the gap between the maximum and the runner-up score. */
+    double top_gap = INFINITY;
+    for (int j = 0; j < n; ++j)
+      if (R->s[j] != R->M && R->M - R->s[j] < top_gap) top_gap = R->M - R->s[j];
     for (int j = 0; j < n; ++j) {
       const size_t idx = ((size_t)bh * T + i) * T + j;
       const int ov = J->ov && J->ov->bins;
@@ -274,9 +279,10 @@ static void row_forward(const job_t* J, int bh, int i, row_t* R) {
       R->wL[j] = R->wN[j] = w;
       R->code_l[j] = bf16_low_byte(zb);
       R->code_r[j] = bf16_low_byte(w);
-      /* z = 0 (the row max) is itself a boundary: every z of either sign near 0 has its own
-       * bfloat16 code, so a row max that another key ties within rounding moves it */
-      double mg = 0.0;
+      /* z = 0 (the row max) is a boundary in its own way: every z of either sign near 0 has
+       * its own bfloat16 code, so the row max key's code moves when a runner-up within
+       * rounding takes over as the maximum: its margin is the top-two gap */
+      double mg = top_gap;
       if (R->z[j] != 0.0) mg = bf16_margin(R->z[j]);
       if (ez > 0.0 && ez != 1.0) {
         const double me = bf16_margin(ez) / ez; /* relative: in z units */
