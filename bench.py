@@ -178,6 +178,69 @@ def cpu_oracle_rate(n_heads: int, min_seconds: float = 0.0):
     return reps * 6 * unit_flops(1, n_heads, T, d) / dt / 1e12, dt, threads, reps
 
 
+def bench_parity(Q, K, V, dO):
+    """The timed workload's outputs against the fp64 oracle (outside the timed region, in
+    the CPU-baseline leg): decisions, flip fraction, normwise errors, zero-sum residual."""
+    from paper_2609_33591_gb300 import kint
+    from tests import parity
+    cfg = kint.Config(**VARIANT)
+    rep, err = {}, None
+    t0 = time.perf_counter()
+    try:
+        parity.check(Q, K, V, dO, cfg, kint.PREC_TF32, heads_per_chunk=12, report=rep, case="bench")
+    except AssertionError as e:
+        err = str(e)[:400]
+    keys = ("flip_fraction", "bins_flips", "ivals_flips", "valid", "arg_max_flips", "errors", "p99_rel",
+            "zero_sum_gpu", "zero_sum_oracle", "band")
+    out = {"passed": err is None, "tol": parity.TOL[kint.PREC_TF32], "prec": "tf32",
+           "oracle": "fp64 CPU oracle on the whole workload, 12 heads per chunk, decision-aligned",
+           "seconds": time.perf_counter() - t0, **{k: rep.get(k) for k in keys}}
+    if err:
+        out["failure"] = err
+    return out
+
+
+def cublas_tf32_tflops(dev, n=8192, reps=10):
+    """cuBLAS fp32 GEMM with TF32 tensor cores, n^3, best of `reps` (a measured TF32 peak on
+    this GPU, beside the nominal-ratio one)."""
+    import torch
+    old = torch.backends.cuda.matmul.allow_tf32
+    torch.backends.cuda.matmul.allow_tf32 = True
+    try:
+        a = torch.randn(n, n, device=dev)
+        b = torch.randn(n, n, device=dev)
+        c = torch.empty(n, n, device=dev)
+        for _ in range(3):
+            torch.matmul(a, b, out=c)
+        best = float("inf")
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            torch.matmul(a, b, out=c)
+            e1.record()
+            torch.cuda.synchronize()
+            best = min(best, e0.elapsed_time(e1))
+        del a, b, c
+        return 2.0 * n ** 3 / (best * 1e-3) / 1e12
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = old
+
+
+# The other single-GPU workloads of the benchmark's configurations, timed like the headline
+# (inputs larger than L2, CUDA events, warm-up first): name -> shape, seed, peaked-row
+# fraction, operator, and whether the softmax comparator runs beside it.
+OTHER_CONFIGS = {
+    "1b_scale": dict(shape=(4, 16, 2048, 128), seed=3, peaked=0.05, softmax=False,
+                     variant=dict(Kint=4, calib=1, tau=8.0, recon=1, ste=0, grad=0),
+                     workload="1B-scale attention: B=4, H=16, T=2048, d=128, 5% peaked rows (+12 score); K=4, "
+                              "FWM tau=8, Nearest, Weight-STE, full; TF32"),
+    "long_context": dict(shape=(1, 16, 16384, 128), seed=4, peaked=0.0, softmax=True,
+                         variant=dict(Kint=16, calib=0, tau=8.0, recon=0, ste=1, grad=0),
+                         workload="long context: B=1, H=16, T=16384, d=128; K=16, MinMax, LERP, Prob-STE, full; "
+                                  "TF32"),
+}
+
+
 def run_reference(args, world, rank):
     """The oracle as the reference arm, on a bounded sample per step."""
     if rank != 0:
@@ -449,12 +512,57 @@ def run_cuda(args, world, rank, local):
                    "copies_only_ms_per_step": ms_link, "link_bound_frac": ms_link / ms_e2e}
     kint.check_status()
 
+    # the other configurations' workloads, one at a time (their inputs replace these)
+    del sets, O, grads, st, ws_f, ws_b, ins, outs, pin_in, pin_out
+    torch.cuda.empty_cache()
+    if not args.headline_only:
+        line["other_configs"] = {}
+        for name, spec in OTHER_CONFIGS.items():
+            B2, H2, T2, d2 = spec["shape"]
+            Q2, K2, V2, dO2 = (torch.from_numpy(x).to(dev) for x in
+                               make_qkvdo(B2, H2, T2, d2, seed=spec["seed"], peaked_frac=spec["peaked"]))
+            O2 = torch.empty_like(Q2)
+            g2 = tuple(torch.empty_like(Q2) for _ in range(3))
+            c2 = kint.Config(**spec["variant"])
+            st2 = kint.alloc_rowstats(B2, H2, T2, d2, dev, c2.prob)
+            wf2 = kint.workspace(B2, H2, T2, d2, prec, 0, dev)
+            wb2 = kint.workspace(B2, H2, T2, d2, prec, 1, dev)
+
+            def step2(i, c=c2):
+                kint.forward(Q2, K2, V2, c, prec, O=O2, stats=st2, ws=wf2)
+                kint.backward(Q2, K2, V2, O2, dO2, st2, c, prec, grads=g2, ws=wb2)
+
+            for i in range(3):
+                step2(i)
+            n2 = 5 if T2 <= 4096 else 3
+            ms2 = timed(n2, step2)
+            f2 = 6 * unit_flops(B2, H2, T2, d2)
+            rec = {"workload": spec["workload"], "value": job_value(f2, world, ms2), "unit": UNIT,
+                   "ms_per_step": ms2, "steps": n2, "warmup": 3, "tf32_peak_frac": f2 / (ms2 * 1e-3) / 1e12 / tf32_peak,
+                   "l2": "inputs larger than the 129 MB L2 (one input set)"}
+            if spec["softmax"]:
+                for i in range(3):
+                    step2(i, soft)
+                ms_s = timed(n2, lambda i: step2(i, soft))
+                rec["softmax_comparator"] = {"value": job_value(f2, world, ms_s), "unit": UNIT, "ms_per_step": ms_s}
+            kint.check_status()
+            line["other_configs"][name] = rec
+            del Q2, K2, V2, dO2, O2, g2, st2, wf2, wb2
+            torch.cuda.empty_cache()
+    # a measured TF32 tensor peak on this GPU (cuBLAS), beside the nominal-ratio denominator
+    tf32_meas = cublas_tf32_tflops(dev)
+    roof["cublas_tf32_measured"] = tf32_meas
+    roof["frac_of_cublas_tf32"] = roof["achieved"] / tf32_meas if roof["unit"] == "TFLOP/s" else None
+    line["tf32_peak_frac_of_cublas"] = value / world / tf32_meas
+
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         heads = SHAPE["B"] * SHAPE["H"]
         rate, dt, threads, reps = cpu_oracle_rate(heads, min_seconds=10.0)
         line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
                                 "sample": f"the whole workload ({heads} (b,h) heads at T=1024, fwd+bwd) x {reps}, "
                                           f"fp64 oracle, {dt:.1f} s wall on {threads} threads"}
+        # the same oracle checks the timed workload's outputs (outside the timed region)
+        line["parity"] = bench_parity(Qh, Kh, Vh, dOh)
     if rank == 0:
         print(json.dumps(line), flush=True)
     return 0
@@ -467,6 +575,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--headline-only", action="store_true", help="skip the other configurations' lines")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world, rank, local = dist_setup(args.gpus)

@@ -122,6 +122,17 @@ typedef struct {
                         detach, detach_proj and for softmax */
   float* c_m;        /* optional side output of kint_attn_bwd: c_m = sum_j gamma_j dw_j/dm
                         (MinMax; 0 otherwise) */
+  /* Optional side outputs of kint_attn_bwd (NULL: not written), [B,H,T] each: the row sums
+   * sum_j dS_ij (dS_sum) and sum_j |dS_ij| (dS_abs) of the score gradient that the dK
+   * contraction uses, extremum terms, tie split and the P1 projection included.  Eq. (full)
+   * makes sum_j dS_ij zero in exact arithmetic in every full mode (the three per-key terms
+   * cancel, Sec. 3 after Eq. full); the detached mode breaks it (App. B "Detach (legacy)").
+   * |dS_sum| / dS_abs per row is the zero-sum residual of the paper's gradient-consistency
+   * diagnostics.  Accumulated with fp32 atomics in an order that is not fixed; the call
+   * zeroes them first.  Either may be NULL; giving one selects a slower diagnostic variant
+   * of the dK/dV kernel.  16-byte aligned. */
+  float* dS_sum;
+  float* dS_abs;
 } kint_rowstats;
 
 /*
@@ -226,6 +237,19 @@ const char* kint_strerror(int code);
 void kint_set_wait_timeout_ns(unsigned long long ns);
 
 /*
+ * Test hook of the bounded waits (the paper has no counterpart).  The next `count`
+ * calls that run the row-statistics pass (kint_attn_fwd, kint_attn_fwd_noalloc,
+ * kint_attn_debug_bins, kint_attn_probe) make that kernel's first wait, which comes
+ * before it issues any copy or product, wait on a barrier that nothing completes.  The
+ * wait gives up after the kint_set_wait_timeout_ns limit: the kernel sets bit 4 (CTA
+ * sync timed out) in the status word, releases its tensor memory and leaves, so
+ * kint_get_status then returns KINT_ERR_DEVICE and the context stays usable.  The
+ * outputs of such a call are not defined.  Nothing faults, traps or hangs.  count <= 0
+ * cancels pending requests.  Process-wide.
+ */
+void kint_test_expire_next_wait(int count);
+
+/*
  * Launch tracing (a profiling aid with no counterpart in the paper).  When set,
  * cb(kernel_name, phase, stream, user) is called on the host immediately before
  * (phase 0) and after (phase 1) every kernel launch this library makes, with
@@ -251,7 +275,10 @@ void kint_set_launch_callback(kint_launch_cb cb, void* user);
  *     array's device address; make that first call before any stream capture.
  *   - Problems whose forward workspace, kint_attn_workspace_bytes(..., 0),
  *     exceeds KINT_NOALLOC_SCRATCH_BYTES return KINT_ERR_SCRATCH_LIMIT before
- *     any work is enqueued (TF32 at d = 64 fits B*H*T up to 131072).
+ *     any work is enqueued.  That workspace is B*H*d*round_up(T, 32)*4 bytes in
+ *     TF32 (so at d = 64 the limit is B*H*round_up(T, 32) <= 131072) and about
+ *     four times as much in 3xTF32; compare kint_attn_workspace_bytes(..., 0)
+ *     with KINT_NOALLOC_SCRATCH_BYTES to know in advance.
  *   - All calls share the one array: calls whose work overlaps on the GPU
  *     (different streams, or concurrent host threads) race and must be
  *     serialised by the caller.  The array keeps the previous call's contents;

@@ -6,6 +6,7 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include <cuda.h>
@@ -30,6 +31,7 @@ unsigned* g_status_ptr[kMaxDevices] = {nullptr};
 int g_dev_ok[kMaxDevices] = {0};  // 0 unknown, 1 sm_103, -1 other
 int g_num_sms[kMaxDevices] = {0};
 unsigned long long g_wait_ns = 2000000000ull;
+std::atomic<int> g_expire_waits{0};  // test hook: forward calls whose first kernel's first wait runs out
 constexpr int kSmemLimit = 232448;  // opt-in maximum per CTA on sm_103
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
@@ -226,7 +228,7 @@ int plan_stats(Params& p) {
   p.sm_stage_bytes = parts * tile;
   p.nstage = 2;
   p.sm_rows = p.sm_stage0 + p.nstage * p.sm_stage_bytes;  // the 6 x 128 exchange words
-  const int total = finish_plan(p, p.sm_rows + 6 * 128 * 4, 6 + 2 * p.nstage);
+  const int total = finish_plan(p, p.sm_rows + 6 * 128 * 4, 8 + 2 * p.nstage);
   // CTAs loop over the items, as many as are resident at once (two per SM when they fit)
   const int per_sm = (2 * total <= 228 * 1024) ? 2 : 1;
   p.ngrid = std::min(p.nitems, per_sm * num_sms());
@@ -244,7 +246,7 @@ int plan_probe(Params& p) {
   p.nstage = 2;
   p.sm_rows = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
   p.sm_table = p.sm_rows + 8 * 128 * 4;
-  const int total = finish_plan(p, p.sm_table + 2 * 128 * (p.Kint + 2) * 4, 6 + 2 * p.nstage);
+  const int total = finish_plan(p, p.sm_table + 2 * 128 * (p.Kint + 2) * 4, 7 + 2 * p.nstage);
   p.ngrid = std::min(p.nitems, num_sms());
   return total;
 }
@@ -271,7 +273,7 @@ int plan_main(Params& p, int mode) {
       p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
       p.sm_ostage = persist ? round_up(p.sm_table + table, 1024) : p.sm_stage0;
       const int end = persist ? p.sm_ostage + ostage : p.sm_table + table;
-      const int total = std::max(finish_plan(p, end, 9 + 2 * p.nstage), kOneCtaPerSm);
+      const int total = std::max(finish_plan(p, end, 10 + 2 * p.nstage), kOneCtaPerSm);
       if (total <= kSmemLimit) {
         // Issuing S(kb+1) before P V(kb) needs tile kb+1 in a second stage while
         // tile kb's V^T is still being read; with one stage the two would wait on
@@ -306,7 +308,7 @@ int plan_dq(Params& p) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
     p.sm_ostage = 0;
-    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 3 * p.nstage + 10), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 3 * p.nstage + 11), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       p.ngrid = std::min(p.nitems, num_sms());
@@ -335,7 +337,7 @@ int plan_dkdv(Params& p, int sel) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     // FWM Nearest: the half-bin table, 2K + 3 entries of 8 bytes
     const int table = (p.calib == KINT_CALIB_FWM || p.calib == KINT_CALIB_FWM_RESOLVED) ? 2048 : 1024;
-    const int total = std::max(finish_plan(p, p.sm_table + table, 4 * p.nstage + 8), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_table + table, 4 * p.nstage + 9), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       // one CTA per SM looping over the (key block, head) items
@@ -400,6 +402,11 @@ int forward_prologue(const float* Q, const float* K, const float* V, const Param
   if (!ok) return KINT_ERR_LAUNCH;
   Params ps = p;
   const int smem = plan_stats(ps);
+  // test hook of the bounded waits: consume one pending request
+  int pending = g_expire_waits.load();
+  while (pending > 0 && !g_expire_waits.compare_exchange_weak(pending, pending - 1)) {
+  }
+  ps.expire_wait = pending > 0 ? 1 : 0;
   return launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem, s); }));
 }
 
@@ -412,6 +419,7 @@ int check_stats(const kint_rowstats* st, bool prob) {
     if (!aligned16(q)) return KINT_ERR_ALIGN;
   if (prob && (!aligned16(st->W_lerp) || !aligned16(st->O_lerp))) return KINT_ERR_ALIGN;
   if ((st->c_M && !aligned16(st->c_M)) || (st->c_m && !aligned16(st->c_m))) return KINT_ERR_ALIGN;
+  if ((st->dS_sum && !aligned16(st->dS_sum)) || (st->dS_abs && !aligned16(st->dS_abs))) return KINT_ERR_ALIGN;
   return KINT_OK;
 }
 
@@ -428,11 +436,41 @@ void set_stats(Params& p, const kint_rowstats* st) {
   p.n_max = st->n_max; p.n_min = st->n_min;
   p.W = st->W; p.W_lerp = st->W_lerp; p.O_lerp = st->O_lerp;
   p.cM_out = st->c_M; p.cm_out = st->c_m;
+  p.dsum_out = st->dS_sum; p.dabs_out = st->dS_abs;
 }
 
 bool is_prob(const Common& c) {
   return c.calib != KINT_CALIB_SOFTMAX && c.calib != KINT_CALIB_EXP_FP8 && c.calib != KINT_CALIB_EXP_BF16 &&
          c.recon == KINT_RECON_NEAREST && c.ste == KINT_STE_PROB;
+}
+
+// The forward's launches once the arguments are checked and the scratch memory is known
+// (the caller's workspace, or the library's fixed array): operand prep and pass 1, then
+// pass 2 (and, for 3xTF32 Prob-STE, its second launch for O_lerp and W_lerp).
+int forward_launches(const float* Q, const float* K, const float* V, float* O, const kint_rowstats* st,
+                     const Common& c, unsigned* status, void* scratch, cudaStream_t s) {
+  const bool prob = is_prob(c);
+  Params p = base_params(c, status);
+  set_stats(p, st);
+  p.Q = Q; p.K = K; p.V = V; p.Out = O;
+  const Workspace w = plan_workspace(static_cast<char*>(scratch), p.BH, c.T, c.d, p.x3 != 0, false);
+  Maps maps;
+  int rc = forward_prologue(Q, K, V, p, w, maps, s);
+  if (rc) return rc;
+  if (!map_fwd_outputs(maps, p)) return KINT_ERR_LAUNCH;
+  Params pm = p;
+  pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
+  const int smem = plan_main(pm, pm.pv_sel);
+  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
+  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
+  if (prob && p.x3) {
+    Params pl = p;
+    pl.pv_sel = PV_LERP;
+    const int smem2 = plan_main(pl, PV_LERP);
+    if (smem2 < 0) return KINT_ERR_UNSUPPORTED;
+    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s); })))) return rc;
+  }
+  return KINT_OK;
 }
 
 }  // namespace
@@ -464,29 +502,7 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
   if (!aligned16(workspace)) return KINT_ERR_ALIGN;
   unsigned* status = nullptr;
   if ((rc = device_setup(&status))) return rc;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-
-  Params p = base_params(c, status);
-  set_stats(p, st);
-  p.Q = Q; p.K = K; p.V = V; p.Out = O;
-  const Workspace w = plan_workspace(static_cast<char*>(workspace), p.BH, T, d, p.x3 != 0, false);
-  Maps maps;
-  if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
-  if (!map_fwd_outputs(maps, p)) return KINT_ERR_LAUNCH;
-
-  Params pm = p;
-  pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
-  const int smem = plan_main(pm, pm.pv_sel);
-  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
-  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
-  if (prob && p.x3) {
-    Params pl = p;
-    pl.pv_sel = PV_LERP;
-    const int smem2 = plan_main(pl, PV_LERP);
-    if (smem2 < 0) return KINT_ERR_UNSUPPORTED;
-    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s); })))) return rc;
-  }
-  return KINT_OK;
+  return forward_launches(Q, K, V, O, st, c, status, workspace, static_cast<cudaStream_t>(stream));
 }
 
 int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O, const float* dO,
@@ -522,6 +538,9 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   p.gbar = w.gbar;
   p.nqt = (T + 63) / 64;
   if (cudaMemsetAsync(p.tileflags, 0, (size_t)BH * p.nqt * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+  // the optional per-row dS sums are accumulated by the dK/dV pass
+  if (p.dsum_out && cudaMemsetAsync(p.dsum_out, 0, (size_t)BH * T * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+  if (p.dabs_out && cudaMemsetAsync(p.dabs_out, 0, (size_t)BH * T * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
 
   // Operand copies: K-major transposes (and 3xTF32 splits).
   PrepList pl;
@@ -693,6 +712,8 @@ const char* kint_strerror(int code) {
 
 void kint_set_wait_timeout_ns(unsigned long long ns) { g_wait_ns = ns < 1000ull ? 1000ull : ns; }
 
+void kint_test_expire_next_wait(int count) { g_expire_waits.store(count > 0 ? count : 0); }
+
 void kint_set_launch_callback(kint_launch_cb cb, void* user) {
   g_cb_user = user;
   g_cb = cb;
@@ -747,28 +768,7 @@ int kint_attn_fwd_noalloc(const float* Q, const float* K, const float* V, float*
   if ((rc = device_setup(&status))) return rc;
   void* scratch = nullptr;
   if ((rc = noalloc_scratch(&scratch))) return rc;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-
-  Params p = base_params(c, status);
-  set_stats(p, st);
-  p.Q = Q; p.K = K; p.V = V; p.Out = O;
-  const Workspace w = plan_workspace(static_cast<char*>(scratch), p.BH, T, d, p.x3 != 0, false);
-  Maps maps;
-  if ((rc = forward_prologue(Q, K, V, p, w, maps, s))) return rc;
-  if (!map_fwd_outputs(maps, p)) return KINT_ERR_LAUNCH;
-  Params pm = p;
-  pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
-  const int smem = plan_main(pm, pm.pv_sel);
-  if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
-  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
-  if (prob && p.x3) {
-    Params pl = p;
-    pl.pv_sel = PV_LERP;
-    const int smem2 = plan_main(pl, PV_LERP);
-    if (smem2 < 0) return KINT_ERR_UNSUPPORTED;
-    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s); })))) return rc;
-  }
-  return KINT_OK;
+  return forward_launches(Q, K, V, O, st, c, status, scratch, static_cast<cudaStream_t>(stream));
 }
 
 }  // extern "C"

@@ -100,6 +100,41 @@ struct RingPos {
   }
 };
 
+// Clean-up before a kernel leaves (also after a wait ran out): the last n loads issued
+// into a ring of NS stages, `next` being the ring position of the load that would come
+// next, have landed, so no copy still writes into shared memory.  Each of those loads was
+// the last one into its stage, so waiting on the parity of its phase returns at once when
+// it completed long ago.  Bounded like every wait; warp-collective.
+__device__ __forceinline__ void drain_ring(uint64_t* bar_full, RingPos next, int n, int NS, uint64_t timeout_ns,
+                                           unsigned* status) {
+  for (int k = 1; k <= n && k <= NS; ++k) {
+    int i = next.i - k;
+    uint32_t ph = next.ph;
+    if (i < 0) {  // the previous lap of the ring (k <= NS: at most one wrap)
+      i += NS;
+      ph ^= 1u;
+    }
+    mbar_wait_warp(&bar_full[i], ph, timeout_ns, status, DEV_ERR_TIMEOUT_TMA);
+  }
+}
+// Clean-up of an MMA-issuing warp: every tcgen05.mma it issued has completed (one commit
+// onto `bar`, a barrier used for nothing else, whose first phase counts `arrivals` such
+// commits), so the TMEM they write can be released.  Bounded; warp-collective.
+__device__ __forceinline__ void drain_mma(uint64_t* bar, uint64_t timeout_ns, unsigned* status) {
+  mma_commit(bar);
+  mbar_wait_warp(bar, 0, timeout_ns, status, DEV_ERR_TIMEOUT_MMA);
+}
+
+// Test hook of the bounded waits (Params::expire_wait): thread 0 waits on `bar`, a
+// barrier nothing ever arrives at, until the wait limit runs out and flags the status
+// word; the whole CTA learns of it and skips its work (nothing has been issued yet, so
+// nothing is in flight).  Returns true when the CTA must skip.
+__device__ __forceinline__ bool expire_first_wait(const Params& p, uint64_t* bar) {
+  bool ok = true;
+  if (p.expire_wait && threadIdx.x == 0) ok = mbar_wait(bar, 0, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC);
+  return p.expire_wait ? cta_any(!ok) : false;
+}
+
 // n-th work item of this CTA when the grid loops over items sorted longest first:
 // rounds of gridDim.x items taken in alternating directions (CTA 0 takes the longest
 // item of even rounds and the shortest of odd ones), which evens out the per-CTA

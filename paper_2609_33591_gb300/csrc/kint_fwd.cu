@@ -211,7 +211,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   uint64_t* bar_s = bars + 1 + 2 * NS;      // [2] S_b computed
   uint64_t* bar_sfree = bars + 3 + 2 * NS;  // [2] S_b read by every compute warp
   uint64_t* bar_qfree = bars + 5 + 2 * NS;  // the item's last product complete: Q may be reloaded
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 6 + 2 * NS);
+  uint64_t* bar_never = bars + 6 + 2 * NS;  // nothing arrives (test hook of the bounded waits)
+  uint64_t* bar_drain = bars + 7 + 2 * NS;  // the MMA warp's clean-up commit
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 8 + 2 * NS);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [6][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
 
@@ -226,6 +228,8 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
       mbar_init(&bar_sfree[b], NCOMP / 32);
     }
     mbar_init(bar_qfree, 1);
+    mbar_init(bar_never, 1);
+    mbar_init(bar_drain, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -238,9 +242,12 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   pdl_trigger();
   pdl_wait();  // everything below may read what the previous kernel wrote
   const uint32_t tmem = *tslot;
+  const bool skip = expire_first_wait(p, bar_never);
 
   // Work items as in pass 2: (query block, head), longest first, strided over the grid.
-  if (warp == PRODUCER_WARP) {
+  if (skip) {
+    // (the test hook's wait ran out before anything was issued)
+  } else if (warp == PRODUCER_WARP) {
     int g = 0, n = 0;
     RingPos ld;  // stage of the next K tile loaded
     bool ok = true;
@@ -262,6 +269,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
         if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
       }
     }
+    // clean-up: the last K tiles and Q tile issued have landed
+    drain_ring(bar_full, ld, g, NS, p.wait_ns, p.status);
+    if (n > 0) mbar_wait_warp(bar_q, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
   } else if (warp == MMA_WARP) {
     int g = 0, n = 0;
     RingPos cs;  // stage of the current K tile
@@ -296,6 +306,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
       }
       g += nkb;
     }
+    drain_mma(bar_drain, p.wait_ns, p.status);  // clean-up: no product still writes TMEM
   } else {
     const int row = tid & 127, cg = tid >> 7;
     int g = 0, n = 0;
@@ -552,7 +563,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   uint64_t* bar_done = bars + 6 + 2 * NS;     // every product of the item complete
   uint64_t* bar_qfree = bars + 7 + 2 * NS;    // the item's last S product complete: Q may be reloaded
   uint64_t* bar_ofree = bars + 8 + 2 * NS;    // O / O_lerp read out of TMEM by every compute warp
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 9 + 2 * NS);
+  uint64_t* bar_drain = bars + 9 + 2 * NS;    // the MMA warp's clean-up commit
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 10 + 2 * NS);
   uint8_t* ostg = sm + p.sm_ostage;
   float* xch = reinterpret_cast<float*>(ostg);  // [4][128], written before the staging tiles each item
   const int tid = threadIdx.x, warp = warp_id_uniform();
@@ -573,6 +585,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
     mbar_init(bar_done, 1);
     mbar_init(bar_qfree, 1);
     mbar_init(bar_ofree, NCOMP / 32);
+    mbar_init(bar_drain, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -616,6 +629,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
         }
       }
     }
+    // clean-up: the last K/V tiles and Q tile issued have landed
+    drain_ring(bar_full, ld, g, NS, p.wait_ns, p.status);
+    if (n > 0) mbar_wait_warp(bar_q, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     int g = 0, n = 0;
@@ -666,6 +682,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       g += nkb;
       mma_commit(bar_done);
     }
+    drain_mma(bar_drain, p.wait_ns, p.status);  // clean-up: no product still writes TMEM
   } else {
     const int row = tid & 127, cg = tid >> 7;
     const float Kf = (float)Kq;

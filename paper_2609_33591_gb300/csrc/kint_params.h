@@ -46,6 +46,7 @@ struct Params {
   float fwm_hl, fwm_b0l;  // (tau / K) log2 e and -tau log2 e (resolved grid below the window)
   float fwm_e[KMAX + 2];  // FWM grid values e^{-tau + r tau/K}, r = 0..K (host fp64 -> fp32)
   int pv_sel, dkv_sel, debug;
+  int expire_wait;  // test hook: the launch's first wait is on a barrier that nothing completes
   unsigned long long wait_ns;
   unsigned* status;
 
@@ -71,6 +72,7 @@ struct Params {
   float* tie_acc;           // [2][BH*T][d] sums of tied keys (workspace, touched only on ties)
   const float* gbar;        // [BH*T] <g>_{P*} = dO_i . O*_i (workspace, written by the dO prep)
   float *cM_out, *cm_out;   // optional [BH*T] side outputs of the backward: c_M, c_m per row
+  float *dsum_out, *dabs_out;  // optional [BH*T] side outputs of the backward: sum_j dS_ij, sum_j |dS_ij|
   float* probe;             // [7][BH*T] geometry probe outputs
   uint8_t *bins, *ivals;
 };

@@ -79,7 +79,8 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_probe(const __grid_constant__ M
   uint64_t* bar_s = bars + 1 + 2 * NS;      // [2] S_b computed
   uint64_t* bar_sfree = bars + 3 + 2 * NS;  // [2] S_b read by every compute warp
   uint64_t* bar_qfree = bars + 5 + 2 * NS;  // the item's last product complete: Q may be reloaded
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 6 + 2 * NS);
+  uint64_t* bar_drain = bars + 6 + 2 * NS;  // the MMA warp's clean-up commit
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 7 + 2 * NS);
   float* xch = reinterpret_cast<float*>(sm + p.sm_rows);  // [8][128]
   const int tid = threadIdx.x, warp = warp_id_uniform();
 
@@ -94,6 +95,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_probe(const __grid_constant__ M
       mbar_init(&bar_sfree[b], NCOMP / 32);
     }
     mbar_init(bar_qfree, 1);
+    mbar_init(bar_drain, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -129,6 +131,9 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_probe(const __grid_constant__ M
         if (p.x3) load_rows_tile(dst + tile, &maps.k_lo, &bar_full[s], D, 128, 0, kb * 128, bh);
       }
     }
+    // clean-up: the last K tiles and Q tile issued have landed
+    drain_ring(bar_full, ld, g, NS, p.wait_ns, p.status);
+    if (n > 0) mbar_wait_warp(bar_q, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
   } else if (warp == MMA_WARP) {
     int g = 0, n = 0;
     RingPos cs;
@@ -162,6 +167,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_probe(const __grid_constant__ M
       }
       g += nt;
     }
+    drain_mma(bar_drain, p.wait_ns, p.status);  // clean-up: no product still writes TMEM
   } else if (warp < NCOMP / 32) {
     const int row = tid & 127, cg = tid >> 7;
     float* hist = reinterpret_cast<float*>(sm + p.sm_table) + (size_t)(cg * 128 + row) * NB;

@@ -32,7 +32,7 @@ NOALLOC_SCRATCH_BYTES = 32 << 20
 # Every symbol include/kint_attn.h declares.
 EXPORTS = ("kint_attn_workspace_bytes", "kint_attn_fwd", "kint_attn_bwd", "kint_attn_debug_bins", "kint_attn_probe",
            "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns", "kint_set_launch_callback",
-           "kint_attn_fwd_noalloc")
+           "kint_attn_fwd_noalloc", "kint_test_expire_next_wait")
 
 LAUNCH_CB = ctypes.CFUNCTYPE(None, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p)
 
@@ -45,7 +45,7 @@ class KintError(RuntimeError):
 
 class kint_rowstats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in ("row_max", "row_min", "arg_max", "arg_min", "n_max", "n_min", "W",
-                                               "W_lerp", "O_lerp", "c_M", "c_m")]
+                                               "W_lerp", "O_lerp", "c_M", "c_m", "dS_sum", "dS_abs")]
 
 
 _lock = threading.Lock()
@@ -89,6 +89,8 @@ def load(build_if_missing: bool = True):
             lib.kint_attn_fwd_noalloc.argtypes = [vp, vp, vp, vp, ctypes.POINTER(kint_rowstats), i, i, i, i, i, i,
                                                   f, i, i, i, i, i, vp]
             lib.kint_attn_fwd_noalloc.restype = i
+            lib.kint_test_expire_next_wait.argtypes = [i]
+            lib.kint_test_expire_next_wait.restype = None
             _lib = lib
     return _lib
 
@@ -196,6 +198,10 @@ def kint_set_wait_timeout_ns(ns: int) -> None:
     load().kint_set_wait_timeout_ns(int(ns))
 
 
+def kint_test_expire_next_wait(count: int) -> None:
+    load().kint_test_expire_next_wait(int(count))
+
+
 _cb_keep = None
 
 
@@ -217,21 +223,24 @@ def kint_set_launch_callback(fn) -> None:
 
 # ---- conveniences that allocate with torch ---------------------------------------------------
 
-def alloc_rowstats(B, H, T, d, device, prob: bool, calib_sums: bool = False) -> dict:
+def alloc_rowstats(B, H, T, d, device, prob: bool, calib_sums: bool = False, row_sums: bool = False) -> dict:
     """Row statistics for one forward/backward pair.  ``calib_sums`` adds the backward's
-    optional per-row outputs c_M and c_m."""
+    optional per-row outputs c_M and c_m, ``row_sums`` its per-row sums of dS and |dS|."""
     f = dict(device=device, dtype=torch.float32)
     i = dict(device=device, dtype=torch.int32)
     st = {"row_max": torch.empty(B, H, T, **f), "row_min": torch.empty(B, H, T, **f),
           "arg_max": torch.empty(B, H, T, **i), "arg_min": torch.empty(B, H, T, **i),
           "n_max": torch.empty(B, H, T, **i), "n_min": torch.empty(B, H, T, **i), "W": torch.empty(B, H, T, **f),
-          "W_lerp": None, "O_lerp": None, "c_M": None, "c_m": None}
+          "W_lerp": None, "O_lerp": None, "c_M": None, "c_m": None, "dS_sum": None, "dS_abs": None}
     if prob:
         st["W_lerp"] = torch.empty(B, H, T, **f)
         st["O_lerp"] = torch.empty(B, H, T, d, **f)
     if calib_sums:
         st["c_M"] = torch.empty(B, H, T, **f)
         st["c_m"] = torch.empty(B, H, T, **f)
+    if row_sums:
+        st["dS_sum"] = torch.empty(B, H, T, **f)
+        st["dS_abs"] = torch.empty(B, H, T, **f)
     return st
 
 
