@@ -278,6 +278,29 @@ KERNEL_WORK = {
 }
 
 
+PROFILE_VARIANTS = {"kint": VARIANT, "softmax": dict(Kint=4, calib=2, tau=8.0, recon=0, ste=0, grad=0),
+                    "exp_fp8": dict(Kint=4, calib=4, tau=8.0, recon=0, ste=0, grad=0)}
+
+
+def profile_steps(args, dev):
+    """W + K plain fwd+bwd steps (stream launches, nothing else) of the workload with
+    B = --batch and the operator --variant: the program the ncu captures profile."""
+    import torch
+    from paper_2609_33591_gb300 import kint
+    from paper_2609_33591_gb300.inputs import make_qkvdo
+    B, H, T, d = args.batch, SHAPE["H"], SHAPE["T"], SHAPE["d"]
+    cfg = kint.Config(**PROFILE_VARIANTS[args.variant])
+    q, k, v, do = (torch.from_numpy(x).to(dev) for x in make_qkvdo(B, H, T, d, seed=1))
+    for i in range(args.warmup + args.steps):
+        O, st = kint.forward(q, k, v, cfg, kint.PREC_TF32)
+        kint.backward(q, k, v, O, do, st, cfg, kint.PREC_TF32)
+    torch.cuda.synchronize()
+    kint.check_status()
+    print(json.dumps({"profile_steps": args.warmup + args.steps, "B": B, "H": H, "T": T, "d": d,
+                      "variant": args.variant}), flush=True)
+    return 0
+
+
 def run_cuda(args, world, rank, local):
     import torch
     from paper_2609_33591_gb300 import kint
@@ -289,6 +312,8 @@ def run_cuda(args, world, rank, local):
     B, H, T, d = SHAPE["B"], SHAPE["H"], SHAPE["T"], SHAPE["d"]
     cfg = kint.Config(**VARIANT)
     prec = kint.PREC_TF32
+    if args.profile_steps:
+        return profile_steps(args, dev)
     Qh, Kh, Vh, dOh = make_qkvdo(B, H, T, d, seed=1)
     sets = []
     for _ in range(N_INPUT_SETS):
@@ -576,6 +601,10 @@ def main():
     ap.add_argument("--impl", choices=["cuda", "reference"], default="cuda")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--headline-only", action="store_true", help="skip the other configurations' lines")
+    ap.add_argument("--profile-steps", action="store_true",
+                    help="only run warmup + steps plain fwd+bwd steps (B = --batch, operator --variant) for ncu")
+    ap.add_argument("--batch", type=int, default=SHAPE["B"])
+    ap.add_argument("--variant", choices=sorted(PROFILE_VARIANTS), default="kint")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world, rank, local = dist_setup(args.gpus)
