@@ -41,11 +41,15 @@ BAND_REL = {kint.PREC_3XTF32: 16 * 2.0 ** -22, kint.PREC_TF32: 16 * 2.0 ** -11}
 # over up to T keys, against the tensor-core sums of the outputs).  The per-row dS sums
 # (the zero-sum diagnostic) are held to the same bar against the same scale.
 SUM_TOL_FACTOR = 4.0
-# The BF16 exponential baseline computes its score gradient in bfloat16 (dL/dz = bf16(bf16(gamma) w)):
-# a gamma within the GPU's rounding of a bfloat16 midpoint rounds to the other neighbour, one
-# bfloat16 unit (2^-8 relative) on that key, twice at most; dQ, dK and the calibration sums are
-# held to that, 2^-7 normwise.
-BF16_GRAD_TOL = 2.0 ** -7
+# The BF16 exponential baseline computes its score gradient in bfloat16 (dL/dz = bf16(bf16(gamma) w)).
+# Each backward kernel forms gamma from its own recomputed scores and rounds it, so a gamma within the
+# fp32 error of a bfloat16 rounding midpoint may round to the other neighbour (one bfloat16 unit,
+# 2^-8 of that key's dS) in either kernel, independently; no decision dump can align the oracle with
+# both.  In TF32 these flips hide under the 5e-3 bar; in 3xTF32 gamma's error is ~2^-20 relative, so a
+# flip needs gamma within ~2^-20 of a midpoint (about one key in 2^11) and moves one term of a dQ or dK
+# row by at most 2^-8 of itself: dQ, dK and the row sums are held to 2^-14 there (measured: 2-3e-5 at
+# T = 300).
+BF16_GRAD_TOL_X3 = 2.0 ** -14
 P99_FLOOR = 1e-3  # elementwise relative errors are taken against max(|ref|, P99_FLOOR * max |ref|)
 
 
@@ -258,7 +262,8 @@ def check(Q, K, V, dO, cfg: kint.Config, prec, *, want_bwd=True, tol=None, repor
         report.update(rep)
     for n, e in errs.items():
         t = tol * SUM_TOL_FACTOR if n in ("c_M", "c_m", "dS_sum") else tol
-        if cfg.calib == kint.CALIB_EXP_BF16 and n in ("dQ", "dK", "c_M", "c_m", "dS_sum", "dS_abs"):
-            t = max(t, BF16_GRAD_TOL)
+        if cfg.calib == kint.CALIB_EXP_BF16 and prec == kint.PREC_3XTF32 and \
+                n in ("dQ", "dK", "c_M", "c_m", "dS_sum", "dS_abs"):
+            t = max(t, BF16_GRAD_TOL_X3)
         assert e <= t, f"{n}: normwise error {e:.3g} > {t:g} ({rep})"
     return rep

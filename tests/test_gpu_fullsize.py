@@ -83,3 +83,19 @@ def test_sweep_3xtf32_k4(c, r, s, g):
     rep = parity.check(Q, K, V, dO, kint.Config(Kint=4, calib=c, tau=8.0, recon=r, ste=s, grad=g), X3,
                        heads_per_chunk=CHUNK)
     _zero_sum_bar(rep, g)
+
+
+@pytest.mark.parametrize("c,r,s", [(FW, NE, WE), (MM, NE, PR)])
+def test_head_dim_128_long_peaked_rows(c, r, s):
+    """The 1B-scale layer's heads (d = 128, T = 2048) with 5% peaked rows (one key per chosen row
+    raised by +12 in score, which pushes the rest of the row toward FWM's tail), two heads, TF32."""
+    Q, K, V, dO = make_qkvdo(1, 2, 2048, 128, seed=3, peaked_frac=0.05)
+    parity.check(Q, K, V, dO, kint.Config(Kint=4, calib=c, tau=8.0, recon=r, ste=s, grad=FU), TF,
+                 heads_per_chunk=1)
+
+
+def test_long_context_rows():
+    """The long-context operator (K = 16, MinMax, LERP, d = 128) on one head of 8192 rows, TF32:
+    the longest accumulation chains the oracle checks element by element."""
+    Q, K, V, dO = make_qkvdo(1, 1, 8192, 128, seed=4)
+    parity.check(Q, K, V, dO, kint.Config(Kint=16, calib=MM, tau=8.0, recon=LE, ste=PR, grad=FU), TF)
