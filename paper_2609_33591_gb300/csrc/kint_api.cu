@@ -33,6 +33,7 @@ int g_num_sms[kMaxDevices] = {0};
 unsigned long long g_wait_ns = 2000000000ull;
 std::atomic<int> g_expire_waits{0};  // test hook: forward calls whose first kernel's first wait runs out
 constexpr int kSmemLimit = 232448;  // opt-in maximum per CTA on sm_103
+constexpr int NCOMP_THREADS = 256;  // compute threads of the warp-specialised kernels (kint_dev.cuh NCOMP)
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -307,8 +308,9 @@ int plan_dq(Params& p) {
   for (p.nstage = 4; p.nstage >= 1; --p.nstage) {
     p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
     p.sm_rows = p.sm_table + table;
+    p.sm_rstat = p.sm_rows + 8 * 128 * 4;
     p.sm_ostage = 0;
-    const int total = std::max(finish_plan(p, p.sm_rows + 8 * 128 * 4, 3 * p.nstage + 11), kOneCtaPerSm);
+    const int total = std::max(finish_plan(p, p.sm_rstat + 9 * NCOMP_THREADS * 4, 3 * p.nstage + 11), kOneCtaPerSm);
     if (total <= kSmemLimit) {
       if (p.nstage == 1) p.nbuf = 1;
       p.ngrid = std::min(p.nitems, num_sms());

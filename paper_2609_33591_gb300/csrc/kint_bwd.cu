@@ -234,18 +234,19 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
     int gt = 0, n = 0;
     RingPos ld;  // stage of the next tile loaded
     bool ok = true;
+    // Q / dO of this CTA's k-th item into the staging area (TF32 at d = 64)
+    int staged = 0;  // staging loads issued
+    auto stage_ops = [&](int k) {
+      const int it_ = snake_item(k), qb_ = p.nqb - 1 - it_ / p.BH, bh_ = it_ % p.BH;
+      mbar_arrive_expect_tx(bar_stg, 2 * 128 * D * 4);
+      load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb_ * 128, bh_);
+      load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb_ * 128, bh_);
+      staged = k + 1;
+    };
+    if (p.ops_smem && snake_item(0) < p.nitems) stage_ops(0);
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH;
       const int nkt = min(2 * qb + 2, (p.T + BT - 1) / BT);
-      if (p.ops_smem) {
-        // the staging tiles of the previous item have been copied into TMEM
-        if (n > 0 && !mbar_wait_warp(bar_ops, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-        // the dQ tile of item n - 2, staged in this area since, leaves first
-        if (n >= 2 && !store_staged_dq(maps, p, bar_ostg, n - 2, sm + p.sm_a)) break;
-        mbar_arrive_expect_tx(bar_stg, 2 * 128 * D * 4);
-        load_rows_tile_boxed(sm + p.sm_a, &maps.q, bar_stg, D, 128, BT, 0, qb * 128, bh);
-        load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.dout, bar_stg, D, 128, BT, 0, qb * 128, bh);
-      }
       for (int kt = 0; kt < nkt; ++kt, ++gt, ld.next(NS)) {
         const int s = ld.i;
         if (gt >= NS && !mbar_wait_warp(&bar_emptyA[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
@@ -267,6 +268,18 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
         }
         load_rows_tile(dst + 2 * parts * ktile, &maps.kt, b, BT, D, kt * BT, 0, bh);
         if (p.x3) load_rows_tile(dst + 2 * parts * ktile + ktile, &maps.kt_lo, b, BT, D, kt * BT, 0, bh);
+        // The next item's Q / dO, as soon as the stage ring holds this item's first tiles: it needs
+        // this item's Q / dO copied out into TMEM and the previous item's dQ tile, staged in the
+        // same area since, stored; both happen at the end of the previous item, so the load has
+        // this whole item to land.
+        if (p.ops_smem && kt == min(nkt, NS) - 1 && snake_item(n + 1) < p.nitems) {
+          if (!mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) ||
+              (n >= 1 && !store_staged_dq(maps, p, bar_ostg, n - 1, sm + p.sm_a))) {
+            ok = false;
+            break;
+          }
+          stage_ops(n + 1);
+        }
       }
     }
     // the last-but-one item's tile (the last item's is stored by the compute warps)
@@ -274,7 +287,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
     tma_store_wait_all();
     // clean-up: the last tiles issued have landed
     drain_ring(bar_full, ld, gt, NS, p.wait_ns, p.status);
-    if (p.ops_smem && n > 0) mbar_wait_warp(bar_stg, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+    if (staged > 0) mbar_wait_warp(bar_stg, (staged - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
   } else if (warp == MMA_WARP) {
     // S, g of every tile, into score buffer b once the dQ product that read the buffer's
     // previous dS has completed (bar_dqdone)
@@ -359,22 +372,40 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
       float M = 0.f, m = 0.f, Wf = 1.f, Ws = 1.f, Dg = 0.f;
       int nmax = 1, nmin = 1, amax = 0, amin = 0;
     };
-    auto load_row_stats = [&](int n) {
-      RowIn r;
+    // They arrive by asynchronous copies into this thread's slot of a [9][NCOMP] word array,
+    // issued at the start of the previous item, so their latency hides under its tiles.
+    const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && !gridless(CAL));
+    const uint32_t rslot = smem_u32(sm + p.sm_rstat) + 4u * (uint32_t)tid;
+    auto prefetch_row_stats = [&](int n) {
       const int item = snake_item(n);
       const int i = (p.nqb - 1 - item / p.BH) * 128 + row;
       if (i < p.T) {
         const size_t rw = (size_t)(item % p.BH) * p.T + i;
-        r.M = p.row_max[rw];
-        r.m = p.row_min[rw];
-        r.Wf = p.W[rw];
-        r.nmax = p.n_max[rw];
-        r.nmin = p.n_min[rw];
-        r.amax = p.arg_max[rw];
-        r.amin = p.arg_min[rw];
-        r.Dg = p.gbar[rw];  // <g>_{P*} = dO_i . O*_i
-        const bool prob = (p.recon == REC_NEAREST && p.ste == 1 && !gridless(CAL));
-        r.Ws = prob ? p.W_lerp[rw] : r.Wf;
+        const void* src[9] = {p.row_max + rw, p.row_min + rw, p.W + rw, p.n_max + rw, p.n_min + rw,
+                              p.arg_max + rw, p.arg_min + rw, p.gbar + rw, (prob ? p.W_lerp : p.W) + rw};
+#pragma unroll
+        for (int k = 0; k < 9; ++k)
+          asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(rslot + (uint32_t)k * 4u * NCOMP),
+                       "l"(src[k])
+                       : "memory");
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    auto load_row_stats = [&](int n) {
+      RowIn r;
+      const int item = snake_item(n);
+      const int i = (p.nqb - 1 - item / p.BH) * 128 + row;
+      asm volatile("cp.async.wait_all;" ::: "memory");
+      if (i < p.T) {
+        r.M = lds_f32(rslot);
+        r.m = lds_f32(rslot + 4u * NCOMP);
+        r.Wf = lds_f32(rslot + 8u * NCOMP);
+        r.nmax = __float_as_int(lds_f32(rslot + 12u * NCOMP));
+        r.nmin = __float_as_int(lds_f32(rslot + 16u * NCOMP));
+        r.amax = __float_as_int(lds_f32(rslot + 20u * NCOMP));
+        r.amin = __float_as_int(lds_f32(rslot + 24u * NCOMP));
+        r.Dg = lds_f32(rslot + 28u * NCOMP);  // <g>_{P*} = dO_i . O*_i
+        r.Ws = lds_f32(rslot + 32u * NCOMP);
       }
       return r;
     };
@@ -383,6 +414,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
     bool failed = false;
     RowIn nx;
     if (snake_item(0) < p.nitems) {
+      prefetch_row_stats(0);
       ops_to_tmem(0);
       nx = load_row_stats(0);
     }
@@ -395,6 +427,7 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
       const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
       const float M = nx.M, m = nx.m, Wf = nx.Wf, Ws = nx.Ws, Dg = nx.Dg;
       const int nmax = nx.nmax, nmin = nx.nmin, amax = nx.amax, amin = nx.amin;
+      if (snake_item(n + 1) < p.nitems) prefetch_row_stats(n + 1);  // (the slot was just read)
       const RowGrid g = row_grid(p, M, m);
       if constexpr (fwm_like(CAL)) {  // the same for every item
         if (n == 0 && tid < 2 * Kq + 1 + kHalfTail)

@@ -276,18 +276,19 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     RingPos nf, nT;  // ring positions after the last first-half and transposed-half loads issued
     int cf = 0, cT = 0;  // how many of each were issued
     bool ok = true;
+    // K / V of this CTA's k-th item into the staging area (TF32 at d = 64)
+    int staged = 0;  // staging loads issued
+    auto stage_ops = [&](int k) {
+      const int it_ = snake_item(k), kb_ = it_ / p.BH, bh_ = it_ % p.BH;
+      mbar_arrive_expect_tx(bar_stg, (needV ? 2 : 1) * 128 * D * 4);
+      load_rows_tile_boxed(sm + p.sm_a, &maps.k, bar_stg, D, 128, BT, 0, kb_ * 128, bh_);
+      if (needV) load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.v, bar_stg, D, 128, BT, 0, kb_ * 128, bh_);
+      staged = k + 1;
+    };
+    if (p.ops_smem && snake_item(0) < p.nitems) stage_ops(0);
     for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
-      if (p.ops_smem) {
-        // the staged K / V of the previous item have been copied into TMEM
-        if (n > 0 && !mbar_wait_warp(bar_ops, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
-        // the dV / dK tiles of item n - 2, staged in this area since, leave first
-        if (n >= 2 && !store_staged_dkdv(maps, p, bar_ostg, n - 2, sm + p.sm_a, doDV, doDK)) break;
-        mbar_arrive_expect_tx(bar_stg, (needV ? 2 : 1) * 128 * D * 4);
-        load_rows_tile_boxed(sm + p.sm_a, &maps.k, bar_stg, D, 128, BT, 0, kb * 128, bh);
-        if (needV) load_rows_tile_boxed(sm + p.sm_a + 128 * D * 4, &maps.v, bar_stg, D, 128, BT, 0, kb * 128, bh);
-      }
       for (int it = 0; it < nit; ++it, ++gt, ld.next(NS)) {
         const int s = ld.i, q0 = (qt0 + it) * BT;
         if (gt >= NS && !mbar_wait_warp(&bar_emptyA[s], ld.ph ^ 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
@@ -328,6 +329,18 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
         }
         nT.next(NS);
         ++cT;
+        // The next item's K / V, as soon as the stage ring holds this item's first tiles: it needs
+        // this item's K / V copied out into TMEM and the previous item's dV / dK tiles, staged in
+        // the same area since, stored; both happen at the end of the previous item, so the load
+        // has this whole item to land.
+        if (p.ops_smem && it == min(nit, NS) - 1 && snake_item(n + 1) < p.nitems) {
+          if (!mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) ||
+              (n >= 1 && !store_staged_dkdv(maps, p, bar_ostg, n - 1, sm + p.sm_a, doDV, doDK))) {
+            ok = false;
+            break;
+          }
+          stage_ops(n + 1);
+        }
       }
     }
     // the last-but-one item's tiles (the last item's are stored by the compute warps)
@@ -336,7 +349,7 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
     // clean-up: the last tiles issued have landed
     drain_ring(bar_full, nf, cf, NS, p.wait_ns, p.status);
     drain_ring(bar_fullT, nT, cT, NS, p.wait_ns, p.status);
-    if (p.ops_smem && n > 0) mbar_wait_warp(bar_stg, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
+    if (staged > 0) mbar_wait_warp(bar_stg, (staged - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
   } else if (warp == MMA_WARP) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t cKa = tmem + cK, cVa = tmem + cV, cSG = tmem + base;

@@ -52,6 +52,7 @@ struct Params {
 
   // smem plan (byte offsets from the 1024-aligned base), set by the host
   int sm_a, sm_stage0, sm_stage_bytes, nstage, sm_table, sm_rows, sm_bars;
+  int sm_rstat;  // dQ kernel: the next item's row statistics, [9][256] words
   int nbuf;  // score buffers in TMEM (2: the next tile's product runs under this tile's element work)
   int nitems;     // work items (128-row query or key block, head), longest first
   int ngrid;      // CTAs launched: nitems, or one per SM when the kernel loops over items
