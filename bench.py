@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "3c0af8e07a6451c9", "k_prep": 82473856, "k_fwd_stats": 50369536, "k_fwd_main": 93726976,
-           "k_bwd_dq": 194415616, "k_bwd_dkdv": 274723840}
+TRAFFIC = {"src": "2760b45424ab1f5b", "k_prep": 82348576, "k_fwd_stats": 50404659, "k_fwd_main": 92283994,
+           "k_bwd_dq": 191385203, "k_bwd_dkdv": 264280154}
 
 
 def kernel_source_digest() -> str:
@@ -288,9 +288,16 @@ def profile_steps(args, dev):
     import torch
     from paper_2609_33591_gb300 import kint
     from paper_2609_33591_gb300.inputs import make_qkvdo
-    B, H, T, d = args.batch, SHAPE["H"], SHAPE["T"], SHAPE["d"]
-    cfg = kint.Config(**PROFILE_VARIANTS[args.variant])
-    q, k, v, do = (torch.from_numpy(x).to(dev) for x in make_qkvdo(B, H, T, d, seed=1))
+    if args.workload == "long":  # the long-context operator (K=16, MinMax, LERP) on --heads heads of T=16384, d=128
+        spec = OTHER_CONFIGS["long_context"]
+        B, H, T, d = 1, args.heads, spec["shape"][2], spec["shape"][3]
+        var = dict(spec["variant"]) if args.variant == "kint" else PROFILE_VARIANTS[args.variant]
+        cfg = kint.Config(**var)
+        q, k, v, do = (torch.from_numpy(x).to(dev) for x in make_qkvdo(B, H, T, d, seed=spec["seed"]))
+    else:
+        B, H, T, d = args.batch, SHAPE["H"], SHAPE["T"], SHAPE["d"]
+        cfg = kint.Config(**PROFILE_VARIANTS[args.variant])
+        q, k, v, do = (torch.from_numpy(x).to(dev) for x in make_qkvdo(B, H, T, d, seed=1))
     for i in range(args.warmup + args.steps):
         O, st = kint.forward(q, k, v, cfg, kint.PREC_TF32)
         kint.backward(q, k, v, O, do, st, cfg, kint.PREC_TF32)
@@ -605,6 +612,8 @@ def main():
                     help="only run warmup + steps plain fwd+bwd steps (B = --batch, operator --variant) for ncu")
     ap.add_argument("--batch", type=int, default=SHAPE["B"])
     ap.add_argument("--variant", choices=sorted(PROFILE_VARIANTS), default="kint")
+    ap.add_argument("--workload", choices=["gpt2", "long"], default="gpt2", help="--profile-steps workload")
+    ap.add_argument("--heads", type=int, default=8, help="--profile-steps --workload long: heads of T=16384")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world, rank, local = dist_setup(args.gpus)
