@@ -173,6 +173,13 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
  *     detach_proj);
  *   dQ = dS K / sqrt(d), dK = dS^T Q / sqrt(d), dV = P^T dO with the forward P.
  * dQ, dK, dV are overwritten.
+ * Two implementations (kint_set_backward_path): TF32 at d = 64 with any calibration but
+ * MinMax and any mode but detach_proj, and without dS_sum / dS_abs, runs a single pass
+ * over the (key block, query tile) pairs that adds its dQ partial sums, and then the
+ * extremum terms, in fp32 in global memory: the order of those additions is not fixed,
+ * so dQ (and dK under the extremum terms) may differ in the last bits from call to call.
+ * Everything else, and calls where some row has tied maxima, runs two passes (dQ, then
+ * dK/dV) whose results are bit-reproducible.
  *   O        in:  forward output
  *   dO       in:  [B,H,T,d]
  *   st       in:  row statistics written by kint_attn_fwd
@@ -248,6 +255,14 @@ void kint_set_wait_timeout_ns(unsigned long long ns);
  * cancels pending requests.  Process-wide.
  */
 void kint_test_expire_next_wait(int count);
+
+/*
+ * Backward implementation choice (process-wide; the paper has no counterpart): 0 (default)
+ * uses the single-pass backward wherever kint_attn_bwd describes it as applying, 1 always
+ * the two-pass kernels (bit-reproducible).  Other values act as 0.  Do not change it
+ * while another thread is inside an entry point.
+ */
+void kint_set_backward_path(int path);
 
 /*
  * Launch tracing (a profiling aid with no counterpart in the paper).  When set,

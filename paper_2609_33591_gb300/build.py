@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libkint.so")
-SOURCES = ["kint_api.cu", "kint_fwd.cu", "kint_bwd.cu", "kint_bwd_dkdv.cu", "kint_bwd_dkdv_rs.cu", "kint_probe.cu"]
+SOURCES = ["kint_api.cu", "kint_fwd.cu", "kint_bwd.cu", "kint_bwd_dkdv.cu", "kint_bwd_dkdv_rs.cu", "kint_bwd_fused.cu", "kint_probe.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

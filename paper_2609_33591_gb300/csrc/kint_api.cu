@@ -31,7 +31,8 @@ unsigned* g_status_ptr[kMaxDevices] = {nullptr};
 int g_dev_ok[kMaxDevices] = {0};  // 0 unknown, 1 sm_103, -1 other
 int g_num_sms[kMaxDevices] = {0};
 unsigned long long g_wait_ns = 2000000000ull;
-std::atomic<int> g_expire_waits{0};  // test hook: forward calls whose first kernel's first wait runs out
+std::atomic<int> g_expire_waits{0};
+int g_bwd_path = 0;  // 0: single-pass backward where it applies, 1: always the two-pass kernels  // test hook: forward calls whose first kernel's first wait runs out
 constexpr int kSmemLimit = 232448;  // opt-in maximum per CTA on sm_103
 constexpr int NCOMP_THREADS = 256;  // compute threads of the warp-specialised kernels (kint_dev.cuh NCOMP)
 
@@ -119,6 +120,11 @@ struct Workspace {
   float* rtab = nullptr;  // [BHT][KMAX] (e_r, e_{r+1}) MinMax grid pairs
   float* tie = nullptr;   // [2][BHT][d] sums of tied arg-extremum keys
   int* tileflags = nullptr;  // [BH][ceil(T/64)]
+  int* tie_any = nullptr;    // after tileflags (zeroed with them): the ties overflow the tie list
+  int *tie_count = nullptr, *tie_total = nullptr;  // (also zeroed with the tile flags)
+  int2* tie_list = nullptr;  // [BHT] (row, key) pairs of tied maxima (single-pass backward)
+  void* frec = nullptr;      // [BHT] 16-byte rows records of the single-pass backward
+  float* rsum = nullptr;     // [BHT] its row sums of gamma Delta
   float* gbar = nullptr;     // [BHT] <g>_{P*} = dO_i . O*_i
 };
 
@@ -150,7 +156,16 @@ Workspace plan_workspace(char* base, int BH, int T, int d, bool x3, bool bwd) {
     w.rec = take(rows * 16);
     w.rtab = take(rows * 2 * KMAX);
     w.tie = take(2 * nat);
-    w.tileflags = reinterpret_cast<int*>(take((size_t)BH * ((T + 63) / 64) * 4));
+    const size_t ntf = (size_t)BH * ((T + 63) / 64);
+    w.tileflags = reinterpret_cast<int*>(take((ntf + 4) * 4));
+    if (w.tileflags) {
+      w.tie_any = w.tileflags + ntf;
+      w.tie_count = w.tileflags + ntf + 1;
+      w.tie_total = w.tileflags + ntf + 2;
+    }
+    w.frec = take(rows * 4);
+    w.rsum = take(rows);
+    w.tie_list = reinterpret_cast<int2*>(take(rows * 2));  // one (row, key) pair per row
     w.gbar = take(rows);
   }
   w.bytes = off;
@@ -351,6 +366,28 @@ int plan_dkdv(Params& p, int sel) {
   return -1;
 }
 
+// Single-pass backward (TF32, d = 64): two stages of Q | dO | Q^T | dO^T tiles and their
+// 16-byte row records, the item's V and K^T tiles, eight 2 KB dQ reduce slices, the FWM
+// table; one CTA per SM.
+int plan_fused(Params& p) {
+  const int qtile = 64 * 64 * 4;
+  p.nstage = 2;
+  p.nbuf = 2;
+  p.ops_smem = 0;
+  p.sm_a = 0;
+  p.sm_stage0 = 0;
+  p.sm_stage_bytes = 4 * qtile + 64 * 16;
+  p.sm_v = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
+  p.sm_kt = p.sm_v + 128 * 64 * 4;
+  p.sm_ostage = p.sm_kt + 128 * 64 * 4;  // the compute warps' 2 KB dQ reduce slices
+  p.sm_table = p.sm_ostage + 8 * 2048;
+  const int total = std::max(finish_plan(p, p.sm_table + 2048, 5 * p.nstage + 13), kOneCtaPerSm);
+  if (total > kSmemLimit) return -1;
+  p.nitems = p.nqb * p.BH;
+  p.ngrid = std::min(p.nitems, num_sms());
+  return total;
+}
+
 int launch_rc(cudaError_t e) { return e == cudaSuccess ? KINT_OK : KINT_ERR_LAUNCH; }
 
 kint_launch_cb g_cb = nullptr;
@@ -539,7 +576,7 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   p.tileflags = w.tileflags;
   p.gbar = w.gbar;
   p.nqt = (T + 63) / 64;
-  if (cudaMemsetAsync(p.tileflags, 0, (size_t)BH * p.nqt * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
+  if (cudaMemsetAsync(p.tileflags, 0, ((size_t)BH * p.nqt + 3) * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
   // the optional per-row dS sums are accumulated by the dK/dV pass
   if (p.dsum_out && cudaMemsetAsync(p.dsum_out, 0, (size_t)BH * T * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
   if (p.dabs_out && cudaMemsetAsync(p.dabs_out, 0, (size_t)BH * T * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
@@ -577,6 +614,41 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   ok = ok && map_nat(&maps.dq, dQ, BH, T, d, 64) && map_nat(&maps.dk, dK, BH, T, d, 64) &&
        map_nat(&maps.dv, dV, BH, T, d, 64);
   if (!ok) return KINT_ERR_LAUNCH;
+
+  // Single-pass backward: TF32 at d = 64 on the FWM grids and the exponentials, without the
+  // P1 projection and the row-sum side outputs (those stay on the two-pass kernels).  Tied
+  // maxima are found during the pass and listed (one entry per tied key) for k_bwd_ext; when
+  // the rows hold more ties than the list has room for (one per row of the call), which
+  // k_rowrec finds out, the whole call runs the two-pass kernels instead: both sets are
+  // launched, gated on that flag.
+  const bool single = g_bwd_path == 0 && !p.x3 && d == 64 && c.calib != KINT_CALIB_MINMAX &&
+                      c.grad != KINT_GRAD_DETACH_PROJ && !p.dsum_out && !p.dabs_out;
+  if (single) {
+    Params pf = p;
+    pf.frec = w.frec;
+    pf.rsum = w.rsum;
+    pf.tie_any = w.tie_any;
+    pf.tie_count = w.tie_count;
+    pf.tie_total = w.tie_total;
+    pf.tie_list = w.tie_list;
+    pf.tie_cap = BH * T;
+    const bool ext = c.calib != KINT_CALIB_SOFTMAX && c.grad != KINT_GRAD_DETACH;
+    if (!map_nat(&maps.dq16, dQ, BH, T, d, 16) || !map_nat(&maps.dk32, dK, BH, T, d, 32) ||
+        !map_nat(&maps.dv32, dV, BH, T, d, 32))
+      return KINT_ERR_LAUNCH;
+    if ((rc = launch_rc(traced("k_rowrec", s, [&] { return launch_rowrec(pf, num_sms(), s); })))) return rc;
+    const int smem_f = plan_fused(pf);
+    if (smem_f < 0) return KINT_ERR_UNSUPPORTED;
+    if (ext) {
+      pf.gate = w.tie_any;
+      pf.gate_on = 0;
+    }
+    if ((rc = launch_rc(traced("k_bwd_fused", s, [&] { return launch_bwd_fused(maps, pf, smem_f, s); })))) return rc;
+    if (!ext) return KINT_OK;
+    if ((rc = launch_rc(traced("k_bwd_ext", s, [&] { return launch_bwd_ext(pf, num_sms(), s); })))) return rc;
+    p.gate = w.tie_any;
+    p.gate_on = 1;
+  }
 
   // P1 projection: key prefix sums into the tie-sum buffer (unused by the detached modes)
   if (c.grad == KINT_GRAD_DETACH_PROJ && c.calib != KINT_CALIB_SOFTMAX)
@@ -715,6 +787,8 @@ const char* kint_strerror(int code) {
 void kint_set_wait_timeout_ns(unsigned long long ns) { g_wait_ns = ns < 1000ull ? 1000ull : ns; }
 
 void kint_test_expire_next_wait(int count) { g_expire_waits.store(count > 0 ? count : 0); }
+
+void kint_set_backward_path(int path) { g_bwd_path = path == 1 ? 1 : 0; }
 
 void kint_set_launch_callback(kint_launch_cb cb, void* user) {
   g_cb_user = user;

@@ -229,6 +229,12 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
   constexpr uint32_t tmem = 0;
+  if (gated_off(p)) {  // the single-pass backward ran instead
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+    return;
+  }
 
   if (warp == PRODUCER_WARP) {
     int gt = 0, n = 0;

@@ -266,6 +266,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
   constexpr uint32_t tmem = 0;
+  if (gated_off(p)) {  // the single-pass backward ran instead
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+    return;
+  }
 
   // Work items are (128-key block kb, head) pairs, longest first (kb = 0 meets every
   // query tile); a CTA takes the items snake_item(0), snake_item(1), ...  Tile counters

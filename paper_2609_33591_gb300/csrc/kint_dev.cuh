@@ -135,6 +135,13 @@ __device__ __forceinline__ bool expire_first_wait(const Params& p, uint64_t* bar
   return p.expire_wait ? cta_any(!ok) : false;
 }
 
+// A gated launch (Params::gate) on the side of a device-side decision that was not
+// taken: the kernel does no work.  Read after pdl_wait, so the writer of the decision
+// (an earlier kernel of the stream) has finished.
+__device__ __forceinline__ bool gated_off(const Params& p) {
+  return p.gate != nullptr && ((*reinterpret_cast<const volatile int*>(p.gate) != 0) != (p.gate_on != 0));
+}
+
 // n-th work item of this CTA when the grid loops over items sorted longest first:
 // rounds of gridDim.x items taken in alternating directions (CTA 0 takes the longest
 // item of even rounds and the shortest of odd ones), which evens out the per-CTA

@@ -46,6 +46,11 @@ cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, c
 // Geometry probe: per-row span, width, softmax entropy, share below -6, top-bucket mass,
 // effective buckets and total variation to softmax, into p.probe
 cudaError_t launch_fwd_probe(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
+// Single-pass backward (TF32, d = 64): the row records, rows sums and zeroed dQ, the
+// pass itself, and the extremum terms it leaves for afterwards
+cudaError_t launch_rowrec(const Params& p, int nsm, cudaStream_t s);
+cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
+cudaError_t launch_bwd_ext(const Params& p, int nsm, cudaStream_t s);
 // C = running sums of the key rows of every head, [BH][T][d] (the P1 projection)
 cudaError_t launch_kcum(const float* K, float* C, int BH, int T, int d, cudaStream_t s);
 

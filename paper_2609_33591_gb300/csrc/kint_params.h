@@ -36,6 +36,7 @@ struct Maps {
   CUtensorMap q, q_lo, k, k_lo, v, v_lo, dout, dout_lo;  // natural
   CUtensorMap kt, kt_lo, vt, vt_lo, qt, qt_lo, dot, dot_lo;  // transposed
   CUtensorMap out, out_lerp, dq, dk, dv;  // outputs (natural, box 32 x 64 rows) for TMA stores
+  CUtensorMap dq16, dk32, dv32;  // single-pass backward: dQ reduce boxes of 16 rows, dK / dV stores of 32
 };
 
 struct Params {
@@ -58,6 +59,11 @@ struct Params {
   int ngrid;      // CTAs launched: nitems, or one per SM when the kernel loops over items
   int sm_ostage;  // smem tile(s) the epilogue stages outputs in for TMA stores
   int ops_smem;  // backward: the 128-row TMEM operands (Q, dO / K, V) are staged in smem by TMA first
+  int sm_v, sm_kt;  // single-pass backward: the V tile (A operand of g^T) and the K^T tile (B operand of dQ)
+  // Launch gate of the backward kernels that run on one side of a device-side decision:
+  // with gate set, the kernel does its work only if (*gate != 0) == (gate_on != 0)
+  const int* gate;
+  int gate_on;
 
   // tensors (device pointers)
   const float *Q, *K, *V, *O, *dO, *Ostar;
@@ -74,6 +80,13 @@ struct Params {
   const float* gbar;        // [BH*T] <g>_{P*} = dO_i . O*_i (workspace, written by the dO prep)
   float *cM_out, *cm_out;   // optional [BH*T] side outputs of the backward: c_M, c_m per row
   float *dsum_out, *dabs_out;  // optional [BH*T] side outputs of the backward: sum_j dS_ij, sum_j |dS_ij|
+  void* frec;               // [B*H*T] 16-byte row records of the single-pass backward (k_rowrec)
+  float* rsum;              // [B*H*T] single-pass backward: sum_j gamma_ij Delta_ij per row
+  int* tie_any;             // single-pass backward: set when the rows' ties exceed the tie list
+  int* tie_count;           // single-pass backward: entries in tie_list; tie_total: the ties the rows hold
+  int* tie_total;
+  int2* tie_list;           // [tie_cap] (row, key) pairs of tied maxima found by k_bwd_fused
+  int tie_cap;
   float* probe;             // [7][BH*T] geometry probe outputs
   uint8_t *bins, *ivals;
 };

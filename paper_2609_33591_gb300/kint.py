@@ -32,7 +32,7 @@ NOALLOC_SCRATCH_BYTES = 32 << 20
 # Every symbol include/kint_attn.h declares.
 EXPORTS = ("kint_attn_workspace_bytes", "kint_attn_fwd", "kint_attn_bwd", "kint_attn_debug_bins", "kint_attn_probe",
            "kint_get_status", "kint_strerror", "kint_set_wait_timeout_ns", "kint_set_launch_callback",
-           "kint_attn_fwd_noalloc", "kint_test_expire_next_wait")
+           "kint_attn_fwd_noalloc", "kint_test_expire_next_wait", "kint_set_backward_path")
 
 LAUNCH_CB = ctypes.CFUNCTYPE(None, ctypes.c_char_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p)
 
@@ -200,6 +200,13 @@ def kint_set_wait_timeout_ns(ns: int) -> None:
 
 def kint_test_expire_next_wait(count: int) -> None:
     load().kint_test_expire_next_wait(int(count))
+
+
+BWD_AUTO, BWD_TWO_PASS = 0, 1
+
+
+def kint_set_backward_path(path: int) -> None:
+    load().kint_set_backward_path(int(path))
 
 
 _cb_keep = None

@@ -19,6 +19,7 @@ configuration, flips, errors, zero-sum residuals) to that file.
 """
 from __future__ import annotations
 
+import contextlib
 import json
 import os
 
@@ -57,11 +58,32 @@ def to_oracle_cfg(cfg: kint.Config) -> oracle.Config:
     return oracle.Config(Kint=cfg.Kint, calib=cfg.calib, tau=cfg.tau, recon=cfg.recon, ste=cfg.ste, grad=cfg.grad)
 
 
+def single_pass_applies(cfg: kint.Config, prec, d) -> bool:
+    """Whether kint_attn_bwd takes its single-pass backward for this configuration (the
+    rule stated at kint_attn_bwd in include/kint_attn.h; calls without row-sum outputs,
+    and only when no row has tied maxima)."""
+    return prec == kint.PREC_TF32 and d == 64 and cfg.calib != kint.CALIB_MINMAX and \
+        cfg.grad != kint.GRAD_DETACH_PROJ
+
+
+@contextlib.contextmanager
+def backward_path(path):
+    """Run the block with kint_set_backward_path(path), then back to the default."""
+    kint.kint_set_backward_path(path)
+    try:
+        yield
+    finally:
+        kint.kint_set_backward_path(kint.BWD_AUTO)
+
+
 def run_gpu(Q, K, V, dO, cfg: kint.Config, prec, *, want_bins=True, want_bwd=True, row_sums=None):
     """Forward, decision dump and backward on cuda:0 through the C ABI.  With
     ``row_sums`` (default: with the backward) the backward runs a second time with the
-    per-row dS sums requested (the diagnostic variant of the dK/dV kernel); its dQ, dK,
-    dV must equal those of the plain run bit for bit."""
+    per-row dS sums requested, which always runs the two-pass kernels (the diagnostic
+    variant of the dK/dV kernel).  Where the plain run took the single-pass backward, its
+    dV must equal the two-pass dV bit for bit (the same weights and products) and the
+    two-pass dQ, dK come back as dQ_2p, dK_2p for their own comparison with the oracle;
+    otherwise all three must equal those of the plain run bit for bit."""
     dev = torch.device("cuda:0")
     q, k, v, do = (torch.from_numpy(np.ascontiguousarray(x)).to(dev) for x in (Q, K, V, dO))
     B, H, T, d = q.shape
@@ -80,8 +102,12 @@ def run_gpu(Q, K, V, dO, cfg: kint.Config, prec, *, want_bins=True, want_bwd=Tru
         st2["c_M"], st2["c_m"] = None, None
         g2 = kint.backward(q, k, v, O, do, st2, cfg, prec)
         torch.cuda.synchronize()
+        single = single_pass_applies(cfg, prec, d)
         for n, t in zip(("dQ", "dK", "dV"), g2):
-            assert torch.equal(t, out[n]), f"{n}: the row-sum variant of the backward differs from the plain one"
+            if single and n != "dV":
+                out[n + "_2p"] = t
+            else:
+                assert torch.equal(t, out[n]), f"{n}: the row-sum variant of the backward differs from the plain one"
         out["dS_sum"], out["dS_abs"] = st2["dS_sum"], st2["dS_abs"]
     torch.cuda.synchronize()
     kint.check_status()
@@ -190,8 +216,9 @@ def _compare_chunk(Q, K, V, dO, g, cfg, ocfg, prec, want_bwd, cnt, acc, rho):
     if not want_bwd:
         return
     b = oracle.backward(Q, K, V, dO, ocfg, override=ov)
-    for n in ("dQ", "dK", "dV"):
-        acc[n].add(g[n], b[n])
+    for n in ("dQ", "dK", "dV", "dQ_2p", "dK_2p"):
+        if n in g:
+            acc[n].add(g[n], b[n[:2]])
     # the per-row calibration sums of Eq. (full), exactly zero where they are not formed
     scale = float(np.max(b["dabs"] + np.abs(b["cM"]) + np.abs(b["cm"]))) if b["dabs"].size else 0.0
     for n, on in (("c_M", "cM"), ("c_m", "cm")):
@@ -228,7 +255,7 @@ def check(Q, K, V, dO, cfg: kint.Config, prec, *, want_bwd=True, tol=None, repor
     BH = B * H
     step = BH if not heads_per_chunk else max(1, int(heads_per_chunk))
     names = ["O", "W"] + (["O_lerp", "W_lerp"] if cfg.prob else []) + \
-        (["dQ", "dK", "dV", "c_M", "c_m", "dS_sum", "dS_abs"] if want_bwd else [])
+        (["dQ", "dK", "dV", "dQ_2p", "dK_2p", "c_M", "c_m", "dS_sum", "dS_abs"] if want_bwd else [])
     acc = {n: _Acc() for n in names}
     cnt = dict(band=0.0, score_err=0.0, arg_max_flips=0, arg_min_flips=0, bins_flips=0, ivals_flips=0, valid=0)
     rho = {"gpu": [], "oracle": []}
@@ -263,7 +290,7 @@ def check(Q, K, V, dO, cfg: kint.Config, prec, *, want_bwd=True, tol=None, repor
     for n, e in errs.items():
         t = tol * SUM_TOL_FACTOR if n in ("c_M", "c_m", "dS_sum") else tol
         if cfg.calib == kint.CALIB_EXP_BF16 and prec == kint.PREC_3XTF32 and \
-                n in ("dQ", "dK", "c_M", "c_m", "dS_sum", "dS_abs"):
+                n in ("dQ", "dK", "dQ_2p", "dK_2p", "c_M", "c_m", "dS_sum", "dS_abs"):
             t = max(t, BF16_GRAD_TOL_X3)
         assert e <= t, f"{n}: normwise error {e:.3g} > {t:g} ({rep})"
     return rep

@@ -159,6 +159,25 @@ def test_degenerate_and_tied_rows():
         parity.check(Q * 3, Kd, V, dO, cfg, X3)
 
 
+@pytest.mark.parametrize("calib", [FW, E8])
+def test_single_pass_tied_maxima(calib):
+    """TF32 single-pass backward with a few rows whose maximum is tied (three identical
+    keys that those rows point at): the pass lists the tied keys and splits c_M over them
+    (Eq. full).  Q = 0 makes every row all-equal, more ties than the list holds: the call
+    runs the two-pass kernels instead.  Both against the oracle."""
+    Q, K, V, dO = make_qkvdo(1, 2, 140, 64, seed=31)
+    Kd = K.copy()
+    for h in range(2):
+        Kd[0, h, 5] = Kd[0, h, 2]
+        Kd[0, h, 130] = Kd[0, h, 2]
+        u = Kd[0, h, 2] / np.linalg.norm(Kd[0, h, 2])
+        for i in (10, 50, 100, 135):
+            Q[0, h, i] = (2.5 * 8.0 * u).astype(np.float32)
+    cfg = _cfg(calib, NE, PR, FU)
+    parity.check(Q, Kd, V, dO, cfg, TF)
+    parity.check(np.zeros_like(Q), K, V, dO, cfg, TF)
+
+
 def test_fwm_far_tail():
     """Scores spread far beyond tau: every key but the maximum falls in the zero tail."""
     Q, K, V, dO = make_qkvdo(1, 1, 150, 64, seed=9)
