@@ -273,13 +273,13 @@ KERNEL_WORK = {
     "k_bwd_dq": ("tensor", 2),     # dP = dO V^T, dQ = dS K
     "k_bwd_dkdv": ("tensor", 2),   # dV = P^T dO, dK = dS^T Q (S^T, dP^T are recomputations)
     "k_bwd_fused": ("tensor", 4),  # single pass: dP^T, dV, dK, dQ (S^T is a recomputation)
-    # single pass, HBM passes over [B,H,T,d] fp32: the zeroed dQ (1); the extremum terms read
-    # Q, K at the arg-max rows and dQ, write dQ and add to dK (5)
-    "k_rowrec": ("hbm", 1),
+    # single pass, HBM passes over [B,H,T,d] fp32: the extremum terms read Q, K at the arg-max
+    # rows and dQ, write dQ and add to dK (5)
     "k_bwd_ext": ("hbm", 5),
     # per launch, [B,H,T,d] fp32 tensor passes: the forward launch reads V and writes V^T (2),
-    # the backward one reads Q, K, dO and O* and writes three transposes (7); 4.5 on average
-    "k_prep": ("hbm", 4.5),
+    # the backward one reads Q, K, dO and O*, writes three transposes and (single pass) zeroes
+    # dQ (8); 5 on average
+    "k_prep": ("hbm", 5),
 }
 
 

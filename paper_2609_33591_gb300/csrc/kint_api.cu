@@ -581,7 +581,17 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
   if (p.dsum_out && cudaMemsetAsync(p.dsum_out, 0, (size_t)BH * T * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
   if (p.dabs_out && cudaMemsetAsync(p.dabs_out, 0, (size_t)BH * T * 4, s) != cudaSuccess) return KINT_ERR_LAUNCH;
 
-  // Operand copies: K-major transposes (and 3xTF32 splits).
+  // Single-pass backward: TF32 at d = 64 on the FWM grids and the exponentials, without the
+  // P1 projection and the row-sum side outputs (those stay on the two-pass kernels).  Tied
+  // maxima are found during the pass and listed (one entry per tied key) for k_bwd_ext; when
+  // the rows hold more ties than the list has room for (one per row of the call), which the
+  // dO prep job finds out, the whole call runs the two-pass kernels instead: both sets are
+  // launched, gated on that flag.
+  const bool single = g_bwd_path == 0 && !p.x3 && d == 64 && c.calib != KINT_CALIB_MINMAX &&
+                      c.grad != KINT_GRAD_DETACH_PROJ && !p.dsum_out && !p.dabs_out;
+
+  // Operand copies: K-major transposes (and 3xTF32 splits); for the single pass, the dO job
+  // also writes its row records and zeroes dQ and the row sums.
   PrepList pl;
   if (p.x3) {
     pl.add(Q, w.qh, w.ql, w.qth, w.qtl);
@@ -592,6 +602,29 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     pl.add(Q, nullptr, nullptr, w.qth, nullptr);
     pl.add(K, nullptr, nullptr, w.kth, nullptr);
     pl.add(dO, nullptr, nullptr, w.doth, nullptr, p.Ostar, w.gbar);
+  }
+  if (single) {
+    RecJob& R = pl.jobs.rec;
+    R.frec = reinterpret_cast<float4*>(w.frec);
+    R.rsum = w.rsum;
+    R.dQ = dQ;
+    R.cM_out = p.cM_out;
+    R.cm_out = p.cm_out;
+    R.row_max = st->row_max;
+    R.W = st->W;
+    R.Ws = prob ? st->W_lerp : st->W;
+    R.n_max = st->n_max;
+    R.tileflags = w.tileflags;
+    R.tie_total = w.tie_total;
+    R.tie_any = w.tie_any;
+    R.nqt = p.nqt;
+    R.tie_cap = BH * T;
+    const bool fwm = c.calib == KINT_CALIB_FWM || c.calib == KINT_CALIB_FWM_RESOLVED;
+    R.c0_kind = (c.calib == KINT_CALIB_SOFTMAX || c.calib == KINT_CALIB_EXP_FP8) ? 0 : (fwm ? 1 : 2);
+    R.half = fwm && c.recon == KINT_RECON_NEAREST;
+    R.softmax = c.calib == KINT_CALIB_SOFTMAX;
+    R.tau = p.tau;
+    R.inv_h = p.fwm_inv_h;
   }
   if (prep(pl, BH, T, Tp, d, p.x3 != 0, s) != cudaSuccess) return KINT_ERR_LAUNCH;
   Maps maps;
@@ -615,14 +648,6 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
        map_nat(&maps.dv, dV, BH, T, d, 64);
   if (!ok) return KINT_ERR_LAUNCH;
 
-  // Single-pass backward: TF32 at d = 64 on the FWM grids and the exponentials, without the
-  // P1 projection and the row-sum side outputs (those stay on the two-pass kernels).  Tied
-  // maxima are found during the pass and listed (one entry per tied key) for k_bwd_ext; when
-  // the rows hold more ties than the list has room for (one per row of the call), which
-  // k_rowrec finds out, the whole call runs the two-pass kernels instead: both sets are
-  // launched, gated on that flag.
-  const bool single = g_bwd_path == 0 && !p.x3 && d == 64 && c.calib != KINT_CALIB_MINMAX &&
-                      c.grad != KINT_GRAD_DETACH_PROJ && !p.dsum_out && !p.dabs_out;
   if (single) {
     Params pf = p;
     pf.frec = w.frec;
@@ -636,7 +661,6 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     if (!map_nat(&maps.dq16, dQ, BH, T, d, 16) || !map_nat(&maps.dk32, dK, BH, T, d, 32) ||
         !map_nat(&maps.dv32, dV, BH, T, d, 32))
       return KINT_ERR_LAUNCH;
-    if ((rc = launch_rc(traced("k_rowrec", s, [&] { return launch_rowrec(pf, num_sms(), s); })))) return rc;
     const int smem_f = plan_fused(pf);
     if (smem_f < 0) return KINT_ERR_UNSUPPORTED;
     if (ext) {
@@ -645,7 +669,7 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     }
     if ((rc = launch_rc(traced("k_bwd_fused", s, [&] { return launch_bwd_fused(maps, pf, smem_f, s); })))) return rc;
     if (!ext) return KINT_OK;
-    if ((rc = launch_rc(traced("k_bwd_ext", s, [&] { return launch_bwd_ext(pf, num_sms(), s); })))) return rc;
+    if ((rc = launch_rc(traced("k_bwd_ext", s, [&] { return launch_bwd_ext(pf, s); })))) return rc;
     p.gate = w.tie_any;
     p.gate_on = 1;
   }

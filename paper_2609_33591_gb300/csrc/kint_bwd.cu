@@ -174,6 +174,12 @@ __device__ __forceinline__ bool store_staged_dq(const Maps& maps, const Params& 
 template <int CAL, bool FULLG>
 __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
+  if (p.gate != nullptr) {
+    // launched on one side of a device-side decision: when the single-pass backward ran
+    // instead, leave before any set-up (no barrier, no tensor memory)
+    pdl_wait();
+    if (gated_off(p)) return;
+  }
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int ktile = BT * D * 4;
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + p.sm_bars);
@@ -229,12 +235,6 @@ __global__ void __launch_bounds__(NTHR_DQ, 1) k_bwd_dq(const __grid_constant__ M
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
   constexpr uint32_t tmem = 0;
-  if (gated_off(p)) {  // the single-pass backward ran instead
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, 512);
-    return;
-  }
 
   if (warp == PRODUCER_WARP) {
     int gt = 0, n = 0;

@@ -8,7 +8,6 @@
 namespace kint {
 
 constexpr int BT = 64;  // keys per tile (k_bwd_dq), queries per tile (k_bwd_dkdv)
-constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ __forceinline__ int4 lds_i4(uint32_t addr) {
   int4 v;

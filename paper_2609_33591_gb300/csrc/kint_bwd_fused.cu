@@ -20,8 +20,9 @@
 
 namespace kint {
 
-// 16-byte row record of this pass (k_rowrec): u = acc * k1 + c0 with k1 the same for
-// every row of a launch (FWM, the exponentials), forward 1/W, gamma = g * ga + gb.
+// 16-byte row record of this pass (written by the backward's dO prep job, RecJob):
+// u = acc * k1 + c0 with k1 the same for every row of a launch (FWM, the exponentials),
+// forward 1/W, gamma = g * ga + gb.
 struct FRec {
   float c0, invWf, ga, gb;
 };
@@ -31,49 +32,6 @@ __device__ __forceinline__ float fused_k1(const Params& p) {
   const RowGrid g = row_grid(p, 0.0f, 0.0f);
   if (exp_like(p.calib)) return p.scale * kLog2e;
   return (fwm_like(p.calib) && p.recon == REC_NEAREST) ? 2.0f * g.k1 : g.k1;
-}
-
-// ---------------------------------------------------------------------------
-// Row records, the zeroed row sums, dQ and calibration-sum outputs, the query tiles that
-// hold tied maxima, and the flag for ties beyond the tie list.  One thread per row
-// (grid-stride) for the records; the dQ zeroing runs over float4 words.
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_rowrec(const Params p) {
-  pdl_wait();
-  pdl_trigger();
-  const size_t nrows = (size_t)p.BH * p.T;
-  const bool prob = p.recon == REC_NEAREST && p.ste == 1 && !gridless(p.calib);
-  const bool half = fwm_like(p.calib) && p.recon == REC_NEAREST;
-  const size_t stride = (size_t)gridDim.x * blockDim.x;
-  bool tie = false;
-  for (size_t r = (size_t)blockIdx.x * blockDim.x + threadIdx.x; r < nrows; r += stride) {
-    const float M = p.row_max[r], Wf = p.W[r], Ws = prob ? p.W_lerp[r] : Wf, Dg = p.gbar[r];
-    const RowGrid g = row_grid(p, M, p.row_min[r]);
-    FRec f;
-    f.ga = p.calib == CAL_SOFTMAX ? 1.0f : 1.0f / Ws;
-    f.gb = p.calib == CAL_SOFTMAX ? -Dg : -Dg * f.ga;
-    f.invWf = 1.0f / Wf;
-    f.c0 = exp_like(p.calib) ? -M * kLog2e : (half ? 2.0f * g.c0 : g.c0);
-    reinterpret_cast<FRec*>(p.frec)[r] = f;
-    p.rsum[r] = 0.0f;
-    // the calibration-sum outputs: 0 unless k_bwd_ext writes them (modes without them)
-    if (p.cM_out) p.cM_out[r] = 0.0f;
-    if (p.cm_out) p.cm_out[r] = 0.0f;
-    const int nm = p.n_max[r];
-    if (nm > 1) {
-      // a row with tied maxima: its 64-row query tile takes the tie search of k_bwd_fused, and
-      // its ties must fit in the list
-      const int bh = (int)(r / (size_t)p.T), i = (int)(r - (size_t)bh * p.T);
-      p.tileflags[(size_t)bh * p.nqt + i / BT] = 1;
-      const int old = atomicAdd(p.tie_total, nm);
-      tie = tie || old + nm > p.tie_cap;
-    }
-  }
-  float4* dq = reinterpret_cast<float4*>(p.dQ);
-  const size_t n4 = nrows * (size_t)p.d / 4;
-  for (size_t k = (size_t)blockIdx.x * blockDim.x + threadIdx.x; k < n4; k += stride)
-    dq[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (__any_sync(0xffffffffu, tie) && (threadIdx.x & 31) == 0) atomicOr(p.tie_any, 1);
 }
 
 // ---------------------------------------------------------------------------
@@ -641,54 +599,78 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
 
 // ---------------------------------------------------------------------------
 // The extremum terms of Eq. (full) after the single pass: c_M = -sum_j gamma_ij Delta_ij
-// (the row sums k_bwd_fused accumulated), split over n_max = 1 arg-max key (rows with
-// tied maxima run the two-pass kernels instead):
-//   dQ_i += s c_M K_amax(i),   dK_amax(i) += s c_M Q_i   (USE_M: not in min_only, where
-// FWM-like grids have no minimum channel), both as fp32 additions at L2, and the c_M / c_m
-// side outputs.  16 threads per row, four columns each, one row per 16 threads.
+// (the row sums k_bwd_fused accumulated), split over the n_max arg-max keys:
+//   dQ_i += s (c_M / n_max) K_j,   dK_j += s (c_M / n_max) Q_i   for each arg-max key j
+// (USE_M: not in min_only, where FWM-like grids have no minimum channel), both as fp32
+// additions at L2, and the c_M / c_m side outputs.  The first blocks take rows with one
+// maximum (arg_max), 64 rows per block, 16 threads per row with four columns each and
+// four rows per thread, all loads issued before the additions; the last EXT_TIE_BLOCKS
+// blocks take the tied maxima that k_bwd_fused listed as (row, key) pairs.
 // ---------------------------------------------------------------------------
+constexpr int EXT_TIE_BLOCKS = 64;
+
 template <bool USE_M>
 __global__ void __launch_bounds__(256) k_bwd_ext(const Params p) {
   pdl_wait();
   pdl_trigger();
   if (gated_off(p)) return;
-  const int nrows = p.BH * p.T, l = threadIdx.x & 15;
-  const int r = blockIdx.x * 16 + (threadIdx.x >> 4);
-  if (r >= nrows) return;
-  const float cM = -p.rsum[r];
-  if (l == 0) {
-    if (p.cM_out) p.cM_out[r] = cM;
-    if (p.cm_out) p.cm_out[r] = 0.f;
-  }
-  if constexpr (USE_M) {
-    const int nm = p.n_max[r];
-    if (nm > 1) return;  // its keys come from the tie list
-    const int bh = r / p.T, am = p.arg_max[r];
-    const float c = cM * p.scale;
-    const size_t kr = ((size_t)bh * p.T + am) * 64 + 4 * l, qr = (size_t)r * 64 + 4 * l;
-    const float4 k4 = __ldg(reinterpret_cast<const float4*>(p.K + kr));
-    const float4 q4 = __ldg(reinterpret_cast<const float4*>(p.Q + qr));
-    red_add_v4(p.dQ + qr, c * k4.x, c * k4.y, c * k4.z, c * k4.w);
-    red_add_v4(p.dK + kr, c * q4.x, c * q4.y, c * q4.z, c * q4.w);
-  }
-}
-
-// The tied-maxima entries of k_bwd_ext: c_M / n_max of row i at each listed key j.
-template <bool USE_M>
-__global__ void __launch_bounds__(256) k_bwd_ext_ties(const Params p) {
-  pdl_wait();
-  pdl_trigger();
-  if (gated_off(p) || !USE_M) return;
-  const int cnt = min(*p.tie_count, p.tie_cap), l = threadIdx.x & 15;
-  for (int e = blockIdx.x * 16 + (threadIdx.x >> 4); e < cnt; e += gridDim.x * 16) {
-    const int2 rj = p.tie_list[e];
-    const int r = rj.x, bh = r / p.T;
-    const float c = -p.rsum[r] / (float)p.n_max[r] * p.scale;
-    const size_t kr = ((size_t)bh * p.T + rj.y) * 64 + 4 * l, qr = (size_t)r * 64 + 4 * l;
-    const float4 k4 = __ldg(reinterpret_cast<const float4*>(p.K + kr));
-    const float4 q4 = __ldg(reinterpret_cast<const float4*>(p.Q + qr));
-    red_add_v4(p.dQ + qr, c * k4.x, c * k4.y, c * k4.z, c * k4.w);
-    red_add_v4(p.dK + kr, c * q4.x, c * q4.y, c * q4.z, c * q4.w);
+  const int nrows = p.BH * p.T, l = threadIdx.x & 15, grp = threadIdx.x >> 4;
+  const int nrb = (nrows + 63) / 64;
+  if ((int)blockIdx.x < nrb) {
+    int r[4], am[4];
+    float c[4];
+    bool act[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      r[k] = blockIdx.x * 64 + 16 * k + grp;
+      act[k] = r[k] < nrows;
+      c[k] = 0.f;
+      am[k] = 0;
+      if (act[k]) {
+        const float cM = -p.rsum[r[k]];
+        if (l == 0) {
+          if (p.cM_out) p.cM_out[r[k]] = cM;
+          if (p.cm_out) p.cm_out[r[k]] = 0.f;
+        }
+        c[k] = cM * p.scale;
+        act[k] = USE_M && p.n_max[r[k]] == 1;  // tied rows' keys come from the tie list
+        am[k] = p.arg_max[r[k]];
+      }
+    }
+    if constexpr (USE_M) {
+      float4 k4[4], q4[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        if (act[k]) {
+          const int bh = r[k] / p.T;
+          k4[k] = __ldg(reinterpret_cast<const float4*>(p.K + ((size_t)bh * p.T + am[k]) * 64 + 4 * l));
+          q4[k] = __ldg(reinterpret_cast<const float4*>(p.Q + (size_t)r[k] * 64 + 4 * l));
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        if (act[k]) {
+          const int bh = r[k] / p.T;
+          red_add_v4(p.dQ + (size_t)r[k] * 64 + 4 * l, c[k] * k4[k].x, c[k] * k4[k].y, c[k] * k4[k].z,
+                     c[k] * k4[k].w);
+          red_add_v4(p.dK + ((size_t)bh * p.T + am[k]) * 64 + 4 * l, c[k] * q4[k].x, c[k] * q4[k].y,
+                     c[k] * q4[k].z, c[k] * q4[k].w);
+        }
+      }
+    }
+  } else if constexpr (USE_M) {
+    // the tied maxima: c_M / n_max of row i at each listed key j
+    const int cnt = min(*p.tie_count, p.tie_cap);
+    for (int e = (blockIdx.x - nrb) * 16 + grp; e < cnt; e += EXT_TIE_BLOCKS * 16) {
+      const int2 rj = p.tie_list[e];
+      const int rr = rj.x, bh = rr / p.T;
+      const float cc = -p.rsum[rr] / (float)p.n_max[rr] * p.scale;
+      const size_t kr = ((size_t)bh * p.T + rj.y) * 64 + 4 * l, qr = (size_t)rr * 64 + 4 * l;
+      const float4 k4 = __ldg(reinterpret_cast<const float4*>(p.K + kr));
+      const float4 q4 = __ldg(reinterpret_cast<const float4*>(p.Q + qr));
+      red_add_v4(p.dQ + qr, cc * k4.x, cc * k4.y, cc * k4.z, cc * k4.w);
+      red_add_v4(p.dK + kr, cc * q4.x, cc * q4.y, cc * q4.z, cc * q4.w);
+    }
   }
 }
 
@@ -701,10 +683,6 @@ static cudaError_t launch_fused_modes(dim3 grid, const Maps& maps, const Params&
     return full ? launch3(k_bwd_fused<CAL, REC, true>, grid, maps, p, smem_bytes, s, NTHR_FUSED)
                 : launch3(k_bwd_fused<CAL, REC, false>, grid, maps, p, smem_bytes, s, NTHR_FUSED);
   }
-}
-
-cudaError_t launch_rowrec(const Params& p, int nsm, cudaStream_t s) {
-  return launch_pdl(k_rowrec, dim3((unsigned)(4 * nsm)), dim3(256), 0, s, p);
 }
 
 cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
@@ -724,13 +702,11 @@ cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, 
   }
 }
 
-cudaError_t launch_bwd_ext(const Params& p, int nsm, cudaStream_t s) {
-  const dim3 grid((unsigned)(((size_t)p.BH * p.T + 15) / 16)), block(256);
+cudaError_t launch_bwd_ext(const Params& p, cudaStream_t s) {
+  const int nrb = (int)(((size_t)p.BH * p.T + 63) / 64);
   const bool use_M = p.grad != GRAD_MIN_ONLY;
-  cudaError_t e = use_M ? launch_pdl(k_bwd_ext<true>, grid, block, 0, s, p)
-                        : launch_pdl(k_bwd_ext<false>, grid, block, 0, s, p);
-  if (e != cudaSuccess || !use_M) return e;
-  return launch_pdl(k_bwd_ext_ties<true>, dim3((unsigned)nsm), block, 0, s, p);
+  const dim3 grid((unsigned)(nrb + (use_M ? EXT_TIE_BLOCKS : 0))), block(256);
+  return use_M ? launch_pdl(k_bwd_ext<true>, grid, block, 0, s, p) : launch_pdl(k_bwd_ext<false>, grid, block, 0, s, p);
 }
 
 }  // namespace kint

@@ -197,6 +197,12 @@ __device__ __forceinline__ bool store_staged_dkdv(const Maps& maps, const Params
 template <int CAL, int REC, bool FULLG, bool PROJ = false, bool RS = false>
 __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
+  if (p.gate != nullptr) {
+    // launched on one side of a device-side decision: when the single-pass backward ran
+    // instead, leave before any set-up (no barrier, no tensor memory)
+    pdl_wait();
+    if (gated_off(p)) return;
+  }
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int qtile = BT * D * 4;
   const bool doDV = p.dkv_sel != DKV_DK, doDK = p.dkv_sel != DKV_DV, needV = doDK;
@@ -266,12 +272,6 @@ __global__ void __launch_bounds__(NTHR, 1) k_bwd_dkdv(const __grid_constant__ Ma
   // compile-time base keeps the TMEM addresses of the issue paths in uniform registers.
   if (threadIdx.x == 0 && *tslot != 0u) dev_flag(p.status, DEV_ERR_BOUNDS);
   constexpr uint32_t tmem = 0;
-  if (gated_off(p)) {  // the single-pass backward ran instead
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(tmem, 512);
-    return;
-  }
 
   // Work items are (128-key block kb, head) pairs, longest first (kb = 0 meets every
   // query tile); a CTA takes the items snake_item(0), snake_item(1), ...  Tile counters

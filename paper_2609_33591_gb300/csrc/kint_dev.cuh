@@ -10,6 +10,8 @@
 
 namespace kint {
 
+constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
+
 constexpr int NT = 128;              // threads per CTA; thread t owns TMEM lane t
 constexpr int SW = 128;              // bytes of one swizzled panel row (32 fp32)
 

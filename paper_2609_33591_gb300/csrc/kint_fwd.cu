@@ -10,6 +10,34 @@
 
 namespace kint {
 
+// Row record of the single-pass backward for row rw (position t of head bh) from its row
+// max M, forward normalizer Wf, the W* of gamma Ws, tie count nm and <g>_{P*} = dg;
+// returns whether this row's tied keys overflow the tie list.
+__device__ __forceinline__ bool prep_row_record(const RecJob& R, size_t rw, int bh, int t, float M, float Wf, float Ws,
+                                                int nm, float dg) {
+  float4 f;
+  f.z = R.softmax ? 1.0f : 1.0f / Ws;  // gamma = g * f.z + f.w
+  f.w = R.softmax ? -dg : -dg * f.z;
+  f.y = 1.0f / Wf;
+  if (R.c0_kind == 0) {
+    f.x = -M * kLog2e;
+  } else if (R.c0_kind == 1) {
+    const float c0 = __fmul_rn(__fsub_rn(R.tau, M), R.inv_h);
+    f.x = R.half ? 2.0f * c0 : c0;
+  } else {
+    f.x = -M;
+  }
+  R.frec[rw] = f;
+  R.rsum[rw] = 0.0f;
+  // the calibration-sum outputs stay 0 in the modes whose extremum pass does not write them
+  if (R.cM_out) R.cM_out[rw] = 0.0f;
+  if (R.cm_out) R.cm_out[rw] = 0.0f;
+  if (nm <= 1) return false;
+  // a row with tied maxima: its 64-row query tile takes the single pass's tie search
+  R.tileflags[(size_t)bh * R.nqt + t / 64] = 1;
+  return atomicAdd(R.tie_total, nm) + nm > R.tie_cap;
+}
+
 // ---------------------------------------------------------------------------
 // Operand preparation (HBM-bound).  tcgen05.mma kind::tf32 reads both operands
 // K-major, so every second-stage product (P V, dS K, P^T dO, dS^T Q) reads a
@@ -26,6 +54,7 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
                                               int BH) {
   __shared__ float hs[32][65];
   __shared__ float ls[SPLIT ? 32 : 1][65];
+  __shared__ float dots[32];
   const int tid = threadIdx.x;
   const int r = tid >> 4, c4 = tid & 15;  // load phase: rows r + 8 q, columns 4 c4 .. 4 c4 + 3
   const int k = tid >> 3, tq = tid & 7;   // store phase: output rows k + 16 q, keys 4 tq .. 4 tq + 3
@@ -36,6 +65,25 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
     const int bh = (u % per_job) / ntb, t0 = (u % ntb) * 32;
     const size_t nat = (size_t)bh * T * d, tr = (size_t)bh * d * Tp;
     const bool dotj = J.Y != nullptr;
+    const RecJob& R = jobs.rec;
+    const bool recj = dotj && R.frec != nullptr;
+    // single-pass set-up: this unit's row statistics load under the transposes, and its dQ
+    // rows start at zero (the single pass adds its partial sums to them)
+    float rM = 0.f, rW = 1.f, rWs = 1.f;
+    int rnm = 0;
+    if (recj) {
+      const int t = t0 + tid;
+      if (tid < 32 && t < T) {
+        const size_t rw = (size_t)bh * T + t;
+        rM = R.row_max[rw];
+        rW = R.W[rw];
+        rWs = R.Ws[rw];
+        rnm = R.n_max[rw];
+      }
+      const int nr = min(32, T - t0);
+      float4* dq = reinterpret_cast<float4*>(R.dQ + nat + (size_t)t0 * d);
+      for (int k4 = tid; k4 < nr * d / 4; k4 += 128) dq[k4] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     float dacc[4] = {0.f, 0.f, 0.f, 0.f};
     for (int k0 = 0; k0 < d; k0 += 64) {
       float4 x[4];
@@ -102,7 +150,17 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
 #pragma unroll
         for (int o = 8; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
         const int t = t0 + r + 8 * q;
-        if (c4 == 0 && t < T) J.dot[(size_t)bh * T + t] = v;
+        if (c4 == 0 && t < T) {
+          J.dot[(size_t)bh * T + t] = v;
+          dots[r + 8 * q] = v;
+        }
+      }
+      if (recj) {
+        __syncthreads();  // dots[] (the next unit writes it only after the syncs of its own loop)
+        const int t = t0 + tid;
+        if (tid < 32 && t < T &&
+            prep_row_record(R, (size_t)bh * T + t, bh, t, rM, rW, rWs, rnm, dots[tid]))
+          atomicOr(R.tie_any, 1);
       }
     }
   }

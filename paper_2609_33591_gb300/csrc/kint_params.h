@@ -80,7 +80,7 @@ struct Params {
   const float* gbar;        // [BH*T] <g>_{P*} = dO_i . O*_i (workspace, written by the dO prep)
   float *cM_out, *cm_out;   // optional [BH*T] side outputs of the backward: c_M, c_m per row
   float *dsum_out, *dabs_out;  // optional [BH*T] side outputs of the backward: sum_j dS_ij, sum_j |dS_ij|
-  void* frec;               // [B*H*T] 16-byte row records of the single-pass backward (k_rowrec)
+  void* frec;               // [B*H*T] 16-byte row records of the single-pass backward (RecJob of k_prep)
   float* rsum;              // [B*H*T] single-pass backward: sum_j gamma_ij Delta_ij per row
   int* tie_any;             // single-pass backward: set when the rows' ties exceed the tie list
   int* tie_count;           // single-pass backward: entries in tie_list; tie_total: the ties the rows hold
