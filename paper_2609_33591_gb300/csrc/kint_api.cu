@@ -95,6 +95,17 @@ bool map_nat(CUtensorMap* m, const float* X, int BH, int T, int d, int rows) {
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+// X [BH][T][d] with a box of (cols, rows) and the 64-byte swizzle (cols = 16): the single-pass
+// backward's dQ reduce and dV / dK stores, 16 columns per compute warp.
+bool map_nat_sw64(CUtensorMap* m, const float* X, int BH, int T, int d, int cols, int rows) {
+  cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)T, (cuuint64_t)BH};
+  cuuint64_t strides[2] = {(cuuint64_t)d * 4, (cuuint64_t)T * d * 4};
+  cuuint32_t box[3] = {(cuuint32_t)cols, (cuuint32_t)rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float*>(X), dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 // Transposed view of X^T [BH][d][Tp] (valid columns T): box (32 keys, d rows).
 bool map_tr(CUtensorMap* m, const float* XT, int BH, int T, int Tp, int d) {
   cuuint64_t dims[3] = {(cuuint64_t)T, (cuuint64_t)d, (cuuint64_t)BH};
@@ -367,7 +378,7 @@ int plan_dkdv(Params& p, int sel) {
 }
 
 // Single-pass backward (TF32, d = 64): two stages of Q | dO | Q^T | dO^T tiles and their
-// 16-byte row records, the item's V and K^T tiles, eight 2 KB dQ reduce slices, the FWM
+// 16-byte row records, the item's V and K^T tiles, sixteen 1 KB dQ reduce slices, the FWM
 // table; one CTA per SM.
 int plan_fused(Params& p) {
   const int qtile = 64 * 64 * 4;
@@ -379,8 +390,8 @@ int plan_fused(Params& p) {
   p.sm_stage_bytes = 4 * qtile + 64 * 16;
   p.sm_v = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
   p.sm_kt = p.sm_v + 128 * 64 * 4;
-  p.sm_ostage = p.sm_kt + 128 * 64 * 4;  // the compute warps' 2 KB dQ reduce slices
-  p.sm_table = p.sm_ostage + 8 * 2048;
+  p.sm_ostage = p.sm_kt + 128 * 64 * 4;  // the compute warps' 1 KB dQ reduce slices
+  p.sm_table = p.sm_ostage + 16 * 1024;
   const int total = std::max(finish_plan(p, p.sm_table + 2048, 5 * p.nstage + 13), kOneCtaPerSm);
   if (total > kSmemLimit) return -1;
   p.nitems = p.nqb * p.BH;
@@ -658,8 +669,8 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     pf.tie_list = w.tie_list;
     pf.tie_cap = BH * T;
     const bool ext = c.calib != KINT_CALIB_SOFTMAX && c.grad != KINT_GRAD_DETACH;
-    if (!map_nat(&maps.dq16, dQ, BH, T, d, 16) || !map_nat(&maps.dk32, dK, BH, T, d, 32) ||
-        !map_nat(&maps.dv32, dV, BH, T, d, 32))
+    if (!map_nat_sw64(&maps.dq16, dQ, BH, T, d, 16, 16) || !map_nat_sw64(&maps.dk32, dK, BH, T, d, 16, 32) ||
+        !map_nat_sw64(&maps.dv32, dV, BH, T, d, 16, 32))
       return KINT_ERR_LAUNCH;
     const int smem_f = plan_fused(pf);
     if (smem_f < 0) return KINT_ERR_UNSUPPORTED;

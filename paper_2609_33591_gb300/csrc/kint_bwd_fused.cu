@@ -132,10 +132,12 @@ __device__ __forceinline__ void rowsum_red(const float (&v)[16], float* dst, siz
 
 
 // ---------------------------------------------------------------------------
-// k_bwd_fused (352 threads: 8 compute warps, the MMA warp, two producer warps).  Work
+// k_bwd_fused (608 threads: 16 compute warps, the MMA warp, two producer warps).  Work
 // items are (128-key block kb, head) pairs, longest first; a CTA
-// takes snake_item(0), snake_item(1), ...  Thread t (< 256) owns key j = kb*128 + t%128
-// (TMEM lane t%128) and the query half t/128 of each 64-query tile.
+// takes snake_item(0), snake_item(1), ...  Thread t (< 512) owns key j = kb*128 + t%128
+// (TMEM lane t%128) and the 16 query columns 16 (t/128) .. +15 of each 64-query tile:
+// four compute warps per SM sub-partition, so that one warp's latencies (TMEM and
+// shared-memory loads, shuffles) hide under the others' element work.
 // TMEM: K [0, 64) (A operand of S^T), per buffer b: S^T_b at 64 + 128 b and g^T_b 64
 // columns further (P^T overwrites S^T_b, dS^T overwrites g^T_b: the A operands of dV, dK),
 // dV [320, 384), dK [384, 448), the 64-query dQ partial [448, 512) (M = 64: query row r
@@ -147,11 +149,20 @@ __device__ __forceinline__ void rowsum_red(const float (&v)[16], float* dst, siz
 // for tile u + 2 as soon as the element work of tile u is done, and that stage's Q^T | dO^T
 // half takes tile u + 1's tiles once dQ of tile u has read dS.  The item's V tile (A
 // operand of g^T) also stages the next item's K rows on their way into TMEM; its K^T tile
-// (B operand of dQ) stages the dV, dK rows of the epilogue for TMA stores; each compute
-// warp has a 2 KB slice for its 16 rows x 32 columns of the dQ partial, added to dQ by a
-// TMA reduce.
+// (B operand of dQ) stages the dV, dK rows of the epilogue (32 keys x 16 columns per warp,
+// 64-byte swizzle) for TMA stores; each compute warp has a 1 KB slice for its 16 rows x 16
+// columns of the dQ partial (64-byte swizzle), added to dQ by a TMA reduce.
 // ---------------------------------------------------------------------------
-constexpr int PRODUCER2_WARP = NCOMP / 32 + 2, NTHR_FUSED = NTHR + 32;
+constexpr int NCOMP_F = 512;  // compute threads
+constexpr int MMA_WARP_F = NCOMP_F / 32, PRODUCER_WARP_F = NCOMP_F / 32 + 1, PRODUCER2_WARP_F = NCOMP_F / 32 + 2;
+constexpr int NTHR_FUSED = NCOMP_F + 96;
+
+// Byte offset of 16-byte chunk c of row r in a tile of 64-byte rows under the 64-byte
+// swizzle (chunk index XOR bits 1..2 of the row), the layout TMA reads for the dQ reduce
+// and the dV / dK stores.
+__device__ __forceinline__ uint32_t sw64_off(int r, int c) {
+  return (uint32_t)r * 64u + (uint32_t)((c ^ ((r >> 1) & 3)) << 4);
+}
 
 template <int CAL, int REC, bool FULLG>
 __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_constant__ Maps maps, const Params p) {
@@ -186,23 +197,23 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
   if (tid == 0) {
     for (int s = 0; s < NS; ++s) {
       mbar_init(&bar_full[s], 1);
-      mbar_init(&bar_emptyA[s], NCOMP / 32);
+      mbar_init(&bar_emptyA[s], NCOMP_F / 32);
       mbar_init(&bar_fullT[s], 1);
       mbar_init(&bar_empty[s], 1);
       mbar_init(&bar_tfree[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_sfull[b], 1);
-      mbar_init(&bar_pready[b], NCOMP / 32);
+      mbar_init(&bar_pready[b], NCOMP_F / 32);
     }
     mbar_init(bar_dqfull, 1);
     mbar_init(bar_done, 1);
     mbar_init(bar_kst, 1);
-    mbar_init(bar_ops, NCOMP / 32);
+    mbar_init(bar_ops, NCOMP_F / 32);
     mbar_init(bar_v, 1);
     mbar_init(bar_vfree, 1);
     mbar_init(bar_kt, 1);
-    mbar_init(bar_ktfree, NCOMP / 32);
+    mbar_init(bar_ktfree, NCOMP_F / 32);
     mbar_init(bar_drain, 1);
     fence_mbar_init();
   }
@@ -225,15 +236,15 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     return;
   }
 
-  // Two producer warps: PRODUCER_WARP loads the Q | dO halves with their records and the
-  // items' K rows and V tiles, PRODUCER2_WARP the Q^T | dO^T halves and the K^T tiles, so
+  // Two producer warps: PRODUCER_WARP_F loads the Q | dO halves with their records and the
+  // items' K rows and V tiles, PRODUCER2_WARP_F the Q^T | dO^T halves and the K^T tiles, so
   // that neither kind of load waits behind the other's condition.
   auto item_of = [&](int k, int& kb_, int& bh_) {
     const int it_ = snake_item(k);
     kb_ = it_ / p.BH;
     bh_ = it_ % p.BH;
   };
-  if (warp == PRODUCER_WARP) {
+  if (warp == PRODUCER_WARP_F) {
     int gt = 0, n = 0;
     RingPos ld, nf;
     int cf = 0, nks = 0, nv = 0;
@@ -294,7 +305,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     drain_ring(bar_full, nf, cf, NS, p.wait_ns, p.status);
     if (nks > 0) mbar_wait_warp(bar_kst, (nks - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
     if (nv > 0) mbar_wait_warp(bar_v, (nv - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-  } else if (warp == PRODUCER2_WARP) {
+  } else if (warp == PRODUCER2_WARP_F) {
     int gt = 0, n = 0;
     RingPos ld, nT;
     int cT = 0, nkt = 0;
@@ -338,7 +349,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     // clean-up: the last loads issued have landed
     drain_ring(bar_fullT, nT, cT, NS, p.wait_ns, p.status);
     if (nkt > 0) mbar_wait_warp(bar_kt, (nkt - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
-  } else if (warp == MMA_WARP) {
+  } else if (warp == MMA_WARP_F) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t idq = idesc_tf32(64, D, 0, 0);
     int n = 0;
@@ -398,55 +409,52 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
       mma_commit(bar_done);
     }
     drain_mma(bar_drain, p.wait_ns, p.status);  // clean-up: no product still writes TMEM
-  } else if (warp < NCOMP / 32) {
-    const int row = tid & 127, cg = tid >> 7, q4 = warp & 3, lane = tid & 31;
-    uint8_t* dqs = sm + p.sm_ostage + warp * 2048;  // this warp's dQ reduce slice (16 rows x 32)
-    uint8_t* ostg = sm + p.sm_kt + (q4 * 2 + cg) * 4096;  // its epilogue slice (32 rows x 32)
-    // the k-th item's K rows from the V buffer into TMEM (each column group half of the
+  } else if (warp < NCOMP_F / 32) {
+    const int row = tid & 127, cq = tid >> 7, q4 = warp & 3, lane = tid & 31;
+    uint8_t* dqs = sm + p.sm_ostage + warp * 1024;      // this warp's dQ reduce slice (16 rows x 16)
+    uint8_t* ostg = sm + p.sm_kt + (q4 * 4 + cq) * 2048;  // its epilogue slice (32 rows x 16)
+    // the k-th item's K rows from the V buffer into TMEM (each warp 16 of its keys' 64
     // columns), handed to the MMA warp (and the producer) through bar_ops
     auto ops_to_tmem = [&](int k) {
       const bool okk = mbar_wait(bar_kst, k & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
       if (okk) {
-        const uint32_t base = smem_u32(sm + p.sm_v) + (uint32_t)cg * 128u * SW + (uint32_t)row * SW;
+        const uint32_t base = smem_u32(sm + p.sm_v) + (uint32_t)(cq >> 1) * 128u * SW + (uint32_t)row * SW;
+        float v[16];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          float v[16];
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const int chunk = h * 4 + c;
-            const float4 x = lds_f4(base + (uint32_t)((chunk ^ (row & 7)) << 4));
-            v[4 * c] = x.x;
-            v[4 * c + 1] = x.y;
-            v[4 * c + 2] = x.z;
-            v[4 * c + 3] = x.w;
-          }
-          tmem_st16(lane_addr(tmem, cK + 32 * cg + 16 * h), v);
+        for (int c = 0; c < 4; ++c) {
+          const int chunk = (cq & 1) * 4 + c;
+          const float4 x = lds_f4(base + (uint32_t)((chunk ^ (row & 7)) << 4));
+          v[4 * c] = x.x;
+          v[4 * c + 1] = x.y;
+          v[4 * c + 2] = x.z;
+          v[4 * c + 3] = x.w;
         }
+        tmem_st16(lane_addr(tmem, cK + 16 * cq), v);
       }
       tmem_st_wait();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_ops);
     };
-    // the dQ partial of tile q0 (this warp's 16 rows in its lanes 0..15, this column half),
+    // the dQ partial of tile q0 (this warp's 16 rows in its lanes 0..15, its 16 columns),
     // scaled, staged in the warp's slice and added to dQ by a TMA reduce
     auto dq_out = [&](int bh_, int q0) {
-      float v[32];
-      tmem_ld32(lane_addr(tmem, cdQ + 32 * cg), v);
+      float v[16];
+      tmem_ld16(lane_addr(tmem, cdQ + 16 * cq), v);
       tmem_ld_wait();
       tma_store_wait_read();  // the slice's previous reduce has read it
       if (lane < 16) {
-        const uint32_t base = smem_u32(dqs) + (uint32_t)lane * SW;
+        const uint32_t base = smem_u32(dqs);
 #pragma unroll
-        for (int c = 0; c < 8; ++c)
-          asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(base + (uint32_t)((c ^ (lane & 7)) << 4)),
+        for (int c = 0; c < 4; ++c)
+          asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(base + sw64_off(lane, c)),
                        "f"(v[4 * c] * p.scale), "f"(v[4 * c + 1] * p.scale), "f"(v[4 * c + 2] * p.scale),
                        "f"(v[4 * c + 3] * p.scale)
                        : "memory");
       }
       fence_async_smem();
       __syncwarp();
-      tma_reduce_add_3d(&maps.dq16, dqs, 32 * cg, q0 + 16 * q4, bh_);
+      tma_reduce_add_3d(&maps.dq16, dqs, 16 * cq, q0 + 16 * q4, bh_);
       tma_store_commit();
     };
     // (i, j) pairs of a row with tied maxima whose score at key j equals its maximum, into the
@@ -474,10 +482,11 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     }
     const float Kf = (float)(half ? 2 * Kq : Kq), k1 = fused_k1(p);
     const uint32_t fwtab = smem_u32(sm + p.sm_table) + (half ? 8u * kHalfTail : 0u) - 0x58000000u;
-    group_sync(BAR_COMPUTE, NCOMP);  // the FWM table
+    group_sync(BAR_COMPUTE, NCOMP_F);  // the FWM table
     bool failed = false;
     int n = 0, gu = 0;  // gu: tiles so far over the CTA's run (stage parity, bar_dqfull, bar_tfree)
     RingPos cs, cb;
+    const int c0 = cq * 16;  // this thread's query columns in every tile
     for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
@@ -503,9 +512,8 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         const uint32_t dsb = smem_u32(sm + p.sm_stage0 + (s ^ 1) * p.sm_stage_bytes + oQT) + (uint32_t)q4 * PNL_DS +
                              (uint32_t)(lane & 3) * 4u;
         const uint32_t dchunk = (uint32_t)(lane >> 2);
-#pragma unroll 1
-        for (int h = 0; h < 2; ++h) {
-          const int c0 = cg * 32 + h * 16, i0h = q0 + c0;
+        const int i0h = q0 + c0;
+        {
           const uint32_t recs = smem_u32(st + oRec) + c0 * 16;
           const int cS = cSG + 128 * b + c0, cG = cS + 64;
           float sv[16], gv[16], pa[16], da[16];
@@ -526,9 +534,8 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
           tmem_stw<16>(lane_addr(tmem, cS), pa);
           tmem_stw<16>(lane_addr(tmem, cG), da);
           // dS goes where the previous tile's Q^T, dO^T were, once dV, dK have read them
-          if (h == 0 && gu >= 1 &&
-              !mbar_wait(&bar_tfree[s ^ 1], (uint32_t)((gu - 1) >> 1) & 1u, p.wait_ns, p.status,
-                         DEV_ERR_TIMEOUT_MMA)) {
+          if (gu >= 1 &&
+              !mbar_wait(&bar_tfree[s ^ 1], (uint32_t)((gu - 1) >> 1) & 1u, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
             failed = true;
             break;
           }
@@ -540,7 +547,6 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
                          : "memory");
           }
         }
-        if (failed) break;
         // the tile's records and Q, dO are no longer needed
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar_emptyA[s]);
@@ -562,28 +568,28 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         if (it + 1 == nit && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
       }
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
-      failed = group_any(BAR_COMPUTE, NCOMP, !dok);
+      failed = group_any(BAR_COMPUTE, NCOMP_F, !dok);
       if (!failed) {
         tc_fence_after();
         dq_out(bh, (qt0 + nit - 1) * BT);
-        // dV, then dK (scaled): this warp's 32 rows x 32 columns through its slice of the
+        // dV, then dK (scaled): this warp's 32 rows x 16 columns through its slice of the
         // K^T buffer (every product of the item has completed) and a TMA store
         for (int pass = 0; pass < 2; ++pass) {
-          float v[32];
-          tmem_ld32(lane_addr(tmem, (pass == 0 ? cdV : cdK) + 32 * cg), v);
+          float v[16];
+          tmem_ld16(lane_addr(tmem, (pass == 0 ? cdV : cdK) + 16 * cq), v);
           tmem_ld_wait();
           const float mul = pass == 0 ? 1.0f : p.scale;
           if (pass == 1) tma_store_wait_read();  // dV has left the slice
-          const uint32_t base = smem_u32(ostg) + (uint32_t)lane * SW;
+          const uint32_t base = smem_u32(ostg);
 #pragma unroll
-          for (int c = 0; c < 8; ++c)
-            asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(base + (uint32_t)((c ^ (lane & 7)) << 4)),
+          for (int c = 0; c < 4; ++c)
+            asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(base + sw64_off(lane, c)),
                          "f"(v[4 * c] * mul), "f"(v[4 * c + 1] * mul), "f"(v[4 * c + 2] * mul),
                          "f"(v[4 * c + 3] * mul)
                          : "memory");
           fence_async_smem();
           __syncwarp();
-          tma_store_3d(pass == 0 ? &maps.dv32 : &maps.dk32, ostg, 32 * cg, kb * 128 + 32 * q4, bh);
+          tma_store_3d(pass == 0 ? &maps.dv32 : &maps.dk32, ostg, 16 * cq, kb * 128 + 32 * q4, bh);
           tma_store_commit();
         }
         tma_store_wait_read();

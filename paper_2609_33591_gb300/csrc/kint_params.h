@@ -36,7 +36,7 @@ struct Maps {
   CUtensorMap q, q_lo, k, k_lo, v, v_lo, dout, dout_lo;  // natural
   CUtensorMap kt, kt_lo, vt, vt_lo, qt, qt_lo, dot, dot_lo;  // transposed
   CUtensorMap out, out_lerp, dq, dk, dv;  // outputs (natural, box 32 x 64 rows) for TMA stores
-  CUtensorMap dq16, dk32, dv32;  // single-pass backward: dQ reduce boxes of 16 rows, dK / dV stores of 32
+  CUtensorMap dq16, dk32, dv32;  // single-pass backward: 16-column boxes (64-byte swizzle), dQ reduces of 16 rows, dK / dV stores of 32
 };
 
 struct Params {
