@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "2760b45424ab1f5b", "k_prep": 82348576, "k_fwd_stats": 50404659, "k_fwd_main": 92283994,
-           "k_bwd_dq": 191385203, "k_bwd_dkdv": 264280154}
+TRAFFIC = {"src": "aff76cf58171ef16", "k_prep": 90550304, "k_fwd_stats": 50402458, "k_fwd_main": 92317171,
+           "k_bwd_fused": 423584435, "k_bwd_ext": 73675046}
 
 
 def kernel_source_digest() -> str:
