@@ -45,7 +45,7 @@ __device__ __forceinline__ bool prep_row_record(const RecJob& R, size_t rw, int 
 // with Y also forms the row dot products dot[t] = X_t . Y_t (the backward's
 // <g>_{P*} = dO_i . O*_i, App. B) from the rows it already holds.
 // One launch serves up to four tensors.  The work units (job, head, 32-row block)
-// are spread over a grid of a few CTAs per SM that loop over them, so the launch
+// are spread over a grid of sixteen CTAs per SM that loop over them, so the launch
 // has no partial last wave; a unit moves all d columns in 64-column steps through a
 // padded 32 x 65 shared tile (128 threads, four float4 loads and stores each).
 // ---------------------------------------------------------------------------
@@ -169,7 +169,9 @@ __global__ void __launch_bounds__(128) k_prep(const __grid_constant__ PrepJobs j
 cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool split, int nsm, cudaStream_t s) {
   if (jobs.n <= 0) return cudaSuccess;
   const int units = jobs.n * BH * (Tp / 32);
-  dim3 grid((unsigned)(units < 6 * nsm ? units : 6 * nsm)), block(128);
+  // sixteen 128-thread CTAs per SM (the most that are resident): a unit's loads, transpose
+  // and stores run one after the other, so the SM hides their latency with other CTAs' units
+  dim3 grid((unsigned)(units < 16 * nsm ? units : 16 * nsm)), block(128);
   return launch_pdl(split ? k_prep<true> : k_prep<false>, grid, block, 0, s, jobs, T, Tp, d, BH);
 }
 
