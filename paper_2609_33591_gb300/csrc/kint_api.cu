@@ -300,7 +300,7 @@ int plan_main(Params& p, int mode) {
       p.sm_table = p.sm_stage0 + p.nstage * p.sm_stage_bytes;
       p.sm_ostage = persist ? round_up(p.sm_table + table, 1024) : p.sm_stage0;
       const int end = persist ? p.sm_ostage + ostage : p.sm_table + table;
-      const int total = std::max(finish_plan(p, end, 10 + 2 * p.nstage), kOneCtaPerSm);
+      const int total = std::max(finish_plan(p, end, 11 + 2 * p.nstage), kOneCtaPerSm);
       if (total <= kSmemLimit) {
         // Issuing S(kb+1) before P V(kb) needs tile kb+1 in a second stage while
         // tile kb's V^T is still being read; with one stage the two would wait on

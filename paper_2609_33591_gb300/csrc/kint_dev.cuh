@@ -221,6 +221,19 @@ __device__ __forceinline__ void decode_u(float u, float Kf, float& t, uint32_t& 
   rb = __float_as_uint(fr);
 }
 
+// decode_u for FWM's forward with its zero tail folded into the table: u is clamped to
+// [-1, K] instead of [0, K], so a tail key (u < 0) rounds down to one of the two float
+// patterns just below 2^23 (2^23 - 1, 2^23 - 1/2), which address two zero entries placed
+// ahead of r = 0 (table base 16 bytes further on); u = 0 and u = -0.0 stay at r = 0, as
+// the strict cutoff wants.  In the tail t lies in [0, 1/2) and both weights read 0.
+constexpr int kFwdTail = 2;  // zero entries ahead of r = 0 in the forward FWM pair table
+__device__ __forceinline__ void decode_u_tail(float u, float Kf, float& t, uint32_t& rb) {
+  const float uc = fminf(fmaxf(u, -1.0f), Kf);
+  const float fr = fminf(__fadd_rd(uc, kMagic), kMagic + (Kf - 1.0f));
+  t = __fsub_rn(uc, __fsub_rn(fr, kMagic));
+  rb = __float_as_uint(fr);
+}
+
 // ---------------------------------------------------------------------------
 // FWM half-bin index.  With v = 2u (formed exactly as acc * 2k1 + 2c0) and
 // u = r + t, floor(v) = 2r + [t >= 1/2]: one floor gives both the bin r = q >> 1

@@ -484,9 +484,14 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
       wm = bf16_exp_weight(__fadd_rn(__fmul_rn(v[jj], g.k1), g.c0), zb);  // bf16(e^{bf16(s - M)})
     } else {
       const float u = __fmaf_rn(v[jj], g.k1, g.c0);
-      float t, rf;
+      float t;
       uint32_t rb;
-      decode_u(u, Kf, t, rb, rf);
+      if constexpr (CAL == CAL_FWM) {
+        decode_u_tail(u, Kf, t, rb);  // the tail reads the zero entries ahead of r = 0
+      } else {
+        float rf;
+        decode_u(u, Kf, t, rb, rf);
+      }
       // MinMax: this row's table, rows 1024 bytes apart; FWM: one shared table, entries 8 bytes apart
       float2 e = lds_f2(fwm_like(CAL) ? tab + rb * 8u : tab + rb * 1024u);
       if constexpr (CAL == CAL_FWMR) {
@@ -498,11 +503,6 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
       }
       wl = __fmaf_rn(t, __fsub_rn(e.y, e.x), e.x);
       float wn = (t >= 0.5f) ? e.y : e.x;
-      if constexpr (CAL == CAL_FWM) {
-        const bool tail = u < 0.0f;
-        wl = tail ? 0.f : wl;
-        wn = tail ? 0.f : wn;
-      }
       if constexpr (CAL == CAL_MINMAX) {
         wl = g.nogrid ? 1.f : wl;
         wn = g.nogrid ? 1.f : wn;
@@ -607,8 +607,15 @@ __device__ __forceinline__ bool main_issue_s(const Params& p, RingPos stg, int b
   return true;
 }
 
+// MODE 1 (Nearest weights for O, LERP weights for O_lerp) in TF32 issues its two P V
+// products from two warps on different SM sub-partitions: P V with the S products from
+// MMA_WARP, P^L V from MMA2_WARP, which frees the single A2 buffer (w^L) for the next
+// tile sooner than one warp issuing 32 MMAs back to back would.
+template <int MODE>
+constexpr int main_threads() { return MODE == 1 ? NTHR_DQ : NTHR; }
+
 template <int CAL, int REC, int MODE>
-__global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p) {
   uint8_t* sm = smem_base();
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int qtile = D * 512, vtile = D * 512;
@@ -624,28 +631,31 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
   uint64_t* bar_qfree = bars + 7 + 2 * NS;    // the item's last S product complete: Q may be reloaded
   uint64_t* bar_ofree = bars + 8 + 2 * NS;    // O / O_lerp read out of TMEM by every compute warp
   uint64_t* bar_drain = bars + 9 + 2 * NS;    // the MMA warp's clean-up commit
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 10 + 2 * NS);
+  uint64_t* bar_drain2 = bars + 10 + 2 * NS;  // MMA2_WARP's clean-up commit
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 11 + 2 * NS);
   uint8_t* ostg = sm + p.sm_ostage;
   float* xch = reinterpret_cast<float*>(ostg);  // [4][128], written before the staging tiles each item
   const int tid = threadIdx.x, warp = warp_id_uniform();
   const bool useA2 = (MODE == 1) || p.x3;
+  const bool split = MODE == 1 && !p.x3;  // P^L V from MMA2_WARP
   const int cA2 = 128 * nbuf, cO = cA2 + (useA2 ? 128 : 0), cOL = cO + D;
 
   if (tid == 0) {
     mbar_init(bar_q, 1);
     for (int s = 0; s < NS; ++s) {
       mbar_init(&bar_full[s], 1);
-      mbar_init(&bar_empty[s], 1);
+      mbar_init(&bar_empty[s], split ? 2 : 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar_s[b], 1);
       mbar_init(&bar_pready[b], NCOMP / 32);
     }
     mbar_init(bar_pv, 1);
-    mbar_init(bar_done, 1);
+    mbar_init(bar_done, split ? 2 : 1);
     mbar_init(bar_qfree, 1);
     mbar_init(bar_ofree, NCOMP / 32);
     mbar_init(bar_drain, 1);
+    mbar_init(bar_drain2, 1);
     fence_mbar_init();
   }
   if (warp == 0) {
@@ -726,10 +736,10 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
           mma_tmem_smem(tmem + cO, a, vt + vtile, D, 128, true);   // A_hi V_lo
           mma_tmem_smem(tmem + cO, a, vt, D, 128, true);           // A_hi V_hi
         } else {
-          if (MODE == 1) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);  // frees A2 first
+          if (MODE == 1 && !split) mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, acc);  // frees A2 first
           mma_tmem_smem(tmem + cO, a, vt, D, 128, acc);
         }
-        mma_commit(bar_pv);
+        if (!split) mma_commit(bar_pv);
         mma_commit(&bar_empty[s]);
         // one buffer: S(kb+1) overwrites the weights P V(kb) reads, in issue order after it
         if (nbuf == 1 && kb + 1 < nkb) {
@@ -743,6 +753,32 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       mma_commit(bar_done);
     }
     drain_mma(bar_drain, p.wait_ns, p.status);  // clean-up: no product still writes TMEM
+  } else if (warp == MMA2_WARP) {
+    // P^L V of every tile (split only): O_lerp += w^L V once the tile's weights are stored
+    if (split) {
+      int n = 0;
+      RingPos cs, cb;
+      bool ok = true;
+      for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+        const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
+        for (int kb = 0; kb < nkb; ++kb, cs.next(NS), cb.next(nbuf)) {
+          // the tile's K / V^T stage has landed: its weights, which need S, are stored
+          if (!mbar_wait_warp(&bar_pready[cb.i], cb.ph, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) ||
+              (kb == 0 && n > 0 && !mbar_wait_warp(bar_ofree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint8_t* vt = sm + p.sm_stage0 + cs.i * p.sm_stage_bytes + qtile;
+          mma_tmem_smem(tmem + cOL, tmem + cA2, vt, D, 128, kb > 0);
+          mma_commit(bar_pv);
+          mma_commit(&bar_empty[cs.i]);
+        }
+        if (!ok) break;
+        mma_commit(bar_done);
+      }
+      drain_mma(bar_drain2, p.wait_ns, p.status);  // clean-up: no product still writes TMEM
+    }
   } else {
     const int row = tid & 127, cg = tid >> 7;
     const float Kf = (float)Kq;
@@ -773,9 +809,12 @@ __global__ void __launch_bounds__(NTHR, 1) k_fwd_main(const __grid_constant__ Ma
       // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r).
       uint32_t tab;
       if constexpr (fwm_like(CAL)) {
-        tab = smem_u32(sm + p.sm_table) - 0x58000000u;
+        // entries r = 0 .. K-1 after kFwdTail zero entries (FWM's tail, decode_u_tail)
+        tab = smem_u32(sm + p.sm_table) + 8u * kFwdTail - 0x58000000u;
         if (n == 0 && tid < Kq)
-          *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+          *reinterpret_cast<float2*>(sm + p.sm_table + 8 * kFwdTail + tid * 8) =
+              make_float2(p.fwm_e[tid], p.fwm_e[tid + 1]);
+        if (n == 0 && tid < kFwdTail) *reinterpret_cast<float2*>(sm + p.sm_table + tid * 8) = make_float2(0.f, 0.f);
       } else {
         tab = smem_u32(sm + p.sm_table) + (uint32_t)row * 8u;
         if constexpr (CAL == CAL_MINMAX) {
@@ -897,7 +936,7 @@ static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_byt
   auto kern = k_fwd_main<CAL, REC, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kern, launch_grid(p), dim3(NTHR), smem_bytes, s, maps, p);
+  return launch_pdl(kern, launch_grid(p), dim3(main_threads<MODE>()), smem_bytes, s, maps, p);
 }
 
 cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
