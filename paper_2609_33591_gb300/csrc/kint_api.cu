@@ -7,7 +7,9 @@
 #include <cstdint>
 #include <cstring>
 #include <atomic>
+#include <memory>
 #include <mutex>
+#include <vector>
 
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -31,13 +33,78 @@ unsigned* g_status_ptr[kMaxDevices] = {nullptr};
 int g_dev_ok[kMaxDevices] = {0};  // 0 unknown, 1 sm_103, -1 other
 int g_num_sms[kMaxDevices] = {0};
 unsigned long long g_wait_ns = 2000000000ull;
-std::atomic<int> g_expire_waits{0};
-int g_bwd_path = 0;  // 0: single-pass backward where it applies, 1: always the two-pass kernels  // test hook: forward calls whose first kernel's first wait runs out
+std::atomic<int> g_expire_waits{0};  // test hook: forward calls whose first kernel's first wait runs out
+int g_bwd_path = 0;  // 0: single-pass backward where it applies, 1: always the two-pass kernels
 constexpr int kSmemLimit = 232448;  // opt-in maximum per CTA on sm_103
 constexpr int NCOMP_THREADS = 256;  // compute threads of the warp-specialised kernels (kint_dev.cuh NCOMP)
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Item schedules of the persistent kernels (Sched), longest processing time first: an
+// item costs a + tiles (a = its fixed cost in tiles: operand loads, epilogue, measured
+// per CTA), and items in decreasing cost each go to the CTA with the least work so far,
+// ties to the lower CTA.  Built once per kernel and shape and kept.
+enum SchedKind { SCHED_STATS = 0, SCHED_MAIN = 1, SCHED_FUSED = 2 };
+
+struct SchedEntry {
+  int kind, nitems, ngrid, BH, nqb, nqt;
+  Sched sch;
+};
+std::vector<std::unique_ptr<SchedEntry>> g_sched;
+
+const Sched& sched_for(int kind, const Params& p) {
+  static const Sched none = [] { Sched z; std::memset(&z, 0, sizeof(z)); return z; }();
+  if (p.ngrid >= p.nitems || p.ngrid > SCHED_MAX_CTAS || p.nitems > SCHED_MAX_ITEMS) return none;
+  const int nqt = kind == SCHED_FUSED ? p.nqt : 0;
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (const auto& e : g_sched)
+    if (e->kind == kind && e->nitems == p.nitems && e->ngrid == p.ngrid && e->BH == p.BH && e->nqb == p.nqb &&
+        e->nqt == nqt)
+      return e->sch;
+  if (g_sched.size() >= 256) return none;  // entries are never released: bound their number
+  // tiles and fixed cost of item i: query blocks (longest first) for the forward passes, key
+  // blocks with their 64-row query tiles for the single-pass backward
+  const double fixed = kind == SCHED_MAIN ? 2.6 : 2.0;
+  std::vector<double> cost(p.nitems);
+  for (int i = 0; i < p.nitems; ++i) {
+    int tiles;
+    if (kind == SCHED_FUSED)
+      tiles = p.nqt - (i / p.BH) * 2;
+    else
+      tiles = p.nqb - i / p.BH;
+    cost[i] = fixed + tiles;
+  }
+  std::vector<int> order(p.nitems);
+  for (int i = 0; i < p.nitems; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return cost[a] > cost[b]; });
+  std::vector<double> load(p.ngrid, 0.0);
+  std::vector<std::vector<int>> lists(p.ngrid);
+  for (int i : order) {
+    int best = 0;
+    for (int c = 1; c < p.ngrid; ++c)
+      if (load[c] < load[best]) best = c;
+    load[best] += cost[i];
+    lists[best].push_back(i);
+  }
+  auto e = std::make_unique<SchedEntry>();
+  std::memset(&e->sch, 0, sizeof(Sched));
+  e->kind = kind;
+  e->nitems = p.nitems;
+  e->ngrid = p.ngrid;
+  e->BH = p.BH;
+  e->nqb = p.nqb;
+  e->nqt = nqt;
+  int k = 0;
+  for (int c = 0; c < p.ngrid; ++c) {
+    e->sch.off[c] = (uint16_t)k;
+    for (int i : lists[c]) e->sch.idx[k++] = (uint16_t)i;
+  }
+  e->sch.off[p.ngrid] = (uint16_t)k;
+  e->sch.n = p.nitems;
+  g_sched.push_back(std::move(e));
+  return g_sched.back()->sch;
+}
 
 // Resolve the device-dependent handles once per device.
 int num_sms() {
@@ -457,7 +524,7 @@ int forward_prologue(const float* Q, const float* K, const float* V, const Param
   while (pending > 0 && !g_expire_waits.compare_exchange_weak(pending, pending - 1)) {
   }
   ps.expire_wait = pending > 0 ? 1 : 0;
-  return launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem, s); }));
+  return launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem, s, sched_for(SCHED_STATS, ps)); }));
 }
 
 int check_stats(const kint_rowstats* st, bool prob) {
@@ -512,13 +579,13 @@ int forward_launches(const float* Q, const float* K, const float* V, float* O, c
   pm.pv_sel = (prob && !p.x3) ? PV_MAIN_LERP : PV_MAIN;
   const int smem = plan_main(pm, pm.pv_sel);
   if (smem < 0 || smem > kSmemLimit) return KINT_ERR_UNSUPPORTED;
-  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); })))) return rc;
+  if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s, sched_for(SCHED_MAIN, pm)); })))) return rc;
   if (prob && p.x3) {
     Params pl = p;
     pl.pv_sel = PV_LERP;
     const int smem2 = plan_main(pl, PV_LERP);
     if (smem2 < 0) return KINT_ERR_UNSUPPORTED;
-    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s); })))) return rc;
+    if ((rc = launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pl, smem2, s, sched_for(SCHED_MAIN, pl)); })))) return rc;
   }
   return KINT_OK;
 }
@@ -678,7 +745,7 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
       pf.gate = w.tie_any;
       pf.gate_on = 0;
     }
-    if ((rc = launch_rc(traced("k_bwd_fused", s, [&] { return launch_bwd_fused(maps, pf, smem_f, s); })))) return rc;
+    if ((rc = launch_rc(traced("k_bwd_fused", s, [&] { return launch_bwd_fused(maps, pf, smem_f, s, sched_for(SCHED_FUSED, pf)); })))) return rc;
     if (!ext) return KINT_OK;
     if ((rc = launch_rc(traced("k_bwd_ext", s, [&] { return launch_bwd_ext(pf, s); })))) return rc;
     p.gate = w.tie_any;
@@ -741,7 +808,7 @@ int kint_attn_debug_bins(const float* Q, const float* K, const float* V, const k
   pm.debug = 1;
   pm.bins = bins;
   pm.ivals = ivals;
-  return launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s); }));
+  return launch_rc(traced("k_fwd_main", s, [&] { return launch_fwd_main(maps, pm, smem, s, sched_for(SCHED_MAIN, pm)); }));
 }
 
 int kint_attn_probe(const float* Q, const float* K, const kint_rowstats* st, float* probe, int B, int H, int T,
@@ -783,7 +850,7 @@ int kint_attn_probe(const float* Q, const float* K, const kint_rowstats* st, flo
   // pass 1 (row extrema), then the probe's two sweeps
   Params ps = p;
   const int smem_s = plan_stats(ps);
-  if ((rc = launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem_s, s); })))) return rc;
+  if ((rc = launch_rc(traced("k_fwd_stats", s, [&] { return launch_fwd_stats(maps, ps, smem_s, s, sched_for(SCHED_STATS, ps)); })))) return rc;
   Params pp = p;
   const int smem_p = plan_probe(pp);
   if (smem_p < 0 || smem_p > kSmemLimit) return KINT_ERR_UNSUPPORTED;

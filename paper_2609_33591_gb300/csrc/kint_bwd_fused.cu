@@ -134,7 +134,7 @@ __device__ __forceinline__ void rowsum_red(const float (&v)[16], float* dst, siz
 // ---------------------------------------------------------------------------
 // k_bwd_fused (608 threads: 16 compute warps, the MMA warp, two producer warps).  Work
 // items are (128-key block kb, head) pairs, longest first; a CTA
-// takes snake_item(0), snake_item(1), ...  Thread t (< 512) owns key j = kb*128 + t%128
+// takes sched_item(sch, 0), sched_item(sch, 1), ...  Thread t (< 512) owns key j = kb*128 + t%128
 // (TMEM lane t%128) and the 16 query columns 16 (t/128) .. +15 of each 64-query tile:
 // four compute warps per SM sub-partition, so that one warp's latencies (TMEM and
 // shared-memory loads, shuffles) hide under the others' element work.
@@ -165,7 +165,8 @@ __device__ __forceinline__ uint32_t sw64_off(int r, int c) {
 }
 
 template <int CAL, int REC, bool FULLG>
-__global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_constant__ Maps maps, const Params p,
+                                                           const __grid_constant__ Sched sch) {
   uint8_t* sm = smem_base();
   constexpr int D = 64, NS = 2;
   constexpr int qtile = BT * D * 4;
@@ -240,7 +241,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
   // items' K rows and V tiles, PRODUCER2_WARP_F the Q^T | dO^T halves and the K^T tiles, so
   // that neither kind of load waits behind the other's condition.
   auto item_of = [&](int k, int& kb_, int& bh_) {
-    const int it_ = snake_item(k);
+    const int it_ = sched_item(sch, k);
     kb_ = it_ / p.BH;
     bh_ = it_ % p.BH;
   };
@@ -263,8 +264,8 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
       load_rows_tile_boxed(sm + p.sm_v, &maps.v, bar_v, D, 128, BT, 0, kb_ * 128, bh_);
       ++nv;
     };
-    if (snake_item(0) < p.nitems) load_k(0);
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    if (sched_item(sch, 0) < p.nitems) load_k(0);
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
       for (int it = 0; it < nit; ++it, ++gt, ld.next(NS)) {
@@ -293,7 +294,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         }
       }
       // the next item's K rows, once this item's last g^T has read V
-      if (ok && snake_item(n + 1) < p.nitems) {
+      if (ok && sched_item(sch, n + 1) < p.nitems) {
         if (!mbar_wait_warp(bar_vfree, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA)) {
           ok = false;
           break;
@@ -317,7 +318,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
       load_rows_tile(sm + p.sm_kt, &maps.kt, bar_kt, 128, D, kb_ * 128, 0, bh_);
       ++nkt;
     };
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
       for (int it = 0; it < nit; ++it, ++gt, ld.next(NS)) {
@@ -369,7 +370,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
       ib.next(2);
       return true;
     };
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int kb = item / p.BH, nit = nqt - (kb * 128) / BT;
       ok = mbar_wait_warp(bar_ops, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC) &&
            mbar_wait_warp(bar_v, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
@@ -472,7 +473,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         }
       }
     };
-    if (snake_item(0) < p.nitems) ops_to_tmem(0);
+    if (sched_item(sch, 0) < p.nitems) ops_to_tmem(0);
     constexpr bool half = fwm_like(CAL) && REC == REC_NEAREST;
     if constexpr (fwm_like(CAL)) {
       if (half && tid < 2 * Kq + 1 + kHalfTail)
@@ -487,7 +488,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     int n = 0, gu = 0;  // gu: tiles so far over the CTA's run (stage parity, bar_dqfull, bar_tfree)
     RingPos cs, cb;
     const int c0 = cq * 16;  // this thread's query columns in every tile
-    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && !failed; item = sched_item(sch, ++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
       const int j = kb * 128 + row;
@@ -565,7 +566,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         __syncwarp();
         if (lane == 0) mbar_arrive(&bar_pready[b]);
         // the item's last S^T has completed: the next item's K rows may replace these
-        if (it + 1 == nit && snake_item(n + 1) < p.nitems) ops_to_tmem(n + 1);
+        if (it + 1 == nit && sched_item(sch, n + 1) < p.nitems) ops_to_tmem(n + 1);
       }
       const bool dok = !failed && mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       failed = group_any(BAR_COMPUTE, NCOMP_F, !dok);
@@ -680,30 +681,39 @@ __global__ void __launch_bounds__(256) k_bwd_ext(const Params p) {
   }
 }
 
+template <class K>
+static cudaError_t launch_fused_k(K kern, dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s,
+                                  const Sched& sch) {
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(kern, grid, dim3(NTHR_FUSED), smem_bytes, s, maps, p, sch);
+}
+
 template <int CAL, int REC>
-static cudaError_t launch_fused_modes(dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+static cudaError_t launch_fused_modes(dim3 grid, const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s,
+                                      const Sched& sch) {
   const bool full = p.grad != GRAD_DETACH && p.grad != GRAD_DETACH_PROJ;
   if constexpr (CAL == CAL_SOFTMAX) {
-    return launch3(k_bwd_fused<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s, NTHR_FUSED);
+    return launch_fused_k(k_bwd_fused<CAL_SOFTMAX, REC_LERP, false>, grid, maps, p, smem_bytes, s, sch);
   } else {
-    return full ? launch3(k_bwd_fused<CAL, REC, true>, grid, maps, p, smem_bytes, s, NTHR_FUSED)
-                : launch3(k_bwd_fused<CAL, REC, false>, grid, maps, p, smem_bytes, s, NTHR_FUSED);
+    return full ? launch_fused_k(k_bwd_fused<CAL, REC, true>, grid, maps, p, smem_bytes, s, sch)
+                : launch_fused_k(k_bwd_fused<CAL, REC, false>, grid, maps, p, smem_bytes, s, sch);
   }
 }
 
-cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch) {
   const dim3 grid((unsigned)p.ngrid);
   const bool near = p.recon == REC_NEAREST;
   switch (p.calib) {
-    case CAL_SOFTMAX: return launch_fused_modes<CAL_SOFTMAX, REC_LERP>(grid, maps, p, smem_bytes, s);
-    case CAL_EXP8: return launch_fused_modes<CAL_EXP8, REC_LERP>(grid, maps, p, smem_bytes, s);
-    case CAL_EXPB: return launch_fused_modes<CAL_EXPB, REC_LERP>(grid, maps, p, smem_bytes, s);
+    case CAL_SOFTMAX: return launch_fused_modes<CAL_SOFTMAX, REC_LERP>(grid, maps, p, smem_bytes, s, sch);
+    case CAL_EXP8: return launch_fused_modes<CAL_EXP8, REC_LERP>(grid, maps, p, smem_bytes, s, sch);
+    case CAL_EXPB: return launch_fused_modes<CAL_EXPB, REC_LERP>(grid, maps, p, smem_bytes, s, sch);
     case CAL_FWMR:
-      return near ? launch_fused_modes<CAL_FWMR, REC_NEAREST>(grid, maps, p, smem_bytes, s)
-                  : launch_fused_modes<CAL_FWMR, REC_LERP>(grid, maps, p, smem_bytes, s);
+      return near ? launch_fused_modes<CAL_FWMR, REC_NEAREST>(grid, maps, p, smem_bytes, s, sch)
+                  : launch_fused_modes<CAL_FWMR, REC_LERP>(grid, maps, p, smem_bytes, s, sch);
     case CAL_FWM:
-      return near ? launch_fused_modes<CAL_FWM, REC_NEAREST>(grid, maps, p, smem_bytes, s)
-                  : launch_fused_modes<CAL_FWM, REC_LERP>(grid, maps, p, smem_bytes, s);
+      return near ? launch_fused_modes<CAL_FWM, REC_NEAREST>(grid, maps, p, smem_bytes, s, sch)
+                  : launch_fused_modes<CAL_FWM, REC_LERP>(grid, maps, p, smem_bytes, s, sch);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -153,6 +153,14 @@ __device__ __forceinline__ int snake_item(int n) {
   return n * G + ((n & 1) ? G - 1 - c : c);
 }
 
+// n-th work item of this CTA under a host schedule (Sched), or in snake order without
+// one; past the CTA's last item it returns a value above every item index.
+__device__ __forceinline__ int sched_item(const Sched& s, int n) {
+  if (s.n == 0) return snake_item(n);
+  const int k = s.off[blockIdx.x] + n;
+  return k < s.off[blockIdx.x + 1] ? (int)s.idx[k] : 0x7fffffff;
+}
+
 // ---------------------------------------------------------------------------
 // Row grid.  Scores s are fp32 values of acc * scale.  The position of a key in
 // grid units is u = s * inv_h + c0:

@@ -260,7 +260,8 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
 static dim3 launch_grid(const Params& p) { return dim3((unsigned)p.ngrid); }
 
 template <bool MIN>
-__global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ Maps maps, const Params p,
+                                                         const __grid_constant__ Sched sch) {
   uint8_t* sm = smem_base();
   const int D = p.d, tile = D * 512, parts = p.x3 ? 2 : 1, NS = p.nstage;
   uint8_t* sQ = sm + p.sm_a;
@@ -311,7 +312,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
     int g = 0, n = 0;
     RingPos ld;  // stage of the next K tile loaded
     bool ok = true;
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       if (n > 0 && !mbar_wait_warp(bar_qfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
       mbar_arrive_expect_tx(bar_q, parts * tile);
@@ -336,7 +337,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
     int g = 0, n = 0;
     RingPos cs;  // stage of the current K tile
     bool ok = true;
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
       ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
       for (int kb = 0; kb < nkb && ok; ++kb, cs.next(NS)) {
@@ -371,7 +372,7 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
     const int row = tid & 127, cg = tid >> 7;
     int g = 0, n = 0;
     bool failed = false;
-    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && !failed; item = sched_item(sch, ++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       const int i = qb * 128 + row;
       float M = -FLT_MAX, m = FLT_MAX;
@@ -453,11 +454,11 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
   if (warp == 0) tmem_dealloc(tmem, 256);
 }
 
-cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch) {
   auto kern = p.calib == CAL_MINMAX ? k_fwd_stats<true> : k_fwd_stats<false>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kern, launch_grid(p), dim3(NTHR), smem_bytes, s, maps, p);
+  return launch_pdl(kern, launch_grid(p), dim3(NTHR), smem_bytes, s, maps, p, sch);
 }
 
 // ---------------------------------------------------------------------------
@@ -574,7 +575,7 @@ __device__ void fwd_debug_codes(const Params& p, const float (&v)[32], int j0, i
 // ---------------------------------------------------------------------------
 // Pass 2: reconstruction, normalization and P V (App. A).
 // Work items are (128-row query block, head) pairs, longest blocks first; a CTA
-// takes the items snake_item(0), snake_item(1), ... (one item per CTA when the
+// takes the items sched_item(sch, 0), sched_item(sch, 1), ... (one item per CTA when the
 // grid covers them all).  Tile counters run on across items, so the next item's Q
 // and first K/V tiles load while the current one finishes.
 // TMEM: score buffers S_b at [128 b, 128 b + 128), b < nbuf (the weights
@@ -615,7 +616,8 @@ template <int MODE>
 constexpr int main_threads() { return MODE == 1 ? NTHR_DQ : NTHR; }
 
 template <int CAL, int REC, int MODE>
-__global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p) {
+__global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __grid_constant__ Maps maps, const Params p,
+                                                                   const __grid_constant__ Sched sch) {
   uint8_t* sm = smem_base();
   const int D = p.d, Kq = p.Kint, parts = p.x3 ? 2 : 1, NS = p.nstage, nbuf = p.nbuf;
   const int qtile = D * 512, vtile = D * 512;
@@ -676,7 +678,7 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
     int g = 0, n = 0;
     RingPos ld;  // stage of the next K/V tile loaded
     bool ok = true;
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       // Q of the previous item is an operand until its last S product completes
       if (n > 0 && !mbar_wait_warp(bar_qfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) break;
@@ -707,7 +709,7 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
     int g = 0, n = 0;
     RingPos is, ib, cs, cb;  // stage / buffer of the next S product and of the tile being finished
     bool ok = true;
-    for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+    for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
       ok = mbar_wait_warp(bar_q, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA) &&
            main_issue_s(p, is, ib.i, bar_full, bar_s, st0, sQ, tmem, qtile);
@@ -759,7 +761,7 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
       int n = 0;
       RingPos cs, cb;
       bool ok = true;
-      for (int item = snake_item(n); item < p.nitems && ok; item = snake_item(++n)) {
+      for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
         const int qb = p.nqb - 1 - item / p.BH, nkb = qb + 1;
         for (int kb = 0; kb < nkb; ++kb, cs.next(NS), cb.next(nbuf)) {
           // the tile's K / V^T stage has landed: its weights, which need S, are stored
@@ -787,15 +789,15 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
     bool failed = false;
     // the row extrema of an item, loaded one item ahead (under the previous item's epilogue)
     auto load_extrema = [&](int n, float& M, float& m) {
-      const int item = snake_item(n);
+      const int item = sched_item(sch, n);
       const int i = (p.nqb - 1 - item / p.BH) * 128 + row;
       const size_t rw = (size_t)(item % p.BH) * p.T + i;
       M = i < p.T ? p.row_max[rw] : 0.0f;
       m = i < p.T ? p.row_min[rw] : 0.0f;
     };
     float nM = 0.f, nm = 0.f;
-    if (snake_item(0) < p.nitems) load_extrema(0, nM, nm);
-    for (int item = snake_item(n); item < p.nitems && !failed; item = snake_item(++n)) {
+    if (sched_item(sch, 0) < p.nitems) load_extrema(0, nM, nm);
+    for (int item = sched_item(sch, n); item < p.nitems && !failed; item = sched_item(sch, ++n)) {
       const int qb = p.nqb - 1 - item / p.BH, bh = item % p.BH, nkb = qb + 1;
       const int i = qb * 128 + row;
       const bool row_ok = i < p.T;
@@ -871,7 +873,7 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
         if ((tid & 31) == 0) mbar_arrive(&bar_pready[b]);
       }
       g += nkb;
-      if (snake_item(n + 1) < p.nitems) load_extrema(n + 1, nM, nm);
+      if (sched_item(sch, n + 1) < p.nitems) load_extrema(n + 1, nM, nm);
       if (!failed) failed = !mbar_wait(bar_done, n & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_MMA);
       failed = group_any(BAR_COMPUTE, NCOMP, failed);
       if (failed) break;
@@ -932,34 +934,34 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
 }
 
 template <int CAL, int REC, int MODE>
-static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+static cudaError_t launch_main_t(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch) {
   auto kern = k_fwd_main<CAL, REC, MODE>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kern, launch_grid(p), dim3(main_threads<MODE>()), smem_bytes, s, maps, p);
+  return launch_pdl(kern, launch_grid(p), dim3(main_threads<MODE>()), smem_bytes, s, maps, p, sch);
 }
 
-cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s) {
+cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch) {
   const int mode = p.pv_sel;
-  if (p.calib == CAL_SOFTMAX) return launch_main_t<CAL_SOFTMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
-  if (p.calib == CAL_EXP8) return launch_main_t<CAL_EXP8, REC_LERP, 0>(maps, p, smem_bytes, s);
-  if (p.calib == CAL_EXPB) return launch_main_t<CAL_EXPB, REC_LERP, 0>(maps, p, smem_bytes, s);
+  if (p.calib == CAL_SOFTMAX) return launch_main_t<CAL_SOFTMAX, REC_LERP, 0>(maps, p, smem_bytes, s, sch);
+  if (p.calib == CAL_EXP8) return launch_main_t<CAL_EXP8, REC_LERP, 0>(maps, p, smem_bytes, s, sch);
+  if (p.calib == CAL_EXPB) return launch_main_t<CAL_EXPB, REC_LERP, 0>(maps, p, smem_bytes, s, sch);
   if (p.calib == CAL_MINMAX) {
-    if (p.recon == REC_LERP) return launch_main_t<CAL_MINMAX, REC_LERP, 0>(maps, p, smem_bytes, s);
-    if (mode == PV_MAIN) return launch_main_t<CAL_MINMAX, REC_NEAREST, 0>(maps, p, smem_bytes, s);
-    if (mode == PV_MAIN_LERP) return launch_main_t<CAL_MINMAX, REC_NEAREST, 1>(maps, p, smem_bytes, s);
-    return launch_main_t<CAL_MINMAX, REC_NEAREST, 2>(maps, p, smem_bytes, s);
+    if (p.recon == REC_LERP) return launch_main_t<CAL_MINMAX, REC_LERP, 0>(maps, p, smem_bytes, s, sch);
+    if (mode == PV_MAIN) return launch_main_t<CAL_MINMAX, REC_NEAREST, 0>(maps, p, smem_bytes, s, sch);
+    if (mode == PV_MAIN_LERP) return launch_main_t<CAL_MINMAX, REC_NEAREST, 1>(maps, p, smem_bytes, s, sch);
+    return launch_main_t<CAL_MINMAX, REC_NEAREST, 2>(maps, p, smem_bytes, s, sch);
   }
   if (p.calib == CAL_FWMR) {
-    if (p.recon == REC_LERP) return launch_main_t<CAL_FWMR, REC_LERP, 0>(maps, p, smem_bytes, s);
-    if (mode == PV_MAIN) return launch_main_t<CAL_FWMR, REC_NEAREST, 0>(maps, p, smem_bytes, s);
-    if (mode == PV_MAIN_LERP) return launch_main_t<CAL_FWMR, REC_NEAREST, 1>(maps, p, smem_bytes, s);
-    return launch_main_t<CAL_FWMR, REC_NEAREST, 2>(maps, p, smem_bytes, s);
+    if (p.recon == REC_LERP) return launch_main_t<CAL_FWMR, REC_LERP, 0>(maps, p, smem_bytes, s, sch);
+    if (mode == PV_MAIN) return launch_main_t<CAL_FWMR, REC_NEAREST, 0>(maps, p, smem_bytes, s, sch);
+    if (mode == PV_MAIN_LERP) return launch_main_t<CAL_FWMR, REC_NEAREST, 1>(maps, p, smem_bytes, s, sch);
+    return launch_main_t<CAL_FWMR, REC_NEAREST, 2>(maps, p, smem_bytes, s, sch);
   }
-  if (p.recon == REC_LERP) return launch_main_t<CAL_FWM, REC_LERP, 0>(maps, p, smem_bytes, s);
-  if (mode == PV_MAIN) return launch_main_t<CAL_FWM, REC_NEAREST, 0>(maps, p, smem_bytes, s);
-  if (mode == PV_MAIN_LERP) return launch_main_t<CAL_FWM, REC_NEAREST, 1>(maps, p, smem_bytes, s);
-  return launch_main_t<CAL_FWM, REC_NEAREST, 2>(maps, p, smem_bytes, s);
+  if (p.recon == REC_LERP) return launch_main_t<CAL_FWM, REC_LERP, 0>(maps, p, smem_bytes, s, sch);
+  if (mode == PV_MAIN) return launch_main_t<CAL_FWM, REC_NEAREST, 0>(maps, p, smem_bytes, s, sch);
+  if (mode == PV_MAIN_LERP) return launch_main_t<CAL_FWM, REC_NEAREST, 1>(maps, p, smem_bytes, s, sch);
+  return launch_main_t<CAL_FWM, REC_NEAREST, 2>(maps, p, smem_bytes, s, sch);
 }
 
 }  // namespace kint

@@ -57,8 +57,9 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, dim3 block, int smem, cudaStream_t 
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
-cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
-cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
+// sch: the host item schedule of the persistent kernels (Sched::n == 0: snake order)
+cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch);
+cudaError_t launch_fwd_main(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch);
 cudaError_t launch_bwd_dq(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 // Geometry probe: per-row span, width, softmax entropy, share below -6, top-bucket mass,
@@ -66,7 +67,7 @@ cudaError_t launch_bwd_dkdv(const Maps& maps, const Params& p, int smem_bytes, c
 cudaError_t launch_fwd_probe(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
 // Single-pass backward (TF32, d = 64; its row records come from the dO prep job, RecJob):
 // the pass itself, and the extremum terms it leaves for afterwards
-cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s);
+cudaError_t launch_bwd_fused(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch);
 cudaError_t launch_bwd_ext(const Params& p, cudaStream_t s);
 // C = running sums of the key rows of every head, [BH][T][d] (the P1 projection)
 cudaError_t launch_kcum(const float* K, float* C, int BH, int T, int d, cudaStream_t s);

@@ -39,6 +39,16 @@ struct Maps {
   CUtensorMap dq16, dk32, dv32;  // single-pass backward: 16-column boxes (64-byte swizzle), dQ reduces of 16 rows, dK / dV stores of 32
 };
 
+// Static item schedule of a persistent kernel, computed on the host (longest processing
+// time first over the launch's CTAs): CTA c takes the items idx[off[c]] .. idx[off[c+1] - 1]
+// in that order.  n == 0: no schedule, the snake order (snake_item) instead.
+constexpr int SCHED_MAX_CTAS = 304, SCHED_MAX_ITEMS = 1536;
+struct Sched {
+  int n;
+  uint16_t off[SCHED_MAX_CTAS + 1];
+  uint16_t idx[SCHED_MAX_ITEMS];
+};
+
 struct Params {
   int B, H, T, d, Kint, calib, recon, ste, grad, x3;
   int BH, nqb;  // number of 128-row query blocks
