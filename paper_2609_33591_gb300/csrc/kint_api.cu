@@ -349,8 +349,11 @@ int plan_probe(Params& p) {
 // and the deepest K/V ring that fit.
 int plan_main(Params& p, int mode) {
   const int parts = p.x3 ? 2 : 1, tile = p.d * 512;
-  // (e_r, e_{r+1}) pairs: per row for MinMax ([K][128]), one shared [K] for FWM
-  const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024 : (p.calib == KINT_CALIB_FWM || p.calib == KINT_CALIB_FWM_RESOLVED ? 1024 : 0);
+  // (e_r, e_{r+1}) pairs: per row for MinMax ([K][128]), one shared [K] for FWMR; FWM's
+  // half-bin table of 16-byte entries, q in [-2, 2K]
+  const int table = p.calib == KINT_CALIB_MINMAX ? p.Kint * 1024
+                    : p.calib == KINT_CALIB_FWM  ? std::max(1024, round_up((2 * p.Kint + 3) * 16, 128))
+                    : p.calib == KINT_CALIB_FWM_RESOLVED ? 1024 : 0;
   const bool useA2 = mode == PV_MAIN_LERP || p.x3;
   const int cols1 = 128 + (useA2 ? 128 : 0) + p.d + (mode == PV_MAIN_LERP ? p.d : 0);
   const int ostage = (mode == PV_MAIN_LERP ? 2 : 1) * 128 * p.d * 4;  // O (and O_lerp) staging tiles

@@ -229,18 +229,8 @@ __device__ __forceinline__ void decode_u(float u, float Kf, float& t, uint32_t& 
   rb = __float_as_uint(fr);
 }
 
-// decode_u for FWM's forward with its zero tail folded into the table: u is clamped to
-// [-1, K] instead of [0, K], so a tail key (u < 0) rounds down to one of the two float
-// patterns just below 2^23 (2^23 - 1, 2^23 - 1/2), which address two zero entries placed
-// ahead of r = 0 (table base 16 bytes further on); u = 0 and u = -0.0 stay at r = 0, as
-// the strict cutoff wants.  In the tail t lies in [0, 1/2) and both weights read 0.
-constexpr int kFwdTail = 2;  // zero entries ahead of r = 0 in the forward FWM pair table
-__device__ __forceinline__ void decode_u_tail(float u, float Kf, float& t, uint32_t& rb) {
-  const float uc = fminf(fmaxf(u, -1.0f), Kf);
-  const float fr = fminf(__fadd_rd(uc, kMagic), kMagic + (Kf - 1.0f));
-  t = __fsub_rn(uc, __fsub_rn(fr, kMagic));
-  rb = __float_as_uint(fr);
-}
+// Zero entries ahead of r = 0 in the pair table of the resolved policy's forward (FWMR).
+constexpr int kFwdTail = 2;
 
 // ---------------------------------------------------------------------------
 // FWM half-bin index.  With v = 2u (formed exactly as acc * 2k1 + 2c0) and
@@ -263,6 +253,18 @@ __device__ __forceinline__ float2 fwm_half_entry(const Params& p, int q) {
   const int r = min(q >> 1, p.Kint - 1);
   const float dlt = __fmul_rn(__fsub_rn(p.fwm_e[r + 1], p.fwm_e[r]), p.fwm_inv_h);
   return make_float2(p.fwm_e[(q + 1) >> 1], dlt);
+}
+
+// Entry q in [-2, 2K] of the forward's FWM half-bin table: {alpha, beta, w^N, 0} with
+// r = min(q >> 1, K - 1), beta = (e_{r+1} - e_r) / 2 and alpha = e_r - 2 r beta, so that
+// the LERP weight e_r + (u - r)(e_{r+1} - e_r) is the bin's line alpha + v beta at v = 2u
+// and w^N = e_{(q+1) >> 1} is the Nearest endpoint; the tail entries (q < 0) are zero, so a
+// key below the window reads w^L = w^N = 0 whatever its v.
+__device__ __forceinline__ float4 fwm_line_entry(const Params& p, int q) {
+  if (q < 0) return make_float4(0.f, 0.f, 0.f, 0.f);
+  const int r = min(q >> 1, p.Kint - 1);
+  const float beta = 0.5f * __fsub_rn(p.fwm_e[r + 1], p.fwm_e[r]);
+  return make_float4(__fmaf_rn(-2.0f * (float)r, beta, p.fwm_e[r]), beta, p.fwm_e[(q + 1) >> 1], 0.f);
 }
 
 __device__ __forceinline__ float lds_f32(uint32_t addr) {

@@ -483,17 +483,32 @@ __device__ __forceinline__ void fwd_chunk(const float (&v)[32], float (&a1)[32],
     } else if constexpr (CAL == CAL_EXPB) {
       float zb;
       wm = bf16_exp_weight(__fadd_rn(__fmul_rn(v[jj], g.k1), g.c0), zb);  // bf16(e^{bf16(s - M)})
+    } else if constexpr (CAL == CAL_FWM) {
+      // v = 2u = acc * 2k1 + 2c0 (sk1, sc0) clamped to [-1, 2K]; floor(v) = q = 2r + [t >= 1/2]
+      // indexes the half-bin table {alpha, beta, w^N, 0} by the float bits of its round-down
+      // (entry q at tab + 16 bits), with the tail (u < 0) on the two zero entries below q = 0:
+      // w^L = alpha + v beta, w^N = the Nearest endpoint.  Same decisions as decode_u.
+      constexpr bool need_wn = REC == REC_NEAREST && MODE != 2;
+      constexpr bool need_wl = REC == REC_LERP || MODE != 0;
+      const float vc = fminf(fmaxf(__fmaf_rn(v[jj], sk1, sc0), -1.0f), 2.0f * Kf);
+      const uint32_t a = tab + (__float_as_uint(__fadd_rd(vc, kMagic)) << 4);
+      if constexpr (need_wn && need_wl) {
+        const float2 e = lds_f2(a);
+        wl = __fmaf_rn(vc, e.y, e.x);
+        wm = lds_f32(a + 8u);
+      } else if constexpr (need_wn) {
+        wm = lds_f32(a + 8u);
+      } else {
+        const float2 e = lds_f2(a);
+        wl = __fmaf_rn(vc, e.y, e.x);
+        wm = wl;
+      }
     } else {
       const float u = __fmaf_rn(v[jj], g.k1, g.c0);
-      float t;
+      float t, rf;
       uint32_t rb;
-      if constexpr (CAL == CAL_FWM) {
-        decode_u_tail(u, Kf, t, rb);  // the tail reads the zero entries ahead of r = 0
-      } else {
-        float rf;
-        decode_u(u, Kf, t, rb, rf);
-      }
-      // MinMax: this row's table, rows 1024 bytes apart; FWM: one shared table, entries 8 bytes apart
+      decode_u(u, Kf, t, rb, rf);
+      // MinMax: this row's table, rows 1024 bytes apart; FWMR: one shared table, entries 8 bytes apart
       float2 e = lds_f2(fwm_like(CAL) ? tab + rb * 8u : tab + rb * 1024u);
       if constexpr (CAL == CAL_FWMR) {
         // below the window: the continued grid (negative r)
@@ -804,14 +819,24 @@ __global__ void __launch_bounds__(main_threads<MODE>(), 1) k_fwd_main(const __gr
       const size_t rw = (size_t)bh * p.T + (row_ok ? i : 0);
       const float M = nM, m = nm;
       const RowGrid gr = row_grid(p, M, m);
-      const float sk1 = p.scale * 1.4426950408889634f, sc0 = -M * 1.4426950408889634f;  // softmax, base 2
+      // softmax: base-2 exponent coefficients; FWM: the half-bin position v = 2u = acc * 2k1 + 2c0
+      // (an exact doubling of u)
+      const float sk1 = CAL == CAL_FWM ? 2.0f * gr.k1 : p.scale * 1.4426950408889634f;
+      const float sc0 = CAL == CAL_FWM ? 2.0f * gr.c0 : -M * 1.4426950408889634f;
       // Pair tables, entry r = (e_r, e_{r+1}), r = 0..K-1, addressed by the float bits
       // rb = 0x4B000000 + r of the floored position: MinMax keeps one table per row
-      // ([K][128], 1024 bytes per r: rb * 1024 wraps to r * 1024); FWM's grid is the
-      // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r).
+      // ([K][128], 1024 bytes per r: rb * 1024 wraps to r * 1024); FWMR's grid is the
+      // same for every row, so one [K] table serves all (rb * 8 = 0x58000000 + 8 r), and
+      // FWM's one half-bin table of line coefficients.
       uint32_t tab;
-      if constexpr (fwm_like(CAL)) {
-        // entries r = 0 .. K-1 after kFwdTail zero entries (FWM's tail, decode_u_tail)
+      if constexpr (CAL == CAL_FWM) {
+        // the half-bin table, entry q in [-2, 2K] at sm_table + 16 (q + 2); the float bits
+        // 0x4B000000 + q of the rounded-down position times 16 wrap to 0xB0000000 + 16 q
+        tab = smem_u32(sm + p.sm_table) + 16u * kHalfTail - 0xB0000000u;
+        if (n == 0 && tid < 2 * Kq + 1 + kHalfTail)
+          *reinterpret_cast<float4*>(sm + p.sm_table + tid * 16) = fwm_line_entry(p, tid - kHalfTail);
+      } else if constexpr (CAL == CAL_FWMR) {
+        // entries r = 0 .. K-1 after kFwdTail zero entries
         tab = smem_u32(sm + p.sm_table) + 8u * kFwdTail - 0x58000000u;
         if (n == 0 && tid < Kq)
           *reinterpret_cast<float2*>(sm + p.sm_table + 8 * kFwdTail + tid * 8) =
