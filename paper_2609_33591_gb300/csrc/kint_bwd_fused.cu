@@ -132,7 +132,7 @@ __device__ __forceinline__ void rowsum_red(const float (&v)[16], float* dst, siz
 
 
 // ---------------------------------------------------------------------------
-// k_bwd_fused (608 threads: 16 compute warps, the MMA warp, two producer warps).  Work
+// k_bwd_fused (640 threads: 16 compute warps, the MMA warp, two producer warps, an idle warp).  Work
 // items are (128-key block kb, head) pairs, longest first; a CTA
 // takes sched_item(sch, 0), sched_item(sch, 1), ...  Thread t (< 512) owns key j = kb*128 + t%128
 // (TMEM lane t%128) and the 16 query columns 16 (t/128) .. +15 of each 64-query tile:
@@ -155,7 +155,13 @@ __device__ __forceinline__ void rowsum_red(const float (&v)[16], float* dst, siz
 // ---------------------------------------------------------------------------
 constexpr int NCOMP_F = 512;  // compute threads
 constexpr int MMA_WARP_F = NCOMP_F / 32, PRODUCER_WARP_F = NCOMP_F / 32 + 1, PRODUCER2_WARP_F = NCOMP_F / 32 + 2;
-constexpr int NTHR_FUSED = NCOMP_F + 96;
+// The MMA warp, the two producer warps and a fourth, idle warp form the fifth warpgroup, which
+// gives registers to the four compute warpgroups: launched at 96 per thread (640 threads),
+// it keeps 64 and the compute warps take 104 (512 x 104 + 128 x 64 = 640 x 96).
+constexpr int NTHR_FUSED = NCOMP_F + 128;
+constexpr int REG_LAUNCH_F = 96, REG_COMP_F = 104, REG_AUX_F = 64;
+static_assert(NCOMP_F * REG_COMP_F + (NTHR_FUSED - NCOMP_F) * REG_AUX_F <= NTHR_FUSED * REG_LAUNCH_F,
+              "register shares exceed the launch allocation");
 
 // Byte offset of 16-byte chunk c of row r in a tile of 64-byte rows under the 64-byte
 // swizzle (chunk index XOR bits 1..2 of the row), the layout TMA reads for the dQ reduce
@@ -236,6 +242,11 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     if (warp == 0) tmem_dealloc(tmem, 512);
     return;
   }
+
+  if (warp < NCOMP_F / 32)
+    setmaxnreg_inc<REG_COMP_F>();
+  else
+    setmaxnreg_dec<REG_AUX_F>();
 
   // Two producer warps: PRODUCER_WARP_F loads the Q | dO halves with their records and the
   // items' K rows and V tiles, PRODUCER2_WARP_F the Q^T | dO^T halves and the K^T tiles, so
