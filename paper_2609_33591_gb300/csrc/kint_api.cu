@@ -681,7 +681,9 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     pl.add(dO, w.doh, w.dol, w.doth, w.dotl, p.Ostar, w.gbar);
   } else {
     pl.add(Q, nullptr, nullptr, w.qth, nullptr);
-    pl.add(K, nullptr, nullptr, w.kth, nullptr);
+    // the single pass forms its K^T tiles from the K rows it holds in TMEM (k_bwd_ext writes K^T
+    // for the two-pass kernels if they run instead)
+    if (!single) pl.add(K, nullptr, nullptr, w.kth, nullptr);
     pl.add(dO, nullptr, nullptr, w.doth, nullptr, p.Ostar, w.gbar);
   }
   if (single) {
@@ -738,6 +740,7 @@ int kint_attn_bwd(const float* Q, const float* K, const float* V, const float* O
     pf.tie_total = w.tie_total;
     pf.tie_list = w.tie_list;
     pf.tie_cap = BH * T;
+    pf.kt_out = w.kth;
     const bool ext = c.calib != KINT_CALIB_SOFTMAX && c.grad != KINT_GRAD_DETACH;
     if (!map_nat_sw64(&maps.dq16, dQ, BH, T, d, 16, 16) || !map_nat_sw64(&maps.dk32, dK, BH, T, d, 16, 32) ||
         !map_nat_sw64(&maps.dv32, dV, BH, T, d, 16, 32))

@@ -149,9 +149,11 @@ __device__ __forceinline__ void rowsum_red(const float (&v)[16], float* dst, siz
 // for tile u + 2 as soon as the element work of tile u is done, and that stage's Q^T | dO^T
 // half takes tile u + 1's tiles once dQ of tile u has read dS.  The item's V tile (A
 // operand of g^T) also stages the next item's K rows on their way into TMEM; its K^T tile
-// (B operand of dQ) stages the dV, dK rows of the epilogue (32 keys x 16 columns per warp,
-// 64-byte swizzle) for TMA stores; each compute warp has a 1 KB slice for its 16 rows x 16
-// columns of the dQ partial (64-byte swizzle), added to dQ by a TMA reduce.
+// (B operand of dQ), which the compute warps write from the K rows in TMEM, stages the dV,
+// dK rows of the epilogue (32 keys x 16 columns per warp, 64-byte swizzle) for TMA stores,
+// after which each warp writes its part of the next item's K^T there; each compute warp
+// has a 1 KB slice for its 16 rows x 16 columns of the dQ partial (64-byte swizzle), added
+// to dQ by a TMA reduce.
 // ---------------------------------------------------------------------------
 constexpr int NCOMP_F = 512;  // compute threads
 constexpr int MMA_WARP_F = NCOMP_F / 32, PRODUCER_WARP_F = NCOMP_F / 32 + 1, PRODUCER2_WARP_F = NCOMP_F / 32 + 2;
@@ -194,8 +196,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
   uint64_t* bar_ops = bars + 5 * NS + 7;     // the item's K rows in TMEM (the V buffer free)
   uint64_t* bar_v = bars + 5 * NS + 8;       // the item's V tile landed
   uint64_t* bar_vfree = bars + 5 * NS + 9;   // the item's last g^T completed
-  uint64_t* bar_kt = bars + 5 * NS + 10;     // the item's K^T tile landed
-  uint64_t* bar_ktfree = bars + 5 * NS + 11; // the item's dV, dK rows stored out of the K^T buffer
+  uint64_t* bar_kt = bars + 5 * NS + 10;     // the item's K^T tile written by every compute warp
   uint64_t* bar_drain = bars + 5 * NS + 12;  // the MMA warp's clean-up commit
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 5 * NS + 13);
   const int tid = threadIdx.x, warp = warp_id_uniform();
@@ -219,8 +220,7 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     mbar_init(bar_ops, NCOMP_F / 32);
     mbar_init(bar_v, 1);
     mbar_init(bar_vfree, 1);
-    mbar_init(bar_kt, 1);
-    mbar_init(bar_ktfree, NCOMP_F / 32);
+    mbar_init(bar_kt, NCOMP_F / 32);
     mbar_init(bar_drain, 1);
     fence_mbar_init();
   }
@@ -249,8 +249,8 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
     setmaxnreg_dec<REG_AUX_F>();
 
   // Two producer warps: PRODUCER_WARP_F loads the Q | dO halves with their records and the
-  // items' K rows and V tiles, PRODUCER2_WARP_F the Q^T | dO^T halves and the K^T tiles, so
-  // that neither kind of load waits behind the other's condition.
+  // items' K rows and V tiles, PRODUCER2_WARP_F the Q^T | dO^T halves, so that neither kind
+  // of load waits behind the other's condition.
   auto item_of = [&](int k, int& kb_, int& bh_) {
     const int it_ = sched_item(sch, k);
     kb_ = it_ / p.BH;
@@ -320,15 +320,8 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
   } else if (warp == PRODUCER2_WARP_F) {
     int gt = 0, n = 0;
     RingPos ld, nT;
-    int cT = 0, nkt = 0;
+    int cT = 0;
     bool ok = true;
-    auto load_kt = [&](int k) {
-      int kb_, bh_;
-      item_of(k, kb_, bh_);
-      mbar_arrive_expect_tx(bar_kt, 128 * D * 4);
-      load_rows_tile(sm + p.sm_kt, &maps.kt, bar_kt, 128, D, kb_ * 128, 0, bh_);
-      ++nkt;
-    };
     for (int item = sched_item(sch, n); item < p.nitems && ok; item = sched_item(sch, ++n)) {
       const int kb = item / p.BH, bh = item % p.BH;
       const int qt0 = (kb * 128) / BT, nit = nqt - qt0;
@@ -347,20 +340,10 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         load_rows_tile(dst + odOT, &maps.dot, bt, BT, D, q0, 0, bh);
         nT.next(NS);
         ++cT;
-        // this item's K^T, once the previous item's dV, dK rows have left the K^T buffer: before
-        // the next wait above, which waits for this item's first dQ product, which reads K^T
-        if (it == 0) {
-          if (n > 0 && !mbar_wait_warp(bar_ktfree, (n - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_SYNC)) {
-            ok = false;
-            break;
-          }
-          load_kt(n);
-        }
       }
     }
     // clean-up: the last loads issued have landed
     drain_ring(bar_fullT, nT, cT, NS, p.wait_ns, p.status);
-    if (nkt > 0) mbar_wait_warp(bar_kt, (nkt - 1) & 1, p.wait_ns, p.status, DEV_ERR_TIMEOUT_TMA);
   } else if (warp == MMA_WARP_F) {
     const uint8_t* st0 = sm + p.sm_stage0;
     const uint32_t idq = idesc_tf32(64, D, 0, 0);
@@ -448,6 +431,25 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(bar_ops);
     };
+    // The item's K^T tile (the B operand of every dQ product: 64 rows d, 128 keys, four 32-key
+    // panels under the 128-byte swizzle) from its K rows in TMEM: this thread's key (TMEM lane)
+    // at its 16 columns d = 16 cq .. 16 cq + 15, which in that layout are rows 16 cq + k of panel
+    // q4, the 2 KB of the warp's own epilogue slice.  Handed to the MMA warp through bar_kt.
+    auto kt_out = [&]() {
+      float v[16];
+      tmem_ld16(lane_addr(tmem, cK + 16 * cq), v);
+      tmem_ld_wait();
+      const uint32_t base = smem_u32(ostg) + (uint32_t)(lane & 3) * 4u;
+#pragma unroll
+      for (int k = 0; k < 16; ++k)
+        asm volatile("st.shared.f32 [%0], %1;" ::"r"(base + (uint32_t)k * (uint32_t)SW +
+                                                     ((((uint32_t)lane >> 2) ^ (uint32_t)(k & 7)) << 4)),
+                     "f"(v[k])
+                     : "memory");
+      fence_async_smem();  // read by the tensor core
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar_kt);
+    };
     // the dQ partial of tile q0 (this warp's 16 rows in its lanes 0..15, its 16 columns),
     // scaled, staged in the warp's slice and added to dQ by a TMA reduce
     auto dq_out = [&](int bh_, int q0) {
@@ -484,7 +486,10 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
         }
       }
     };
-    if (sched_item(sch, 0) < p.nitems) ops_to_tmem(0);
+    if (sched_item(sch, 0) < p.nitems) {
+      ops_to_tmem(0);
+      kt_out();
+    }
     constexpr bool half = fwm_like(CAL) && REC == REC_NEAREST;
     if constexpr (fwm_like(CAL)) {
       if (half && tid < 2 * Kq + 1 + kHalfTail)
@@ -605,7 +610,8 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
           tma_store_commit();
         }
         tma_store_wait_read();
-        if (lane == 0) mbar_arrive(bar_ktfree);
+        // the next item's K^T into the slice the stores have read (its K rows are in TMEM)
+        if (sched_item(sch, n + 1) < p.nitems) kt_out();
         tc_fence_before();
       }
     }
@@ -627,11 +633,34 @@ __global__ void __launch_bounds__(NTHR_FUSED, 1) k_bwd_fused(const __grid_consta
 // ---------------------------------------------------------------------------
 constexpr int EXT_TIE_BLOCKS = 64;
 
+// K^T [BH][64][Tp] (keys past T zero) for the two-pass kernels that run in place of the
+// single pass: 32-key blocks through a padded shared tile, grid-stride.
+__device__ void ext_kt_fallback(const Params& p) {
+  __shared__ float ts[32][65];
+  const int Tp = (p.T + 31) & ~31, ntb = Tp / 32, tid = threadIdx.x;
+  for (int u = blockIdx.x; u < p.BH * ntb; u += gridDim.x) {
+    const int bh = u / ntb, t0 = (u % ntb) * 32;
+    const int r = tid >> 3, c8 = (tid & 7) * 8;
+    const int t = t0 + r;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) ts[r][c8 + k] = t < p.T ? p.K[((size_t)bh * p.T + t) * 64 + c8 + k] : 0.f;
+    __syncthreads();
+    const int dd = tid >> 2, k8 = (tid & 3) * 8;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) p.kt_out[((size_t)bh * 64 + dd) * Tp + t0 + k8 + k] = ts[k8 + k][dd];
+    __syncthreads();
+  }
+}
+
 template <bool USE_M>
 __global__ void __launch_bounds__(256) k_bwd_ext(const Params p) {
   pdl_wait();
   pdl_trigger();
-  if (gated_off(p)) return;
+  if (gated_off(p)) {
+    // the two-pass kernels run instead of this pass's result: they read K^T
+    if (p.kt_out) ext_kt_fallback(p);
+    return;
+  }
   const int nrows = p.BH * p.T, l = threadIdx.x & 15, grp = threadIdx.x >> 4;
   const int nrb = (nrows + 63) / 64;
   if ((int)blockIdx.x < nrb) {

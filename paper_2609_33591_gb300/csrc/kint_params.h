@@ -97,6 +97,8 @@ struct Params {
   int* tie_total;
   int2* tie_list;           // [tie_cap] (row, key) pairs of tied maxima found by k_bwd_fused
   int tie_cap;
+  float* kt_out;            // [BH][d][Tp] K^T for the two-pass kernels, written by k_bwd_ext when the
+                            // single pass gives way to them (the single pass forms its K^T tiles itself)
   float* probe;             // [7][BH*T] geometry probe outputs
   uint8_t *bins, *ivals;
 };
