@@ -190,13 +190,18 @@ cudaError_t launch_prep(const PrepJobs& jobs, int BH, int T, int Tp, int d, bool
 // reaches their running extremum count the chunk's equal keys with a bit mask;
 // its lowest set bit is the lowest index.  Masked keys (j > i) take -inf / +inf.
 // MIN: also the minimum side, which only the MinMax grid spans (FWM and the softmax
-// comparator are anchored at M alone).
-template <bool DIAG, bool MIN>
+// comparator are anchored at M alone).  RAW: the scale is a power of two (d = 64: 2^-3), so
+// the chunk compares the unscaled dot products, whose order and equalities are those of
+// the scaled scores (exact scaling: only scores below 2^-123 in magnitude, subnormal after
+// scaling, could merge), and M, m are scaled once when the row is stored.
+template <bool DIAG, bool MIN, bool RAW>
 __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float scale, float& M, float& m,
                                             int& amax, int& amin, int& nmax, int& nmin) {
   float hi[16], lo[16];
+  if constexpr (!RAW) {
 #pragma unroll
-  for (int jj = 0; jj < 32; ++jj) v[jj] = __fmul_rn(v[jj], scale);
+    for (int jj = 0; jj < 32; ++jj) v[jj] = __fmul_rn(v[jj], scale);
+  }
 #pragma unroll
   for (int jj = 0; jj < 16; ++jj) {
     float a = v[jj], b = v[jj + 16], a2 = a, b2 = b;
@@ -259,7 +264,7 @@ __device__ __forceinline__ void stats_chunk(float (&v)[32], int j0, int i, float
 
 static dim3 launch_grid(const Params& p) { return dim3((unsigned)p.ngrid); }
 
-template <bool MIN>
+template <bool MIN, bool RAW>
 __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ Maps maps, const Params p,
                                                          const __grid_constant__ Sched sch) {
   uint8_t* sm = smem_base();
@@ -393,9 +398,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
           tmem_ld_wait();
           const int j0 = kb * 128 + c * 32;
           if (diag)
-            stats_chunk<true, MIN>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+            stats_chunk<true, MIN, RAW>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
           else
-            stats_chunk<false, MIN>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
+            stats_chunk<false, MIN, RAW>(v, j0, i, p.scale, M, m, amax, amin, nmax, nmin);
         }
         tc_fence_before();
         __syncwarp();
@@ -438,6 +443,10 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
           amin = -1;
           nmin = 0;
         }
+        if constexpr (RAW) {
+          M = __fmul_rn(M, p.scale);
+          m = __fmul_rn(m, p.scale);  // (+inf stays +inf when the minimum is not computed)
+        }
         const size_t rw = (size_t)bh * p.T + i;
         p.row_max[rw] = M;
         p.row_min[rw] = m;
@@ -455,7 +464,9 @@ __global__ void __launch_bounds__(NTHR, 2) k_fwd_stats(const __grid_constant__ M
 }
 
 cudaError_t launch_fwd_stats(const Maps& maps, const Params& p, int smem_bytes, cudaStream_t s, const Sched& sch) {
-  auto kern = p.calib == CAL_MINMAX ? k_fwd_stats<true> : k_fwd_stats<false>;
+  // d = 64: scale 1/8, a power of two (RAW)
+  auto kern = p.calib == CAL_MINMAX ? (p.d == 64 ? k_fwd_stats<true, true> : k_fwd_stats<true, false>)
+                                    : (p.d == 64 ? k_fwd_stats<false, true> : k_fwd_stats<false, false>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
   if (e != cudaSuccess) return e;
   return launch_pdl(kern, launch_grid(p), dim3(NTHR), smem_bytes, s, maps, p, sch);
