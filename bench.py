@@ -41,8 +41,8 @@ TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 : BF16 tensor rate of GB300 (1.
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of each kernel from
 # one ncu capture of this workload (profiles/traffic_gpt2_tf32.md), valid only for the
 # kernel sources they were taken from.
-TRAFFIC = {"src": "ee2ac705c39a31db", "k_prep": 89492947, "k_fwd_stats": 50400768, "k_fwd_main": 92099622,
-           "k_bwd_fused": 422984256, "k_bwd_ext": 73672499}
+TRAFFIC = {"src": "893f13747009898a", "k_prep": 65120486, "k_fwd_stats": 50400448, "k_fwd_main": 91583501,
+           "k_bwd_fused": 378647168, "k_bwd_ext": 73677402}
 
 
 def kernel_source_digest() -> str:
