@@ -178,8 +178,9 @@ int kint_attn_fwd(const float* Q, const float* K, const float* V, float* O, cons
  * over the (key block, query tile) pairs that adds its dQ partial sums, and then the
  * extremum terms, in fp32 in global memory: the order of those additions is not fixed,
  * so dQ (and dK under the extremum terms) may differ in the last bits from call to call.
- * Everything else, and calls where some row has tied maxima, runs two passes (dQ, then
- * dK/dV) whose results are bit-reproducible.
+ * Everything else, and calls whose rows hold more tied maximum keys in all than the call
+ * has rows (the single pass lists each tied key), runs two passes (dQ, then dK/dV) whose
+ * results are bit-reproducible.
  *   O        in:  forward output
  *   dO       in:  [B,H,T,d]
  *   st       in:  row statistics written by kint_attn_fwd
